@@ -1,0 +1,224 @@
+"""Plain CPU oracle of the Bi-GCN layer forward (Wang et al., CVPR 2021).
+
+TEST INFRASTRUCTURE. Only the tests, ``__graft_entry__.smoke()`` and the
+benchmark's CPU-baseline leg import this package; the product path never does,
+and the two share no code. The arithmetic lives in ``bigcn_oracle.c``; this
+module marshals numpy arrays into it and composes the steps in the paper's
+order:
+
+    step 1  centring (Sec. 6.2)            oracle_centre
+    step 2  F = sign(Y), row scale (Eq. 8, Eq. 7)       oracle_sign, oracle_row_scale
+    step 3  B = sign(W), column scale (Eq. 3, Eq. 4)    oracle_weight_binarize
+    step 4  zeta = alpha beta (F . B) (Eq. 11, Eq. 12)  oracle_binary_dot, oracle_zeta
+    step 5  H = A~ zeta (Eq. 13, Eq. 1)                 oracle_aggregate
+
+Naming follows the layer's C interface: ``alpha`` is the per-node scale (the
+paper's beta, Eq. 7) and ``beta`` the per-weight-column scale (the paper's
+alpha, Eq. 4). Floating-point results are float64; the only fp32 arithmetic is
+the centring, whose result decides the sign bits and so must round exactly as
+the kernel's does.
+"""
+from __future__ import annotations
+
+import ctypes
+import threading
+
+import numpy as np
+
+from . import build as _build
+
+_lib = None
+_lock = threading.Lock()
+
+_f32p = np.ctypeslib.ndpointer(np.float32, flags="C_CONTIGUOUS")
+_f64p = np.ctypeslib.ndpointer(np.float64, flags="C_CONTIGUOUS")
+_i8p = np.ctypeslib.ndpointer(np.int8, flags="C_CONTIGUOUS")
+_i32p = np.ctypeslib.ndpointer(np.int32, flags="C_CONTIGUOUS")
+_i64p = np.ctypeslib.ndpointer(np.int64, flags="C_CONTIGUOUS")
+_u64p = np.ctypeslib.ndpointer(np.uint64, flags="C_CONTIGUOUS")
+_vp = ctypes.c_void_p
+_i32 = ctypes.c_int32
+_i64 = ctypes.c_int64
+
+
+def lib() -> ctypes.CDLL:
+    """Load (building first if needed) the oracle's shared library."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            h = ctypes.CDLL(_build.build())
+            h.oracle_centre.argtypes = [_f32p, _i64, _i32, _i64, _vp, _vp, _f32p]
+            h.oracle_centre.restype = None
+            h.oracle_sign.argtypes = [_f32p, _i64, _i8p]
+            h.oracle_sign.restype = None
+            h.oracle_row_scale.argtypes = [_f32p, _i64, _i32, _f64p]
+            h.oracle_row_scale.restype = None
+            h.oracle_weight_binarize.argtypes = [_f32p, _i32, _i32, _i64, _i8p, _f64p]
+            h.oracle_weight_binarize.restype = None
+            h.oracle_pack.argtypes = [_i8p, _i64, _i32, _i32, _u64p]
+            h.oracle_pack.restype = None
+            h.oracle_binary_dot.argtypes = [_i8p, _i64, _i8p, _i32, _i32, _i32p]
+            h.oracle_binary_dot.restype = None
+            h.oracle_zeta.argtypes = [_i32p, _f64p, _f64p, _i64, _i32, _f64p]
+            h.oracle_zeta.restype = None
+            h.oracle_degree.argtypes = [_i64p, _i64, _f64p]
+            h.oracle_degree.restype = None
+            h.oracle_aggregate.argtypes = [_i64p, _i32p, _i64, _f64p, _i32, _vp, _i64,
+                                           _f64p, _vp]
+            h.oracle_aggregate.restype = ctypes.c_int
+            _lib = h
+    return _lib
+
+
+def words_for(K: int) -> int:
+    """Number of 64-bit words that hold K packed signs."""
+    return (int(K) + 63) // 64
+
+
+def _c(a, dtype):
+    return np.ascontiguousarray(a, dtype=dtype)
+
+
+# ---------------------------------------------------------------- step 1 ----
+def centre(X, s=None, t=None) -> np.ndarray:
+    """Sec. 6.2: Y = fmaf(X, s, t) per feature, fp32; identity when s is None."""
+    X = _c(X, np.float32)
+    N, K = X.shape
+    Y = np.empty((N, K), np.float32)
+    if s is None:
+        lib().oracle_centre(X, N, K, K, None, None, Y)
+    else:
+        s = _c(s, np.float32)
+        t = _c(t, np.float32)
+        assert s.shape == (K,) and t.shape == (K,)
+        lib().oracle_centre(X, N, K, K, s.ctypes.data, t.ctypes.data, Y)
+    return Y
+
+
+# ------------------------------------------------------------ steps 2, 3 ----
+def sign(V) -> np.ndarray:
+    """Eq. 3 / Eq. 8: +1 where v >= 0 (sign(0) = +1), else -1, as int8."""
+    V = _c(V, np.float32)
+    S = np.empty(V.shape, np.int8)
+    lib().oracle_sign(V.reshape(-1), V.size, S.reshape(-1))
+    return S
+
+
+def row_scale(Y) -> np.ndarray:
+    """Eq. 7 read as the mean |y| over the row's d_in entries (float64)."""
+    Y = _c(Y, np.float32)
+    N, K = Y.shape
+    alpha = np.empty(N, np.float64)
+    lib().oracle_row_scale(Y, N, K, alpha)
+    return alpha
+
+
+def weight_binarize(Wt):
+    """Eq. 3 and Eq. 4 on W (K x F): returns (SB as F x K int8, beta float64)."""
+    Wt = _c(Wt, np.float32)
+    K, F = Wt.shape
+    SB = np.empty((F, K), np.int8)
+    beta = np.empty(F, np.float64)
+    lib().oracle_weight_binarize(Wt, K, F, F, SB, beta)
+    return SB, beta
+
+
+def pack(S, words=None) -> np.ndarray:
+    """Store a +-1 matrix (n x K) in the interface's packed layout (n x words)."""
+    S = _c(S, np.int8)
+    n, K = S.shape
+    words = words_for(K) if words is None else int(words)
+    bits = np.empty((n, words), np.uint64)
+    lib().oracle_pack(S, n, K, words, bits)
+    return bits
+
+
+# ---------------------------------------------------------------- step 4 ----
+def binary_dot(SF, SB) -> np.ndarray:
+    """Eq. 11's inner products F_i . B_j of +-1 vectors (int32, N x F)."""
+    SF = _c(SF, np.int8)
+    SB = _c(SB, np.int8)
+    N, K = SF.shape
+    F, K2 = SB.shape
+    assert K == K2
+    dot = np.empty((N, F), np.int32)
+    lib().oracle_binary_dot(SF, N, SB, F, K, dot)
+    return dot
+
+
+def zeta(dot, alpha, beta) -> np.ndarray:
+    """Eq. 11/12: zeta_ij = alpha_i beta_j dot_ij (float64)."""
+    dot = _c(dot, np.int32)
+    N, F = dot.shape
+    out = np.empty((N, F), np.float64)
+    lib().oracle_zeta(dot, _c(alpha, np.float64), _c(beta, np.float64), N, F, out)
+    return out
+
+
+# ---------------------------------------------------------------- step 5 ----
+def degree(rowptr) -> np.ndarray:
+    """Sec. 3.1: dhat_i = 1 + |N(i)| (the self-loop of A + I included)."""
+    rowptr = _c(rowptr, np.int64)
+    N = rowptr.shape[0] - 1
+    d = np.empty(N, np.float64)
+    lib().oracle_degree(rowptr, N, d)
+    return d
+
+
+def aggregate(rowptr, colidx, zeta_, rows=None, with_absterm=False):
+    """Eq. 13: H = A~ zeta with A~ = D^-1/2 (A + I) D^-1/2 (Eq. 1), float64.
+
+    ``rows`` restricts the output to those rows (in that order). With
+    ``with_absterm`` also returns the per-element sum of |terms|.
+    """
+    rowptr = _c(rowptr, np.int64)
+    colidx = _c(colidx, np.int32)
+    z = _c(zeta_, np.float64)
+    N = rowptr.shape[0] - 1
+    assert z.shape[0] == N
+    F = z.shape[1]
+    if rows is None:
+        rows_arr, nrows, rows_ptr = None, N, None
+    else:
+        rows_arr = _c(rows, np.int64)
+        nrows = rows_arr.shape[0]
+        rows_ptr = rows_arr.ctypes.data
+    H = np.empty((nrows, F), np.float64)
+    A = np.empty((nrows, F), np.float64) if with_absterm else None
+    if colidx.size == 0:
+        colidx = np.zeros(1, np.int32)  # a valid pointer; never read when nnz == 0
+    rc = lib().oracle_aggregate(rowptr, colidx, N, z, F, rows_ptr, nrows, H,
+                                None if A is None else A.ctypes.data)
+    if rc != 0:
+        raise ValueError("malformed CSR or row index")
+    return (H, A) if with_absterm else H
+
+
+# ----------------------------------------------------------- composition ----
+def layer_forward(X, Wt, rowptr, colidx, s=None, t=None, rows=None) -> dict:
+    """One binarized graph-convolution layer, Eq. 10-13, every step kept.
+
+    With ``rows`` only the aggregation is restricted to those rows; every
+    other step runs on all N rows (the aggregation reads zeta of neighbours).
+    """
+    Y = centre(X, s, t)
+    SF = sign(Y)
+    alpha = row_scale(Y)
+    SB, beta = weight_binarize(Wt)
+    dot = binary_dot(SF, SB)
+    z = zeta(dot, alpha, beta)
+    H, absterm = aggregate(rowptr, colidx, z, rows=rows, with_absterm=True)
+    return dict(Y=Y, SF=SF, alpha=alpha, bits=pack(SF), SB=SB, beta=beta,
+                wbits=pack(SB), dot=dot, zeta=z, H=H, absterm=absterm)
+
+
+def forward_2layer(X, s, t, W1, W2, rowptr, colidx) -> dict:
+    """The 2-layer Bi-GCN of Sec. 6.2: layer 1 centred, layer 2 on H1 raw.
+
+    The layer interface carries fp32, so H1 is rounded to fp32 before it
+    becomes layer 2's input (no activation between layers, Sec. 4.1.2).
+    """
+    l1 = layer_forward(X, W1, rowptr, colidx, s, t)
+    H1 = l1["H"].astype(np.float32)
+    l2 = layer_forward(H1, W2, rowptr, colidx)
+    return dict(layer1=l1, layer2=l2, H1=H1, logits=l2["H"])

@@ -1,0 +1,81 @@
+/*
+ * bigcn_oracle.h -- plain CPU oracle of the Bi-GCN binarized graph-convolution
+ * layer forward (Wang et al., "Bi-GCN: Binary Graph Convolutional Network",
+ * CVPR 2021, arXiv:2010.07565).
+ *
+ * TEST INFRASTRUCTURE. Only the test suite, the smoke check and the
+ * benchmark's CPU-baseline leg load this library. It shares no source, header,
+ * table or helper with the CUDA path, and the CUDA path never calls it.
+ *
+ * Every routine is a slow, element-by-element restatement of one definition of
+ * the paper, in its order, with floating point carried in double except where
+ * a decision (a sign bit) must be taken in the same fp32 precision as the
+ * kernel. All arrays are host memory owned by the caller; row-major.
+ *
+ * Naming: this library follows the naming of the layer's C interface, which
+ * swaps the paper's letters. Here alpha_i is the per-NODE scale (the paper's
+ * beta_i, Eq. 7) and beta_j is the per-WEIGHT-COLUMN scale (the paper's
+ * alpha_j, Eq. 4).
+ */
+#ifndef BIGCN_ORACLE_H
+#define BIGCN_ORACLE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Step 1 -- input batch normalisation in inference form (Sec. 6.2):
+ * Y[i,k] = fmaf(X[i,k], s[k], t[k]) in fp32, one rounding. s == t == NULL
+ * means the identity (layer 2 binarizes its input raw, Sec. 4.1.2). */
+void oracle_centre(const float *X, int64_t N, int32_t K, int64_t ldx,
+                   const float *s, const float *t, float *Y);
+
+/* Eq. 8 (F_i = sign(H_i,:)) and Eq. 3 (B_j = sign(W_:,j)): +1 where v >= 0
+ * (so sign(0) = sign(-0) = +1), else -1. */
+void oracle_sign(const float *V, int64_t n, int8_t *S);
+
+/* Eq. 7 read as mean |y_i| (the bucket is the whole row, Sec. 4.1):
+ * alpha[i] = (sum_k |Y[i,k]|) / K, summed in double. */
+void oracle_row_scale(const float *Y, int64_t N, int32_t K, double *alpha);
+
+/* Eq. 3 and Eq. 4 for the weight matrix Wt (K x F, row stride ldw):
+ * SB[j,k] = sign(Wt[k,j]) (F x K, i.e. transposed) and
+ * beta[j] = (sum_k |Wt[k,j]|) / K in double. */
+void oracle_weight_binarize(const float *Wt, int32_t K, int32_t F, int64_t ldw,
+                            int8_t *SB, double *beta);
+
+/* Storage of a sign matrix S (n x K, entries +-1) in the interface's packed
+ * layout: element k of row r is bit (k % 64) of 64-bit word r*words + k/64,
+ * set for +1; bits at k >= K are 0. */
+void oracle_pack(const int8_t *S, int64_t n, int32_t K, int32_t words,
+                 uint64_t *bits);
+
+/* Eq. 11, the integer part: dot[i,j] = sum_k SF[i,k] * SB[j,k]. */
+void oracle_binary_dot(const int8_t *SF, int64_t N, const int8_t *SB, int32_t F,
+                       int32_t K, int32_t *dot);
+
+/* Eq. 11/12, the scaled result: zeta[i,j] = alpha[i] * beta[j] * dot[i,j]. */
+void oracle_zeta(const int32_t *dot, const double *alpha, const double *beta,
+                 int64_t N, int32_t F, double *zeta);
+
+/* Sec. 3.1: dhat[i] = sum_j ahat[i,j] with Ahat = A + I and a_ij = 1 on the
+ * CSR's entries, i.e. 1 + (rowptr[i+1] - rowptr[i]). */
+void oracle_degree(const int64_t *rowptr, int64_t N, double *dhat);
+
+/* Eq. 13 with Eq. 1's operator: H[r,:] = sum over j in N(i) u {i} of
+ * zeta[j,:] / sqrt(dhat_i * dhat_j), for each requested row i = rows[r]
+ * (rows == NULL: all N rows, r = i). absterm[r,:] (nullable) receives the sum
+ * of the absolute values of the same terms, the scale of the rounding error
+ * of any evaluation order. Returns 0, or -1 if the CSR is malformed (rowptr
+ * not monotone from 0 to its end, or a column index outside [0, N)). */
+int oracle_aggregate(const int64_t *rowptr, const int32_t *colidx, int64_t N,
+                     const double *zeta, int32_t F, const int64_t *rows,
+                     int64_t nrows, double *H, double *absterm);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BIGCN_ORACLE_H */
