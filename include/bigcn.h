@@ -1,0 +1,195 @@
+/*
+ * bigcn.h -- C interface of the GB300 (sm_103a) Bi-GCN layer forward.
+ *
+ * Bi-GCN (Wang et al., "Bi-GCN: Binary Graph Convolutional Network", CVPR
+ * 2021, arXiv:2010.07565) replaces the feature-extraction product H W of a
+ * graph-convolution layer (Eq. 1) by a product of sign matrices scaled per
+ * row and per column (Eqs. 10-12), then aggregates with the normalised
+ * adjacency (Eq. 13). One layer is five steps, each one call below:
+ *
+ *   1+2  bigcn_pack_rows     centre (Sec. 6.2), sign-pack rows, row scale (Eqs. 7-8)
+ *   3    bigcn_pack_weights  sign-pack weight columns, column scale (Eqs. 3-4)
+ *   4    bigcn_xnor_gemm     XNOR/popcount product, scaled (Eqs. 11-12)
+ *   5    bigcn_spmm_norm     H = D^-1/2 (A + I) D^-1/2 Z (Eqs. 1, 13)
+ *        bigcn_layer_forward all five, fused where the layout allows
+ *
+ * Naming. The interface follows the layer's own naming, which swaps the
+ * paper's letters: alpha_i is the per-NODE scale (the paper's beta_i, Eq. 7)
+ * and beta_j is the per-WEIGHT-COLUMN scale (the paper's alpha_j, Eq. 4).
+ * Both scales are the mean absolute value over the d_in = K entries of the
+ * row / column (the least-squares optimum of the sign approximation; Eq. 4
+ * and Eq. 7 as printed divide by d_out and N, which is read as a misprint).
+ *
+ * Conventions for every call:
+ *  - Array pointers are DEVICE pointers owned by the caller. The library
+ *    allocates no memory and keeps no state besides a per-device cache of
+ *    the device's properties.
+ *  - Every call is asynchronous on `stream` (a cudaStream_t; NULL = the
+ *    legacy default stream). Outputs are valid once the stream reaches the
+ *    call; inputs must stay valid until then.
+ *  - Matrices are row-major with a leading dimension (row stride) in
+ *    elements. Pointers must be aligned to their element size; faster
+ *    vectorised paths are chosen internally when alignment allows.
+ *  - Argument errors are detected on the host before any launch; the
+ *    outputs are then untouched and nothing is enqueued.
+ *  - Packed sign layout: element k of a packed row is bit (k % 64) of the
+ *    row's 64-bit word k / 64, set for +1 and clear for -1, with
+ *    sign(v) = +1 for v >= 0 (so +0 and -0 give +1; NaN gives -1). Rows
+ *    hold `words` >= ceil(K / 64) words; every bit at k >= K is written 0.
+ *  - Floating point is IEEE fp32 with round-to-nearest; the centring is one
+ *    fused multiply-add, so the sign bits are reproducible bit for bit.
+ *  - NaN or infinite inputs are not supported (results are unspecified, but
+ *    every access stays in bounds).
+ */
+#ifndef BIGCN_H
+#define BIGCN_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum bigcn_status {
+    BIGCN_OK = 0,
+    BIGCN_ERR_INVALID_ARG = 1,  /* null pointer, bad size, aliasing, short workspace */
+    BIGCN_ERR_MISALIGNED = 2,   /* a pointer not aligned as documented */
+    BIGCN_ERR_CUDA = 3,         /* a CUDA runtime error (launch or device query) */
+    BIGCN_ERR_UNSUPPORTED = 4   /* the current device is not sm_103 */
+} bigcn_status;
+
+/* Human-readable name of a status code (static storage; never NULL). */
+const char *bigcn_status_string(int status);
+
+/* ceil(K / 64): the minimum `words` of a packed row of K signs (0 if K <= 0). */
+int32_t bigcn_words(int32_t K);
+
+/*
+ * Steps 1+2. Centring (Sec. 6.2: batch normalisation of the input features,
+ * inference form, as one fp32 fma per element) fused with the sign
+ * binarization of node features (Eq. 8) and the per-node scale (Eq. 7):
+ *
+ *   y[i,k]    = fmaf(X[i,k], scale[k], shift[k])   (y = X if both are NULL)
+ *   bits[i]   = packed sign(y[i,:])
+ *   alpha[i]  = (1/K) sum_k |y[i,k]|
+ *
+ * X      N x K fp32, row stride ldx >= K.
+ * scale, shift  K fp32 each, or both NULL (identity: layer 2 and beyond
+ *        binarize their input raw, Sec. 4.1.2). Exactly one NULL is an error.
+ * bits   N x words uint64, row stride `words` >= ceil(K/64).
+ * alpha  N fp32.
+ * N >= 0 (N == 0 enqueues nothing), 1 <= K, N * ldx and N * words < 2^62.
+ */
+bigcn_status bigcn_pack_rows(const float *X, int64_t N, int32_t K, int64_t ldx,
+                             const float *scale, const float *shift,
+                             uint64_t *bits, int32_t words, float *alpha,
+                             void *stream);
+
+/*
+ * Step 3. Sign binarization of the weight columns (Eq. 3) and the
+ * per-column scale (Eq. 4):
+ *
+ *   bits[j]  = packed sign(Wt[:, j])   (column j becomes packed row j)
+ *   beta[j]  = (1/K) sum_k |Wt[k, j]|
+ *
+ * Wt     K x F fp32 (the layer's W, d_in x d_out), row stride ldw >= F.
+ * bits   F x words uint64, words >= ceil(K/64).   beta  F fp32.
+ * 1 <= K, 1 <= F.
+ */
+bigcn_status bigcn_pack_weights(const float *Wt, int32_t K, int32_t F, int64_t ldw,
+                                uint64_t *bits, int32_t words, float *beta,
+                                void *stream);
+
+/*
+ * Step 4. The binary feature extraction of Eqs. 11-12: the +-1 inner
+ * product of packed row i of A with packed row j of B, evaluated as
+ *
+ *   dot[i,j] = K - 2 popcount(a_i XOR b_j)       (= sum_k sign * sign)
+ *   Z[i,j]   = (alpha[i] * beta[j]) * (float)dot[i,j]
+ *
+ * a_bits N x words, alpha N;  b_bits F x words, beta F (from the two pack
+ * calls, same K and words; all bits at k >= K must be 0, as they write).
+ * Z      N x F fp32, row stride ldz >= F.
+ * dots   nullable; if given, N x F int32 (row stride F) receives dot.
+ * 0 <= N, 1 <= F, 1 <= K <= 64 * words. Z must not overlap the inputs.
+ */
+bigcn_status bigcn_xnor_gemm(const uint64_t *a_bits, const float *alpha, int64_t N,
+                             const uint64_t *b_bits, const float *beta, int32_t F,
+                             int32_t K, int32_t words, float *Z, int64_t ldz,
+                             int32_t *dots, void *stream);
+
+/*
+ * Step 5. Aggregation with the normalised adjacency of Eq. 1 (Eq. 13):
+ *
+ *   H[i,:] = sum over j in N(i) u {i} of Z[j,:] / sqrt(dhat_i * dhat_j),
+ *   dhat_i = 1 + (rowptr[i+1] - rowptr[i])     (A + I, Sec. 3.1)
+ *
+ * rowptr N+1 int64, colidx nnz int32: the CSR of A, unweighted, without
+ *        self-loops (the call adds I). Symmetry is the caller's contract;
+ *        the formula is evaluated for any CSR. rowptr[0] = 0,
+ *        rowptr[N] = nnz, non-decreasing, 0 <= colidx < N. The kernel
+ *        clamps row ranges to [0, nnz] and skips out-of-range column
+ *        indices, so a malformed CSR gives wrong numbers, never a fault.
+ * Z      N x F fp32, row stride ldz >= F.   H  N x F fp32, stride ldh >= F.
+ * 0 <= N < 2^31, 0 <= nnz, 1 <= F. H must not overlap Z.
+ */
+bigcn_status bigcn_spmm_norm(const int64_t *rowptr, const int32_t *colidx,
+                             int64_t N, int64_t nnz, const float *Z, int64_t ldz,
+                             int32_t F, float *H, int64_t ldh, void *stream);
+
+/*
+ * Steps 4 and 5 with the degree normalisation split between them, as
+ * bigcn_layer_forward runs them: D^-1/2 (A + I) D^-1/2 Z = D^-1/2 (A + I) Z'
+ * with Z' = D^-1/2 Z (Eq. 1). bigcn_xnor_gemm_degscaled writes
+ *
+ *   Z'[i,j] = (alpha[i] * (1 / sqrt(dhat_i))) * (beta[j] * (float)dot[i,j]),
+ *   dhat_i  = 1 + rowptr[i+1] - rowptr[i],
+ *
+ * and bigcn_spmm_prescaled then computes
+ *
+ *   H[i,:] = (1 / sqrt(dhat_i)) * sum over j in N(i) u {i} of Z'[j,:],
+ *
+ * which saves the aggregation one random read of the row pointers per edge.
+ * Arguments, layouts and errors are those of bigcn_xnor_gemm (plus `rowptr`,
+ * N+1 int64, required) and of bigcn_spmm_norm.
+ */
+bigcn_status bigcn_xnor_gemm_degscaled(const uint64_t *a_bits, const float *alpha, int64_t N,
+                                       const uint64_t *b_bits, const float *beta, int32_t F,
+                                       int32_t K, int32_t words, const int64_t *rowptr,
+                                       float *Z, int64_t ldz, void *stream);
+
+bigcn_status bigcn_spmm_prescaled(const int64_t *rowptr, const int32_t *colidx,
+                                  int64_t N, int64_t nnz, const float *Z, int64_t ldz,
+                                  int32_t F, float *H, int64_t ldh, void *stream);
+
+/* Bytes of device workspace bigcn_layer_forward needs for (N, K, F); 0 on
+ * invalid sizes. */
+size_t bigcn_layer_workspace_bytes(int64_t N, int32_t K, int32_t F);
+
+/*
+ * One binarized graph-convolution layer, H = A~ zeta (Eq. 13), with zeta from
+ * the centred (scale/shift, as in bigcn_pack_rows) and binarized X and the
+ * binarized W (Eqs. 3-12). The result equals the composition of the four
+ * calls above within fp32 rounding; it runs exactly bigcn_pack_rows,
+ * bigcn_pack_weights, bigcn_xnor_gemm_degscaled and bigcn_spmm_prescaled on
+ * `stream`. No activation follows (Sec. 4.1.2).
+ *
+ * X N x K (ldx), Wt K x F (ldw), CSR as in bigcn_spmm_norm, H N x F (ldh).
+ * workspace  device memory of at least bigcn_layer_workspace_bytes(N, K, F)
+ *            bytes, 256-byte aligned, not overlapping any argument; its
+ *            contents on entry do not matter and on exit are unspecified.
+ * H must not overlap the workspace; it may not be X either.
+ */
+bigcn_status bigcn_layer_forward(const float *X, int64_t N, int32_t K, int64_t ldx,
+                                 const float *scale, const float *shift,
+                                 const float *Wt, int32_t F, int64_t ldw,
+                                 const int64_t *rowptr, const int32_t *colidx,
+                                 int64_t nnz, void *workspace, size_t ws_bytes,
+                                 float *H, int64_t ldh, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BIGCN_H */

@@ -1,0 +1,62 @@
+// Internal helpers shared by the Bi-GCN CUDA translation units: argument
+// checks, the per-device property cache, launch-status mapping and warp-level
+// reductions. Not part of the public interface (include/bigcn.h).
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <cstddef>
+#include <cstdint>
+
+#include "bigcn.h"
+
+namespace bigcn {
+
+constexpr unsigned kFullMask = 0xffffffffu;
+constexpr int64_t kMaxElems = int64_t(1) << 62;
+
+struct DeviceInfo {
+    int device;
+    int sm_count;
+    int max_smem_optin;  // bytes of shared memory a block may opt in to
+};
+
+// Properties of the current device, queried once per device and cached.
+// Returns BIGCN_ERR_UNSUPPORTED unless the device is sm_103.
+bigcn_status current_device(DeviceInfo *info);
+
+// Maps the launch result (cudaGetLastError) to a status.
+bigcn_status launch_status();
+
+inline bool aligned_to(const void *p, size_t a) {
+    return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0;
+}
+
+// True when the byte ranges [a, a + na) and [b, b + nb) intersect.
+inline bool overlaps(const void *a, size_t na, const void *b, size_t nb) {
+    if (a == nullptr || b == nullptr || na == 0 || nb == 0) return false;
+    uintptr_t pa = reinterpret_cast<uintptr_t>(a), pb = reinterpret_cast<uintptr_t>(b);
+    return pa < pb + nb && pb < pa + na;
+}
+
+// Bytes spanned by a rows x cols matrix of elem-byte elements with row stride ld.
+inline size_t span_bytes(int64_t rows, int64_t cols, int64_t ld, size_t elem) {
+    if (rows <= 0 || cols <= 0) return 0;
+    return size_t((rows - 1) * ld + cols) * elem;
+}
+
+inline cudaStream_t as_stream(void *s) { return reinterpret_cast<cudaStream_t>(s); }
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFullMask, v, o);
+    return v;
+}
+
+// 1 / sqrt(1 + row length): the D^-1/2 factor of A + I (Sec. 3.1, Eq. 1),
+// with IEEE-rounded sqrt and division.
+__device__ __forceinline__ float inv_sqrt_degree(int64_t row_len) {
+    return 1.0f / sqrtf(1.0f + float(row_len));
+}
+
+}  // namespace bigcn

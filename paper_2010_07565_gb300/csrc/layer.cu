@@ -1,0 +1,154 @@
+// The fused Bi-GCN layer (Wang et al., CVPR 2021, Eq. 13 with zeta from
+// Eqs. 11-12) and the interface's small helpers: status strings, the packed
+// row width, the per-device property cache and the workspace layout.
+//
+// bigcn_layer_forward enqueues, on one stream:
+//   pack_rows (centre + sign + alpha) -> pack_weights (sign + beta)
+//   -> xnor_gemm whose epilogue also multiplies row j by 1/sqrt(dhat_j)
+//   -> spmm over the pre-scaled rows, which multiplies by 1/sqrt(dhat_i).
+// Folding the source-side degree factor into the product's epilogue saves the
+// aggregation one random read of the CSR row pointers per edge.
+#include <mutex>
+
+#include "launch.cuh"
+
+namespace bigcn {
+
+namespace {
+constexpr int kMaxDevices = 64;
+DeviceInfo g_info[kMaxDevices];
+bigcn_status g_info_status[kMaxDevices];
+std::once_flag g_info_once[kMaxDevices];
+
+void query_device(int dev) {
+    DeviceInfo &d = g_info[dev];
+    d.device = dev;
+    int major = 0, minor = 0;
+    if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&d.sm_count, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&d.max_smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) !=
+            cudaSuccess) {
+        cudaGetLastError();
+        g_info_status[dev] = BIGCN_ERR_CUDA;
+        return;
+    }
+    g_info_status[dev] = (major == 10 && minor == 3) ? BIGCN_OK : BIGCN_ERR_UNSUPPORTED;
+}
+
+constexpr size_t kAlign = 256;
+size_t round_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+
+// Workspace carve-up of the fused layer; every piece 256-byte aligned.
+struct LayerWorkspace {
+    size_t a_bits, alpha, b_bits, beta, z, total;
+};
+
+bool layer_workspace(int64_t N, int32_t K, int32_t F, LayerWorkspace *w) {
+    if (N < 0 || K < 1 || F < 1) return false;
+    const int64_t words = bigcn_words(K);
+    if (N > kMaxElems / (words > F ? words : F)) return false;
+    size_t off = 0;
+    w->a_bits = off; off = round_up(off + size_t(N) * size_t(words) * 8);
+    w->alpha = off;  off = round_up(off + size_t(N) * 4);
+    w->b_bits = off; off = round_up(off + size_t(F) * size_t(words) * 8);
+    w->beta = off;   off = round_up(off + size_t(F) * 4);
+    w->z = off;      off = round_up(off + size_t(N) * size_t(F) * 4);
+    w->total = off;
+    return true;
+}
+}  // namespace
+
+bigcn_status current_device(DeviceInfo *info) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        cudaGetLastError();
+        return BIGCN_ERR_CUDA;
+    }
+    if (dev < 0 || dev >= kMaxDevices) return BIGCN_ERR_UNSUPPORTED;
+    std::call_once(g_info_once[dev], query_device, dev);
+    if (g_info_status[dev] != BIGCN_OK) return g_info_status[dev];
+    *info = g_info[dev];
+    return BIGCN_OK;
+}
+
+bigcn_status launch_status() {
+    return cudaGetLastError() == cudaSuccess ? BIGCN_OK : BIGCN_ERR_CUDA;
+}
+
+}  // namespace bigcn
+
+using namespace bigcn;
+
+extern "C" const char *bigcn_status_string(int status) {
+    switch (status) {
+        case BIGCN_OK: return "BIGCN_OK";
+        case BIGCN_ERR_INVALID_ARG: return "BIGCN_ERR_INVALID_ARG";
+        case BIGCN_ERR_MISALIGNED: return "BIGCN_ERR_MISALIGNED";
+        case BIGCN_ERR_CUDA: return "BIGCN_ERR_CUDA";
+        case BIGCN_ERR_UNSUPPORTED: return "BIGCN_ERR_UNSUPPORTED";
+        default: return "BIGCN_ERR_UNKNOWN";
+    }
+}
+
+extern "C" int32_t bigcn_words(int32_t K) { return K <= 0 ? 0 : int32_t((int64_t(K) + 63) / 64); }
+
+extern "C" size_t bigcn_layer_workspace_bytes(int64_t N, int32_t K, int32_t F) {
+    LayerWorkspace w;
+    return layer_workspace(N, K, F, &w) ? w.total : 0;
+}
+
+extern "C" bigcn_status bigcn_layer_forward(const float *X, int64_t N, int32_t K, int64_t ldx,
+                                            const float *scale, const float *shift,
+                                            const float *Wt, int32_t F, int64_t ldw,
+                                            const int64_t *rowptr, const int32_t *colidx,
+                                            int64_t nnz, void *workspace, size_t ws_bytes,
+                                            float *H, int64_t ldh, void *stream) {
+    LayerWorkspace w;
+    if (N < 0 || N > int64_t(INT32_MAX) || K < 1 || F < 1 || ldx < K || ldw < F || ldh < F ||
+        nnz < 0)
+        return BIGCN_ERR_INVALID_ARG;
+    if ((scale == nullptr) != (shift == nullptr)) return BIGCN_ERR_INVALID_ARG;
+    if (!layer_workspace(N, K, F, &w)) return BIGCN_ERR_INVALID_ARG;
+    if (N > 0 && (N > kMaxElems / ldx || N > kMaxElems / ldh)) return BIGCN_ERR_INVALID_ARG;
+    if (int64_t(K) > kMaxElems / ldw) return BIGCN_ERR_INVALID_ARG;
+    if (N == 0) return BIGCN_OK;
+    if (!X || !Wt || !rowptr || !H || !workspace || (nnz > 0 && !colidx))
+        return BIGCN_ERR_INVALID_ARG;
+    if (ws_bytes < w.total) return BIGCN_ERR_INVALID_ARG;
+    if (!aligned_to(X, 4) || !aligned_to(Wt, 4) || !aligned_to(rowptr, 8) ||
+        (colidx && !aligned_to(colidx, 4)) || !aligned_to(H, 4) || !aligned_to(workspace, kAlign) ||
+        (scale && (!aligned_to(scale, 4) || !aligned_to(shift, 4))))
+        return BIGCN_ERR_MISALIGNED;
+    const size_t xb = span_bytes(N, K, ldx, 4), hb = span_bytes(N, F, ldh, 4);
+    const size_t wb = span_bytes(K, F, ldw, 4);
+    const void *inputs[] = {X, Wt, rowptr, colidx, scale, shift};
+    const size_t in_bytes[] = {xb, wb, size_t(N + 1) * 8, size_t(nnz) * 4, size_t(K) * 4,
+                               size_t(K) * 4};
+    for (int q = 0; q < 6; ++q) {
+        if (overlaps(workspace, w.total, inputs[q], in_bytes[q])) return BIGCN_ERR_INVALID_ARG;
+        if (overlaps(H, hb, inputs[q], in_bytes[q])) return BIGCN_ERR_INVALID_ARG;
+    }
+    if (overlaps(H, hb, workspace, w.total)) return BIGCN_ERR_INVALID_ARG;
+
+    DeviceInfo dev;
+    bigcn_status st = current_device(&dev);
+    if (st != BIGCN_OK) return st;
+
+    char *ws = static_cast<char *>(workspace);
+    uint64_t *a_bits = reinterpret_cast<uint64_t *>(ws + w.a_bits);
+    float *alpha = reinterpret_cast<float *>(ws + w.alpha);
+    uint64_t *b_bits = reinterpret_cast<uint64_t *>(ws + w.b_bits);
+    float *beta = reinterpret_cast<float *>(ws + w.beta);
+    float *Zs = reinterpret_cast<float *>(ws + w.z);
+    const int words = bigcn_words(K);
+    cudaStream_t s = as_stream(stream);
+
+    launch_pack_rows(X, N, K, ldx, scale, shift, a_bits, words, alpha, dev, s);
+    launch_pack_weights(Wt, K, F, ldw, b_bits, words, beta, s);
+    GemmArgs g{a_bits, alpha, N, b_bits, beta, F, K, words, Zs, F, nullptr, rowptr};
+    launch_xnor_gemm(g, dev, s);
+    SpmmArgs a{rowptr, colidx, N, nnz, Zs, F, F, H, ldh, true};
+    launch_spmm_norm(a, dev, s);
+    return launch_status();
+}

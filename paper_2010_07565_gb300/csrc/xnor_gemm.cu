@@ -1,0 +1,203 @@
+// Step 4 of the Bi-GCN layer forward (Wang et al., CVPR 2021, Eqs. 11-12):
+// the +-1 inner products of packed node rows with packed weight columns,
+//   dot[i,j] = K - 2 popcount(a_i XOR b_j),  Z[i,j] = alpha_i beta_j dot[i,j].
+//
+// CUDA-core path: a 128 x (16*TN) output tile per 256-thread block, the two
+// packed operand tiles staged in shared memory 8 words (512 signs) at a time
+// with register double buffering; each thread accumulates TM x TN mismatch
+// counts with XOR + POPC. Thread (tx, ty) owns rows ty + 16 i and columns
+// tx + 16 j, which keeps the shared-memory reads free of bank conflicts (odd
+// row pitch) and the Z stores coalesced along the columns.
+//
+// The epilogue optionally multiplies row i by dinv_i = 1/sqrt(1 + deg_i), the
+// source-side factor of D^-1/2 (A + I) D^-1/2, so that the aggregation that
+// follows in the fused layer reads pre-scaled rows.
+#include "launch.cuh"
+
+namespace bigcn {
+namespace {
+
+constexpr int kBM = 128;     // rows per block tile
+constexpr int kBKW = 8;      // 64-bit words per k-step
+constexpr int kPitch = kBKW + 1;
+constexpr int kTM = 8;       // rows per thread
+constexpr int kThreads = 256;
+
+template <int TN, bool kDegreeScale>
+__global__ void __launch_bounds__(kThreads)
+xnor_gemm_popc_kernel(const uint64_t *__restrict__ A, const float *__restrict__ alpha, int64_t N,
+                      const uint64_t *__restrict__ B, const float *__restrict__ beta, int F,
+                      int K, int words, float *__restrict__ Z, int64_t ldz,
+                      int32_t *__restrict__ dots, const int64_t *__restrict__ rowptr) {
+    constexpr int BN = 16 * TN;
+    constexpr int kALoads = kBM * kBKW / kThreads;                         // 4
+    constexpr int kBLoads = (BN * kBKW + kThreads - 1) / kThreads;          // 1..2
+    __shared__ uint64_t As[kBM][kPitch];
+    __shared__ uint64_t Bs[BN][kPitch];
+
+    const int tid = threadIdx.x;
+    const int tx = tid & 15, ty = tid >> 4;
+    const int64_t m0 = int64_t(blockIdx.x) * kBM;
+    const int n0 = blockIdx.y * BN;
+
+    uint64_t ra[kALoads], rb[kBLoads];
+    auto load_tile = [&](int k0) {
+#pragma unroll
+        for (int q = 0; q < kALoads; ++q) {
+            const int e = tid + q * kThreads;
+            const int r = e / kBKW, kw = e % kBKW;
+            const int64_t row = m0 + r;
+            ra[q] = (row < N && k0 + kw < words) ? __ldg(A + row * words + k0 + kw) : 0ull;
+        }
+#pragma unroll
+        for (int q = 0; q < kBLoads; ++q) {
+            const int e = tid + q * kThreads;
+            const int c = e / kBKW, kw = e % kBKW;
+            rb[q] = (e < BN * kBKW && n0 + c < F && k0 + kw < words)
+                        ? __ldg(B + int64_t(n0 + c) * words + k0 + kw) : 0ull;
+        }
+    };
+    auto store_tile = [&]() {
+#pragma unroll
+        for (int q = 0; q < kALoads; ++q) {
+            const int e = tid + q * kThreads;
+            As[e / kBKW][e % kBKW] = ra[q];
+        }
+#pragma unroll
+        for (int q = 0; q < kBLoads; ++q) {
+            const int e = tid + q * kThreads;
+            if (e < BN * kBKW) Bs[e / kBKW][e % kBKW] = rb[q];
+        }
+    };
+
+    int mism[kTM][TN];
+#pragma unroll
+    for (int i = 0; i < kTM; ++i)
+#pragma unroll
+        for (int j = 0; j < TN; ++j) mism[i][j] = 0;
+
+    load_tile(0);
+    for (int k0 = 0; k0 < words; k0 += kBKW) {
+        __syncthreads();
+        store_tile();
+        __syncthreads();
+        if (k0 + kBKW < words) load_tile(k0 + kBKW);
+#pragma unroll
+        for (int kw = 0; kw < kBKW; ++kw) {
+            uint64_t a[kTM], b[TN];
+#pragma unroll
+            for (int i = 0; i < kTM; ++i) a[i] = As[ty + 16 * i][kw];
+#pragma unroll
+            for (int j = 0; j < TN; ++j) b[j] = Bs[tx + 16 * j][kw];
+#pragma unroll
+            for (int i = 0; i < kTM; ++i)
+#pragma unroll
+                for (int j = 0; j < TN; ++j) mism[i][j] += __popcll(a[i] ^ b[j]);
+        }
+    }
+
+#pragma unroll
+    for (int i = 0; i < kTM; ++i) {
+        const int64_t row = m0 + ty + 16 * i;
+        if (row >= N) continue;
+        float ai = __ldg(alpha + row);
+        if (kDegreeScale) ai *= inv_sqrt_degree(__ldg(rowptr + row + 1) - __ldg(rowptr + row));
+#pragma unroll
+        for (int j = 0; j < TN; ++j) {
+            const int col = n0 + tx + 16 * j;
+            if (col >= F) continue;
+            const int d = K - 2 * mism[i][j];
+            if (kDegreeScale)
+                Z[row * ldz + col] = ai * (__ldg(beta + col) * float(d));
+            else
+                Z[row * ldz + col] = (ai * __ldg(beta + col)) * float(d);
+            if (dots != nullptr) dots[row * F + col] = d;
+        }
+    }
+}
+
+template <int TN, bool kDeg>
+void launch_tn(const GemmArgs &g, cudaStream_t s) {
+    dim3 grid(unsigned((g.N + kBM - 1) / kBM), unsigned((g.F + 16 * TN - 1) / (16 * TN)));
+    xnor_gemm_popc_kernel<TN, kDeg><<<grid, kThreads, 0, s>>>(
+        g.A, g.alpha, g.N, g.B, g.beta, g.F, g.K, g.words, g.Z, g.ldz, g.dots, g.rowptr);
+}
+
+template <bool kDeg>
+void launch_deg(const GemmArgs &g, cudaStream_t s) {
+    if (g.F > 32) launch_tn<4, kDeg>(g, s);
+    else if (g.F > 16) launch_tn<2, kDeg>(g, s);
+    else launch_tn<1, kDeg>(g, s);
+}
+
+}  // namespace
+
+void launch_xnor_gemm(const GemmArgs &g, const DeviceInfo &, cudaStream_t stream) {
+    if (g.N == 0) return;
+    if (g.rowptr != nullptr) launch_deg<true>(g, stream);
+    else launch_deg<false>(g, stream);
+}
+
+}  // namespace bigcn
+
+using namespace bigcn;
+
+namespace {
+bigcn_status check_gemm(const uint64_t *a_bits, const float *alpha, int64_t N,
+                        const uint64_t *b_bits, const float *beta, int32_t F, int32_t K,
+                        int32_t words, const float *Z, int64_t ldz, const int32_t *dots,
+                        const int64_t *rowptr, bool need_rowptr) {
+    if (N < 0 || F < 1 || K < 1 || words < bigcn_words(K) || ldz < F) return BIGCN_ERR_INVALID_ARG;
+    if (N > 0 && (N > kMaxElems / ldz || N > kMaxElems / words)) return BIGCN_ERR_INVALID_ARG;
+    if (N == 0) return BIGCN_OK;
+    if (!a_bits || !alpha || !b_bits || !beta || !Z || (need_rowptr && !rowptr))
+        return BIGCN_ERR_INVALID_ARG;
+    if (!aligned_to(a_bits, 8) || !aligned_to(b_bits, 8) || !aligned_to(alpha, 4) ||
+        !aligned_to(beta, 4) || !aligned_to(Z, 4) || (dots && !aligned_to(dots, 4)) ||
+        (rowptr && !aligned_to(rowptr, 8)))
+        return BIGCN_ERR_MISALIGNED;
+    const size_t zb = span_bytes(N, F, ldz, 4);
+    const size_t ab = size_t(N) * words * 8, bb = size_t(F) * words * 8;
+    if (overlaps(Z, zb, a_bits, ab) || overlaps(Z, zb, b_bits, bb) ||
+        overlaps(Z, zb, alpha, size_t(N) * 4) || overlaps(Z, zb, beta, size_t(F) * 4) ||
+        overlaps(Z, zb, rowptr, size_t(N + 1) * 8))
+        return BIGCN_ERR_INVALID_ARG;
+    if (dots) {
+        const size_t db = size_t(N) * F * 4;
+        if (overlaps(dots, db, Z, zb) || overlaps(dots, db, a_bits, ab) ||
+            overlaps(dots, db, b_bits, bb) || overlaps(dots, db, alpha, size_t(N) * 4) ||
+            overlaps(dots, db, beta, size_t(F) * 4))
+            return BIGCN_ERR_INVALID_ARG;
+    }
+    return BIGCN_OK;
+}
+}  // namespace
+
+extern "C" bigcn_status bigcn_xnor_gemm(const uint64_t *a_bits, const float *alpha, int64_t N,
+                                        const uint64_t *b_bits, const float *beta, int32_t F,
+                                        int32_t K, int32_t words, float *Z, int64_t ldz,
+                                        int32_t *dots, void *stream) {
+    bigcn_status st = check_gemm(a_bits, alpha, N, b_bits, beta, F, K, words, Z, ldz, dots,
+                                 nullptr, false);
+    if (st != BIGCN_OK || N == 0) return st;
+    DeviceInfo dev;
+    if ((st = current_device(&dev)) != BIGCN_OK) return st;
+    GemmArgs g{a_bits, alpha, N, b_bits, beta, F, K, words, Z, ldz, dots, nullptr};
+    launch_xnor_gemm(g, dev, as_stream(stream));
+    return launch_status();
+}
+
+extern "C" bigcn_status bigcn_xnor_gemm_degscaled(const uint64_t *a_bits, const float *alpha,
+                                                  int64_t N, const uint64_t *b_bits,
+                                                  const float *beta, int32_t F, int32_t K,
+                                                  int32_t words, const int64_t *rowptr,
+                                                  float *Z, int64_t ldz, void *stream) {
+    bigcn_status st = check_gemm(a_bits, alpha, N, b_bits, beta, F, K, words, Z, ldz, nullptr,
+                                 rowptr, true);
+    if (st != BIGCN_OK || N == 0) return st;
+    DeviceInfo dev;
+    if ((st = current_device(&dev)) != BIGCN_OK) return st;
+    GemmArgs g{a_bits, alpha, N, b_bits, beta, F, K, words, Z, ldz, nullptr, rowptr};
+    launch_xnor_gemm(g, dev, as_stream(stream));
+    return launch_status();
+}

@@ -145,21 +145,33 @@ def edges_to_csr(u: np.ndarray, v: np.ndarray, N: int):
     """Undirected unique edges (u < v) -> symmetric CSR (rowptr int64, colidx
     int32), both directions stored, columns ascending within a row, no
     self-loops."""
-    rows = np.concatenate([u, v]).astype(np.int64)
-    cols = np.concatenate([v, u]).astype(np.int64)
-    key = np.sort(rows * N + cols)
+    u = np.asarray(u, np.int64)
+    v = np.asarray(v, np.int64)
+    key = np.concatenate([u * N + v, v * N + u])
+    key.sort()
     rows = key // N
-    cols = key - rows * N
     rowptr = np.zeros(N + 1, np.int64)
     np.cumsum(np.bincount(rows, minlength=N), out=rowptr[1:])
-    return rowptr, cols.astype(np.int32)
+    key -= rows * N
+    return rowptr, key.astype(np.int32)
+
+
+def _sorted_unique(keys: np.ndarray) -> np.ndarray:
+    """Distinct values of an int64 array, ascending (sort + adjacent compare)."""
+    keys = np.sort(keys)
+    if keys.size == 0:
+        return keys
+    keep = np.empty(keys.size, bool)
+    keep[0] = True
+    np.not_equal(keys[1:], keys[:-1], out=keep[1:])
+    return keys[keep]
 
 
 def _unique_pairs(a: np.ndarray, b: np.ndarray, N: int) -> np.ndarray:
     lo = np.minimum(a, b).astype(np.int64)
     hi = np.maximum(a, b).astype(np.int64)
     keep = lo != hi
-    return np.unique(lo[keep] * N + hi[keep])
+    return _sorted_unique(lo[keep] * N + hi[keep])
 
 
 def preferential_attachment(N: int, m_choices, m_probs, rng, isolated: int = 0):
@@ -195,40 +207,48 @@ def preferential_attachment(N: int, m_choices, m_probs, rng, isolated: int = 0):
     return keys // N, keys % N
 
 
+def _iid_endpoints(p: np.ndarray, M: int, rng) -> np.ndarray:
+    """M i.i.d. draws from the categorical distribution p, in random order
+    (multinomial counts per category, expanded and shuffled)."""
+    counts = rng.multinomial(M, p)
+    ends = np.repeat(np.arange(p.shape[0], dtype=np.int64), counts)
+    rng.shuffle(ends)
+    return ends
+
+
+def _sample_unique_edges(p: np.ndarray, target_edges: int, rng) -> np.ndarray:
+    """Undirected edge keys lo * N + hi (lo < hi): endpoint pairs drawn i.i.d.
+    from p, self-loops and repeats dropped, topped up and then subsampled to
+    exactly ``target_edges`` distinct edges."""
+    N = p.shape[0]
+    keys = np.empty(0, np.int64)
+    batch = int(target_edges * 1.08) + 64
+    while keys.size < target_edges:
+        fresh = _unique_pairs(_iid_endpoints(p, batch, rng), _iid_endpoints(p, batch, rng), N)
+        keys = fresh if keys.size == 0 else _sorted_unique(np.concatenate([keys, fresh]))
+        batch = max(int((target_edges - keys.size) * 1.5), 1024)
+    if keys.size > target_edges:
+        keep = rng.choice(keys.size, size=target_edges, replace=False)
+        keys = keys[np.sort(keep)]
+    return keys
+
+
 def chung_lu(N: int, target_edges: int, mean_degree: float, max_degree: int, rng,
              exponent: float = 2.5):
     """Chung-Lu graph: expected degrees w_i from a power law (tail exponent
     ``exponent``) truncated at ``max_degree`` and scaled to ``mean_degree``;
     endpoints drawn proportional to w; self-loops and duplicates dropped;
-    topped up until ``target_edges`` unique undirected edges exist."""
+    exactly ``target_edges`` unique undirected edges kept."""
     w = rng.pareto(exponent - 1.0, size=N) + 1.0
     for _ in range(50):
         w = np.minimum(w * (mean_degree / w.mean()), max_degree)
-    cum = np.cumsum(w)
-    total = cum[-1]
-    keys = np.empty(0, np.int64)
-    batch = int(target_edges * 1.05)
-    while keys.size < target_edges:
-        a = np.searchsorted(cum, rng.random(batch) * total, side="right")
-        b = np.searchsorted(cum, rng.random(batch) * total, side="right")
-        a = np.minimum(a, N - 1)
-        b = np.minimum(b, N - 1)
-        keys = np.union1d(keys, _unique_pairs(a, b, N))
-        batch = max(int((target_edges - keys.size) * 1.3), 1024)
-    keys = rng.permutation(keys)[:target_edges]
+    keys = _sample_unique_edges(w / w.sum(), target_edges, rng)
     return keys // N, keys % N
 
 
 def erdos_renyi(N: int, target_edges: int, rng):
     """G(n, m): ``target_edges`` distinct undirected edges chosen uniformly."""
-    keys = np.empty(0, np.int64)
-    batch = int(target_edges * 1.02) + 16
-    while keys.size < target_edges:
-        a = rng.integers(0, N, batch)
-        b = rng.integers(0, N, batch)
-        keys = np.union1d(keys, _unique_pairs(a, b, N))
-        batch = max(int((target_edges - keys.size) * 1.3), 1024)
-    keys = rng.permutation(keys)[:target_edges]
+    keys = _sample_unique_edges(np.full(N, 1.0 / N), target_edges, rng)
     return keys // N, keys % N
 
 
@@ -259,7 +279,8 @@ def random_graph(N: int, mean_degree: float, seed: int, hub_degree: int = 0):
         u = v = np.empty(0, np.int64)
     if hub_degree > 0:
         others = rng.choice(np.arange(1, N), size=min(hub_degree, N - 1), replace=False)
-        keys = np.union1d(u * N + v, _unique_pairs(np.zeros_like(others), others, N))
+        keys = _sorted_unique(np.concatenate([u * N + v,
+                                              _unique_pairs(np.zeros_like(others), others, N)]))
         u, v = keys // N, keys % N
     return edges_to_csr(u, v, N)
 
