@@ -1,0 +1,433 @@
+#!/usr/bin/env python3
+"""Benchmark: the 2-layer Bi-GCN forward (Wang et al., CVPR 2021) on GB300.
+
+One step = one pass of the whole hot path over the workload: for each of the
+two layers, centre + sign-pack the node rows (Sec. 6.2, Eqs. 7-8), sign-pack
+the weight columns (Eqs. 3-4), the XNOR-popcount product (Eqs. 11-12) and the
+normalised-adjacency aggregation (Eqs. 1, 13) -- eight C-ABI kernel launches,
+replayed as one CUDA graph with a timing event between every two kernels.
+
+Default workload: C2 (the Citeseer-shaped 2-layer configuration: N=3327,
+K=3703, hidden 64, out 6). Its inputs (49 MB) fit in L2, so L2 is flushed
+(a 256 MiB memset, outside the timed events) before every step.
+
+Prints one JSON line (rank 0): nodes/s of the device-resident forward, the
+same through host buffers (e2e), per-kernel times and the dominant kernel's
+roofline, the CPU oracle timed on the host as a baseline, and SM clocks
+sampled during the timed region. ``--impl reference`` times the CPU oracle
+itself on the same workload (the reference arm).
+
+Multi-GPU (torchrun): the layer on one graph has no partition without an
+exchange step, so N GPUs run N independent replicas ("replicas only"); value
+= nodes processed by all ranks / the slowest rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+METRIC = "Bi-GCN layer fwd nodes/s; XNOR-GEMM bit-ops/s; SpMM GB/s as % of GB300 peak"
+DEFAULT_WORKLOAD = "C2"
+L2_FLUSH_BYTES = 256 << 20
+POPC_PER_CLK_PER_SM = 16          # 32-bit population counts per clock per SM
+FALLBACK_HBM_GBS = 6800.0
+KERNEL_SOURCES = {"pack_rows": "pack.cu", "pack_weights": "pack.cu",
+                  "xnor_gemm": "xnor_gemm.cu", "spmm": "spmm.cu"}
+
+
+# --------------------------------------------------------------- host logic --
+def dist_env():
+    return (int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)),
+            int(os.environ.get("LOCAL_RANK", 0)))
+
+
+def aggregate_over_ranks(total_ms: float, units: float, world: int):
+    """Max of the per-rank timed totals and the sum of units over ranks
+    (replicas): returns (max_ms, total_units)."""
+    if world == 1:
+        return total_ms, units
+    import torch
+    import torch.distributed as dist
+    dev = torch.device("cuda", torch.cuda.current_device()) if dist.get_backend() == "nccl" \
+        else torch.device("cpu")
+    t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
+    u = torch.tensor([units], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.all_reduce(u, op=dist.ReduceOp.SUM)
+    return float(t.item()), float(u.item())
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        return p, "measured"
+    return {"hbm_gbs": FALLBACK_HBM_GBS, "sm_max_mhz": 2070.0}, "fallback"
+
+
+def induced_subgraph(rowptr, colidx, lo: int, hi: int):
+    """CSR of the subgraph induced by nodes [lo, hi), renumbered from 0."""
+    rp = rowptr[lo:hi + 1] - rowptr[lo]
+    cols = colidx[rowptr[lo]:rowptr[hi]].astype(np.int64)
+    rows = np.repeat(np.arange(hi - lo), np.diff(rp))
+    keep = (cols >= lo) & (cols < hi)
+    counts = np.bincount(rows[keep], minlength=hi - lo)
+    out = np.zeros(hi - lo + 1, np.int64)
+    np.cumsum(counts, out=out[1:])
+    return out, (cols[keep] - lo).astype(np.int32)
+
+
+def kernel_work(N, K, F, nnz, name):
+    """Algorithmic work of one launch: (amount, unit, bound)."""
+    W = (K + 63) // 64
+    if name == "pack_rows":
+        return 4.0 * N * K + 8.0 * N * W + 4.0 * N + 8.0 * K, "bytes", "hbm"
+    if name == "pack_weights":
+        return 4.0 * K * F + 8.0 * F * W + 4.0 * F, "bytes", "hbm"
+    if name == "xnor_gemm":
+        return float(N) * K * F, "bit-ops", "alu"
+    if name == "spmm":
+        return 8.0 * (N + 1) + 4.0 * nnz + 8.0 * N * F, "bytes", "hbm"
+    raise KeyError(name)
+
+
+def source_hash(name):
+    path = os.path.join(ROOT, "paper_2010_07565_gb300", "csrc", KERNEL_SOURCES[name])
+    with open(path, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def profiled_traffic(name, workload):
+    """DRAM bytes per launch from a committed ncu summary, if it was taken on
+    the current source of the kernel (profiles/<kernel>_<workload>.txt lines
+    'source_sha256_16: ...' and 'dram_bytes_per_launch: ...')."""
+    path = os.path.join(ROOT, "profiles", f"{name}_{workload}.txt")
+    if not os.path.exists(path):
+        return None
+    fields = {}
+    with open(path) as f:
+        for line in f:
+            if ":" in line:
+                k, v = line.split(":", 1)
+                fields[k.strip()] = v.strip()
+    if fields.get("source_sha256_16") != source_hash(name):
+        return None
+    try:
+        return float(fields["dram_bytes_per_launch"])
+    except (KeyError, ValueError):
+        return None
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle samples every 200 ms while running."""
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.out = None
+
+    def __enter__(self):
+        try:
+            self.out = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.QUERY}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=self.out, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        if self.proc is None or self.out is None:
+            return None
+        self.out.seek(0)
+        rows = [r.split(",") for r in self.out.read().strip().splitlines() if r.count(",") >= 8]
+        os.unlink(self.out.name)
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].strip().replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for r in rows for n, v in zip(names, r[5:9]) if "Active" in v
+                          and "Not" not in v})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": float(rows[0][2]) if rows[0][2].strip().replace(".", "").isdigit()
+                else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+# ---------------------------------------------------------------- workload --
+def build_workload(name):
+    from paper_2010_07565_gb300 import inputs
+    w = inputs.get_workload(name)
+    X = inputs.features(w)
+    s, t = inputs.bn_stats(X)
+    W1, W2 = inputs.layer_weights(w)
+    rowptr, colidx = inputs.graph(w)
+    return w, dict(X=X, s=s, t=t, W1=W1, W2=W2, rowptr=rowptr, colidx=colidx)
+
+
+def time_oracle(w, data, budget_s, rows=None):
+    """Run the CPU oracle's 2-layer forward on the subgraph induced by the
+    first ``rows`` nodes (all if None) repeatedly for about ``budget_s``;
+    returns (nodes/s, sample description)."""
+    import oracle
+    n = w.N if rows is None else int(min(rows, w.N))
+    rp, ci = (data["rowptr"], data["colidx"]) if n == w.N else \
+        induced_subgraph(data["rowptr"], data["colidx"], 0, n)
+    X = np.ascontiguousarray(data["X"][:n])
+    reps, t0 = 0, time.perf_counter()
+    while True:
+        oracle.forward_2layer(X, data["s"], data["t"], data["W1"], data["W2"], rp, ci)
+        reps += 1
+        el = time.perf_counter() - t0
+        if el >= budget_s:
+            break
+    what = "full" if n == w.N else f"the subgraph induced by nodes [0, {n}) of"
+    return n * reps / el, f"{reps} x the oracle's 2-layer forward on {what} {w.name} ({el:.1f} s)"
+
+
+# ------------------------------------------------------------ reference arm --
+def run_reference(args, rank, world):
+    """The CPU oracle as the reference arm: each step is one oracle forward
+    on a node block of the workload (its induced subgraph), sized so that
+    warm-up plus steps take about two and a half minutes."""
+    if rank != 0:
+        return 0
+    import oracle
+    w, data = build_workload(args.workload)
+    # seconds per node of the oracle, from a small calibration block
+    cal = min(w.N, 128)
+    rp, ci = induced_subgraph(data["rowptr"], data["colidx"], 0, cal)
+    t0 = time.perf_counter()
+    oracle.forward_2layer(np.ascontiguousarray(data["X"][:cal]), data["s"], data["t"],
+                          data["W1"], data["W2"], rp, ci)
+    sec_per_node = (time.perf_counter() - t0) / cal
+    per_step = 150.0 / max(args.steps + args.warmup, 1)
+    n = int(max(16, min(w.N, per_step / max(sec_per_node, 1e-9))))
+    times = []
+    for step in range(args.warmup + args.steps):
+        lo = (step * n) % max(w.N - n + 1, 1)
+        rp, ci = induced_subgraph(data["rowptr"], data["colidx"], lo, lo + n)
+        X = np.ascontiguousarray(data["X"][lo:lo + n])
+        t0 = time.perf_counter()
+        oracle.forward_2layer(X, data["s"], data["t"], data["W1"], data["W2"], rp, ci)
+        if step >= args.warmup:
+            times.append(time.perf_counter() - t0)
+    total = sum(times)
+    value = n * len(times) / total
+    sample = (f"each step: the oracle's 2-layer forward on the subgraph induced by {n} "
+              f"consecutive nodes of {w.name}")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "nodes/s",
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 * total / len(times), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32+b1", "data": "synthetic",
+            "config": {"workload": w.description, "name": w.name, "nodes_per_step": n},
+            "cpu_baseline": {"value": value, "unit": "nodes/s", "cores": 1, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": "nodes/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ----------------------------------------------------------------- our arm --
+def run_gpu(args, rank, world, local_rank):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2010_07565_gb300 import cost_model
+    from paper_2010_07565_gb300.runner import GCN2Forward, STEP_KERNELS
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    w, data = build_workload(args.workload)
+    nnz = int(data["colidx"].shape[0])
+    model = GCN2Forward(w.N, w.K, w.hidden, w.out, nnz, dev)
+    host = {k: torch.from_numpy(np.ascontiguousarray(v)).pin_memory() for k, v in data.items()}
+    model.load(non_blocking=False, **host)
+    torch.cuda.synchronize()
+
+    try:
+        events = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(9)]
+        model.capture(events)
+        launch, how = model.replay, "CUDA graph of the 8 kernel launches, events between kernels"
+    except TypeError:    # torch without external events: plain launches
+        events = [torch.cuda.Event(enable_timing=True) for _ in range(9)]
+        launch, how = (lambda: model.launch(events)), "8 kernel launches, events between kernels"
+
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    for _ in range(args.warmup):
+        flush.zero_()
+        launch()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+
+    per_kernel = [[] for _ in range(8)]
+    step_ms = []
+    with ClockSampler(local_rank) as clocks:
+        for _ in range(args.steps):
+            flush.zero_()
+            launch()
+            events[8].synchronize()
+            ts = [events[k].elapsed_time(events[k + 1]) for k in range(8)]
+            for k in range(8):
+                per_kernel[k].append(ts[k])
+            step_ms.append(events[0].elapsed_time(events[8]))
+        torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    total_ms = float(sum(step_ms))
+    max_ms, units = aggregate_over_ranks(total_ms, float(w.N) * args.steps, world)
+    value = units / (max_ms * 1e-3)
+
+    # End to end through host buffers: pinned inputs -> device, forward, logits -> host.
+    logits_host = torch.empty((w.N, w.out), dtype=torch.float32).pin_memory()
+    h2d = sum(int(v.numel() * v.element_size()) for v in host.values())
+    d2h = int(logits_host.numel() * logits_host.element_size())
+    e2e_steps = max(3, min(args.steps, 200))
+    ea, eb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e2e_ms = []
+    for i in range(e2e_steps + 2):
+        ea.record()
+        model.load(non_blocking=True, **host)
+        launch()
+        logits_host.copy_(model.logits, non_blocking=True)
+        eb.record()
+        eb.synchronize()
+        if i >= 2:
+            e2e_ms.append(ea.elapsed_time(eb))
+    e2e_max, e2e_units = aggregate_over_ranks(float(sum(e2e_ms)), float(w.N) * len(e2e_ms), world)
+
+    if rank != 0:
+        return 0
+
+    peaks, peak_kind = load_peaks()
+    hbm = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+    props = torch.cuda.get_device_properties(dev)
+    sm_max = float(peaks.get("sm_max_mhz", 2070.0))
+    popc_peak = props.multi_processor_count * POPC_PER_CLK_PER_SM * 32 * sm_max * 1e6
+    shapes = [(w.N, w.K, w.hidden), (w.N, w.hidden, w.out)]
+    kernels = []
+    for k in range(8):
+        layer, name = k // 4, STEP_KERNELS[k % 4]
+        N, K, F = shapes[layer]
+        work, unit, bound = kernel_work(N, K, F, nnz, name)
+        mean_ms = statistics.fmean(per_kernel[k])
+        kernels.append(dict(layer=layer + 1, name=name, mean_us=1e3 * mean_ms, work=work,
+                            unit=unit, bound=bound))
+    dom = max(kernels, key=lambda r: r["mean_us"])
+    rate = dom["work"] / (dom["mean_us"] * 1e-6)
+    if dom["bound"] == "hbm":
+        achieved, peak, unit = rate / 1e9, hbm, "GB/s"
+        traffic = profiled_traffic(dom["name"], w.name)
+    else:
+        achieved, peak, unit = rate / 1e12, popc_peak / 1e12, "T bit-ops/s"
+        traffic = profiled_traffic(dom["name"], w.name)
+    gemm1 = kernels[2]
+    spmm1 = kernels[3]
+    spmm_gbs = spmm1["work"] / (spmm1["mean_us"] * 1e-6) / 1e9
+
+    cpu_baseline = None
+    if world == 1 and not args.no_cpu_baseline:
+        v, sample = time_oracle(w, data, budget_s=args.cpu_seconds)
+        cpu_baseline = {"value": v, "unit": "nodes/s", "cores": 1, "kind": "oracle",
+                        "sample": sample}
+
+    dims = [w.K, w.hidden, w.out]
+    line = {
+        "metric": METRIC, "value": value, "unit": "nodes/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": max_ms / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f32+b1", "data": "synthetic",
+        "config": {"workload": w.description, "name": w.name, "N": w.N, "K": w.K,
+                   "hidden": w.hidden, "out": w.out, "nnz": nnz,
+                   "l2": "flushed before every step (256 MiB memset outside the timed events)",
+                   "launch": how, "parallelism": "replicas" if world > 1 else "single GPU"},
+        "components": {
+            "xnor_gemm_bitops_per_s": gemm1["work"] / (gemm1["mean_us"] * 1e-6),
+            "spmm_gbs": spmm_gbs, "spmm_pct_of_hbm_peak": 100.0 * spmm_gbs / hbm,
+            "per_kernel_us": {f"L{r['layer']}.{r['name']}": round(r["mean_us"], 3)
+                              for r in kernels}},
+        "roofline": {"kernel": f"L{dom['layer']}.{dom['name']}", "bound": dom["bound"],
+                     "achieved": achieved, "peak": peak, "unit": unit, "frac": achieved / peak,
+                     "traffic": traffic,
+                     "peak_source": (f"{peak_kind} MEASURED_PEAKS.json hbm_gbs"
+                                     if dom["bound"] == "hbm" else
+                                     f"{POPC_PER_CLK_PER_SM} POPC/clk/SM x {props.multi_processor_count}"
+                                     f" SMs x 32 bits x {sm_max:.0f} MHz")},
+        "cpu_baseline": cpu_baseline,
+        "e2e": {"value": e2e_units / (e2e_max * 1e-3), "unit": "nodes/s",
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": 8 * args.steps,
+        "clocks": clocks.summary(),
+        "paper_context": {
+            "cycle_ops_gcn": cost_model.cycle_ops(w.N, nnz // 2, dims, False),
+            "cycle_ops_bigcn": cost_model.cycle_ops(w.N, nnz // 2, dims, True),
+            "note": "Sec. 5.3's analytic cycle-operation counts for this shape; the paper "
+                    "reports no measured timings"},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["bigcn", "reference"], default="bigcn")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD,
+                    help="C1..C4, or a sweep point such as C5_K4096_F256 (1 layer not supported)")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    if args.warmup < 3:
+        ap.error("--warmup must be at least 3")
+    rank, world, local_rank = dist_env()
+    if args.impl == "reference":
+        return run_reference(args, rank, world)
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if backend == "nccl":
+            torch.cuda.set_device(local_rank)
+        dist.init_process_group(backend=backend)
+    try:
+        return run_gpu(args, rank, world, local_rank)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+            if dist.is_initialized():
+                dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -5,97 +5,131 @@
 //                         per-column scale (Eq. 4)
 //
 // pack_rows is HBM-bound: it reads 4K bytes per node and writes K/8 + 4.
-// One warp walks one row at a time (persistent grid, a multiple of the SM
-// count): lane l of chunk c owns feature 32c + l, so one __ballot_sync gives
-// the 32-bit half-word of the packed row directly, and each lane keeps a
-// running sum of |y| that one warp reduction turns into the scale. Eight
-// chunks' loads are issued before any is consumed to keep 1 KB per warp in
-// flight.
+// Lane l of a 32-feature chunk c owns feature 32c + l, so one __ballot_sync
+// yields the chunk's 32-bit half-word of the packed row directly, and every
+// lane keeps a running sum of |y|. G warps (1, 2, 4 or 8, so that the grid
+// fills the GPU even when N is small) share a row, warp g taking chunks
+// g, g + G, ...; each warp issues eight chunks' loads (1 KB) before it
+// consumes any. The G partial |y| sums are added in a fixed order through
+// shared memory, so alpha does not depend on scheduling.
+//
+// pack_weights reads W (K x F) column-wise: thread (x, y) of a 32 x 8 block
+// owns column 32*bx + x and builds whole 64-bit words from 64 coalesced row
+// reads. The words of a column are spread over a cluster of S <= 8 blocks
+// (grid y); each block reduces its |W| partial sums in shared memory, and
+// block 0 of the cluster adds the S partials through distributed shared
+// memory in rank order (deterministic).
+#include <cooperative_groups.h>
+
 #include "launch.cuh"
 
 namespace bigcn {
 namespace {
 
+namespace cg = cooperative_groups;
+
 constexpr int kPackThreads = 256;
+constexpr int kPackWarps = kPackThreads / 32;
 constexpr int kPackUnroll = 8;
 
 template <bool kAffine>
-__global__ void __launch_bounds__(kPackThreads, 6)
+__global__ void __launch_bounds__(kPackThreads, 4)
 pack_rows_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
                  const float *__restrict__ scale, const float *__restrict__ shift,
-                 uint32_t *__restrict__ bits32, int64_t ld32, float *__restrict__ alpha) {
+                 uint32_t *__restrict__ bits32, int64_t ld32, float *__restrict__ alpha,
+                 int G) {
+    __shared__ float part[kPackWarps];
     const int lane = threadIdx.x & 31;
-    const int64_t warp0 = (int64_t(blockIdx.x) * kPackThreads + threadIdx.x) >> 5;
-    const int64_t nwarps = (int64_t(gridDim.x) * kPackThreads) >> 5;
-    const int nchunks = (K + 31) >> 5;          // 32-bit words that carry signs
-    const float kf = float(K);
+    const int warp = threadIdx.x >> 5;
+    const int sub = warp & (G - 1);
+    const int64_t row = int64_t(blockIdx.x) * (kPackWarps / G) + warp / G;
+    const int nchunks = (K + 31) >> 5;          // 32-bit half-words that carry signs
 
-    for (int64_t row = warp0; row < N; row += nwarps) {
+    float l1 = 0.0f;
+    if (row < N) {
         const float *x = X + row * ldx;
         uint32_t *out = bits32 + row * ld32;
-        float l1 = 0.0f;
-        for (int c0 = 0; c0 < nchunks; c0 += kPackUnroll) {
+        for (int m0 = sub; m0 < nchunks; m0 += G * kPackUnroll) {
             float v[kPackUnroll];
 #pragma unroll
             for (int u = 0; u < kPackUnroll; ++u) {
-                const int k = (c0 + u) * 32 + lane;
+                const int k = (m0 + u * G) * 32 + lane;
                 v[u] = (k < K) ? __ldcs(x + k) : 0.0f;
             }
 #pragma unroll
             for (int u = 0; u < kPackUnroll; ++u) {
-                const int k = (c0 + u) * 32 + lane;
+                const int c = m0 + u * G;
+                const int k = c * 32 + lane;
                 const bool in = k < K;
                 float y = v[u];
                 if (kAffine && in) y = __fmaf_rn(y, __ldg(scale + k), __ldg(shift + k));
                 const unsigned m = __ballot_sync(kFullMask, in && y >= 0.0f);
-                if (c0 + u < nchunks && lane == 0) out[c0 + u] = m;
+                if (c < nchunks && lane == 0) out[c] = m;
                 l1 += in ? fabsf(y) : 0.0f;
             }
         }
         // Pad half-words past the last one that carries signs are zero.
-        for (int64_t q = nchunks + lane; q < ld32; q += 32) out[q] = 0u;
-        l1 = warp_sum(l1);
-        if (lane == 0) alpha[row] = l1 / kf;
+        if (sub == 0)
+            for (int64_t q = nchunks + lane; q < ld32; q += 32) out[q] = 0u;
+    }
+    l1 = warp_sum(l1);
+    if (lane == 0) part[warp] = l1;
+    __syncthreads();
+    if (row < N && sub == 0 && lane == 0) {
+        float s = 0.0f;
+        for (int g = 0; g < G; ++g) s += part[warp + g];
+        alpha[row] = s / float(K);
     }
 }
 
-// Weight columns: thread (x, y) of a 32 x 8 block owns column j = 32*bx + x
-// and the packed words w = y, y + 8, ...; reads of one k are coalesced across
-// the 32 columns. The per-column |W| sums are reduced over y in shared memory.
 constexpr int kWCols = 32;
 constexpr int kWRows = 8;
+constexpr int kMaxCluster = 8;
 
 __global__ void __launch_bounds__(kWCols *kWRows)
 pack_weights_kernel(const float *__restrict__ Wt, int K, int F, int64_t ldw,
                     uint64_t *__restrict__ bits, int words, float *__restrict__ beta) {
     __shared__ float partial[kWRows][kWCols];
+    __shared__ float colsum[kWCols];
+    cg::cluster_group cluster = cg::this_cluster();
+    const int S = int(cluster.num_blocks());
+    const int rank = int(cluster.block_rank());
     const int tx = threadIdx.x, ty = threadIdx.y;
     const int j = blockIdx.x * kWCols + tx;
+
     float l1 = 0.0f;
     if (j < F) {
-        for (int w = ty; w < words; w += kWRows) {
-            uint64_t word = 0;
+        for (int w = rank * kWRows + ty; w < words; w += S * kWRows) {
             const int kb = w * 64;
-#pragma unroll 16
+            float v[64];
+#pragma unroll
+            for (int b = 0; b < 64; ++b)
+                v[b] = (kb + b < K) ? __ldg(Wt + int64_t(kb + b) * ldw + j) : 0.0f;
+            uint64_t word = 0;
+#pragma unroll
             for (int b = 0; b < 64; ++b) {
-                const int k = kb + b;
-                if (k < K) {
-                    const float v = __ldg(Wt + int64_t(k) * ldw + j);
-                    word |= uint64_t(v >= 0.0f) << b;
-                    l1 += fabsf(v);
-                }
+                const bool in = kb + b < K;
+                word |= uint64_t(in && v[b] >= 0.0f) << b;
+                l1 += fabsf(v[b]);
             }
             bits[int64_t(j) * words + w] = word;
         }
     }
     partial[ty][tx] = l1;
     __syncthreads();
-    if (ty == 0 && j < F) {
+    if (ty == 0) {
         float s = 0.0f;
 #pragma unroll
         for (int r = 0; r < kWRows; ++r) s += partial[r][tx];
+        colsum[tx] = s;
+    }
+    cluster.sync();
+    if (rank == 0 && ty == 0 && j < F) {
+        float s = 0.0f;
+        for (int r = 0; r < S; ++r) s += cluster.map_shared_rank(colsum, r)[tx];
         beta[j] = s / float(K);
     }
+    cluster.sync();   // peers keep their shared memory until block 0 has read it
 }
 
 }  // namespace
@@ -104,23 +138,41 @@ void launch_pack_rows(const float *X, int64_t N, int K, int64_t ldx, const float
                       const float *shift, uint64_t *bits, int words, float *alpha,
                       const DeviceInfo &dev, cudaStream_t stream) {
     if (N == 0) return;
-    const int64_t blocks_needed = (N * 32 + kPackThreads - 1) / kPackThreads;
-    const int64_t resident = int64_t(dev.sm_count) * (2048 / kPackThreads);
-    const int grid = int(blocks_needed < resident ? blocks_needed : resident);
+    // Split rows over up to 8 warps while the grid is short of one full wave
+    // of warps, as long as every warp keeps at least one 8-chunk batch.
+    const int nchunks = (K + 31) / 32;
+    const int64_t full_wave = int64_t(dev.sm_count) * 64;
+    int G = 1;
+    while (G < kPackWarps && N * G < full_wave && nchunks >= 2 * G * kPackUnroll) G *= 2;
+    const int rows_per_block = kPackWarps / G;
+    const unsigned grid = unsigned((N + rows_per_block - 1) / rows_per_block);
     uint32_t *b32 = reinterpret_cast<uint32_t *>(bits);
     if (scale)
         pack_rows_kernel<true><<<grid, kPackThreads, 0, stream>>>(
-            X, N, K, ldx, scale, shift, b32, int64_t(words) * 2, alpha);
+            X, N, K, ldx, scale, shift, b32, int64_t(words) * 2, alpha, G);
     else
         pack_rows_kernel<false><<<grid, kPackThreads, 0, stream>>>(
-            X, N, K, ldx, nullptr, nullptr, b32, int64_t(words) * 2, alpha);
+            X, N, K, ldx, nullptr, nullptr, b32, int64_t(words) * 2, alpha, G);
 }
 
 void launch_pack_weights(const float *Wt, int K, int F, int64_t ldw, uint64_t *bits,
                          int words, float *beta, cudaStream_t stream) {
-    dim3 block(kWCols, kWRows);
-    dim3 grid((F + kWCols - 1) / kWCols);
-    pack_weights_kernel<<<grid, block, 0, stream>>>(Wt, K, F, ldw, bits, words, beta);
+    // One block row per 8 words, at most a cluster of 8.
+    int S = (words + kWRows - 1) / kWRows;
+    if (S > kMaxCluster) S = kMaxCluster;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((F + kWCols - 1) / kWCols, S, 1);
+    cfg.blockDim = dim3(kWCols, kWRows, 1);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 1;
+    attr[0].val.clusterDim.y = S;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaLaunchKernelEx(&cfg, pack_weights_kernel, Wt, K, F, ldw, bits, words, beta);
 }
 
 }  // namespace bigcn

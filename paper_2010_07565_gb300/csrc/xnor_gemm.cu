@@ -9,9 +9,18 @@
 // tx + 16 j, which keeps the shared-memory reads free of bank conflicts (odd
 // row pitch) and the Z stores coalesced along the columns.
 //
+// When the output has fewer tiles than the GPU has SMs, the k-steps of each
+// tile are split over a thread-block cluster of S <= 8 blocks (grid z): each
+// block counts mismatches over every S-th k-step, stores its counts in shared
+// memory, and after a cluster barrier each block finishes 1/S of the tile's
+// rows by adding the S partial counts through distributed shared memory. The
+// counts are integers, so the split changes no bit of the result.
+//
 // The epilogue optionally multiplies row i by dinv_i = 1/sqrt(1 + deg_i), the
 // source-side factor of D^-1/2 (A + I) D^-1/2, so that the aggregation that
 // follows in the fused layer reads pre-scaled rows.
+#include <cooperative_groups.h>
+
 #include "launch.cuh"
 
 namespace bigcn {
@@ -23,7 +32,9 @@ constexpr int kPitch = kBKW + 1;
 constexpr int kTM = 8;       // rows per thread
 constexpr int kThreads = 256;
 
-template <int TN, bool kDegreeScale>
+namespace cg = cooperative_groups;
+
+template <int TN, bool kDegreeScale, bool kSplit>
 __global__ void __launch_bounds__(kThreads)
 xnor_gemm_popc_kernel(const uint64_t *__restrict__ A, const float *__restrict__ alpha, int64_t N,
                       const uint64_t *__restrict__ B, const float *__restrict__ beta, int F,
@@ -39,6 +50,8 @@ xnor_gemm_popc_kernel(const uint64_t *__restrict__ A, const float *__restrict__ 
     const int tx = tid & 15, ty = tid >> 4;
     const int64_t m0 = int64_t(blockIdx.x) * kBM;
     const int n0 = blockIdx.y * BN;
+    const int S = kSplit ? int(gridDim.z) : 1;
+    const int rank = kSplit ? int(blockIdx.z) : 0;
 
     uint64_t ra[kALoads], rb[kBLoads];
     auto load_tile = [&](int k0) {
@@ -76,12 +89,12 @@ xnor_gemm_popc_kernel(const uint64_t *__restrict__ A, const float *__restrict__ 
 #pragma unroll
         for (int j = 0; j < TN; ++j) mism[i][j] = 0;
 
-    load_tile(0);
-    for (int k0 = 0; k0 < words; k0 += kBKW) {
+    load_tile(rank * kBKW);
+    for (int k0 = rank * kBKW; k0 < words; k0 += S * kBKW) {
         __syncthreads();
         store_tile();
         __syncthreads();
-        if (k0 + kBKW < words) load_tile(k0 + kBKW);
+        if (k0 + S * kBKW < words) load_tile(k0 + S * kBKW);
 #pragma unroll
         for (int kw = 0; kw < kBKW; ++kw) {
             uint64_t a[kTM], b[TN];
@@ -96,8 +109,31 @@ xnor_gemm_popc_kernel(const uint64_t *__restrict__ A, const float *__restrict__ 
         }
     }
 
+    if constexpr (kSplit) {
+        __shared__ int red[kBM * BN];
+        cg::cluster_group cluster = cg::this_cluster();
+#pragma unroll
+        for (int i = 0; i < kTM; ++i)
+#pragma unroll
+            for (int j = 0; j < TN; ++j) red[(ty + 16 * i) * BN + tx + 16 * j] = mism[i][j];
+        cluster.sync();
+#pragma unroll
+        for (int i = 0; i < kTM; ++i) {
+            if (i % S != rank) continue;
+#pragma unroll
+            for (int j = 0; j < TN; ++j) {
+                int total = 0;
+                for (int r = 0; r < S; ++r)
+                    total += cluster.map_shared_rank(red, r)[(ty + 16 * i) * BN + tx + 16 * j];
+                mism[i][j] = total;
+            }
+        }
+        cluster.sync();   // peers keep their counts until every block has read them
+    }
+
 #pragma unroll
     for (int i = 0; i < kTM; ++i) {
+        if (kSplit && i % S != rank) continue;
         const int64_t row = m0 + ty + 16 * i;
         if (row >= N) continue;
         float ai = __ldg(alpha + row);
@@ -117,25 +153,50 @@ xnor_gemm_popc_kernel(const uint64_t *__restrict__ A, const float *__restrict__ 
 }
 
 template <int TN, bool kDeg>
-void launch_tn(const GemmArgs &g, cudaStream_t s) {
-    dim3 grid(unsigned((g.N + kBM - 1) / kBM), unsigned((g.F + 16 * TN - 1) / (16 * TN)));
-    xnor_gemm_popc_kernel<TN, kDeg><<<grid, kThreads, 0, s>>>(
-        g.A, g.alpha, g.N, g.B, g.beta, g.F, g.K, g.words, g.Z, g.ldz, g.dots, g.rowptr);
+void launch_tn(const GemmArgs &g, const DeviceInfo &dev, cudaStream_t s) {
+    constexpr int BN = 16 * TN;
+    const unsigned gx = unsigned((g.N + kBM - 1) / kBM), gy = unsigned((g.F + BN - 1) / BN);
+    const int ksteps = (g.words + kBKW - 1) / kBKW;
+    const int64_t tiles = int64_t(gx) * gy;
+    int S = 1;
+    if (tiles < dev.sm_count && ksteps > 1) {
+        const int64_t want = (2 * int64_t(dev.sm_count) + tiles - 1) / tiles;
+        S = int(want < 8 ? want : 8);
+        if (S > ksteps) S = ksteps;
+    }
+    if (S == 1) {
+        xnor_gemm_popc_kernel<TN, kDeg, false><<<dim3(gx, gy), kThreads, 0, s>>>(
+            g.A, g.alpha, g.N, g.B, g.beta, g.F, g.K, g.words, g.Z, g.ldz, g.dots, g.rowptr);
+        return;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(gx, gy, S);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 1;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = S;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaLaunchKernelEx(&cfg, xnor_gemm_popc_kernel<TN, kDeg, true>, g.A, g.alpha, g.N, g.B,
+                       g.beta, g.F, g.K, g.words, g.Z, g.ldz, g.dots, g.rowptr);
 }
 
 template <bool kDeg>
-void launch_deg(const GemmArgs &g, cudaStream_t s) {
-    if (g.F > 32) launch_tn<4, kDeg>(g, s);
-    else if (g.F > 16) launch_tn<2, kDeg>(g, s);
-    else launch_tn<1, kDeg>(g, s);
+void launch_deg(const GemmArgs &g, const DeviceInfo &dev, cudaStream_t s) {
+    if (g.F > 32) launch_tn<4, kDeg>(g, dev, s);
+    else if (g.F > 16) launch_tn<2, kDeg>(g, dev, s);
+    else launch_tn<1, kDeg>(g, dev, s);
 }
 
 }  // namespace
 
-void launch_xnor_gemm(const GemmArgs &g, const DeviceInfo &, cudaStream_t stream) {
+void launch_xnor_gemm(const GemmArgs &g, const DeviceInfo &dev, cudaStream_t stream) {
     if (g.N == 0) return;
-    if (g.rowptr != nullptr) launch_deg<true>(g, stream);
-    else launch_deg<false>(g, stream);
+    if (g.rowptr != nullptr) launch_deg<true>(g, dev, stream);
+    else launch_deg<false>(g, dev, stream);
 }
 
 }  // namespace bigcn
