@@ -56,7 +56,8 @@ typedef enum bigcn_status {
     BIGCN_ERR_INVALID_ARG = 1,  /* null pointer, bad size, aliasing, short workspace */
     BIGCN_ERR_MISALIGNED = 2,   /* a pointer not aligned as documented */
     BIGCN_ERR_CUDA = 3,         /* a CUDA runtime error (launch or device query) */
-    BIGCN_ERR_UNSUPPORTED = 4   /* the current device is not sm_103 */
+    BIGCN_ERR_UNSUPPORTED = 4,  /* the current device is not sm_103 */
+    BIGCN_ERR_SCRATCH_LIMIT = 5 /* bigcn_layer_forward_static: workspace > its static scratch */
 } bigcn_status;
 
 /* Human-readable name of a status code (static storage; never NULL). */
@@ -187,6 +188,42 @@ bigcn_status bigcn_layer_forward(const float *X, int64_t N, int32_t K, int64_t l
                                  const int64_t *rowptr, const int32_t *colidx,
                                  int64_t nnz, void *workspace, size_t ws_bytes,
                                  float *H, int64_t ldh, void *stream);
+
+/* Bytes of the device scratch array behind bigcn_layer_forward_static. */
+#define BIGCN_STATIC_SCRATCH_BYTES ((size_t)32 << 20)
+
+/*
+ * bigcn_layer_forward without a caller-supplied workspace, for callers that
+ * cannot allocate device memory: serving loops that forbid cudaMalloc and
+ * cudaFree in steady state because both can stall the whole device,
+ * plug-ins whose host application owns every byte of the device memory
+ * budget, and deployments that must fix their memory footprint when they
+ * load. (The paper has no counterpart: this is an interface convenience.)
+ *
+ * The workspace is a file-scope __device__ array of BIGCN_STATIC_SCRATCH_BYTES
+ * (32 MiB) inside this library. Every GPU on which the library's device code
+ * is loaded holds that array until the process exits. The call allocates
+ * nothing: no cudaMalloc, no cudaFree, no allocating library routine.
+ *
+ * Arguments, results and errors are those of bigcn_layer_forward minus
+ * `workspace` and `ws_bytes`, plus: when bigcn_layer_workspace_bytes(N, K, F)
+ * exceeds BIGCN_STATIC_SCRATCH_BYTES the call returns
+ * BIGCN_ERR_SCRATCH_LIMIT and enqueues nothing. (Roughly: N * (K/8 + 4F)
+ * bytes must fit, e.g. 90,000 nodes with K = 602 and F = 64.)
+ *
+ * The first call on a device, with that device current, looks up the array's
+ * device address (cudaGetSymbolAddress) and caches it for the device; make
+ * that first call before any stream capture begins. Every call on a device
+ * shares the one array and overwrites it; the layer writes every scratch
+ * byte it reads, so nothing has to start at zero, but two calls whose
+ * kernels overlap on the GPU (e.g. on two streams, or on one device from two
+ * threads without ordering) race on the array and give wrong results.
+ */
+bigcn_status bigcn_layer_forward_static(const float *X, int64_t N, int32_t K, int64_t ldx,
+                                        const float *scale, const float *shift,
+                                        const float *Wt, int32_t F, int64_t ldw,
+                                        const int64_t *rowptr, const int32_t *colidx,
+                                        int64_t nnz, float *H, int64_t ldh, void *stream);
 
 #ifdef __cplusplus
 }

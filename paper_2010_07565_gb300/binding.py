@@ -25,7 +25,8 @@ _lock = threading.Lock()
 
 BIGCN_OK = 0
 STATUS_NAMES = {0: "BIGCN_OK", 1: "BIGCN_ERR_INVALID_ARG", 2: "BIGCN_ERR_MISALIGNED",
-                3: "BIGCN_ERR_CUDA", 4: "BIGCN_ERR_UNSUPPORTED"}
+                3: "BIGCN_ERR_CUDA", 4: "BIGCN_ERR_UNSUPPORTED", 5: "BIGCN_ERR_SCRATCH_LIMIT"}
+STATIC_SCRATCH_BYTES = 32 << 20   # BIGCN_STATIC_SCRATCH_BYTES
 
 _p = ctypes.c_void_p
 _i32 = ctypes.c_int32
@@ -46,6 +47,8 @@ SIGNATURES = {
     "bigcn_layer_workspace_bytes": ([_i64, _i32, _i32], _sz),
     "bigcn_layer_forward": ([_p, _i64, _i32, _i64, _p, _p, _p, _i32, _i64, _p, _p, _i64, _p,
                              _sz, _p, _i64, _p], ctypes.c_int),
+    "bigcn_layer_forward_static": ([_p, _i64, _i32, _i64, _p, _p, _p, _i32, _i64, _p, _p, _i64,
+                                    _p, _i64, _p], ctypes.c_int),
 }
 
 
@@ -180,6 +183,18 @@ def bigcn_layer_forward(X, scale, shift, Wt, rowptr, colidx, workspace, H, strea
         _ptr(X), N, K, _ld(X), _ptr(scale), _ptr(shift), _ptr(Wt), F, _ld(Wt), _ptr(rowptr),
         _ptr(colidx) if colidx.numel() else None, colidx.numel(), _ptr(workspace),
         workspace.numel() * workspace.element_size(), _ptr(H), _ld(H), _stream(stream)))
+
+
+def bigcn_layer_forward_static(X, scale, shift, Wt, rowptr, colidx, H, stream=None):
+    """The layer on the library's own static device scratch, for callers that
+    cannot allocate device memory (no workspace argument; layers whose
+    workspace exceeds STATIC_SCRATCH_BYTES are refused)."""
+    N, K = X.shape
+    F = Wt.shape[1]
+    _check("bigcn_layer_forward_static", lib().bigcn_layer_forward_static(
+        _ptr(X), N, K, _ld(X), _ptr(scale), _ptr(shift), _ptr(Wt), F, _ld(Wt), _ptr(rowptr),
+        _ptr(colidx) if colidx.numel() else None, colidx.numel(), _ptr(H), _ld(H),
+        _stream(stream)))
 
 
 # ------------------------------------------------- allocating conveniences ---

@@ -87,6 +87,7 @@ extern "C" const char *bigcn_status_string(int status) {
         case BIGCN_ERR_MISALIGNED: return "BIGCN_ERR_MISALIGNED";
         case BIGCN_ERR_CUDA: return "BIGCN_ERR_CUDA";
         case BIGCN_ERR_UNSUPPORTED: return "BIGCN_ERR_UNSUPPORTED";
+        case BIGCN_ERR_SCRATCH_LIMIT: return "BIGCN_ERR_SCRATCH_LIMIT";
         default: return "BIGCN_ERR_UNKNOWN";
     }
 }
@@ -151,4 +152,45 @@ extern "C" bigcn_status bigcn_layer_forward(const float *X, int64_t N, int32_t K
     SpmmArgs a{rowptr, colidx, N, nnz, Zs, F, F, H, ldh, true};
     launch_spmm_norm(a, dev, s);
     return launch_status();
+}
+
+// ---------------------------------------------------------------------------
+// bigcn_layer_forward_static: the layer for callers that cannot allocate.
+//
+// Its workspace is this file-scope device array. In host code the name
+// g_static_scratch is only a host-side shadow of the symbol, not a device
+// address, so the address a kernel may use is looked up once per device with
+// cudaGetSymbolAddress (with that device current) and cached.
+namespace {
+static __device__ __align__(256) unsigned char g_static_scratch[BIGCN_STATIC_SCRATCH_BYTES];
+
+std::once_flag g_scratch_once[kMaxDevices];
+void *g_scratch_addr[kMaxDevices];
+cudaError_t g_scratch_err[kMaxDevices];
+
+void resolve_static_scratch(int dev) {
+    g_scratch_err[dev] = cudaGetSymbolAddress(&g_scratch_addr[dev], g_static_scratch);
+    if (g_scratch_err[dev] != cudaSuccess) {
+        g_scratch_addr[dev] = nullptr;
+        cudaGetLastError();
+    }
+}
+}  // namespace
+
+extern "C" bigcn_status bigcn_layer_forward_static(const float *X, int64_t N, int32_t K,
+                                                   int64_t ldx, const float *scale,
+                                                   const float *shift, const float *Wt,
+                                                   int32_t F, int64_t ldw, const int64_t *rowptr,
+                                                   const int32_t *colidx, int64_t nnz, float *H,
+                                                   int64_t ldh, void *stream) {
+    const size_t need = bigcn_layer_workspace_bytes(N, K, F);
+    if (need > BIGCN_STATIC_SCRATCH_BYTES) return BIGCN_ERR_SCRATCH_LIMIT;
+    DeviceInfo dev;
+    bigcn_status st = current_device(&dev);
+    if (st != BIGCN_OK) return st;
+    std::call_once(g_scratch_once[dev.device], resolve_static_scratch, dev.device);
+    if (g_scratch_err[dev.device] != cudaSuccess) return BIGCN_ERR_CUDA;
+    return bigcn_layer_forward(X, N, K, ldx, scale, shift, Wt, F, ldw, rowptr, colidx, nnz,
+                               g_scratch_addr[dev.device], BIGCN_STATIC_SCRATCH_BYTES, H, ldh,
+                               stream);
 }
