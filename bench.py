@@ -4,12 +4,17 @@
 One step = one pass of the whole hot path over the workload: for each of the
 two layers, centre + sign-pack the node rows (Sec. 6.2, Eqs. 7-8), sign-pack
 the weight columns (Eqs. 3-4), the XNOR-popcount product (Eqs. 11-12) and the
-normalised-adjacency aggregation (Eqs. 1, 13) -- eight C-ABI kernel launches,
-replayed as one CUDA graph with a timing event between every two kernels.
+normalised-adjacency aggregation (Eqs. 1, 13) -- one bigcn_forward_2layer
+call (5 kernels for the usual widths), replayed as a CUDA graph with timing
+events around it. Per-kernel durations come from a second pass of the same
+forward with an event between kernels.
 
 Default workload: C2 (the Citeseer-shaped 2-layer configuration: N=3327,
 K=3703, hidden 64, out 6). Its inputs (49 MB) fit in L2, so L2 is flushed
-(a 256 MiB memset, outside the timed events) before every step.
+before every step, outside the timed events: a 256 MiB buffer is written and
+its first half read back, which leaves L2 holding clean lines of that buffer
+(the inputs come from HBM, and the step does not pay for writing back the
+flush's dirty lines).
 
 Prints one JSON line (rank 0): nodes/s of the device-resident forward, the
 same through host buffers (e2e), per-kernel times and the dominant kernel's
@@ -44,8 +49,6 @@ DEFAULT_WORKLOAD = "C2"
 L2_FLUSH_BYTES = 256 << 20
 POPC_PER_CLK_PER_SM = 16          # 32-bit population counts per clock per SM
 FALLBACK_HBM_GBS = 6800.0
-KERNEL_SOURCES = {"pack_rows": "pack.cu", "pack_weights": "pack.cu",
-                  "xnor_gemm": "xnor_gemm.cu", "spmm": "spmm.cu"}
 
 
 # --------------------------------------------------------------- host logic --
@@ -91,22 +94,34 @@ def induced_subgraph(rowptr, colidx, lo: int, hi: int):
     return out, (cols[keep] - lo).astype(np.int32)
 
 
-def kernel_work(N, K, F, nnz, name):
-    """Algorithmic work of one launch: (amount, unit, bound)."""
-    W = (K + 63) // 64
-    if name == "pack_rows":
-        return 4.0 * N * K + 8.0 * N * W + 4.0 * N + 8.0 * K, "bytes", "hbm"
-    if name == "pack_weights":
-        return 4.0 * K * F + 8.0 * F * W + 4.0 * F, "bytes", "hbm"
-    if name == "xnor_gemm":
-        return float(N) * K * F, "bit-ops", "alu"
-    if name == "spmm":
-        return 8.0 * (N + 1) + 4.0 * nnz + 8.0 * N * F, "bytes", "hbm"
-    raise KeyError(name)
+def kernel_work(w, nnz, name):
+    """Algorithmic work of one launch of the named kernel of the 2-layer
+    forward: (amount, unit, bound)."""
+    N, K, Fh, Fo = w.N, w.K, w.hidden, w.out
+    W1, W2 = (K + 63) // 64, (Fh + 63) // 64
+    csr = 8.0 * (N + 1) + 4.0 * nnz
+    table = {
+        "pack_weights(W1,W2)": (4.0 * K * Fh + 8.0 * Fh * W1 + 4.0 * Fh + 4.0 * Fh * Fo
+                                + 8.0 * Fo * W2 + 4.0 * Fo, "bytes", "hbm"),
+        "L1.pack_rows": (4.0 * N * K + 8.0 * N * W1 + 4.0 * N + 8.0 * K, "bytes", "hbm"),
+        "L1.xnor_gemm": (float(N) * K * Fh, "bit-ops", "alu"),
+        "L1.spmm+L2.pack_rows+L2.xnor_gemm": (csr + 4.0 * N * Fh + 4.0 * N * Fo, "bytes", "hbm"),
+        "L1.spmm": (csr + 8.0 * N * Fh, "bytes", "hbm"),
+        "L2.pack_rows": (4.0 * N * Fh + 8.0 * N * W2 + 4.0 * N, "bytes", "hbm"),
+        "L2.xnor_gemm": (float(N) * Fh * Fo, "bit-ops", "alu"),
+        "L2.spmm": (csr + 8.0 * N * Fo, "bytes", "hbm"),
+    }
+    return table[name]
+
+
+KERNEL_FILES = {"pack_weights(W1,W2)": "pack.cu", "L1.pack_rows": "pack.cu",
+                "L2.pack_rows": "pack.cu", "L1.xnor_gemm": "xnor_gemm.cu",
+                "L2.xnor_gemm": "xnor_gemm.cu", "L1.spmm": "spmm.cu", "L2.spmm": "spmm.cu",
+                "L1.spmm+L2.pack_rows+L2.xnor_gemm": "spmm.cu"}
 
 
 def source_hash(name):
-    path = os.path.join(ROOT, "paper_2010_07565_gb300", "csrc", KERNEL_SOURCES[name])
+    path = os.path.join(ROOT, "paper_2010_07565_gb300", "csrc", KERNEL_FILES[name])
     with open(path, "rb") as f:
         return hashlib.sha256(f.read()).hexdigest()[:16]
 
@@ -115,7 +130,8 @@ def profiled_traffic(name, workload):
     """DRAM bytes per launch from a committed ncu summary, if it was taken on
     the current source of the kernel (profiles/<kernel>_<workload>.txt lines
     'source_sha256_16: ...' and 'dram_bytes_per_launch: ...')."""
-    path = os.path.join(ROOT, "profiles", f"{name}_{workload}.txt")
+    fname = name.replace("(", "_").replace(")", "").replace(",", "_").replace("+", "_")
+    path = os.path.join(ROOT, "profiles", f"{fname}_{workload}.txt")
     if not os.path.exists(path):
         return None
     fields = {}
@@ -261,45 +277,52 @@ def run_gpu(args, rank, world, local_rank):
     import torch.distributed as dist
 
     from paper_2010_07565_gb300 import cost_model
-    from paper_2010_07565_gb300.runner import GCN2Forward, STEP_KERNELS
+    from paper_2010_07565_gb300.runner import GCN2Forward
 
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
     w, data = build_workload(args.workload)
     nnz = int(data["colidx"].shape[0])
-    model = GCN2Forward(w.N, w.K, w.hidden, w.out, nnz, dev)
     host = {k: torch.from_numpy(np.ascontiguousarray(v)).pin_memory() for k, v in data.items()}
+
+    # The timed forward: one CUDA graph of the whole 2-layer forward, with
+    # timing events only around it (event nodes inside a graph cost ~5 us each).
+    model = GCN2Forward(w.N, w.K, w.hidden, w.out, nnz, dev)
     model.load(non_blocking=False, **host)
+    model.capture()
+    # The per-kernel pass: the same forward with an event between kernels.
+    names = model.kernel_names
+    probe = GCN2Forward(w.N, w.K, w.hidden, w.out, nnz, dev)
+    probe.load(non_blocking=False, **host)
+    kev = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(len(names) + 1)]
+    probe.capture(kev)
     torch.cuda.synchronize()
 
-    try:
-        events = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(9)]
-        model.capture(events)
-        launch, how = model.replay, "CUDA graph of the 8 kernel launches, events between kernels"
-    except TypeError:    # torch without external events: plain launches
-        events = [torch.cuda.Event(enable_timing=True) for _ in range(9)]
-        launch, how = (lambda: model.launch(events)), "8 kernel launches, events between kernels"
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    flush_half = flush[: flush.numel() // 2]
 
-    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
-    for _ in range(args.warmup):
+    def flush_l2():
         flush.zero_()
-        launch()
+        flush_half.sum()
+
+    ea, eb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    for _ in range(args.warmup):
+        flush_l2()
+        model.replay()
     torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
 
-    per_kernel = [[] for _ in range(8)]
     step_ms = []
     with ClockSampler(local_rank) as clocks:
         for _ in range(args.steps):
-            flush.zero_()
-            launch()
-            events[8].synchronize()
-            ts = [events[k].elapsed_time(events[k + 1]) for k in range(8)]
-            for k in range(8):
-                per_kernel[k].append(ts[k])
-            step_ms.append(events[0].elapsed_time(events[8]))
+            flush_l2()
+            ea.record()
+            model.replay()
+            eb.record()
+            eb.synchronize()
+            step_ms.append(ea.elapsed_time(eb))
         torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
@@ -307,17 +330,26 @@ def run_gpu(args, rank, world, local_rank):
     max_ms, units = aggregate_over_ranks(total_ms, float(w.N) * args.steps, world)
     value = units / (max_ms * 1e-3)
 
+    # Per-kernel durations (events between kernels, L2 flushed before each pass).
+    per_kernel = [[] for _ in names]
+    for i in range(min(args.steps, 300) + 3):
+        flush_l2()
+        probe.replay()
+        kev[-1].synchronize()
+        if i >= 3:
+            for k in range(len(names)):
+                per_kernel[k].append(kev[k].elapsed_time(kev[k + 1]))
+
     # End to end through host buffers: pinned inputs -> device, forward, logits -> host.
     logits_host = torch.empty((w.N, w.out), dtype=torch.float32).pin_memory()
     h2d = sum(int(v.numel() * v.element_size()) for v in host.values())
     d2h = int(logits_host.numel() * logits_host.element_size())
     e2e_steps = max(3, min(args.steps, 200))
-    ea, eb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e2e_ms = []
     for i in range(e2e_steps + 2):
         ea.record()
         model.load(non_blocking=True, **host)
-        launch()
+        model.replay()
         logits_host.copy_(model.logits, non_blocking=True)
         eb.record()
         eb.synchronize()
@@ -333,26 +365,22 @@ def run_gpu(args, rank, world, local_rank):
     props = torch.cuda.get_device_properties(dev)
     sm_max = float(peaks.get("sm_max_mhz", 2070.0))
     popc_peak = props.multi_processor_count * POPC_PER_CLK_PER_SM * 32 * sm_max * 1e6
-    shapes = [(w.N, w.K, w.hidden), (w.N, w.hidden, w.out)]
     kernels = []
-    for k in range(8):
-        layer, name = k // 4, STEP_KERNELS[k % 4]
-        N, K, F = shapes[layer]
-        work, unit, bound = kernel_work(N, K, F, nnz, name)
-        mean_ms = statistics.fmean(per_kernel[k])
-        kernels.append(dict(layer=layer + 1, name=name, mean_us=1e3 * mean_ms, work=work,
+    for k, name in enumerate(names):
+        work, unit, bound = kernel_work(w, nnz, name)
+        kernels.append(dict(name=name, mean_us=1e3 * statistics.fmean(per_kernel[k]), work=work,
                             unit=unit, bound=bound))
     dom = max(kernels, key=lambda r: r["mean_us"])
     rate = dom["work"] / (dom["mean_us"] * 1e-6)
     if dom["bound"] == "hbm":
         achieved, peak, unit = rate / 1e9, hbm, "GB/s"
-        traffic = profiled_traffic(dom["name"], w.name)
     else:
         achieved, peak, unit = rate / 1e12, popc_peak / 1e12, "T bit-ops/s"
-        traffic = profiled_traffic(dom["name"], w.name)
-    gemm1 = kernels[2]
-    spmm1 = kernels[3]
-    spmm_gbs = spmm1["work"] / (spmm1["mean_us"] * 1e-6) / 1e9
+    traffic = profiled_traffic(dom["name"], w.name)
+    by_name = {r["name"]: r for r in kernels}
+    gemm1 = by_name["L1.xnor_gemm"]
+    agg1 = by_name.get("L1.spmm+L2.pack_rows+L2.xnor_gemm") or by_name["L1.spmm"]
+    spmm_gbs = agg1["work"] / (agg1["mean_us"] * 1e-6) / 1e9
 
     cpu_baseline = None
     if world == 1 and not args.no_cpu_baseline:
@@ -368,14 +396,17 @@ def run_gpu(args, rank, world, local_rank):
         "dtype": "f32+b1", "data": "synthetic",
         "config": {"workload": w.description, "name": w.name, "N": w.N, "K": w.K,
                    "hidden": w.hidden, "out": w.out, "nnz": nnz,
-                   "l2": "flushed before every step (256 MiB memset outside the timed events)",
-                   "launch": how, "parallelism": "replicas" if world > 1 else "single GPU"},
+                   "l2": "flushed before every step outside the timed events (256 MiB written, "
+                         "its first half read back)",
+                   "launch": f"one CUDA graph per step: bigcn_forward_2layer, {len(names)} kernels",
+                   "parallelism": "replicas" if world > 1 else "single GPU"},
         "components": {
             "xnor_gemm_bitops_per_s": gemm1["work"] / (gemm1["mean_us"] * 1e-6),
             "spmm_gbs": spmm_gbs, "spmm_pct_of_hbm_peak": 100.0 * spmm_gbs / hbm,
-            "per_kernel_us": {f"L{r['layer']}.{r['name']}": round(r["mean_us"], 3)
-                              for r in kernels}},
-        "roofline": {"kernel": f"L{dom['layer']}.{dom['name']}", "bound": dom["bound"],
+            "per_kernel_us": {r["name"]: round(r["mean_us"], 3) for r in kernels},
+            "per_kernel_note": "from a second pass of the same graph with an event node "
+                               "between kernels (each node adds a few us)"},
+        "roofline": {"kernel": dom["name"], "bound": dom["bound"],
                      "achieved": achieved, "peak": peak, "unit": unit, "frac": achieved / peak,
                      "traffic": traffic,
                      "peak_source": (f"{peak_kind} MEASURED_PEAKS.json hbm_gbs"
@@ -385,7 +416,7 @@ def run_gpu(args, rank, world, local_rank):
         "cpu_baseline": cpu_baseline,
         "e2e": {"value": e2e_units / (e2e_max * 1e-3), "unit": "nodes/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-        "gpu_launches": 8 * args.steps,
+        "gpu_launches": len(names) * args.steps,
         "clocks": clocks.summary(),
         "paper_context": {
             "cycle_ops_gcn": cost_model.cycle_ops(w.N, nnz // 2, dims, False),

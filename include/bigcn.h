@@ -189,6 +189,46 @@ bigcn_status bigcn_layer_forward(const float *X, int64_t N, int32_t K, int64_t l
                                  int64_t nnz, void *workspace, size_t ws_bytes,
                                  float *H, int64_t ldh, void *stream);
 
+/*
+ * The two-layer Bi-GCN of Sec. 6.2 in one call: a hidden layer of width Fh on
+ * the centred features (scale/shift as in bigcn_pack_rows) and an output
+ * layer of width Fo on the hidden layer's output taken raw (no activation,
+ * Sec. 4.1.2), both H = A~ zeta (Eq. 13) over the same graph:
+ *
+ *   H1  = D^-1/2 (A + I) D^-1/2 zeta(X centred, W1)      N x Fh
+ *   out = D^-1/2 (A + I) D^-1/2 zeta(H1, W2)             N x Fo (the logits)
+ *
+ * The result equals two bigcn_layer_forward calls within fp32 rounding.
+ * When Fh is a multiple of 4 and at most 128 and Fo <= 64, layer 1's
+ * aggregation kernel also binarizes H1 and computes layer 2's XNOR product
+ * while the row is in registers, so H1 never goes through memory; the call
+ * then launches 5 kernels, otherwise 7 (bigcn_forward_2layer_launches).
+ *
+ * X N x K (ldx), W1 K x Fh (ldw1), W2 Fh x Fo (ldw2), CSR as in
+ * bigcn_spmm_norm, out N x Fo (ldo).
+ * H1         nullable; if given (N x Fh, ldh1) it also receives layer 1's output.
+ * workspace  >= bigcn_forward_2layer_workspace_bytes(N, K, Fh, Fo) bytes of
+ *            device memory, 256-byte aligned, overlapping nothing else.
+ * events     nullable array of n_events cudaEvent_t (as void*): event q is
+ *            recorded on `stream` before kernel q and the last one after the
+ *            last kernel (recorded with cudaEventRecordExternal), for timing
+ *            each kernel; entries beyond launches + 1 are not touched.
+ * out, H1 and the workspace must not overlap each other or any input.
+ */
+size_t bigcn_forward_2layer_workspace_bytes(int64_t N, int32_t K, int32_t Fh, int32_t Fo);
+
+/* Kernel launches bigcn_forward_2layer makes for these widths (5 or 7). */
+int32_t bigcn_forward_2layer_launches(int32_t Fh, int32_t Fo);
+
+bigcn_status bigcn_forward_2layer(const float *X, int64_t N, int32_t K, int64_t ldx,
+                                  const float *scale, const float *shift,
+                                  const float *W1, int32_t Fh, int64_t ldw1,
+                                  const float *W2, int32_t Fo, int64_t ldw2,
+                                  const int64_t *rowptr, const int32_t *colidx, int64_t nnz,
+                                  void *workspace, size_t ws_bytes,
+                                  float *H1, int64_t ldh1, float *out, int64_t ldo,
+                                  void *const *events, int32_t n_events, void *stream);
+
 /* Bytes of the device scratch array behind bigcn_layer_forward_static. */
 #define BIGCN_STATIC_SCRATCH_BYTES ((size_t)32 << 20)
 

@@ -47,6 +47,11 @@ SIGNATURES = {
     "bigcn_layer_workspace_bytes": ([_i64, _i32, _i32], _sz),
     "bigcn_layer_forward": ([_p, _i64, _i32, _i64, _p, _p, _p, _i32, _i64, _p, _p, _i64, _p,
                              _sz, _p, _i64, _p], ctypes.c_int),
+    "bigcn_forward_2layer_workspace_bytes": ([_i64, _i32, _i32, _i32], _sz),
+    "bigcn_forward_2layer_launches": ([_i32, _i32], _i32),
+    "bigcn_forward_2layer": ([_p, _i64, _i32, _i64, _p, _p, _p, _i32, _i64, _p, _i32, _i64, _p,
+                              _p, _i64, _p, _sz, _p, _i64, _p, _i64, _p, _i32, _p],
+                             ctypes.c_int),
     "bigcn_layer_forward_static": ([_p, _i64, _i32, _i64, _p, _p, _p, _i32, _i64, _p, _p, _i64,
                                     _p, _i64, _p], ctypes.c_int),
 }
@@ -183,6 +188,36 @@ def bigcn_layer_forward(X, scale, shift, Wt, rowptr, colidx, workspace, H, strea
         _ptr(X), N, K, _ld(X), _ptr(scale), _ptr(shift), _ptr(Wt), F, _ld(Wt), _ptr(rowptr),
         _ptr(colidx) if colidx.numel() else None, colidx.numel(), _ptr(workspace),
         workspace.numel() * workspace.element_size(), _ptr(H), _ld(H), _stream(stream)))
+
+
+def bigcn_forward_2layer_workspace_bytes(N: int, K: int, Fh: int, Fo: int) -> int:
+    return int(lib().bigcn_forward_2layer_workspace_bytes(N, K, Fh, Fo))
+
+
+def bigcn_forward_2layer_launches(Fh: int, Fo: int) -> int:
+    return int(lib().bigcn_forward_2layer_launches(Fh, Fo))
+
+
+def bigcn_forward_2layer(X, scale, shift, W1, W2, rowptr, colidx, workspace, out, H1=None,
+                         events=None, stream=None):
+    """The two-layer forward of Sec. 6.2 (hidden layer on centred X, output
+    layer on H1 raw). ``events``: torch.cuda.Event objects (created with
+    enable_timing=True, external=True and recorded once) to be recorded
+    before each kernel and after the last."""
+    N, K = X.shape
+    Fh, Fo = W1.shape[1], W2.shape[1]
+    if W2.shape[0] != Fh:
+        raise ValueError("W2 must have as many rows as W1 has columns")
+    if events:
+        ev = (ctypes.c_void_p * len(events))(*[e.cuda_event for e in events])
+        n_ev = len(events)
+    else:
+        ev, n_ev = None, 0
+    _check("bigcn_forward_2layer", lib().bigcn_forward_2layer(
+        _ptr(X), N, K, _ld(X), _ptr(scale), _ptr(shift), _ptr(W1), Fh, _ld(W1), _ptr(W2), Fo,
+        _ld(W2), _ptr(rowptr), _ptr(colidx) if colidx.numel() else None, colidx.numel(),
+        _ptr(workspace), workspace.numel() * workspace.element_size(), _ptr(H1),
+        _ld(H1) if H1 is not None else 0, _ptr(out), _ld(out), ev, n_ev, _stream(stream)))
 
 
 def bigcn_layer_forward_static(X, scale, shift, Wt, rowptr, colidx, H, stream=None):

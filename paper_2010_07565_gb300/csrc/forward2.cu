@@ -1,0 +1,175 @@
+// The two-layer Bi-GCN forward of Sec. 6.2 (Wang et al., CVPR 2021) as one
+// call: layer 1 centred (Sec. 6.2), layer 2 on H1 raw (Sec. 4.1.2), each
+// layer Eq. 13 with zeta of Eqs. 11-12. Kernel sequence on one stream:
+//
+//   0 pack W1 and W2 (one launch)                          Eqs. 3-4
+//   1 pack rows of X, centred                              Sec. 6.2, Eqs. 7-8
+//   2 XNOR GEMM, rows scaled by 1/sqrt(dhat)               Eqs. 11-12
+//   3 aggregation of layer 1 fused with layer 2's row      Eq. 13, then
+//     packing and XNOR GEMM (H1 stays in registers)        Eqs. 7-8, 11-12
+//   4 aggregation of layer 2 -> logits                     Eq. 13
+//
+// When the widths do not fit the fused kernel (hidden width not a multiple
+// of 4 or above 128, or more than 64 outputs) step 3 runs as three kernels:
+// aggregation, packing, GEMM. Either way every step runs on the GPU.
+#include "launch.cuh"
+
+namespace bigcn {
+namespace {
+
+constexpr size_t kAlign = 256;
+size_t round_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+
+struct Forward2Workspace {
+    size_t bits1, alpha1, wbits1, beta1, z1, wbits2, beta2, z2, h1, bits2, alpha2, total;
+};
+
+bool forward2_workspace(int64_t N, int32_t K, int32_t Fh, int32_t Fo, Forward2Workspace *w) {
+    if (N < 0 || K < 1 || Fh < 1 || Fo < 1) return false;
+    const int64_t w1 = bigcn_words(K), w2 = bigcn_words(Fh);
+    int64_t widest = w1;
+    if (Fh > widest) widest = Fh;
+    if (Fo > widest) widest = Fo;
+    if (N > kMaxElems / widest) return false;
+    size_t off = 0;
+    auto take = [&](size_t bytes) { size_t at = off; off = round_up(off + bytes); return at; };
+    w->bits1 = take(size_t(N) * w1 * 8);
+    w->alpha1 = take(size_t(N) * 4);
+    w->wbits1 = take(size_t(Fh) * w1 * 8);
+    w->beta1 = take(size_t(Fh) * 4);
+    w->z1 = take(size_t(N) * Fh * 4);
+    w->wbits2 = take(size_t(Fo) * w2 * 8);
+    w->beta2 = take(size_t(Fo) * 4);
+    w->z2 = take(size_t(N) * Fo * 4);
+    w->h1 = take(size_t(N) * Fh * 4);
+    w->bits2 = take(size_t(N) * w2 * 8);
+    w->alpha2 = take(size_t(N) * 4);
+    w->total = off;
+    return true;
+}
+
+}  // namespace
+}  // namespace bigcn
+
+using namespace bigcn;
+
+extern "C" size_t bigcn_forward_2layer_workspace_bytes(int64_t N, int32_t K, int32_t Fh,
+                                                       int32_t Fo) {
+    Forward2Workspace w;
+    return forward2_workspace(N, K, Fh, Fo, &w) ? w.total : 0;
+}
+
+extern "C" int32_t bigcn_forward_2layer_launches(int32_t Fh, int32_t Fo) {
+    return spmm_pack_gemm_supported(Fh, Fo) ? 5 : 7;
+}
+
+extern "C" bigcn_status bigcn_forward_2layer(
+    const float *X, int64_t N, int32_t K, int64_t ldx, const float *scale, const float *shift,
+    const float *W1, int32_t Fh, int64_t ldw1, const float *W2, int32_t Fo, int64_t ldw2,
+    const int64_t *rowptr, const int32_t *colidx, int64_t nnz, void *workspace, size_t ws_bytes,
+    float *H1, int64_t ldh1, float *out, int64_t ldo, void *const *events, int32_t n_events,
+    void *stream) {
+    Forward2Workspace w;
+    if (N < 0 || N > int64_t(INT32_MAX) || K < 1 || Fh < 1 || Fo < 1 || ldx < K || ldw1 < Fh ||
+        ldw2 < Fo || ldo < Fo || (H1 && ldh1 < Fh) || nnz < 0 || n_events < 0)
+        return BIGCN_ERR_INVALID_ARG;
+    if ((scale == nullptr) != (shift == nullptr)) return BIGCN_ERR_INVALID_ARG;
+    if (!forward2_workspace(N, K, Fh, Fo, &w)) return BIGCN_ERR_INVALID_ARG;
+    if (N > 0 && (N > kMaxElems / ldx || N > kMaxElems / ldo || (H1 && N > kMaxElems / ldh1)))
+        return BIGCN_ERR_INVALID_ARG;
+    if (int64_t(K) > kMaxElems / ldw1 || int64_t(Fh) > kMaxElems / ldw2)
+        return BIGCN_ERR_INVALID_ARG;
+    if (N == 0) return BIGCN_OK;
+    if (!X || !W1 || !W2 || !rowptr || !out || !workspace || (nnz > 0 && !colidx) ||
+        (n_events > 0 && !events))
+        return BIGCN_ERR_INVALID_ARG;
+    if (ws_bytes < w.total) return BIGCN_ERR_INVALID_ARG;
+    if (!aligned_to(X, 4) || !aligned_to(W1, 4) || !aligned_to(W2, 4) || !aligned_to(rowptr, 8) ||
+        (colidx && !aligned_to(colidx, 4)) || !aligned_to(out, 4) || (H1 && !aligned_to(H1, 4)) ||
+        !aligned_to(workspace, kAlign) ||
+        (scale && (!aligned_to(scale, 4) || !aligned_to(shift, 4))))
+        return BIGCN_ERR_MISALIGNED;
+    const void *in[] = {X, W1, W2, rowptr, colidx, scale, shift};
+    const size_t in_bytes[] = {span_bytes(N, K, ldx, 4), span_bytes(K, Fh, ldw1, 4),
+                               span_bytes(Fh, Fo, ldw2, 4), size_t(N + 1) * 8, size_t(nnz) * 4,
+                               size_t(K) * 4, size_t(K) * 4};
+    const void *outs[] = {workspace, out, H1};
+    const size_t out_bytes[] = {w.total, span_bytes(N, Fo, ldo, 4),
+                                H1 ? span_bytes(N, Fh, ldh1, 4) : 0};
+    for (int o = 0; o < 3; ++o) {
+        for (int q = 0; q < 7; ++q)
+            if (overlaps(outs[o], out_bytes[o], in[q], in_bytes[q])) return BIGCN_ERR_INVALID_ARG;
+        for (int p = o + 1; p < 3; ++p)
+            if (overlaps(outs[o], out_bytes[o], outs[p], out_bytes[p])) return BIGCN_ERR_INVALID_ARG;
+    }
+
+    DeviceInfo dev;
+    bigcn_status st = current_device(&dev);
+    if (st != BIGCN_OK) return st;
+
+    char *ws = static_cast<char *>(workspace);
+    auto at = [&](size_t off) { return static_cast<void *>(ws + off); };
+    uint64_t *bits1 = static_cast<uint64_t *>(at(w.bits1));
+    float *alpha1 = static_cast<float *>(at(w.alpha1));
+    uint64_t *wbits1 = static_cast<uint64_t *>(at(w.wbits1));
+    float *beta1 = static_cast<float *>(at(w.beta1));
+    float *Z1 = static_cast<float *>(at(w.z1));
+    uint64_t *wbits2 = static_cast<uint64_t *>(at(w.wbits2));
+    float *beta2 = static_cast<float *>(at(w.beta2));
+    float *Z2 = static_cast<float *>(at(w.z2));
+    const int words1 = bigcn_words(K), words2 = bigcn_words(Fh);
+    cudaStream_t s = as_stream(stream);
+    // Inside a stream capture an event must be recorded as an external node
+    // to be timed later; outside a capture a plain record does that.
+    cudaStreamCaptureStatus capture = cudaStreamCaptureStatusNone;
+    if (n_events > 0 && cudaStreamIsCapturing(s, &capture) != cudaSuccess) {
+        cudaGetLastError();
+        return BIGCN_ERR_CUDA;
+    }
+    int recorded = 0;
+    bool event_failed = false;
+    auto mark = [&]() {
+        if (recorded < n_events) {
+            cudaEvent_t ev = static_cast<cudaEvent_t>(events[recorded]);
+            const cudaError_t r = capture == cudaStreamCaptureStatusActive
+                                      ? cudaEventRecordWithFlags(ev, s, cudaEventRecordExternal)
+                                      : cudaEventRecord(ev, s);
+            if (r != cudaSuccess) event_failed = true;
+        }
+        ++recorded;
+    };
+
+    mark();
+    WeightPack p1{W1, K, Fh, ldw1, wbits1, words1, beta1, 0};
+    WeightPack p2{W2, Fh, Fo, ldw2, wbits2, words2, beta2, 0};
+    launch_pack_weights2(p1, p2, s);
+    mark();
+    launch_pack_rows(X, N, K, ldx, scale, shift, bits1, words1, alpha1, dev, s);
+    mark();
+    GemmArgs g1{bits1, alpha1, N, wbits1, beta1, Fh, K, words1, Z1, Fh, nullptr, rowptr};
+    launch_xnor_gemm(g1, dev, s);
+    mark();
+    if (spmm_pack_gemm_supported(Fh, Fo)) {
+        SpmmPackGemmArgs f{rowptr, colidx, N, nnz, Z1, Fh, H1, ldh1, wbits2, beta2, Fo, Z2, Fo};
+        launch_spmm_pack_gemm(f, s);
+        mark();
+    } else {
+        float *H1w = H1 ? H1 : static_cast<float *>(at(w.h1));
+        const int64_t ldh = H1 ? ldh1 : Fh;
+        uint64_t *bits2 = static_cast<uint64_t *>(at(w.bits2));
+        float *alpha2 = static_cast<float *>(at(w.alpha2));
+        SpmmArgs a1{rowptr, colidx, N, nnz, Z1, Fh, Fh, H1w, ldh, true};
+        launch_spmm_norm(a1, dev, s);
+        mark();
+        launch_pack_rows(H1w, N, Fh, ldh, nullptr, nullptr, bits2, words2, alpha2, dev, s);
+        mark();
+        GemmArgs g2{bits2, alpha2, N, wbits2, beta2, Fo, Fh, words2, Z2, Fo, nullptr, rowptr};
+        launch_xnor_gemm(g2, dev, s);
+        mark();
+    }
+    SpmmArgs a2{rowptr, colidx, N, nnz, Z2, Fo, Fo, out, ldo, true};
+    launch_spmm_norm(a2, dev, s);
+    mark();
+    const bigcn_status ls = launch_status();
+    return event_failed ? BIGCN_ERR_CUDA : ls;
+}

@@ -20,6 +20,21 @@ void launch_pack_rows(const float *X, int64_t N, int K, int64_t ldx, const float
 void launch_pack_weights(const float *Wt, int K, int F, int64_t ldw, uint64_t *bits,
                          int words, float *beta, cudaStream_t stream);
 
+// One weight matrix to pack: W (K x F, row stride ldw) -> bits (F x words), beta.
+struct WeightPack {
+    const float *W;
+    int K;
+    int F;
+    int64_t ldw;
+    uint64_t *bits;
+    int words;
+    float *beta;
+    int tiles;               // set by the launcher
+};
+
+// Step 3 for two matrices in one launch (b.W == nullptr: a only).
+void launch_pack_weights2(const WeightPack &a, const WeightPack &b, cudaStream_t stream);
+
 struct GemmArgs {
     const uint64_t *A;       // N x words packed node rows
     const float *alpha;      // N per-node scales
@@ -53,5 +68,30 @@ struct SpmmArgs {
 
 // Step 5: H = D^-1/2 (A + I) D^-1/2 Z (Eqs. 1, 13).
 void launch_spmm_norm(const SpmmArgs &args, const DeviceInfo &dev, cudaStream_t stream);
+
+// Largest layer-2 output width the fused aggregation handles.
+constexpr int kMaxFusedOut = 64;
+
+struct SpmmPackGemmArgs {
+    const int64_t *rowptr;
+    const int32_t *colidx;
+    int64_t N;
+    int64_t nnz;
+    const float *Z1;         // N x Fh, rows pre-scaled by 1/sqrt(dhat), row stride Fh
+    int Fh;
+    float *H1;               // nullable N x Fh output (row stride ldh)
+    int64_t ldh;
+    const uint64_t *wbits2;  // Fo x ceil(Fh/64) packed columns of W2
+    const float *beta2;      // Fo
+    int Fo;
+    float *Z2;               // N x Fo, rows pre-scaled by 1/sqrt(dhat) (row stride ldz2)
+    int64_t ldz2;
+};
+
+// Whether (Fh, Fo) fit the fused kernel: Fh % 4 == 0, Fh <= 128, Fo <= 64.
+bool spmm_pack_gemm_supported(int Fh, int Fo);
+
+// Layer-1 step 5 fused with layer-2 steps 2 and 4 (see spmm.cu).
+void launch_spmm_pack_gemm(const SpmmPackGemmArgs &args, cudaStream_t stream);
 
 }  // namespace bigcn

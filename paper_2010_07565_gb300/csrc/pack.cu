@@ -14,8 +14,8 @@
 // shared memory, so alpha does not depend on scheduling.
 //
 // pack_weights reads W (K x F) column-wise: thread (x, y) of a 32 x 8 block
-// owns column 32*bx + x and builds whole 64-bit words from 64 coalesced row
-// reads. The words of a column are spread over a cluster of S <= 8 blocks
+// owns one column and builds whole 64-bit words from 64 coalesced row reads;
+// one launch can pack two matrices (both layers' weights). The words of a column are spread over a cluster of S <= 8 blocks
 // (grid y); each block reduces its |W| partial sums in shared memory, and
 // block 0 of the cluster adds the S partials through distributed shared
 // memory in rank order (deterministic).
@@ -86,33 +86,38 @@ constexpr int kWCols = 32;
 constexpr int kWRows = 8;
 constexpr int kMaxCluster = 8;
 
+// Blocks with blockIdx.x < a.tiles pack matrix a, the rest matrix b (one
+// launch can pack both layers' weights); each block owns 32 columns.
 __global__ void __launch_bounds__(kWCols *kWRows)
-pack_weights_kernel(const float *__restrict__ Wt, int K, int F, int64_t ldw,
-                    uint64_t *__restrict__ bits, int words, float *__restrict__ beta) {
+pack_weights_kernel(WeightPack a, WeightPack b) {
     __shared__ float partial[kWRows][kWCols];
     __shared__ float colsum[kWCols];
     cg::cluster_group cluster = cg::this_cluster();
     const int S = int(cluster.num_blocks());
     const int rank = int(cluster.block_rank());
+    const bool first = int(blockIdx.x) < a.tiles;
+    const WeightPack &m = first ? a : b;
+    const int tile = first ? int(blockIdx.x) : int(blockIdx.x) - a.tiles;
     const int tx = threadIdx.x, ty = threadIdx.y;
-    const int j = blockIdx.x * kWCols + tx;
+    const int j = tile * kWCols + tx;
+    const int K = m.K;
 
     float l1 = 0.0f;
-    if (j < F) {
-        for (int w = rank * kWRows + ty; w < words; w += S * kWRows) {
+    if (j < m.F) {
+        for (int w = rank * kWRows + ty; w < m.words; w += S * kWRows) {
             const int kb = w * 64;
             float v[64];
 #pragma unroll
-            for (int b = 0; b < 64; ++b)
-                v[b] = (kb + b < K) ? __ldg(Wt + int64_t(kb + b) * ldw + j) : 0.0f;
+            for (int q = 0; q < 64; ++q)
+                v[q] = (kb + q < K) ? __ldg(m.W + int64_t(kb + q) * m.ldw + j) : 0.0f;
             uint64_t word = 0;
 #pragma unroll
-            for (int b = 0; b < 64; ++b) {
-                const bool in = kb + b < K;
-                word |= uint64_t(in && v[b] >= 0.0f) << b;
-                l1 += fabsf(v[b]);
+            for (int q = 0; q < 64; ++q) {
+                const bool in = kb + q < K;
+                word |= uint64_t(in && v[q] >= 0.0f) << q;
+                l1 += fabsf(v[q]);
             }
-            bits[int64_t(j) * words + w] = word;
+            m.bits[int64_t(j) * m.words + w] = word;
         }
     }
     partial[ty][tx] = l1;
@@ -124,10 +129,10 @@ pack_weights_kernel(const float *__restrict__ Wt, int K, int F, int64_t ldw,
         colsum[tx] = s;
     }
     cluster.sync();
-    if (rank == 0 && ty == 0 && j < F) {
+    if (rank == 0 && ty == 0 && j < m.F) {
         float s = 0.0f;
         for (int r = 0; r < S; ++r) s += cluster.map_shared_rank(colsum, r)[tx];
-        beta[j] = s / float(K);
+        m.beta[j] = s / float(K);
     }
     cluster.sync();   // peers keep their shared memory until block 0 has read it
 }
@@ -155,13 +160,17 @@ void launch_pack_rows(const float *X, int64_t N, int K, int64_t ldx, const float
             X, N, K, ldx, nullptr, nullptr, b32, int64_t(words) * 2, alpha, G);
 }
 
-void launch_pack_weights(const float *Wt, int K, int F, int64_t ldw, uint64_t *bits,
-                         int words, float *beta, cudaStream_t stream) {
-    // One block row per 8 words, at most a cluster of 8.
-    int S = (words + kWRows - 1) / kWRows;
+void launch_pack_weights2(const WeightPack &a, const WeightPack &b, cudaStream_t stream) {
+    // One block row per 8 words of the longer matrix, at most a cluster of 8.
+    auto rows = [](const WeightPack &m) { return (m.words + kWRows - 1) / kWRows; };
+    WeightPack A = a, B = b;
+    A.tiles = (a.F + kWCols - 1) / kWCols;
+    B.tiles = (b.W != nullptr) ? (b.F + kWCols - 1) / kWCols : 0;
+    int S = rows(A);
+    if (B.tiles > 0 && rows(B) > S) S = rows(B);
     if (S > kMaxCluster) S = kMaxCluster;
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((F + kWCols - 1) / kWCols, S, 1);
+    cfg.gridDim = dim3(A.tiles + B.tiles, S, 1);
     cfg.blockDim = dim3(kWCols, kWRows, 1);
     cfg.dynamicSmemBytes = 0;
     cfg.stream = stream;
@@ -172,7 +181,14 @@ void launch_pack_weights(const float *Wt, int K, int F, int64_t ldw, uint64_t *b
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    cudaLaunchKernelEx(&cfg, pack_weights_kernel, Wt, K, F, ldw, bits, words, beta);
+    cudaLaunchKernelEx(&cfg, pack_weights_kernel, A, B);
+}
+
+void launch_pack_weights(const float *Wt, int K, int F, int64_t ldw, uint64_t *bits,
+                         int words, float *beta, cudaStream_t stream) {
+    WeightPack a{Wt, K, F, ldw, bits, words, beta, 0};
+    WeightPack none{nullptr, 1, 0, 0, nullptr, 0, nullptr, 0};
+    launch_pack_weights2(a, none, stream);
 }
 
 }  // namespace bigcn

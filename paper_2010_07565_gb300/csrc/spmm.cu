@@ -136,6 +136,121 @@ spmm_norm_kernel(const int64_t *__restrict__ rowptr, const int32_t *__restrict__
     }
 }
 
+// ---------------------------------------------------------------------------
+// Layer-1 aggregation fused with layer 2's binarization and product.
+//
+// Each warp computes H1_i = dinv_i * sum_j Z1'_j exactly as the kernel above
+// (VEC = 4, one vector per lane, pre-scaled rows), then, without writing H1
+// (unless asked to), takes layer 2's steps on the row while it is still in
+// registers: the signs of its Fh <= 128 features become one or two 64-bit
+// words (four ballots, one per vector component, spread into place), the
+// row scale alpha2_i = mean |H1_i| is one warp reduction, and the XNOR
+// popcount against the (shared-memory) packed columns of W2 gives
+//   Z2'_ij = (alpha2_i * dinv_i) * (beta2_j * (Fh - 2 popc(h_i ^ w_j))),
+// the same expression the product's degree-scaled epilogue evaluates.
+
+// Spreads 16 bits so that bit i lands on bit 4i of a 64-bit word.
+__device__ __forceinline__ uint64_t spread16by4(uint32_t x) {
+    uint64_t v = x & 0xFFFFu;
+    v = (v | (v << 24)) & 0x000000FF000000FFull;
+    v = (v | (v << 12)) & 0x000F000F000F000Full;
+    v = (v | (v << 6)) & 0x0303030303030303ull;
+    v = (v | (v << 3)) & 0x1111111111111111ull;
+    return v;
+}
+
+template <int L>
+__global__ void __launch_bounds__(kSpmmThreads, 4)
+spmm_pack_gemm_kernel(const int64_t *__restrict__ rowptr, const int32_t *__restrict__ colidx,
+                      int64_t N, int64_t nnz, const float *__restrict__ Z1, int Fh,
+                      float *__restrict__ H1, int64_t ldh, const uint64_t *__restrict__ wbits2,
+                      const float *__restrict__ beta2, int Fo, int words2,
+                      float *__restrict__ Z2, int64_t ldz2) {
+    constexpr int P = 32 / L;
+    __shared__ uint64_t sW[kMaxFusedOut * 2];
+    __shared__ float sBeta[kMaxFusedOut];
+    for (int q = threadIdx.x; q < Fo * words2; q += kSpmmThreads) sW[q] = __ldg(wbits2 + q);
+    for (int q = threadIdx.x; q < Fo; q += kSpmmThreads) sBeta[q] = __ldg(beta2 + q);
+    __syncthreads();
+
+    const int lane = threadIdx.x & 31;
+    const int64_t i = (int64_t(blockIdx.x) * kSpmmThreads + threadIdx.x) >> 5;
+    if (i >= N) return;
+    const int g = lane / L, sl = lane % L;
+    const int f = sl * 4;                      // this lane's first feature
+
+    const int64_t rb = __ldg(rowptr + i), re = __ldg(rowptr + i + 1);
+    const int64_t b = min(max(rb, int64_t(0)), nnz);
+    const int64_t e = min(max(re, b), nnz);
+    const float dinv_i = inv_sqrt_degree(e - b);
+    const int64_t total = (e - b) + 1;
+
+    float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+    for (int64_t base = 0; base < total; base += 32) {
+        int j = -1;
+        const int64_t q = base + lane;
+        if (q < total) {
+            j = (q == 0) ? int(i) : __ldg(colidx + b + q - 1);
+            if (j < 0 || j >= N) j = -1;
+        }
+        const int cnt = int(min(total - base, int64_t(32)));
+        for (int t0 = 0; t0 < cnt; t0 += P * kUnroll) {
+            float4 val[kUnroll];
+            bool live[kUnroll];
+#pragma unroll
+            for (int u = 0; u < kUnroll; ++u) {
+                const int src = t0 + u * P + g;
+                const int jj = __shfl_sync(kFullMask, j, src & 31);
+                live[u] = src < cnt && jj >= 0 && f < Fh;
+                val[u] = live[u] ? __ldg(reinterpret_cast<const float4 *>(Z1 + int64_t(jj) * Fh + f))
+                                 : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+#pragma unroll
+            for (int u = 0; u < kUnroll; ++u) {
+                acc[0] += val[u].x;
+                acc[1] += val[u].y;
+                acc[2] += val[u].z;
+                acc[3] += val[u].w;
+            }
+        }
+    }
+#pragma unroll
+    for (int o = L; o < 32; o <<= 1)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) acc[c] += __shfl_xor_sync(kFullMask, acc[c], o);
+
+    float h[4];
+#pragma unroll
+    for (int c = 0; c < 4; ++c) h[c] = acc[c] * dinv_i;
+    if (H1 != nullptr && g == 0) {
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+            if (f + c < Fh) H1[i * ldh + f + c] = h[c];
+    }
+
+    // Layer 2, Eqs. 7-8: signs of H1_i packed LSB-first, and its mean |.|.
+    uint64_t w0 = 0, w1 = 0;
+    float l1 = 0.0f;
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+        const bool in = g == 0 && f + c < Fh;
+        const unsigned m = __ballot_sync(kFullMask, in && h[c] >= 0.0f);
+        w0 |= spread16by4(m) << c;
+        w1 |= spread16by4(m >> 16) << c;
+        l1 += in ? fabsf(h[c]) : 0.0f;
+    }
+    l1 = warp_sum(l1);
+    const float a = (l1 / float(Fh)) * dinv_i;
+
+    // Layer 2, Eqs. 11-12, pre-scaled by this row's 1/sqrt(dhat_i).
+    for (int jo = lane; jo < Fo; jo += 32) {
+        int mism = __popcll(w0 ^ sW[jo * words2]);
+        if (words2 > 1) mism += __popcll(w1 ^ sW[jo * words2 + 1]);
+        const int d = Fh - 2 * mism;
+        Z2[i * ldz2 + jo] = a * (sBeta[jo] * float(d));
+    }
+}
+
 template <int VEC, int L, int NV, bool kPre>
 void launch_cfg(const SpmmArgs &a, cudaStream_t s) {
     constexpr int SLAB = L * NV * VEC;
@@ -175,6 +290,26 @@ void launch_spmm_norm(const SpmmArgs &a, const DeviceInfo &, cudaStream_t stream
     if (a.N == 0) return;
     if (a.prescaled) launch_pre<true>(a, stream);
     else launch_pre<false>(a, stream);
+}
+
+bool spmm_pack_gemm_supported(int Fh, int Fo) {
+    return Fh >= 1 && Fh <= 128 && Fh % 4 == 0 && Fo >= 1 && Fo <= kMaxFusedOut;
+}
+
+void launch_spmm_pack_gemm(const SpmmPackGemmArgs &a, cudaStream_t s) {
+    if (a.N == 0) return;
+    const int nvec = a.Fh / 4;
+    const dim3 grid(unsigned((a.N + kSpmmThreads / 32 - 1) / (kSpmmThreads / 32)));
+    const int words2 = (a.Fh + 63) / 64;
+#define BIGCN_LAUNCH_SPG(LL)                                                                  \
+    spmm_pack_gemm_kernel<LL><<<grid, kSpmmThreads, 0, s>>>(a.rowptr, a.colidx, a.N, a.nnz,   \
+                                                            a.Z1, a.Fh, a.H1, a.ldh, a.wbits2, \
+                                                            a.beta2, a.Fo, words2, a.Z2, a.ldz2)
+    if (nvec <= 4) BIGCN_LAUNCH_SPG(4);
+    else if (nvec <= 8) BIGCN_LAUNCH_SPG(8);
+    else if (nvec <= 16) BIGCN_LAUNCH_SPG(16);
+    else BIGCN_LAUNCH_SPG(32);
+#undef BIGCN_LAUNCH_SPG
 }
 
 }  // namespace bigcn

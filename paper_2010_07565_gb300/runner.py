@@ -1,16 +1,16 @@
-"""Two-layer Bi-GCN forward on one GPU: device buffers and the sequence of
-C-ABI calls, optionally replayed as a CUDA graph.
+"""Two-layer Bi-GCN forward on one GPU: device buffers, the C-ABI calls and
+their CUDA-graph capture.
 
-This is plumbing around libbigcn.so: torch owns the device memory and the
-stream, and every step of the computation is one call of the C interface:
+Plumbing around libbigcn.so: torch owns the device memory and the stream,
+and every step of the computation runs in the library's kernels.
 
-    layer 1:  bigcn_pack_rows (centred)  -> bigcn_pack_weights
-              -> bigcn_xnor_gemm_degscaled -> bigcn_spmm_prescaled
-    layer 2:  the same four calls on H1, without centring (Sec. 4.1.2)
-
-i.e. two bigcn_layer_forward's worth of kernels, issued one by one so that
-callers can put timing events between them. The layer-2 output is the
-logits (no softmax: Eq. 2 belongs to training).
+``launch()`` makes the one call ``bigcn_forward_2layer`` (5 kernels for the
+usual widths: both weight packs, layer-1 row pack, layer-1 XNOR GEMM, layer-1
+aggregation fused with layer 2's pack and GEMM, layer-2 aggregation).
+``launch_steps()`` runs the same forward as eight separate step calls
+(pack_rows, pack_weights, xnor_gemm_degscaled, spmm_prescaled per layer),
+keeping every intermediate in its own buffer, for step-by-step checks.
+The output is the logits (no softmax: Eq. 2 belongs to training).
 """
 from __future__ import annotations
 
@@ -21,28 +21,35 @@ from . import binding as B
 STEP_KERNELS = ("pack_rows", "pack_weights", "xnor_gemm", "spmm")
 
 
+def fused_kernel_names(Fh: int, Fo: int):
+    if B.bigcn_forward_2layer_launches(Fh, Fo) == 5:
+        return ("pack_weights(W1,W2)", "L1.pack_rows", "L1.xnor_gemm",
+                "L1.spmm+L2.pack_rows+L2.xnor_gemm", "L2.spmm")
+    return ("pack_weights(W1,W2)", "L1.pack_rows", "L1.xnor_gemm", "L1.spmm",
+            "L2.pack_rows", "L2.xnor_gemm", "L2.spmm")
+
+
 class GCN2Forward:
     """Buffers and launch sequence of the 2-layer Bi-GCN forward of Sec. 6.2."""
 
-    def __init__(self, N: int, K: int, hidden: int, out: int, nnz: int, device):
+    def __init__(self, N: int, K: int, hidden: int, out: int, nnz: int, device,
+                 keep_h1: bool = False):
         self.N, self.K, self.hidden, self.out, self.nnz = N, K, hidden, out, nnz
         self.device = torch.device(device)
         f32, i64 = torch.float32, torch.int64
         e = lambda *shape, dtype=f32: torch.empty(shape, dtype=dtype, device=self.device)
-        w1, w2 = B.words_for(K), B.words_for(hidden)
         # inputs
         self.X, self.s, self.t = e(N, K), e(K), e(K)
         self.W1, self.W2 = e(K, hidden), e(hidden, out)
         self.rowptr, self.colidx = e(N + 1, dtype=i64), e(max(nnz, 1), dtype=torch.int32)[:nnz]
-        # layer 1 intermediates and output
-        self.bits1, self.alpha1 = e(N, w1, dtype=i64), e(N)
-        self.wbits1, self.beta1 = e(hidden, w1, dtype=i64), e(hidden)
-        self.Z1, self.H1 = e(N, hidden), e(N, hidden)
-        # layer 2
-        self.bits2, self.alpha2 = e(N, w2, dtype=i64), e(N)
-        self.wbits2, self.beta2 = e(out, w2, dtype=i64), e(out)
-        self.Z2, self.logits = e(N, out), e(N, out)
+        # fused forward
+        nbytes = B.bigcn_forward_2layer_workspace_bytes(N, K, hidden, out)
+        self.workspace = torch.empty(max(nbytes, 1), dtype=torch.uint8, device=self.device)
+        self.logits = e(N, out)
+        self.H1 = e(N, hidden) if keep_h1 else None
+        self.kernel_names = fused_kernel_names(hidden, out)
         self.graph = None
+        self._steps = None
 
     def input_tensors(self):
         return dict(X=self.X, s=self.s, t=self.t, W1=self.W1, W2=self.W2,
@@ -55,35 +62,21 @@ class GCN2Forward:
             dst[name].copy_(src, non_blocking=non_blocking)
 
     def launch(self, events=None):
-        """Enqueue the 8 kernels on the current stream. ``events`` (9 or None)
-        are recorded before the first, between each, and after the last."""
-        rec = (lambda k: events[k].record()) if events is not None else (lambda k: None)
-        rec(0)
-        B.bigcn_pack_rows(self.X, self.s, self.t, self.bits1, self.alpha1)
-        rec(1)
-        B.bigcn_pack_weights(self.W1, self.wbits1, self.beta1)
-        rec(2)
-        B.bigcn_xnor_gemm_degscaled(self.bits1, self.alpha1, self.wbits1, self.beta1, self.K,
-                                    self.rowptr, self.Z1)
-        rec(3)
-        B.bigcn_spmm_prescaled(self.rowptr, self.colidx, self.Z1, self.H1)
-        rec(4)
-        B.bigcn_pack_rows(self.H1, None, None, self.bits2, self.alpha2)
-        rec(5)
-        B.bigcn_pack_weights(self.W2, self.wbits2, self.beta2)
-        rec(6)
-        B.bigcn_xnor_gemm_degscaled(self.bits2, self.alpha2, self.wbits2, self.beta2,
-                                    self.hidden, self.rowptr, self.Z2)
-        rec(7)
-        B.bigcn_spmm_prescaled(self.rowptr, self.colidx, self.Z2, self.logits)
-        rec(8)
+        """Enqueue the fused forward on the current stream; ``events`` (len =
+        launches + 1) are recorded before each kernel and after the last."""
+        B.bigcn_forward_2layer(self.X, self.s, self.t, self.W1, self.W2, self.rowptr,
+                               self.colidx, self.workspace, self.logits, H1=self.H1,
+                               events=events)
 
     def capture(self, events=None):
         """Capture launch(events) into a CUDA graph (replayed by replay())."""
+        if events:
+            for ev in events:       # torch creates the CUDA event on first record
+                ev.record()
         s = torch.cuda.Stream(device=self.device)
         s.wait_stream(torch.cuda.current_stream(self.device))
         with torch.cuda.stream(s):
-            self.launch(events)          # warm-up outside the graph
+            self.launch(events)     # warm-up outside the graph
         torch.cuda.current_stream(self.device).wait_stream(s)
         torch.cuda.synchronize(self.device)
         g = torch.cuda.CUDAGraph()
@@ -94,3 +87,32 @@ class GCN2Forward:
 
     def replay(self):
         self.graph.replay()
+
+    # ----------------------------------------------------- step by step ----
+    def _alloc_steps(self):
+        N, K, Fh, Fo = self.N, self.K, self.hidden, self.out
+        f32, i64 = torch.float32, torch.int64
+        e = lambda *shape, dtype=f32: torch.empty(shape, dtype=dtype, device=self.device)
+        w1, w2 = B.words_for(K), B.words_for(Fh)
+        self._steps = True
+        self.bits1, self.alpha1 = e(N, w1, dtype=i64), e(N)
+        self.wbits1, self.beta1 = e(Fh, w1, dtype=i64), e(Fh)
+        self.Z1, self.H1s = e(N, Fh), e(N, Fh)
+        self.bits2, self.alpha2 = e(N, w2, dtype=i64), e(N)
+        self.wbits2, self.beta2 = e(Fo, w2, dtype=i64), e(Fo)
+        self.Z2, self.logits_steps = e(N, Fo), e(N, Fo)
+
+    def launch_steps(self):
+        """The same forward as eight step calls, every intermediate kept."""
+        if self._steps is None:
+            self._alloc_steps()
+        B.bigcn_pack_rows(self.X, self.s, self.t, self.bits1, self.alpha1)
+        B.bigcn_pack_weights(self.W1, self.wbits1, self.beta1)
+        B.bigcn_xnor_gemm_degscaled(self.bits1, self.alpha1, self.wbits1, self.beta1, self.K,
+                                    self.rowptr, self.Z1)
+        B.bigcn_spmm_prescaled(self.rowptr, self.colidx, self.Z1, self.H1s)
+        B.bigcn_pack_rows(self.H1s, None, None, self.bits2, self.alpha2)
+        B.bigcn_pack_weights(self.W2, self.wbits2, self.beta2)
+        B.bigcn_xnor_gemm_degscaled(self.bits2, self.alpha2, self.wbits2, self.beta2,
+                                    self.hidden, self.rowptr, self.Z2)
+        B.bigcn_spmm_prescaled(self.rowptr, self.colidx, self.Z2, self.logits_steps)

@@ -10,8 +10,11 @@ the GPU's only where |H1| is within the fp32 tolerance of zero.
 C4 (Reddit-shaped, 114.6M edges) and the C5 sweep points are checked on
 seeded samples of rows the oracle computes one by one: all packed bits, the
 dots and Z of 2048 sampled rows, and H of 2048 sampled rows from the GPU's
-own Z (per-step parity), through the same launch sequence the benchmark
-times.
+own Z (per-step parity).
+
+Both GPU paths are checked: the eight step calls (every intermediate kept)
+and the fused bigcn_forward_2layer the benchmark times, whose layer-1
+aggregation also packs H1 and runs layer 2's product in registers.
 """
 import numpy as np
 import pytest
@@ -27,9 +30,10 @@ pytestmark = pytest.mark.gpu
 
 def run_model(w, data, device):
     nnz = int(data["colidx"].shape[0])
-    m = GCN2Forward(w.N, w.K, w.hidden, w.out, nnz, device)
+    m = GCN2Forward(w.N, w.K, w.hidden, w.out, nnz, device, keep_h1=True)
     m.load(non_blocking=False, **{k: torch.from_numpy(np.ascontiguousarray(v))
                                   for k, v in data.items()})
+    m.launch_steps()
     m.launch()
     torch.cuda.synchronize()
     return m
@@ -60,10 +64,15 @@ def test_two_layer_forward_full(cuda_device, name):
     m = run_model(w, d, cuda_device)
     dinv = 1.0 / np.sqrt(oracle.degree(d["rowptr"]))
     ref1 = oracle.layer_forward(d["X"], d["W1"], d["rowptr"], d["colidx"], d["s"], d["t"])
-    check_layer(m.bits1, m.alpha1, m.wbits1, m.beta1, m.Z1, m.H1, ref1, dinv)
-    H1 = m.H1.cpu().numpy()
+    check_layer(m.bits1, m.alpha1, m.wbits1, m.beta1, m.Z1, m.H1s, ref1, dinv)
+    H1 = m.H1s.cpu().numpy()
     ref2 = oracle.layer_forward(H1, d["W2"], d["rowptr"], d["colidx"])
-    check_layer(m.bits2, m.alpha2, m.wbits2, m.beta2, m.Z2, m.logits, ref2, dinv)
+    check_layer(m.bits2, m.alpha2, m.wbits2, m.beta2, m.Z2, m.logits_steps, ref2, dinv)
+    # The fused forward: H1 and the logits against the oracle (layer 2 on the
+    # fused path's own H1).
+    assert_close(m.H1, ref1["H"], "fused H1")
+    ref2f = oracle.layer_forward(m.H1.cpu().numpy(), d["W2"], d["rowptr"], d["colidx"])
+    assert_close(m.logits, ref2f["H"], "fused logits")
     # End to end: where the oracle's own H1 takes another sign than the
     # GPU's, the value must be within the tolerance of zero.
     flip = (ref1["H"] >= 0) != (H1 >= 0)
@@ -100,14 +109,15 @@ def test_c4_layer1_sampled(cuda_device, c4):
     # H of the sampled rows from the GPU's own Z (undo the degree factor in double)
     Zg = m.Z1.cpu().numpy().astype(np.float64) / dinv[:, None]
     H = oracle.aggregate(d["rowptr"], d["colidx"], Zg, rows=rows)
-    assert_close(m.H1.cpu().numpy()[rows], H, "H1 (sampled rows)")
+    assert_close(m.H1s.cpu().numpy()[rows], H, "H1 (sampled rows)")
+    assert_close(m.H1.cpu().numpy()[rows], H, "fused H1 (sampled rows)")
 
 
 def test_c4_layer2_sampled(cuda_device, c4):
     w, d = c4
     m = run_model(w, d, cuda_device)
     rows = sample_rows(w.N, 2048, 45)
-    H1 = m.H1.cpu().numpy()
+    H1 = m.H1s.cpu().numpy()
     Y = oracle.centre(H1)
     SF = oracle.sign(Y)
     assert_bits_equal(m.bits2, oracle.pack(SF), "layer-2 packed rows")
@@ -116,8 +126,11 @@ def test_c4_layer2_sampled(cuda_device, c4):
     z = oracle.zeta(oracle.binary_dot(SF[rows], SB), oracle.row_scale(Y[rows]), beta)
     assert_close(m.Z2.cpu().numpy()[rows], z * dinv[rows, None], "layer-2 Z' (sampled)")
     Zg = m.Z2.cpu().numpy().astype(np.float64) / dinv[:, None]
-    assert_close(m.logits.cpu().numpy()[rows],
+    assert_close(m.logits_steps.cpu().numpy()[rows],
                  oracle.aggregate(d["rowptr"], d["colidx"], Zg, rows=rows), "logits (sampled)")
+    # fused path: oracle layer 2 on the fused H1 (all rows), logits sampled
+    ref2 = oracle.layer_forward(m.H1.cpu().numpy(), d["W2"], d["rowptr"], d["colidx"], rows=rows)
+    assert_close(m.logits.cpu().numpy()[rows], ref2["H"], "fused logits (sampled)")
 
 
 @pytest.mark.parametrize("K,F", [(512, 64), (4096, 256)])

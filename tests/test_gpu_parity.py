@@ -280,3 +280,57 @@ def test_invalid_arguments_return_status_and_leave_outputs(cuda_device):
     with pytest.raises(B.BigcnError):                              # workspace too small
         B.bigcn_layer_forward(X, None, None, torch.ones((70, 4), device=cuda_device), rowptr,
                               torch.empty(0, dtype=torch.int32, device=cuda_device), ws, Z)
+
+
+# ------------------------------------------------- fused two-layer forward ---
+@pytest.mark.parametrize("N,K,Fh,Fo,deg,hub", [
+    (1, 1, 4, 1, 0.0, 0),             # a single isolated node
+    (301, 203, 64, 7, 4.0, 40),        # fused path (Fh % 4 == 0, Fo <= 64)
+    (1000, 602, 128, 41, 8.0, 300),    # fused, two packed words per hidden row
+    (517, 130, 16, 3, 3.0, 0),         # fused, narrowest lane groups
+    (400, 150, 30, 5, 4.0, 0),         # Fh not a multiple of 4: unfused path
+    (300, 100, 64, 80, 4.0, 0),        # Fo > 64: unfused path
+    (257, 70, 200, 9, 5.0, 0),         # Fh > 128: unfused path
+])
+def test_forward_2layer_matches_oracle(cuda_device, N, K, Fh, Fo, deg, hub):
+    case = inputs.layer_case(N, K, Fh, seed=N + K + Fh + Fo, mean_degree=deg, hub_degree=hub)
+    W2 = inputs.weights(Fh, Fo, seed=N + 99)
+    d = {k: to_dev(v) for k, v in case.items()}
+    ws = torch.empty(B.bigcn_forward_2layer_workspace_bytes(N, K, Fh, Fo), dtype=torch.uint8,
+                     device=cuda_device)
+    H1 = torch.full((N, Fh), float("nan"), device=cuda_device)
+    out = torch.full((N, Fo), float("nan"), device=cuda_device)
+    B.bigcn_forward_2layer(d["X"], d["s"], d["t"], d["W"], to_dev(W2), d["rowptr"],
+                           d["colidx"], ws, out, H1=H1)
+    ref1 = oracle.layer_forward(case["X"], case["W"], case["rowptr"], case["colidx"],
+                                case["s"], case["t"])
+    assert_close(H1, ref1["H"], "H1")
+    ref2 = oracle.layer_forward(H1.cpu().numpy(), W2, case["rowptr"], case["colidx"])
+    assert_close(out, ref2["H"], "logits")
+    # without H1 requested: the same logits
+    out2 = torch.full((N, Fo), float("nan"), device=cuda_device)
+    B.bigcn_forward_2layer(d["X"], d["s"], d["t"], d["W"], to_dev(W2), d["rowptr"],
+                           d["colidx"], ws, out2)
+    assert torch.equal(out, out2)
+
+
+def test_forward_2layer_records_one_event_per_kernel_boundary(cuda_device):
+    N, K, Fh, Fo = 500, 300, 64, 7
+    case = inputs.layer_case(N, K, Fh, seed=3)
+    d = {k: to_dev(v) for k, v in case.items()}
+    W2 = to_dev(inputs.weights(Fh, Fo, seed=4))
+    n = B.bigcn_forward_2layer_launches(Fh, Fo)
+    assert n == 5 and B.bigcn_forward_2layer_launches(30, 7) == 7
+    events = [torch.cuda.Event(enable_timing=True) for _ in range(n + 1)]
+    for e in events:
+        e.record()
+    torch.cuda.synchronize()
+    ws = torch.empty(B.bigcn_forward_2layer_workspace_bytes(N, K, Fh, Fo), dtype=torch.uint8,
+                     device=cuda_device)
+    out = torch.empty((N, Fo), device=cuda_device)
+    B.bigcn_forward_2layer(d["X"], d["s"], d["t"], d["W"], W2, d["rowptr"], d["colidx"], ws,
+                           out, events=events)
+    torch.cuda.synchronize()
+    spans = [events[q].elapsed_time(events[q + 1]) for q in range(n)]
+    assert all(t >= 0.0 for t in spans)
+    assert events[0].elapsed_time(events[n]) > 0.0
