@@ -199,10 +199,13 @@ bigcn_status bigcn_layer_forward(const float *X, int64_t N, int32_t K, int64_t l
  *   out = D^-1/2 (A + I) D^-1/2 zeta(H1, W2)             N x Fo (the logits)
  *
  * The result equals two bigcn_layer_forward calls within fp32 rounding.
- * When Fh is a multiple of 4 and at most 128 and Fo <= 64, layer 1's
- * aggregation kernel also binarizes H1 and computes layer 2's XNOR product
- * while the row is in registers, so H1 never goes through memory; the call
- * then launches 5 kernels, otherwise 7 (bigcn_forward_2layer_launches).
+ * Fusions, when the widths allow: layer 1's centring, packing and XNOR
+ * product run as one kernel whose packed rows stay in shared memory
+ * (Fh <= 128 and the packed tiles fit); and when Fh is a multiple of 4 and at
+ * most 128 and Fo <= 64, layer 1's aggregation kernel also binarizes H1 and
+ * computes layer 2's XNOR product while the row is in registers, so H1 never
+ * goes through memory. The call launches 4 to 7 kernels
+ * (bigcn_forward_2layer_launches).
  *
  * X N x K (ldx), W1 K x Fh (ldw1), W2 Fh x Fo (ldw2), CSR as in
  * bigcn_spmm_norm, out N x Fo (ldo).
@@ -217,8 +220,9 @@ bigcn_status bigcn_layer_forward(const float *X, int64_t N, int32_t K, int64_t l
  */
 size_t bigcn_forward_2layer_workspace_bytes(int64_t N, int32_t K, int32_t Fh, int32_t Fo);
 
-/* Kernel launches bigcn_forward_2layer makes for these widths (5 or 7). */
-int32_t bigcn_forward_2layer_launches(int32_t Fh, int32_t Fo);
+/* Kernel launches bigcn_forward_2layer makes for these sizes on the current
+ * device (4 to 7), or -1 on invalid sizes or a device error. */
+int32_t bigcn_forward_2layer_launches(int64_t N, int32_t K, int32_t Fh, int32_t Fo);
 
 bigcn_status bigcn_forward_2layer(const float *X, int64_t N, int32_t K, int64_t ldx,
                                   const float *scale, const float *shift,

@@ -48,7 +48,7 @@ SIGNATURES = {
     "bigcn_layer_forward": ([_p, _i64, _i32, _i64, _p, _p, _p, _i32, _i64, _p, _p, _i64, _p,
                              _sz, _p, _i64, _p], ctypes.c_int),
     "bigcn_forward_2layer_workspace_bytes": ([_i64, _i32, _i32, _i32], _sz),
-    "bigcn_forward_2layer_launches": ([_i32, _i32], _i32),
+    "bigcn_forward_2layer_launches": ([_i64, _i32, _i32, _i32], _i32),
     "bigcn_forward_2layer": ([_p, _i64, _i32, _i64, _p, _p, _p, _i32, _i64, _p, _i32, _i64, _p,
                               _p, _i64, _p, _sz, _p, _i64, _p, _i64, _p, _i32, _p],
                              ctypes.c_int),
@@ -194,8 +194,11 @@ def bigcn_forward_2layer_workspace_bytes(N: int, K: int, Fh: int, Fo: int) -> in
     return int(lib().bigcn_forward_2layer_workspace_bytes(N, K, Fh, Fo))
 
 
-def bigcn_forward_2layer_launches(Fh: int, Fo: int) -> int:
-    return int(lib().bigcn_forward_2layer_launches(Fh, Fo))
+def bigcn_forward_2layer_launches(N: int, K: int, Fh: int, Fo: int) -> int:
+    n = int(lib().bigcn_forward_2layer_launches(N, K, Fh, Fo))
+    if n < 0:
+        raise BigcnError("bigcn_forward_2layer_launches", 1)
+    return n
 
 
 def bigcn_forward_2layer(X, scale, shift, W1, W2, rowptr, colidx, workspace, out, H1=None,

@@ -3,15 +3,22 @@
 // layer Eq. 13 with zeta of Eqs. 11-12. Kernel sequence on one stream:
 //
 //   0 pack W1 and W2 (one launch)                          Eqs. 3-4
-//   1 pack rows of X, centred                              Sec. 6.2, Eqs. 7-8
-//   2 XNOR GEMM, rows scaled by 1/sqrt(dhat)               Eqs. 11-12
-//   3 aggregation of layer 1 fused with layer 2's row      Eq. 13, then
+//   1 centre + pack rows of X + XNOR GEMM, rows scaled     Sec. 6.2, Eqs. 7-8,
+//     by 1/sqrt(dhat) (packed rows stay in shared memory)  Eqs. 11-12
+//   2 aggregation of layer 1 fused with layer 2's row      Eq. 13, then
 //     packing and XNOR GEMM (H1 stays in registers)        Eqs. 7-8, 11-12
-//   4 aggregation of layer 2 -> logits                     Eq. 13
+//   3 aggregation of layer 2 -> logits                     Eq. 13
 //
-// When the widths do not fit the fused kernel (hidden width not a multiple
-// of 4 or above 128, or more than 64 outputs) step 3 runs as three kernels:
-// aggregation, packing, GEMM. Either way every step runs on the GPU.
+// Step 1 runs as two kernels (pack rows, then GEMM) when the packed weight
+// tile does not fit in shared memory (hidden width above 128 or very long
+// rows), and step 2 as three (aggregation, packing, GEMM) when the widths do
+// not fit the fused kernel (hidden width not a multiple of 4 or above 128, or
+// more than 64 outputs). Every step runs on the GPU either way.
+//
+// Every kernel after the first is launched with programmatic serialization:
+// it may start while its predecessor drains, and waits (griddepcontrol) only
+// before it reads what an earlier kernel wrote -- the fused front streams and
+// packs X while the weights are still being packed.
 #include "launch.cuh"
 
 namespace bigcn {
@@ -40,7 +47,7 @@ bool forward2_workspace(int64_t N, int32_t K, int32_t Fh, int32_t Fo, Forward2Wo
     w->z1 = take(size_t(N) * Fh * 4);
     w->wbits2 = take(size_t(Fo) * w2 * 8);
     w->beta2 = take(size_t(Fo) * 4);
-    w->z2 = take(size_t(N) * Fo * 4);
+    w->z2 = take(size_t(N) * ((Fo + 3) / 4 * 4) * 4);
     w->h1 = take(size_t(N) * Fh * 4);
     w->bits2 = take(size_t(N) * w2 * 8);
     w->alpha2 = take(size_t(N) * 4);
@@ -59,8 +66,12 @@ extern "C" size_t bigcn_forward_2layer_workspace_bytes(int64_t N, int32_t K, int
     return forward2_workspace(N, K, Fh, Fo, &w) ? w.total : 0;
 }
 
-extern "C" int32_t bigcn_forward_2layer_launches(int32_t Fh, int32_t Fo) {
-    return spmm_pack_gemm_supported(Fh, Fo) ? 5 : 7;
+extern "C" int32_t bigcn_forward_2layer_launches(int64_t N, int32_t K, int32_t Fh, int32_t Fo) {
+    if (N < 0 || K < 1 || Fh < 1 || Fo < 1) return -1;
+    DeviceInfo dev;
+    if (current_device(&dev) != BIGCN_OK) return -1;
+    return 1 + (front_supported(N, K, Fh, dev) ? 1 : 2) +
+           (spmm_pack_gemm_supported(Fh, Fo) ? 1 : 3) + 1;
 }
 
 extern "C" bigcn_status bigcn_forward_2layer(
@@ -118,6 +129,10 @@ extern "C" bigcn_status bigcn_forward_2layer(
     float *beta2 = static_cast<float *>(at(w.beta2));
     float *Z2 = static_cast<float *>(at(w.z2));
     const int words1 = bigcn_words(K), words2 = bigcn_words(Fh);
+    // Z2' rows are padded to a multiple of 4 floats; the fused kernel writes
+    // the padding as zeros, which lets the layer-2 aggregation gather float4s.
+    const int64_t ldz2 = (Fo + 3) / 4 * 4;
+    const bool fused = spmm_pack_gemm_supported(Fh, Fo);
     cudaStream_t s = as_stream(stream);
     // Inside a stream capture an event must be recorded as an external node
     // to be timed later; outside a capture a plain record does that.
@@ -144,31 +159,37 @@ extern "C" bigcn_status bigcn_forward_2layer(
     WeightPack p2{W2, Fh, Fo, ldw2, wbits2, words2, beta2, 0};
     launch_pack_weights2(p1, p2, s);
     mark();
-    launch_pack_rows(X, N, K, ldx, scale, shift, bits1, words1, alpha1, dev, s);
-    mark();
-    GemmArgs g1{bits1, alpha1, N, wbits1, beta1, Fh, K, words1, Z1, Fh, nullptr, rowptr};
-    launch_xnor_gemm(g1, dev, s);
-    mark();
-    if (spmm_pack_gemm_supported(Fh, Fo)) {
-        SpmmPackGemmArgs f{rowptr, colidx, N, nnz, Z1, Fh, H1, ldh1, wbits2, beta2, Fo, Z2, Fo};
-        launch_spmm_pack_gemm(f, s);
+    if (front_supported(N, K, Fh, dev)) {
+        FrontArgs fr{X, N, K, ldx, scale, shift, wbits1, beta1, Fh, words1, rowptr, Z1, Fh};
+        launch_front(fr, dev, s, true);
+        mark();
+    } else {
+        launch_pack_rows(X, N, K, ldx, scale, shift, bits1, words1, alpha1, dev, s, true);
+        mark();
+        GemmArgs g1{bits1, alpha1, N, wbits1, beta1, Fh, K, words1, Z1, Fh, nullptr, rowptr};
+        launch_xnor_gemm(g1, dev, s, true);
+        mark();
+    }
+    if (fused) {
+        SpmmPackGemmArgs f{rowptr, colidx, N, nnz, Z1, Fh, H1, ldh1, wbits2, beta2, Fo, Z2, ldz2};
+        launch_spmm_pack_gemm(f, dev, s, true);
         mark();
     } else {
         float *H1w = H1 ? H1 : static_cast<float *>(at(w.h1));
         const int64_t ldh = H1 ? ldh1 : Fh;
         uint64_t *bits2 = static_cast<uint64_t *>(at(w.bits2));
         float *alpha2 = static_cast<float *>(at(w.alpha2));
-        SpmmArgs a1{rowptr, colidx, N, nnz, Z1, Fh, Fh, H1w, ldh, true};
-        launch_spmm_norm(a1, dev, s);
+        SpmmArgs a1{rowptr, colidx, N, nnz, Z1, Fh, Fh, H1w, ldh, true, false};
+        launch_spmm_norm(a1, dev, s, true);
         mark();
-        launch_pack_rows(H1w, N, Fh, ldh, nullptr, nullptr, bits2, words2, alpha2, dev, s);
+        launch_pack_rows(H1w, N, Fh, ldh, nullptr, nullptr, bits2, words2, alpha2, dev, s, true);
         mark();
-        GemmArgs g2{bits2, alpha2, N, wbits2, beta2, Fo, Fh, words2, Z2, Fo, nullptr, rowptr};
-        launch_xnor_gemm(g2, dev, s);
+        GemmArgs g2{bits2, alpha2, N, wbits2, beta2, Fo, Fh, words2, Z2, ldz2, nullptr, rowptr};
+        launch_xnor_gemm(g2, dev, s, true);
         mark();
     }
-    SpmmArgs a2{rowptr, colidx, N, nnz, Z2, Fo, Fo, out, ldo, true};
-    launch_spmm_norm(a2, dev, s);
+    SpmmArgs a2{rowptr, colidx, N, nnz, Z2, ldz2, Fo, out, ldo, true, fused};
+    launch_spmm_norm(a2, dev, s, true);
     mark();
     const bigcn_status ls = launch_status();
     return event_failed ? BIGCN_ERR_CUDA : ls;

@@ -12,9 +12,10 @@
 namespace bigcn {
 
 // Steps 1+2: centre, sign-pack rows, per-node scale (Sec. 6.2, Eqs. 7-8).
+// `pdl`: launch with programmatic serialization (see grid_dependency_wait).
 void launch_pack_rows(const float *X, int64_t N, int K, int64_t ldx, const float *scale,
                       const float *shift, uint64_t *bits, int words, float *alpha,
-                      const DeviceInfo &dev, cudaStream_t stream);
+                      const DeviceInfo &dev, cudaStream_t stream, bool pdl = false);
 
 // Step 3: sign-pack weight columns, per-column scale (Eqs. 3-4).
 void launch_pack_weights(const float *Wt, int K, int F, int64_t ldw, uint64_t *bits,
@@ -33,6 +34,7 @@ struct WeightPack {
 };
 
 // Step 3 for two matrices in one launch (b.W == nullptr: a only).
+// The kernel lets its dependent launch at once (it is the first of a chain).
 void launch_pack_weights2(const WeightPack &a, const WeightPack &b, cudaStream_t stream);
 
 struct GemmArgs {
@@ -51,7 +53,8 @@ struct GemmArgs {
 };
 
 // Step 4: the XNOR-popcount product and its scaling (Eqs. 11-12).
-void launch_xnor_gemm(const GemmArgs &args, const DeviceInfo &dev, cudaStream_t stream);
+void launch_xnor_gemm(const GemmArgs &args, const DeviceInfo &dev, cudaStream_t stream,
+                      bool pdl = false);
 
 struct SpmmArgs {
     const int64_t *rowptr;   // N + 1
@@ -64,10 +67,36 @@ struct SpmmArgs {
     float *H;                // N x F (row stride ldh)
     int64_t ldh;
     bool prescaled;          // Z rows already carry their 1/sqrt(dhat_j)
+    bool z_pad4;             // Z's columns F .. round_up(F, 4) are readable and finite
 };
 
 // Step 5: H = D^-1/2 (A + I) D^-1/2 Z (Eqs. 1, 13).
-void launch_spmm_norm(const SpmmArgs &args, const DeviceInfo &dev, cudaStream_t stream);
+void launch_spmm_norm(const SpmmArgs &args, const DeviceInfo &dev, cudaStream_t stream,
+                      bool pdl = false);
+
+struct FrontArgs {
+    const float *X;          // N x K (row stride ldx)
+    int64_t N;
+    int K;
+    int64_t ldx;
+    const float *scale;      // nullable (identity centring)
+    const float *shift;
+    const uint64_t *wbits;   // F x words packed weight columns
+    const float *beta;       // F
+    int F;
+    int words;
+    const int64_t *rowptr;   // rows are scaled by 1/sqrt(1 + deg)
+    float *Z;                // N x F (row stride ldz)
+    int64_t ldz;
+};
+
+// Whether the fused pack + XNOR-GEMM kernel fits (F <= 128, packed tiles in
+// shared memory).
+bool front_supported(int64_t N, int K, int F, const DeviceInfo &dev);
+
+// Steps 1, 2 and 4 of one layer in one kernel (see front.cu).
+void launch_front(const FrontArgs &args, const DeviceInfo &dev, cudaStream_t stream,
+                  bool pdl = false);
 
 // Largest layer-2 output width the fused aggregation handles.
 constexpr int kMaxFusedOut = 64;
@@ -84,14 +113,15 @@ struct SpmmPackGemmArgs {
     const uint64_t *wbits2;  // Fo x ceil(Fh/64) packed columns of W2
     const float *beta2;      // Fo
     int Fo;
-    float *Z2;               // N x Fo, rows pre-scaled by 1/sqrt(dhat) (row stride ldz2)
-    int64_t ldz2;
+    float *Z2;               // N x Fo, rows pre-scaled by 1/sqrt(dhat) (row stride ldz2;
+    int64_t ldz2;            // columns Fo .. ldz2 are written as zeros)
 };
 
 // Whether (Fh, Fo) fit the fused kernel: Fh % 4 == 0, Fh <= 128, Fo <= 64.
 bool spmm_pack_gemm_supported(int Fh, int Fo);
 
 // Layer-1 step 5 fused with layer-2 steps 2 and 4 (see spmm.cu).
-void launch_spmm_pack_gemm(const SpmmPackGemmArgs &args, cudaStream_t stream);
+void launch_spmm_pack_gemm(const SpmmPackGemmArgs &args, const DeviceInfo &dev,
+                           cudaStream_t stream, bool pdl = false);
 
 }  // namespace bigcn

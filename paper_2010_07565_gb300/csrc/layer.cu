@@ -149,7 +149,7 @@ extern "C" bigcn_status bigcn_layer_forward(const float *X, int64_t N, int32_t K
     launch_pack_weights(Wt, K, F, ldw, b_bits, words, beta, s);
     GemmArgs g{a_bits, alpha, N, b_bits, beta, F, K, words, Zs, F, nullptr, rowptr};
     launch_xnor_gemm(g, dev, s);
-    SpmmArgs a{rowptr, colidx, N, nnz, Zs, F, F, H, ldh, true};
+    SpmmArgs a{rowptr, colidx, N, nnz, Zs, F, F, H, ldh, true, false};
     launch_spmm_norm(a, dev, s);
     return launch_status();
 }

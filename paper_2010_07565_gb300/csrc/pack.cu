@@ -14,8 +14,10 @@
 // shared memory, so alpha does not depend on scheduling.
 //
 // pack_weights reads W (K x F) column-wise: thread (x, y) of a 32 x 8 block
-// owns one column and builds whole 64-bit words from 64 coalesced row reads;
-// one launch can pack two matrices (both layers' weights). The words of a column are spread over a cluster of S <= 8 blocks
+// owns one column and builds whole 64-bit words from 64 coalesced row reads,
+// all 64 in flight at once (the kernel is latency-bound: few blocks, so it
+// is given registers rather than occupancy); one launch can pack two
+// matrices (both layers' weights). The words of a column are spread over a cluster of S <= 8 blocks
 // (grid y); each block reduces its |W| partial sums in shared memory, and
 // block 0 of the cluster adds the S partials through distributed shared
 // memory in rank order (deterministic).
@@ -39,6 +41,7 @@ pack_rows_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
                  uint32_t *__restrict__ bits32, int64_t ld32, float *__restrict__ alpha,
                  int G) {
     __shared__ float part[kPackWarps];
+    grid_dependency_wait();     // X may be the output of the previous kernel
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
     const int sub = warp & (G - 1);
@@ -88,10 +91,12 @@ constexpr int kMaxCluster = 8;
 
 // Blocks with blockIdx.x < a.tiles pack matrix a, the rest matrix b (one
 // launch can pack both layers' weights); each block owns 32 columns.
-__global__ void __launch_bounds__(kWCols *kWRows)
+__global__ void __launch_bounds__(kWCols *kWRows, 2)
 pack_weights_kernel(WeightPack a, WeightPack b) {
     __shared__ float partial[kWRows][kWCols];
     __shared__ float colsum[kWCols];
+    allow_dependent_launch();   // what follows may start on the call's own inputs
+    grid_dependency_wait();
     cg::cluster_group cluster = cg::this_cluster();
     const int S = int(cluster.num_blocks());
     const int rank = int(cluster.block_rank());
@@ -141,7 +146,7 @@ pack_weights_kernel(WeightPack a, WeightPack b) {
 
 void launch_pack_rows(const float *X, int64_t N, int K, int64_t ldx, const float *scale,
                       const float *shift, uint64_t *bits, int words, float *alpha,
-                      const DeviceInfo &dev, cudaStream_t stream) {
+                      const DeviceInfo &dev, cudaStream_t stream, bool pdl) {
     if (N == 0) return;
     // Split rows over up to 8 warps while the grid is short of one full wave
     // of warps, as long as every warp keeps at least one 8-chunk batch.
@@ -153,11 +158,12 @@ void launch_pack_rows(const float *X, int64_t N, int K, int64_t ldx, const float
     const unsigned grid = unsigned((N + rows_per_block - 1) / rows_per_block);
     uint32_t *b32 = reinterpret_cast<uint32_t *>(bits);
     if (scale)
-        pack_rows_kernel<true><<<grid, kPackThreads, 0, stream>>>(
-            X, N, K, ldx, scale, shift, b32, int64_t(words) * 2, alpha, G);
+        launch_kernel(pack_rows_kernel<true>, dim3(grid), dim3(kPackThreads), 0, stream, pdl,
+                      dim3(1, 1, 1), X, N, K, ldx, scale, shift, b32, int64_t(words) * 2, alpha, G);
     else
-        pack_rows_kernel<false><<<grid, kPackThreads, 0, stream>>>(
-            X, N, K, ldx, nullptr, nullptr, b32, int64_t(words) * 2, alpha, G);
+        launch_kernel(pack_rows_kernel<false>, dim3(grid), dim3(kPackThreads), 0, stream, pdl,
+                      dim3(1, 1, 1), X, N, K, ldx, static_cast<const float *>(nullptr),
+                      static_cast<const float *>(nullptr), b32, int64_t(words) * 2, alpha, G);
 }
 
 void launch_pack_weights2(const WeightPack &a, const WeightPack &b, cudaStream_t stream) {
@@ -169,19 +175,8 @@ void launch_pack_weights2(const WeightPack &a, const WeightPack &b, cudaStream_t
     int S = rows(A);
     if (B.tiles > 0 && rows(B) > S) S = rows(B);
     if (S > kMaxCluster) S = kMaxCluster;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(A.tiles + B.tiles, S, 1);
-    cfg.blockDim = dim3(kWCols, kWRows, 1);
-    cfg.dynamicSmemBytes = 0;
-    cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = 1;
-    attr[0].val.clusterDim.y = S;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    cudaLaunchKernelEx(&cfg, pack_weights_kernel, A, B);
+    launch_kernel(pack_weights_kernel, dim3(A.tiles + B.tiles, S, 1), dim3(kWCols, kWRows, 1), 0,
+                  stream, false, dim3(1, S, 1), A, B);
 }
 
 void launch_pack_weights(const float *Wt, int K, int F, int64_t ldw, uint64_t *bits,

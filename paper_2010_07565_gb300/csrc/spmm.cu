@@ -1,32 +1,44 @@
 // Step 5 of the Bi-GCN layer forward (Wang et al., CVPR 2021, Eq. 13 with
 // the operator of Eq. 1): H = D^-1/2 (A + I) D^-1/2 Z over a CSR graph.
 //
-// One warp per output row. The warp is split into P = 32 / L groups of L
-// lanes; each group gathers a different neighbour's row of Z, lane by lane
-// in VEC-wide vectors (NV per lane), so that rows narrower than a warp still
-// keep all 32 lanes busy. Neighbour indices (and, unless Z is pre-scaled,
-// their 1/sqrt(dhat_j)) are fetched 32 at a time, one per lane, then
-// broadcast with shuffles. The self-loop that A + I adds is the first entry
-// of every row's list. Partial sums are combined across groups with xor
-// shuffles and group 0 writes H_i scaled by 1/sqrt(dhat_i). A grid y
-// dimension splits wide rows into column slabs of L * NV * VEC features.
+// Light rows: one warp per output row. The warp is split into P = 32 / L
+// groups of L lanes; each group gathers a different neighbour's row of Z,
+// lane by lane in VEC-wide vectors (NV per lane), so rows narrower than a
+// warp still keep all 32 lanes busy, and U such gathers are issued before any
+// is consumed (U = 4, or 2 when each lane holds two vectors). Neighbour indices (and, unless Z is pre-scaled, their
+// 1/sqrt(dhat_j)) are fetched 32 at a time, one per lane, then broadcast with
+// shuffles. The self-loop that A + I adds is entry 0 of every row's list.
+// Partial sums are combined across groups with xor shuffles and group 0
+// writes H_i scaled by 1/sqrt(dhat_i).
 //
-// Bounds: the row range is clamped to [0, nnz] and column indices outside
-// [0, N) are skipped, so a malformed CSR cannot make the kernel read out of
-// bounds.
+// Heavy rows (more than kHeavyDegree neighbours, e.g. the hubs of a
+// power-law graph) would make one warp the critical path of the whole
+// launch. The first `heavy_blocks` blocks of every launch therefore scan the
+// row pointers, skip light rows, and give each heavy row to all 8 warps of
+// the block: warp w gathers the w-th eighth of the row's list, the eight
+// partial rows meet in shared memory and warp 0 adds them in warp order
+// (deterministic) before the same epilogue. Light warps skip heavy rows.
+//
+// A grid y dimension splits wide rows into column slabs of L * NV * VEC
+// features. Bounds: the row range is clamped to [0, nnz] and column indices
+// outside [0, N) are skipped, so a malformed CSR cannot make the kernel read
+// out of bounds.
 #include "launch.cuh"
 
 namespace bigcn {
 namespace {
 
 constexpr int kSpmmThreads = 256;
-constexpr int kUnroll = 4;
+constexpr int kSpmmWarps = kSpmmThreads / 32;
+constexpr int64_t kHeavyDegree = 2048;
 
 template <int VEC> struct Vec;
 template <> struct Vec<1> {
     using T = float;
-    static __device__ __forceinline__ void fma(float *acc, const T &v, float w) { acc[0] = fmaf(w, v, acc[0]); }
-    static __device__ __forceinline__ void set(float *acc, T &v) { v = acc[0]; }
+    static __device__ __forceinline__ void fma(float *acc, const T &v, float w) {
+        acc[0] = fmaf(w, v, acc[0]);
+    }
+    static __device__ __forceinline__ T make(const float *a) { return a[0]; }
 };
 template <> struct Vec<2> {
     using T = float2;
@@ -34,7 +46,7 @@ template <> struct Vec<2> {
         acc[0] = fmaf(w, v.x, acc[0]);
         acc[1] = fmaf(w, v.y, acc[1]);
     }
-    static __device__ __forceinline__ void set(float *acc, T &v) { v = make_float2(acc[0], acc[1]); }
+    static __device__ __forceinline__ T make(const float *a) { return make_float2(a[0], a[1]); }
 };
 template <> struct Vec<4> {
     using T = float4;
@@ -44,110 +56,230 @@ template <> struct Vec<4> {
         acc[2] = fmaf(w, v.z, acc[2]);
         acc[3] = fmaf(w, v.w, acc[3]);
     }
-    static __device__ __forceinline__ void set(float *acc, T &v) {
-        v = make_float4(acc[0], acc[1], acc[2], acc[3]);
+    static __device__ __forceinline__ T make(const float *a) {
+        return make_float4(a[0], a[1], a[2], a[3]);
     }
 };
 
-template <int VEC, int L, int NV, bool kPrescaled>
-__global__ void __launch_bounds__(kSpmmThreads)
-spmm_norm_kernel(const int64_t *__restrict__ rowptr, const int32_t *__restrict__ colidx,
-                 int64_t N, int64_t nnz, const float *__restrict__ Z, int64_t ldz, int F,
-                 float *__restrict__ H, int64_t ldh) {
-    using V = typename Vec<VEC>::T;
-    constexpr int P = 32 / L;                 // neighbours gathered in parallel
-    constexpr int SLAB = L * NV * VEC;        // features per column slab
+struct SpmmParams {
+    const int64_t *rowptr;
+    const int32_t *colidx;
+    int64_t N;
+    int64_t nnz;
+    const float *Z;
+    int64_t ldz;
+    int Fload;               // features gathered per row (a multiple of VEC, <= ldz)
+    int F;                   // features stored per row (<= Fload)
+    float *H;
+    int64_t ldh;
+    int heavy_blocks;        // leading blocks that take the heavy rows
+    bool vec_store;          // H rows start VEC-aligned: whole vectors may be stored
+};
 
-    const int lane = threadIdx.x & 31;
-    const int64_t i = (int64_t(blockIdx.x) * kSpmmThreads + threadIdx.x) >> 5;
-    if (i >= N) return;
-    const int g = lane / L, sl = lane % L;
-    const int f0 = blockIdx.y * SLAB;
+// Row i's neighbour list: CSR entries [b, b + total - 1) plus the self-loop.
+struct RowSpan {
+    int64_t b;
+    int64_t total;
+    float dinv;
+};
 
+__device__ __forceinline__ RowSpan row_span(const int64_t *__restrict__ rowptr, int64_t nnz,
+                                            int64_t i) {
     const int64_t rb = __ldg(rowptr + i), re = __ldg(rowptr + i + 1);
     const int64_t b = min(max(rb, int64_t(0)), nnz);
     const int64_t e = min(max(re, b), nnz);
-    const float dinv_i = inv_sqrt_degree(e - b);
-    const int64_t total = (e - b) + 1;        // + the self-loop
+    return RowSpan{b, (e - b) + 1, inv_sqrt_degree(e - b)};
+}
 
-    float acc[NV][VEC];
-#pragma unroll
-    for (int v = 0; v < NV; ++v)
-#pragma unroll
-        for (int c = 0; c < VEC; ++c) acc[v][c] = 0.0f;
-
-    for (int64_t base = 0; base < total; base += 32) {
-        // Lane q fetches entry base + q of the row's list (entry 0 = self).
+// Adds, into acc, the Z rows of entries [q0, q1) of row i's list (entry 0 is
+// the self-loop), weighted by 1/sqrt(dhat_j) unless Z is pre-scaled.
+template <int VEC, int L, int NV, int U, bool kPre>
+__device__ __forceinline__ void gather(const SpmmParams &p, int64_t i, int64_t b, int64_t q0,
+                                       int64_t q1, int f0, float (&acc)[NV][VEC]) {
+    using V = typename Vec<VEC>::T;
+    constexpr int P = 32 / L;
+    const int lane = threadIdx.x & 31;
+    const int g = lane / L, sl = lane % L;
+    for (int64_t base = q0; base < q1; base += 32) {
         int j = -1;
         float wj = 0.0f;
         const int64_t q = base + lane;
-        if (q < total) {
-            j = (q == 0) ? int(i) : __ldg(colidx + b + q - 1);
-            if (j < 0 || j >= N) j = -1;
+        if (q < q1) {
+            j = (q == 0) ? int(i) : __ldg(p.colidx + b + q - 1);
+            if (j < 0 || j >= p.N) j = -1;
             if (j >= 0)
-                wj = kPrescaled ? 1.0f
-                                : inv_sqrt_degree(__ldg(rowptr + j + 1) - __ldg(rowptr + j));
+                wj = kPre ? 1.0f
+                          : inv_sqrt_degree(__ldg(p.rowptr + j + 1) - __ldg(p.rowptr + j));
         }
-        const int cnt = int(min(total - base, int64_t(32)));
-        for (int t0 = 0; t0 < cnt; t0 += P * kUnroll) {
-            V val[kUnroll][NV];
-            float w[kUnroll];
+        const int cnt = int(min(q1 - base, int64_t(32)));
+        for (int t0 = 0; t0 < cnt; t0 += P * U) {
+            V val[U][NV];
+            float w[U];
 #pragma unroll
-            for (int u = 0; u < kUnroll; ++u) {
-                const int src = t0 + u * P + g;          // < 32 always
+            for (int u = 0; u < U; ++u) {
+                const int src = t0 + u * P + g;
                 const int jj = __shfl_sync(kFullMask, j, src & 31);
                 w[u] = __shfl_sync(kFullMask, wj, src & 31);
                 const bool live = src < cnt && jj >= 0;
                 if (!live) w[u] = 0.0f;
-                const float *zr = Z + int64_t(live ? jj : 0) * ldz;
+                const float *zr = p.Z + int64_t(live ? jj : 0) * p.ldz;
 #pragma unroll
                 for (int v = 0; v < NV; ++v) {
                     const int f = f0 + (v * L + sl) * VEC;
-                    if (live && f < F) val[u][v] = __ldg(reinterpret_cast<const V *>(zr + f));
+                    if (live && f < p.Fload) val[u][v] = __ldg(reinterpret_cast<const V *>(zr + f));
                     else val[u][v] = V{};
                 }
             }
 #pragma unroll
-            for (int u = 0; u < kUnroll; ++u)
+            for (int u = 0; u < U; ++u)
 #pragma unroll
                 for (int v = 0; v < NV; ++v) Vec<VEC>::fma(acc[v], val[u][v], w[u]);
         }
     }
+}
 
+template <int VEC, int L, int NV>
+__device__ __forceinline__ void reduce_groups(float (&acc)[NV][VEC]) {
 #pragma unroll
     for (int o = L; o < 32; o <<= 1)
 #pragma unroll
         for (int v = 0; v < NV; ++v)
 #pragma unroll
             for (int c = 0; c < VEC; ++c) acc[v][c] += __shfl_xor_sync(kFullMask, acc[v][c], o);
+}
 
-    if (g == 0) {
+// Epilogue of the plain aggregation: H_i = dinv_i * acc (lanes of group 0).
+template <int VEC, int L, int NV>
+struct StoreRow {
+    __device__ __forceinline__ void prologue() const {}
+    __device__ __forceinline__ void operator()(const SpmmParams &p, int64_t i, float dinv,
+                                               int f0, float (&acc)[NV][VEC]) const {
+        using V = typename Vec<VEC>::T;
+        const int lane = threadIdx.x & 31;
+        if (lane / L != 0) return;
+        const int sl = lane % L;
 #pragma unroll
         for (int v = 0; v < NV; ++v) {
             const int f = f0 + (v * L + sl) * VEC;
-            if (f < F) {
+            float o[VEC];
 #pragma unroll
-                for (int c = 0; c < VEC; ++c) acc[v][c] *= dinv_i;
-                V out;
-                Vec<VEC>::set(acc[v], out);
-                *reinterpret_cast<V *>(H + i * ldh + f) = out;
+            for (int c = 0; c < VEC; ++c) o[c] = acc[v][c] * dinv;
+            float *h = p.H + i * p.ldh + f;
+            if (p.vec_store && f + VEC <= p.F) {
+                *reinterpret_cast<V *>(h) = Vec<VEC>::make(o);
+            } else {
+#pragma unroll
+                for (int c = 0; c < VEC; ++c)
+                    if (f + c < p.F) h[c] = o[c];
             }
         }
     }
+};
+
+template <int VEC, int L, int NV, int U, bool kPre, class Epi>
+__device__ __forceinline__ void light_rows(const SpmmParams &p, const Epi &epi, int f0) {
+    const int warp = threadIdx.x >> 5;
+    const int64_t i = int64_t(blockIdx.x - p.heavy_blocks) * kSpmmWarps + warp;
+    if (i >= p.N) return;
+    const RowSpan sp = row_span(p.rowptr, p.nnz, i);
+    if (p.heavy_blocks > 0 && sp.total - 1 > kHeavyDegree) return;   // a heavy block's row
+    float acc[NV][VEC];
+#pragma unroll
+    for (int v = 0; v < NV; ++v)
+#pragma unroll
+        for (int c = 0; c < VEC; ++c) acc[v][c] = 0.0f;
+    gather<VEC, L, NV, U, kPre>(p, i, sp.b, 0, sp.total, f0, acc);
+    reduce_groups<VEC, L, NV>(acc);
+    epi(p, i, sp.dinv, f0, acc);
+}
+
+template <int VEC, int L, int NV, int U, bool kPre, class Epi>
+__device__ __forceinline__ void heavy_rows(const SpmmParams &p, const Epi &epi, int f0,
+                                           float *part, unsigned *mask) {
+    constexpr int SLAB = L * NV * VEC;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int g = lane / L, sl = lane % L;
+    for (int64_t base = int64_t(blockIdx.x) * kSpmmThreads; base < p.N;
+         base += int64_t(p.heavy_blocks) * kSpmmThreads) {
+        const int64_t r = base + threadIdx.x;
+        bool heavy = false;
+        if (r < p.N) heavy = row_span(p.rowptr, p.nnz, r).total - 1 > kHeavyDegree;
+        const unsigned m = __ballot_sync(kFullMask, heavy);
+        if (lane == 0) mask[warp] = m;
+        __syncthreads();
+        for (int w = 0; w < kSpmmWarps; ++w) {
+            unsigned mm = mask[w];
+            while (mm != 0u) {
+                const int bit = __ffs(mm) - 1;
+                mm &= mm - 1u;
+                const int64_t i = base + w * 32 + bit;
+                const RowSpan sp = row_span(p.rowptr, p.nnz, i);
+                float acc[NV][VEC];
+#pragma unroll
+                for (int v = 0; v < NV; ++v)
+#pragma unroll
+                    for (int c = 0; c < VEC; ++c) acc[v][c] = 0.0f;
+                const int64_t q0 = sp.total * warp / kSpmmWarps;
+                const int64_t q1 = sp.total * (warp + 1) / kSpmmWarps;
+                gather<VEC, L, NV, U, kPre>(p, i, sp.b, q0, q1, f0, acc);
+                reduce_groups<VEC, L, NV>(acc);
+                if (g == 0) {
+#pragma unroll
+                    for (int v = 0; v < NV; ++v)
+#pragma unroll
+                        for (int c = 0; c < VEC; ++c)
+                            part[warp * SLAB + (v * L + sl) * VEC + c] = acc[v][c];
+                }
+                __syncthreads();
+                if (warp == 0) {
+#pragma unroll
+                    for (int v = 0; v < NV; ++v)
+#pragma unroll
+                        for (int c = 0; c < VEC; ++c) {
+                            float t = 0.0f;
+                            if (g == 0)
+                                for (int q = 0; q < kSpmmWarps; ++q)
+                                    t += part[q * SLAB + (v * L + sl) * VEC + c];
+                            acc[v][c] = t;
+                        }
+                    epi(p, i, sp.dinv, f0, acc);
+                }
+                __syncthreads();
+            }
+        }
+        __syncthreads();   // every warp has read this chunk's masks before they change
+    }
+}
+
+template <int VEC, int L, int NV, int U, bool kPre>
+__global__ void __launch_bounds__(kSpmmThreads, 3)
+spmm_norm_kernel(SpmmParams p) {
+    constexpr int SLAB = L * NV * VEC;
+    __shared__ float part[kSpmmWarps * SLAB];
+    __shared__ unsigned mask[kSpmmWarps];
+    grid_dependency_wait();     // Z is the output of the previous kernel
+    const int f0 = blockIdx.y * SLAB;
+    StoreRow<VEC, L, NV> epi;
+    if (int(blockIdx.x) < p.heavy_blocks)
+        heavy_rows<VEC, L, NV, U, kPre>(p, epi, f0, part, mask);
+    else
+        light_rows<VEC, L, NV, U, kPre>(p, epi, f0);
 }
 
 // ---------------------------------------------------------------------------
 // Layer-1 aggregation fused with layer 2's binarization and product.
 //
-// Each warp computes H1_i = dinv_i * sum_j Z1'_j exactly as the kernel above
-// (VEC = 4, one vector per lane, pre-scaled rows), then, without writing H1
-// (unless asked to), takes layer 2's steps on the row while it is still in
-// registers: the signs of its Fh <= 128 features become one or two 64-bit
-// words (four ballots, one per vector component, spread into place), the
-// row scale alpha2_i = mean |H1_i| is one warp reduction, and the XNOR
-// popcount against the (shared-memory) packed columns of W2 gives
+// Each row's H1_i = dinv_i * sum_j Z1'_j is computed exactly as above (VEC = 4,
+// one vector per lane, pre-scaled rows). Then, without writing H1 (unless
+// asked to), layer 2's steps run on the row while it is in registers: the
+// signs of its Fh <= 128 features become one or two 64-bit words (four
+// ballots, one per vector component, spread into place), the row scale
+// alpha2_i = mean |H1_i| is one warp reduction, and the XNOR popcount against
+// the (shared-memory) packed columns of W2 gives
 //   Z2'_ij = (alpha2_i * dinv_i) * (beta2_j * (Fh - 2 popc(h_i ^ w_j))),
-// the same expression the product's degree-scaled epilogue evaluates.
+// the expression the product's degree-scaled epilogue evaluates. Columns of
+// Z2' from Fo up to its row stride are written as zeros, so the layer-2
+// aggregation can gather whole 4-wide vectors.
 
 // Spreads 16 bits so that bit i lands on bit 4i of a 64-bit word.
 __device__ __forceinline__ uint64_t spread16by4(uint32_t x) {
@@ -159,157 +291,159 @@ __device__ __forceinline__ uint64_t spread16by4(uint32_t x) {
     return v;
 }
 
+struct FusedLayer2 {
+    float *H1;
+    int64_t ldh;
+    const uint64_t *sW;       // shared: Fo x words2 packed columns of W2
+    const float *sBeta;       // shared: Fo
+    int Fo;
+    int words2;
+    float *Z2;
+    int64_t ldz2;
+};
+
 template <int L>
-__global__ void __launch_bounds__(kSpmmThreads, 4)
-spmm_pack_gemm_kernel(const int64_t *__restrict__ rowptr, const int32_t *__restrict__ colidx,
-                      int64_t N, int64_t nnz, const float *__restrict__ Z1, int Fh,
-                      float *__restrict__ H1, int64_t ldh, const uint64_t *__restrict__ wbits2,
-                      const float *__restrict__ beta2, int Fo, int words2,
-                      float *__restrict__ Z2, int64_t ldz2) {
-    constexpr int P = 32 / L;
+struct PackGemmRow {
+    FusedLayer2 f;
+    __device__ __forceinline__ void operator()(const SpmmParams &p, int64_t i, float dinv,
+                                               int, float (&acc)[1][4]) const {
+        const int lane = threadIdx.x & 31;
+        const int g = lane / L, sl = lane % L;
+        const int fb = sl * 4;
+        const int Fh = p.F;
+        float h[4];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) h[c] = acc[0][c] * dinv;
+        if (f.H1 != nullptr && g == 0) {
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+                if (fb + c < Fh) f.H1[i * f.ldh + fb + c] = h[c];
+        }
+        // Layer 2, Eqs. 7-8: signs of H1_i packed LSB-first, and its mean |.|.
+        uint64_t w0 = 0, w1 = 0;
+        float l1 = 0.0f;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const bool in = g == 0 && fb + c < Fh;
+            const unsigned m = __ballot_sync(kFullMask, in && h[c] >= 0.0f);
+            w0 |= spread16by4(m) << c;
+            w1 |= spread16by4(m >> 16) << c;
+            l1 += in ? fabsf(h[c]) : 0.0f;
+        }
+        l1 = warp_sum(l1);
+        const float a = (l1 / float(Fh)) * dinv;
+        // Layer 2, Eqs. 11-12, pre-scaled by this row's 1/sqrt(dhat_i).
+        for (int jo = lane; jo < f.ldz2; jo += 32) {
+            float z = 0.0f;
+            if (jo < f.Fo) {
+                int mism = __popcll(w0 ^ f.sW[jo * f.words2]);
+                if (f.words2 > 1) mism += __popcll(w1 ^ f.sW[jo * f.words2 + 1]);
+                z = a * (f.sBeta[jo] * float(Fh - 2 * mism));
+            }
+            f.Z2[i * f.ldz2 + jo] = z;
+        }
+    }
+};
+
+template <int L>
+__global__ void __launch_bounds__(kSpmmThreads, 3)
+spmm_pack_gemm_kernel(SpmmParams p, FusedLayer2 f, const uint64_t *__restrict__ wbits2,
+                      const float *__restrict__ beta2) {
+    constexpr int SLAB = L * 4;
+    __shared__ float part[kSpmmWarps * SLAB];
+    __shared__ unsigned mask[kSpmmWarps];
     __shared__ uint64_t sW[kMaxFusedOut * 2];
     __shared__ float sBeta[kMaxFusedOut];
-    for (int q = threadIdx.x; q < Fo * words2; q += kSpmmThreads) sW[q] = __ldg(wbits2 + q);
-    for (int q = threadIdx.x; q < Fo; q += kSpmmThreads) sBeta[q] = __ldg(beta2 + q);
+    grid_dependency_wait();     // Z1' and the packed W2 come from earlier kernels
+    for (int q = threadIdx.x; q < f.Fo * f.words2; q += kSpmmThreads) sW[q] = __ldg(wbits2 + q);
+    for (int q = threadIdx.x; q < f.Fo; q += kSpmmThreads) sBeta[q] = __ldg(beta2 + q);
     __syncthreads();
+    f.sW = sW;
+    f.sBeta = sBeta;
+    PackGemmRow<L> epi{f};
+    if (int(blockIdx.x) < p.heavy_blocks)
+        heavy_rows<4, L, 1, 4, true>(p, epi, 0, part, mask);
+    else
+        light_rows<4, L, 1, 4, true>(p, epi, 0);
+}
 
-    const int lane = threadIdx.x & 31;
-    const int64_t i = (int64_t(blockIdx.x) * kSpmmThreads + threadIdx.x) >> 5;
-    if (i >= N) return;
-    const int g = lane / L, sl = lane % L;
-    const int f = sl * 4;                      // this lane's first feature
-
-    const int64_t rb = __ldg(rowptr + i), re = __ldg(rowptr + i + 1);
-    const int64_t b = min(max(rb, int64_t(0)), nnz);
-    const int64_t e = min(max(re, b), nnz);
-    const float dinv_i = inv_sqrt_degree(e - b);
-    const int64_t total = (e - b) + 1;
-
-    float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-    for (int64_t base = 0; base < total; base += 32) {
-        int j = -1;
-        const int64_t q = base + lane;
-        if (q < total) {
-            j = (q == 0) ? int(i) : __ldg(colidx + b + q - 1);
-            if (j < 0 || j >= N) j = -1;
-        }
-        const int cnt = int(min(total - base, int64_t(32)));
-        for (int t0 = 0; t0 < cnt; t0 += P * kUnroll) {
-            float4 val[kUnroll];
-            bool live[kUnroll];
-#pragma unroll
-            for (int u = 0; u < kUnroll; ++u) {
-                const int src = t0 + u * P + g;
-                const int jj = __shfl_sync(kFullMask, j, src & 31);
-                live[u] = src < cnt && jj >= 0 && f < Fh;
-                val[u] = live[u] ? __ldg(reinterpret_cast<const float4 *>(Z1 + int64_t(jj) * Fh + f))
-                                 : make_float4(0.f, 0.f, 0.f, 0.f);
-            }
-#pragma unroll
-            for (int u = 0; u < kUnroll; ++u) {
-                acc[0] += val[u].x;
-                acc[1] += val[u].y;
-                acc[2] += val[u].z;
-                acc[3] += val[u].w;
-            }
-        }
-    }
-#pragma unroll
-    for (int o = L; o < 32; o <<= 1)
-#pragma unroll
-        for (int c = 0; c < 4; ++c) acc[c] += __shfl_xor_sync(kFullMask, acc[c], o);
-
-    float h[4];
-#pragma unroll
-    for (int c = 0; c < 4; ++c) h[c] = acc[c] * dinv_i;
-    if (H1 != nullptr && g == 0) {
-#pragma unroll
-        for (int c = 0; c < 4; ++c)
-            if (f + c < Fh) H1[i * ldh + f + c] = h[c];
-    }
-
-    // Layer 2, Eqs. 7-8: signs of H1_i packed LSB-first, and its mean |.|.
-    uint64_t w0 = 0, w1 = 0;
-    float l1 = 0.0f;
-#pragma unroll
-    for (int c = 0; c < 4; ++c) {
-        const bool in = g == 0 && f + c < Fh;
-        const unsigned m = __ballot_sync(kFullMask, in && h[c] >= 0.0f);
-        w0 |= spread16by4(m) << c;
-        w1 |= spread16by4(m >> 16) << c;
-        l1 += in ? fabsf(h[c]) : 0.0f;
-    }
-    l1 = warp_sum(l1);
-    const float a = (l1 / float(Fh)) * dinv_i;
-
-    // Layer 2, Eqs. 11-12, pre-scaled by this row's 1/sqrt(dhat_i).
-    for (int jo = lane; jo < Fo; jo += 32) {
-        int mism = __popcll(w0 ^ sW[jo * words2]);
-        if (words2 > 1) mism += __popcll(w1 ^ sW[jo * words2 + 1]);
-        const int d = Fh - 2 * mism;
-        Z2[i * ldz2 + jo] = a * (sBeta[jo] * float(d));
-    }
+// Leading blocks that look for heavy rows: up to two per SM, one per 256 rows.
+int heavy_block_count(int64_t N, const DeviceInfo &dev) {
+    const int64_t chunks = (N + kSpmmThreads - 1) / kSpmmThreads;
+    const int64_t cap = 2 * int64_t(dev.sm_count);
+    return int(chunks < cap ? chunks : cap);
 }
 
 template <int VEC, int L, int NV, bool kPre>
-void launch_cfg(const SpmmArgs &a, cudaStream_t s) {
+void launch_cfg(const SpmmArgs &a, const DeviceInfo &dev, int Fload, cudaStream_t s, bool pdl) {
     constexpr int SLAB = L * NV * VEC;
-    const int64_t rows_per_block = kSpmmThreads / 32;
-    dim3 grid(unsigned((a.N + rows_per_block - 1) / rows_per_block),
+    constexpr int U = NV == 1 ? 4 : 2;
+    const bool vec_store = a.ldh % VEC == 0 && aligned_to(a.H, size_t(VEC) * 4);
+    SpmmParams p{a.rowptr, a.colidx, a.N, a.nnz, a.Z, a.ldz, Fload, a.F, a.H, a.ldh,
+                 heavy_block_count(a.N, dev), vec_store};
+    dim3 grid(unsigned(p.heavy_blocks + (a.N + kSpmmWarps - 1) / kSpmmWarps),
               unsigned((a.F + SLAB - 1) / SLAB));
-    spmm_norm_kernel<VEC, L, NV, kPre><<<grid, kSpmmThreads, 0, s>>>(
-        a.rowptr, a.colidx, a.N, a.nnz, a.Z, a.ldz, a.F, a.H, a.ldh);
+    launch_kernel(spmm_norm_kernel<VEC, L, NV, U, kPre>, grid, dim3(kSpmmThreads), 0, s, pdl,
+                  dim3(1, 1, 1), p);
 }
 
 // Lanes per neighbour L = the power of two >= the row's vector count (at
 // least 4, at most 32); NV = 2 vectors per lane once a row exceeds 32.
 template <int VEC, bool kPre>
-void launch_vec(const SpmmArgs &a, cudaStream_t s) {
-    const int nvec = (a.F + VEC - 1) / VEC;
-    if (nvec <= 4) launch_cfg<VEC, 4, 1, kPre>(a, s);
-    else if (nvec <= 8) launch_cfg<VEC, 8, 1, kPre>(a, s);
-    else if (nvec <= 16) launch_cfg<VEC, 16, 1, kPre>(a, s);
-    else if (nvec <= 32) launch_cfg<VEC, 32, 1, kPre>(a, s);
-    else launch_cfg<VEC, 32, 2, kPre>(a, s);
+void launch_vec(const SpmmArgs &a, const DeviceInfo &dev, int Fload, cudaStream_t s, bool pdl) {
+    const int nvec = Fload / VEC;
+    if (nvec <= 4) launch_cfg<VEC, 4, 1, kPre>(a, dev, Fload, s, pdl);
+    else if (nvec <= 8) launch_cfg<VEC, 8, 1, kPre>(a, dev, Fload, s, pdl);
+    else if (nvec <= 16) launch_cfg<VEC, 16, 1, kPre>(a, dev, Fload, s, pdl);
+    else if (nvec <= 32) launch_cfg<VEC, 32, 1, kPre>(a, dev, Fload, s, pdl);
+    else launch_cfg<VEC, 32, 2, kPre>(a, dev, Fload, s, pdl);
 }
 
 template <bool kPre>
-void launch_pre(const SpmmArgs &a, cudaStream_t s) {
+void launch_pre(const SpmmArgs &a, const DeviceInfo &dev, cudaStream_t s, bool pdl) {
     auto al = [](const void *p, int n) { return aligned_to(p, size_t(n) * 4); };
-    if (a.F % 4 == 0 && a.ldz % 4 == 0 && a.ldh % 4 == 0 && al(a.Z, 4) && al(a.H, 4))
-        launch_vec<4, kPre>(a, s);
+    // Gathers may read whole vectors past F when the padding up to a multiple
+    // of 4 lies inside the row stride and is declared readable (a.z_pad4).
+    const int F4 = (a.F + 3) / 4 * 4;
+    if (a.ldz % 4 == 0 && al(a.Z, 4) && (a.F % 4 == 0 || (a.z_pad4 && F4 <= a.ldz)))
+        launch_vec<4, kPre>(a, dev, F4, s, pdl);
     else if (a.F % 2 == 0 && a.ldz % 2 == 0 && a.ldh % 2 == 0 && al(a.Z, 2) && al(a.H, 2))
-        launch_vec<2, kPre>(a, s);
+        launch_vec<2, kPre>(a, dev, a.F, s, pdl);
     else
-        launch_vec<1, kPre>(a, s);
+        launch_vec<1, kPre>(a, dev, a.F, s, pdl);
 }
 
 }  // namespace
 
-void launch_spmm_norm(const SpmmArgs &a, const DeviceInfo &, cudaStream_t stream) {
+void launch_spmm_norm(const SpmmArgs &a, const DeviceInfo &dev, cudaStream_t stream, bool pdl) {
     if (a.N == 0) return;
-    if (a.prescaled) launch_pre<true>(a, stream);
-    else launch_pre<false>(a, stream);
+    if (a.prescaled) launch_pre<true>(a, dev, stream, pdl);
+    else launch_pre<false>(a, dev, stream, pdl);
 }
 
 bool spmm_pack_gemm_supported(int Fh, int Fo) {
     return Fh >= 1 && Fh <= 128 && Fh % 4 == 0 && Fo >= 1 && Fo <= kMaxFusedOut;
 }
 
-void launch_spmm_pack_gemm(const SpmmPackGemmArgs &a, cudaStream_t s) {
+void launch_spmm_pack_gemm(const SpmmPackGemmArgs &a, const DeviceInfo &dev, cudaStream_t s,
+                           bool pdl) {
     if (a.N == 0) return;
     const int nvec = a.Fh / 4;
-    const dim3 grid(unsigned((a.N + kSpmmThreads / 32 - 1) / (kSpmmThreads / 32)));
-    const int words2 = (a.Fh + 63) / 64;
-#define BIGCN_LAUNCH_SPG(LL)                                                                  \
-    spmm_pack_gemm_kernel<LL><<<grid, kSpmmThreads, 0, s>>>(a.rowptr, a.colidx, a.N, a.nnz,   \
-                                                            a.Z1, a.Fh, a.H1, a.ldh, a.wbits2, \
-                                                            a.beta2, a.Fo, words2, a.Z2, a.ldz2)
-    if (nvec <= 4) BIGCN_LAUNCH_SPG(4);
-    else if (nvec <= 8) BIGCN_LAUNCH_SPG(8);
-    else if (nvec <= 16) BIGCN_LAUNCH_SPG(16);
-    else BIGCN_LAUNCH_SPG(32);
-#undef BIGCN_LAUNCH_SPG
+    SpmmParams p{a.rowptr, a.colidx, a.N, a.nnz, a.Z1, a.Fh, a.Fh, a.Fh, nullptr, 0,
+                 heavy_block_count(a.N, dev), false};
+    FusedLayer2 f{a.H1, a.ldh, nullptr, nullptr, a.Fo, (a.Fh + 63) / 64, a.Z2, a.ldz2};
+    const dim3 grid(unsigned(p.heavy_blocks + (a.N + kSpmmWarps - 1) / kSpmmWarps));
+    const dim3 one(1, 1, 1), block(kSpmmThreads);
+    if (nvec <= 4)
+        launch_kernel(spmm_pack_gemm_kernel<4>, grid, block, 0, s, pdl, one, p, f, a.wbits2, a.beta2);
+    else if (nvec <= 8)
+        launch_kernel(spmm_pack_gemm_kernel<8>, grid, block, 0, s, pdl, one, p, f, a.wbits2, a.beta2);
+    else if (nvec <= 16)
+        launch_kernel(spmm_pack_gemm_kernel<16>, grid, block, 0, s, pdl, one, p, f, a.wbits2,
+                      a.beta2);
+    else
+        launch_kernel(spmm_pack_gemm_kernel<32>, grid, block, 0, s, pdl, one, p, f, a.wbits2,
+                      a.beta2);
 }
 
 }  // namespace bigcn
@@ -336,7 +470,7 @@ bigcn_status spmm_entry(const int64_t *rowptr, const int32_t *colidx, int64_t N,
     DeviceInfo dev;
     bigcn_status st = current_device(&dev);
     if (st != BIGCN_OK) return st;
-    SpmmArgs a{rowptr, colidx, N, nnz, Z, ldz, F, H, ldh, prescaled};
+    SpmmArgs a{rowptr, colidx, N, nnz, Z, ldz, F, H, ldh, prescaled, false};
     launch_spmm_norm(a, dev, as_stream(stream));
     return launch_status();
 }

@@ -46,6 +46,7 @@ xnor_gemm_popc_kernel(const uint64_t *__restrict__ A, const float *__restrict__ 
     __shared__ uint64_t As[kBM][kPitch];
     __shared__ uint64_t Bs[BN][kPitch];
 
+    grid_dependency_wait();     // the packed operands come from earlier kernels
     const int tid = threadIdx.x;
     const int tx = tid & 15, ty = tid >> 4;
     const int64_t m0 = int64_t(blockIdx.x) * kBM;
@@ -153,7 +154,7 @@ xnor_gemm_popc_kernel(const uint64_t *__restrict__ A, const float *__restrict__ 
 }
 
 template <int TN, bool kDeg>
-void launch_tn(const GemmArgs &g, const DeviceInfo &dev, cudaStream_t s) {
+void launch_tn(const GemmArgs &g, const DeviceInfo &dev, cudaStream_t s, bool pdl) {
     constexpr int BN = 16 * TN;
     const unsigned gx = unsigned((g.N + kBM - 1) / kBM), gy = unsigned((g.F + BN - 1) / BN);
     const int ksteps = (g.words + kBKW - 1) / kBKW;
@@ -165,38 +166,29 @@ void launch_tn(const GemmArgs &g, const DeviceInfo &dev, cudaStream_t s) {
         if (S > ksteps) S = ksteps;
     }
     if (S == 1) {
-        xnor_gemm_popc_kernel<TN, kDeg, false><<<dim3(gx, gy), kThreads, 0, s>>>(
-            g.A, g.alpha, g.N, g.B, g.beta, g.F, g.K, g.words, g.Z, g.ldz, g.dots, g.rowptr);
+        launch_kernel(xnor_gemm_popc_kernel<TN, kDeg, false>, dim3(gx, gy), dim3(kThreads), 0, s,
+                      pdl, dim3(1, 1, 1), g.A, g.alpha, g.N, g.B, g.beta, g.F, g.K, g.words, g.Z,
+                      g.ldz, g.dots, g.rowptr);
         return;
     }
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(gx, gy, S);
-    cfg.blockDim = dim3(kThreads, 1, 1);
-    cfg.stream = s;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = 1;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = S;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    cudaLaunchKernelEx(&cfg, xnor_gemm_popc_kernel<TN, kDeg, true>, g.A, g.alpha, g.N, g.B,
-                       g.beta, g.F, g.K, g.words, g.Z, g.ldz, g.dots, g.rowptr);
+    launch_kernel(xnor_gemm_popc_kernel<TN, kDeg, true>, dim3(gx, gy, S), dim3(kThreads), 0, s,
+                  pdl, dim3(1, 1, S), g.A, g.alpha, g.N, g.B, g.beta, g.F, g.K, g.words, g.Z,
+                  g.ldz, g.dots, g.rowptr);
 }
 
 template <bool kDeg>
-void launch_deg(const GemmArgs &g, const DeviceInfo &dev, cudaStream_t s) {
-    if (g.F > 32) launch_tn<4, kDeg>(g, dev, s);
-    else if (g.F > 16) launch_tn<2, kDeg>(g, dev, s);
-    else launch_tn<1, kDeg>(g, dev, s);
+void launch_deg(const GemmArgs &g, const DeviceInfo &dev, cudaStream_t s, bool pdl) {
+    if (g.F > 32) launch_tn<4, kDeg>(g, dev, s, pdl);
+    else if (g.F > 16) launch_tn<2, kDeg>(g, dev, s, pdl);
+    else launch_tn<1, kDeg>(g, dev, s, pdl);
 }
 
 }  // namespace
 
-void launch_xnor_gemm(const GemmArgs &g, const DeviceInfo &dev, cudaStream_t stream) {
+void launch_xnor_gemm(const GemmArgs &g, const DeviceInfo &dev, cudaStream_t stream, bool pdl) {
     if (g.N == 0) return;
-    if (g.rowptr != nullptr) launch_deg<true>(g, dev, stream);
-    else launch_deg<false>(g, dev, stream);
+    if (g.rowptr != nullptr) launch_deg<true>(g, dev, stream, pdl);
+    else launch_deg<false>(g, dev, stream, pdl);
 }
 
 }  // namespace bigcn

@@ -4,9 +4,9 @@ their CUDA-graph capture.
 Plumbing around libbigcn.so: torch owns the device memory and the stream,
 and every step of the computation runs in the library's kernels.
 
-``launch()`` makes the one call ``bigcn_forward_2layer`` (5 kernels for the
-usual widths: both weight packs, layer-1 row pack, layer-1 XNOR GEMM, layer-1
-aggregation fused with layer 2's pack and GEMM, layer-2 aggregation).
+``launch()`` makes the one call ``bigcn_forward_2layer`` (4 kernels for the
+usual widths: both weight packs; layer-1 centre + pack + XNOR GEMM; layer-1
+aggregation fused with layer 2's pack and GEMM; layer-2 aggregation).
 ``launch_steps()`` runs the same forward as eight separate step calls
 (pack_rows, pack_weights, xnor_gemm_degscaled, spmm_prescaled per layer),
 keeping every intermediate in its own buffer, for step-by-step checks.
@@ -21,12 +21,21 @@ from . import binding as B
 STEP_KERNELS = ("pack_rows", "pack_weights", "xnor_gemm", "spmm")
 
 
-def fused_kernel_names(Fh: int, Fo: int):
-    if B.bigcn_forward_2layer_launches(Fh, Fo) == 5:
-        return ("pack_weights(W1,W2)", "L1.pack_rows", "L1.xnor_gemm",
-                "L1.spmm+L2.pack_rows+L2.xnor_gemm", "L2.spmm")
-    return ("pack_weights(W1,W2)", "L1.pack_rows", "L1.xnor_gemm", "L1.spmm",
-            "L2.pack_rows", "L2.xnor_gemm", "L2.spmm")
+FRONT = "L1.pack_rows+L1.xnor_gemm"
+FUSED_AGG = "L1.spmm+L2.pack_rows+L2.xnor_gemm"
+
+
+def fused_kernel_names(N: int, K: int, Fh: int, Fo: int):
+    """Names of the kernels bigcn_forward_2layer launches for these sizes, in
+    order (4 to 7 of them, depending on which fusions the widths allow)."""
+    n = B.bigcn_forward_2layer_launches(N, K, Fh, Fo)
+    front_fused = n in (4, 6)
+    agg_fused = n in (4, 5)
+    names = ["pack_weights(W1,W2)"]
+    names += [FRONT] if front_fused else ["L1.pack_rows", "L1.xnor_gemm"]
+    names += [FUSED_AGG] if agg_fused else ["L1.spmm", "L2.pack_rows", "L2.xnor_gemm"]
+    names += ["L2.spmm"]
+    return tuple(names)
 
 
 class GCN2Forward:
@@ -47,7 +56,7 @@ class GCN2Forward:
         self.workspace = torch.empty(max(nbytes, 1), dtype=torch.uint8, device=self.device)
         self.logits = e(N, out)
         self.H1 = e(N, hidden) if keep_h1 else None
-        self.kernel_names = fused_kernel_names(hidden, out)
+        self.kernel_names = fused_kernel_names(N, K, hidden, out)
         self.graph = None
         self._steps = None
 

@@ -319,8 +319,10 @@ def test_forward_2layer_records_one_event_per_kernel_boundary(cuda_device):
     case = inputs.layer_case(N, K, Fh, seed=3)
     d = {k: to_dev(v) for k, v in case.items()}
     W2 = to_dev(inputs.weights(Fh, Fo, seed=4))
-    n = B.bigcn_forward_2layer_launches(Fh, Fo)
-    assert n == 5 and B.bigcn_forward_2layer_launches(30, 7) == 7
+    n = B.bigcn_forward_2layer_launches(N, K, Fh, Fo)
+    assert n == 4 and B.bigcn_forward_2layer_launches(N, K, 30, 7) == 6
+    assert B.bigcn_forward_2layer_launches(N, 3000, 64, 7) == 5
+    assert B.bigcn_forward_2layer_launches(N, 8192, 256, 7) == 7
     events = [torch.cuda.Event(enable_timing=True) for _ in range(n + 1)]
     for e in events:
         e.record()
@@ -334,3 +336,59 @@ def test_forward_2layer_records_one_event_per_kernel_boundary(cuda_device):
     spans = [events[q].elapsed_time(events[q + 1]) for q in range(n)]
     assert all(t >= 0.0 for t in spans)
     assert events[0].elapsed_time(events[n]) > 0.0
+
+
+def hub_graph(N, hubs, seed, mean_degree=4.0):
+    """Random graph plus hub rows: (node, degree) pairs joined to random others.
+    Degrees above 2048 take the kernels' whole-block path."""
+    g = rng(seed)
+    rowptr, colidx = inputs.random_graph(N, mean_degree, seed=seed)
+    rows = np.repeat(np.arange(N), np.diff(rowptr))
+    keys = [np.minimum(rows, colidx) * N + np.maximum(rows, colidx)]
+    for node, deg in hubs:
+        others = g.choice(np.delete(np.arange(N), node), size=deg, replace=False)
+        keys.append(np.minimum(node, others) * N + np.maximum(node, others))
+    keys = np.unique(np.concatenate(keys).astype(np.int64))
+    return inputs.edges_to_csr(keys // N, keys % N, N)
+
+
+HUBS = [(3, 2049), (7, 2500), (250, 5000), (256, 2100), (4000, 8190), (8999, 3000)]
+
+
+@pytest.mark.parametrize("F", [1, 6, 41, 128, 300])
+@pytest.mark.parametrize("prescaled", [False, True])
+def test_spmm_many_heavy_rows(cuda_device, F, prescaled):
+    N = 9000
+    rowptr, colidx = hub_graph(N, HUBS, seed=F)
+    deg = np.diff(rowptr)
+    assert (deg > 2048).sum() >= len(HUBS)
+    Z = rng(F + 1).standard_normal((N, F)).astype(np.float32)
+    Zd, H = to_dev(Z), torch.empty((N, F), device=cuda_device)
+    if prescaled:
+        B.bigcn_spmm_prescaled(to_dev(rowptr), to_dev(colidx), Zd, H)
+        dinv = 1.0 / np.sqrt(oracle.degree(rowptr))
+        ref = oracle.aggregate(rowptr, colidx, Z.astype(np.float64) / dinv[:, None])
+    else:
+        B.bigcn_spmm_norm(to_dev(rowptr), to_dev(colidx), Zd, H)
+        ref = oracle.aggregate(rowptr, colidx, Z.astype(np.float64))
+    assert_close(H, ref, f"H (F={F}, heavy rows)")
+
+
+@pytest.mark.parametrize("Fh,Fo", [(128, 41), (64, 7), (16, 3)])
+def test_forward_2layer_heavy_rows(cuda_device, Fh, Fo):
+    N, K = 9000, 300
+    rowptr, colidx = hub_graph(N, HUBS, seed=Fh + Fo)
+    g = rng(Fo)
+    X = g.standard_normal((N, K)).astype(np.float32)
+    s, t = inputs.bn_stats(X)
+    W1, W2 = inputs.weights(K, Fh, seed=5), inputs.weights(Fh, Fo, seed=6)
+    ws = torch.empty(B.bigcn_forward_2layer_workspace_bytes(N, K, Fh, Fo), dtype=torch.uint8,
+                     device=cuda_device)
+    H1 = torch.empty((N, Fh), device=cuda_device)
+    out = torch.empty((N, Fo), device=cuda_device)
+    B.bigcn_forward_2layer(to_dev(X), to_dev(s), to_dev(t), to_dev(W1), to_dev(W2),
+                           to_dev(rowptr), to_dev(colidx), ws, out, H1=H1)
+    ref1 = oracle.layer_forward(X, W1, rowptr, colidx, s, t)
+    assert_close(H1, ref1["H"], "H1 with heavy rows")
+    ref2 = oracle.layer_forward(H1.cpu().numpy(), W2, rowptr, colidx)
+    assert_close(out, ref2["H"], "logits with heavy rows")
