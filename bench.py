@@ -443,6 +443,112 @@ def run_gpu(args, rank, world, local_rank):
     return 0
 
 
+SWEEP_KERNELS = ("pack_rows", "pack_weights", "xnor_gemm", "spmm")
+
+
+def run_sweep(args, rank, world, local_rank):
+    """One Bi-GCN layer on a C5 sweep point (2^20 nodes, K, F): the four step
+    kernels the layer runs (bigcn_pack_rows, bigcn_pack_weights,
+    bigcn_xnor_gemm_degscaled, bigcn_spmm_prescaled), each timed with events
+    on its stream. The features (up to 34 GB) are drawn on the device by
+    torch's seeded generator; the other inputs come from the usual seeds.
+    The inputs are larger than L2, so no flush is needed between steps."""
+    import torch
+
+    from paper_2010_07565_gb300 import binding as B
+    from paper_2010_07565_gb300 import inputs
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    w = inputs.get_workload(args.workload)
+    N, K, F = w.N, w.K, w.hidden
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(1000 + w.index)
+    X = torch.randn((N, K), device=dev, generator=gen)
+    Wt = torch.from_numpy(inputs.weights(K, F, 3000 + w.index)).to(dev)
+    rp, ci = inputs.graph(w)
+    rowptr, colidx = torch.from_numpy(rp).to(dev), torch.from_numpy(ci).to(dev)
+    nnz = int(ci.shape[0])
+    words = B.words_for(K)
+    bits = torch.empty((N, words), dtype=torch.int64, device=dev)
+    alpha = torch.empty(N, device=dev)
+    wbits = torch.empty((F, words), dtype=torch.int64, device=dev)
+    beta = torch.empty(F, device=dev)
+    Z, H = torch.empty((N, F), device=dev), torch.empty((N, F), device=dev)
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
+
+    def step():
+        ev[0].record()
+        B.bigcn_pack_rows(X, None, None, bits, alpha)
+        ev[1].record()
+        B.bigcn_pack_weights(Wt, wbits, beta)
+        ev[2].record()
+        B.bigcn_xnor_gemm_degscaled(bits, alpha, wbits, beta, K, rowptr, Z)
+        ev[3].record()
+        B.bigcn_spmm_prescaled(rowptr, colidx, Z, H)
+        ev[4].record()
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    per_kernel = [[] for _ in SWEEP_KERNELS]
+    step_ms = []
+    with ClockSampler(local_rank) as clocks:
+        for _ in range(args.steps):
+            step()
+            ev[4].synchronize()
+            for k in range(4):
+                per_kernel[k].append(ev[k].elapsed_time(ev[k + 1]))
+            step_ms.append(ev[0].elapsed_time(ev[4]))
+    total_ms = float(sum(step_ms))
+    max_ms, units = aggregate_over_ranks(total_ms, float(N) * args.steps, world)
+    if rank != 0:
+        return 0
+    peaks, peak_kind = load_peaks()
+    hbm = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+    mean_us = [1e3 * statistics.fmean(t) for t in per_kernel]
+    work = {"pack_rows": (4.0 * N * K + 8.0 * N * words + 4.0 * N, "bytes", "hbm"),
+            "pack_weights": (4.0 * K * F + 8.0 * F * words + 4.0 * F, "bytes", "hbm"),
+            "xnor_gemm": (float(N) * K * F, "bit-ops", "tensor"),
+            "spmm": (8.0 * (N + 1) + 4.0 * nnz + 8.0 * N * F, "bytes", "hbm")}
+    k_dom = max(range(4), key=lambda k: mean_us[k])
+    name = SWEEP_KERNELS[k_dom]
+    amount, unit, bound = work[name]
+    rate = amount / (mean_us[k_dom] * 1e-6)
+    if bound == "hbm":
+        achieved, peak, runit = rate / 1e9, hbm, "GB/s"
+        src = f"{peak_kind} MEASURED_PEAKS.json hbm_gbs"
+    else:
+        # FP8 dense tensor peak: the measured bf16 burst figure x 2 (fp8 = 2 x bf16 nominal)
+        achieved, peak, runit = 2.0 * rate / 1e12, 2.0 * float(peaks.get("bf16_tflops", 1900.0)), \
+            "TFLOP/s (fp8, 2 flops per +-1 MAC)"
+        src = f"{peak_kind} MEASURED_PEAKS.json bf16_tflops x 2 (fp8/bf16 nominal ratio)"
+    line = {
+        "metric": METRIC, "value": units / (max_ms * 1e-3), "unit": "nodes/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": max_ms / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32+b1",
+        "data": "synthetic",
+        "config": {"workload": w.description, "name": w.name, "N": N, "K": K, "F": F, "nnz": nnz,
+                   "l2": "inputs larger than L2 (no flush)",
+                   "launch": "bigcn_pack_rows, bigcn_pack_weights, bigcn_xnor_gemm_degscaled, "
+                             "bigcn_spmm_prescaled (the kernels of bigcn_layer_forward)"},
+        "components": {
+            "per_kernel_us": {n: round(t, 3) for n, t in zip(SWEEP_KERNELS, mean_us)},
+            "pack_rows_gbs": work["pack_rows"][0] / (mean_us[0] * 1e-6) / 1e9,
+            "xnor_gemm_bitops_per_s": work["xnor_gemm"][0] / (mean_us[2] * 1e-6),
+            "spmm_gbs": work["spmm"][0] / (mean_us[3] * 1e-6) / 1e9},
+        "roofline": {"kernel": name, "bound": bound, "achieved": achieved, "peak": peak,
+                     "unit": runit, "frac": achieved / peak,
+                     "traffic": profiled_traffic(name, w.name), "peak_source": src},
+        "cpu_baseline": None, "e2e": None,
+        "note": "sweep point: one layer, kernel-level timing; no host-buffer run (the features "
+                "alone are up to 34 GB)",
+        "gpu_launches": 4 * args.steps, "clocks": clocks.summary(),
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def run_forward_only(args):
     """R plain forwards of the workload on cuda:0, nothing timed or printed."""
     import torch
@@ -466,7 +572,7 @@ def main(argv=None):
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["bigcn", "reference"], default="bigcn")
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD,
-                    help="C1..C4, or a sweep point such as C5_K4096_F256 (1 layer not supported)")
+                    help="C1..C4, or a one-layer sweep point such as C5_K4096_F256")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--forward-only", type=int, default=0, metavar="R",
@@ -480,6 +586,8 @@ def main(argv=None):
         return run_reference(args, rank, world)
     if args.forward_only > 0:
         return run_forward_only(args)
+    if args.workload.startswith("C5_"):
+        return run_sweep(args, rank, world, local_rank)
     if world > 1:
         import torch
         import torch.distributed as dist

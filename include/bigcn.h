@@ -164,6 +164,19 @@ bigcn_status bigcn_spmm_prescaled(const int64_t *rowptr, const int32_t *colidx,
                                   int64_t N, int64_t nnz, const float *Z, int64_t ldz,
                                   int32_t F, float *H, int64_t ldh, void *stream);
 
+/*
+ * The XNOR product of step 4 runs on the tensor cores (tcgen05, the signs
+ * as FP8 +-1, exact fp32 integer sums) when K >= 128, F >= 32 and N is at
+ * least 128 rows per SM, and on the CUDA cores (XOR + popcount) otherwise;
+ * the dots are identical either way.
+ * Its kernels wait on shared-memory barriers with a bounded number of
+ * tries. bigcn_device_timeouts synchronizes the current device, returns how
+ * many such waits ran out since its last call (0 in correct operation; a
+ * CTA whose wait ran out writes no output) and resets the count; -1 on a
+ * CUDA error.
+ */
+int32_t bigcn_device_timeouts(void);
+
 /* Bytes of device workspace bigcn_layer_forward needs for (N, K, F); 0 on
  * invalid sizes. */
 size_t bigcn_layer_workspace_bytes(int64_t N, int32_t K, int32_t F);

@@ -44,6 +44,7 @@ SIGNATURES = {
                                   ctypes.c_int),
     "bigcn_spmm_norm": ([_p, _p, _i64, _i64, _p, _i64, _i32, _p, _i64, _p], ctypes.c_int),
     "bigcn_spmm_prescaled": ([_p, _p, _i64, _i64, _p, _i64, _i32, _p, _i64, _p], ctypes.c_int),
+    "bigcn_device_timeouts": ([], _i32),
     "bigcn_layer_workspace_bytes": ([_i64, _i32, _i32], _sz),
     "bigcn_layer_forward": ([_p, _i64, _i32, _i64, _p, _p, _p, _i32, _i64, _p, _p, _i64, _p,
                              _sz, _p, _i64, _p], ctypes.c_int),
@@ -112,6 +113,11 @@ def _check(fn: str, status: int):
 
 def status_string(status: int) -> str:
     return lib().bigcn_status_string(status).decode()
+
+
+def device_timeouts() -> int:
+    """Bounded device waits that ran out since the last call (synchronizes)."""
+    return int(lib().bigcn_device_timeouts())
 
 
 def words_for(K: int) -> int:

@@ -52,6 +52,14 @@ struct GemmArgs {
     const int64_t *rowptr;   // nullable: scale row i by 1/sqrt(1 + deg_i)
 };
 
+// Step 4 on the tensor cores (xnor_gemm_tc.cu): +-1 signs as FP8 E4M3,
+// tcgen05.mma with fp32 accumulators in tensor memory. Used by
+// launch_xnor_gemm when K >= 128, F >= 32 and N gives every SM a 128-row tile.
+bool xnor_gemm_tc_supported(int64_t N, int K, int F, const DeviceInfo &dev);
+struct GemmArgs;
+void launch_xnor_gemm_tc(const GemmArgs &args, const DeviceInfo &dev, cudaStream_t stream,
+                         bool pdl);
+
 // Step 4: the XNOR-popcount product and its scaling (Eqs. 11-12).
 void launch_xnor_gemm(const GemmArgs &args, const DeviceInfo &dev, cudaStream_t stream,
                       bool pdl = false);

@@ -10,7 +10,10 @@
 // lane keeps a running sum of |y|. G warps (1, 2, 4 or 8, so that the grid
 // fills the GPU even when N is small) share a row, warp g taking chunks
 // g, g + G, ...; each warp issues eight chunks' loads (1 KB) before it
-// consumes any. The G partial |y| sums are added in a fixed order through
+// consumes any, and the grids are persistent (eight blocks per SM). The
+// whole-row kernel has no block barrier and stays at full occupancy, which
+// -- not a deeper unroll -- is what overlaps one warp's ballots with the
+// other warps' loads. The G partial |y| sums are added in a fixed order through
 // shared memory, so alpha does not depend on scheduling.
 //
 // pack_weights reads W (K x F) column-wise: thread (x, y) of a 32 x 8 block
@@ -33,55 +36,88 @@ namespace cg = cooperative_groups;
 constexpr int kPackThreads = 256;
 constexpr int kPackWarps = kPackThreads / 32;
 constexpr int kPackUnroll = 8;
+constexpr int kPackBlocksPerSM = 8;   // resident blocks the persistent grids assume
 
+// Packs chunks sub, sub + G, ... of row `row` (lane l of chunk c owns
+// feature 32c + l) and returns this warp's sum of |y| (all lanes).
 template <bool kAffine>
-__global__ void __launch_bounds__(kPackThreads, 4)
+__device__ __forceinline__ float pack_row_chunks(const float *__restrict__ x, int K,
+                                                 const float *__restrict__ scale,
+                                                 const float *__restrict__ shift,
+                                                 uint32_t *__restrict__ out, int64_t ld32, int sub,
+                                                 int G) {
+    const int lane = threadIdx.x & 31;
+    const int nchunks = (K + 31) >> 5;          // 32-bit half-words that carry signs
+    float l1 = 0.0f;
+    for (int m0 = sub; m0 < nchunks; m0 += G * kPackUnroll) {
+        float v[kPackUnroll];
+#pragma unroll
+        for (int u = 0; u < kPackUnroll; ++u) {
+            const int k = (m0 + u * G) * 32 + lane;
+            v[u] = (k < K) ? __ldcs(x + k) : 0.0f;
+        }
+#pragma unroll
+        for (int u = 0; u < kPackUnroll; ++u) {
+            const int c = m0 + u * G;
+            const int k = c * 32 + lane;
+            const bool in = k < K;
+            float y = v[u];
+            if (kAffine && in) y = __fmaf_rn(y, __ldg(scale + k), __ldg(shift + k));
+            const unsigned m = __ballot_sync(kFullMask, in && y >= 0.0f);
+            if (c < nchunks && lane == 0) out[c] = m;
+            l1 += in ? fabsf(y) : 0.0f;
+        }
+    }
+    // Pad half-words past the last one that carries signs are zero.
+    if (sub == 0)
+        for (int64_t q = nchunks + lane; q < ld32; q += 32) out[q] = 0u;
+    return warp_sum(l1);
+}
+
+// Whole rows per warp: every warp walks rows on its own (persistent grid,
+// no block barrier), which keeps the kernel small enough for full occupancy.
+template <bool kAffine>
+__global__ void __launch_bounds__(kPackThreads)
 pack_rows_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
                  const float *__restrict__ scale, const float *__restrict__ shift,
-                 uint32_t *__restrict__ bits32, int64_t ld32, float *__restrict__ alpha,
-                 int G) {
-    __shared__ float part[kPackWarps];
+                 uint32_t *__restrict__ bits32, int64_t ld32, float *__restrict__ alpha) {
     grid_dependency_wait();     // X may be the output of the previous kernel
     const int lane = threadIdx.x & 31;
-    const int warp = threadIdx.x >> 5;
-    const int sub = warp & (G - 1);
-    const int64_t row = int64_t(blockIdx.x) * (kPackWarps / G) + warp / G;
-    const int nchunks = (K + 31) >> 5;          // 32-bit half-words that carry signs
-
-    float l1 = 0.0f;
-    if (row < N) {
-        const float *x = X + row * ldx;
-        uint32_t *out = bits32 + row * ld32;
-        for (int m0 = sub; m0 < nchunks; m0 += G * kPackUnroll) {
-            float v[kPackUnroll];
-#pragma unroll
-            for (int u = 0; u < kPackUnroll; ++u) {
-                const int k = (m0 + u * G) * 32 + lane;
-                v[u] = (k < K) ? __ldcs(x + k) : 0.0f;
-            }
-#pragma unroll
-            for (int u = 0; u < kPackUnroll; ++u) {
-                const int c = m0 + u * G;
-                const int k = c * 32 + lane;
-                const bool in = k < K;
-                float y = v[u];
-                if (kAffine && in) y = __fmaf_rn(y, __ldg(scale + k), __ldg(shift + k));
-                const unsigned m = __ballot_sync(kFullMask, in && y >= 0.0f);
-                if (c < nchunks && lane == 0) out[c] = m;
-                l1 += in ? fabsf(y) : 0.0f;
-            }
-        }
-        // Pad half-words past the last one that carries signs are zero.
-        if (sub == 0)
-            for (int64_t q = nchunks + lane; q < ld32; q += 32) out[q] = 0u;
+    const int64_t nwarps = int64_t(gridDim.x) * kPackWarps;
+    for (int64_t row = int64_t(blockIdx.x) * kPackWarps + (threadIdx.x >> 5); row < N;
+         row += nwarps) {
+        const float l1 =
+            pack_row_chunks<kAffine>(X + row * ldx, K, scale, shift, bits32 + row * ld32, ld32, 0, 1);
+        if (lane == 0) alpha[row] = l1 / float(K);
     }
-    l1 = warp_sum(l1);
-    if (lane == 0) part[warp] = l1;
-    __syncthreads();
-    if (row < N && sub == 0 && lane == 0) {
-        float s = 0.0f;
-        for (int g = 0; g < G; ++g) s += part[warp + g];
-        alpha[row] = s / float(K);
+}
+
+// Rows shared by G > 1 warps (few, long rows): block b takes row groups
+// b, b + gridDim.x, ...; the G partial sums meet in shared memory.
+template <bool kAffine>
+__global__ void __launch_bounds__(kPackThreads)
+pack_rows_split_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
+                       const float *__restrict__ scale, const float *__restrict__ shift,
+                       uint32_t *__restrict__ bits32, int64_t ld32, float *__restrict__ alpha,
+                       int G) {
+    __shared__ float part[kPackWarps];
+    grid_dependency_wait();
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int sub = warp & (G - 1);
+    const int rows_per_block = kPackWarps / G;
+    for (int64_t group = blockIdx.x; group * rows_per_block < N; group += gridDim.x) {
+        const int64_t row = group * rows_per_block + warp / G;
+        const float l1 = (row < N) ? pack_row_chunks<kAffine>(X + row * ldx, K, scale, shift,
+                                                              bits32 + row * ld32, ld32, sub, G)
+                                   : 0.0f;
+        if (lane == 0) part[warp] = l1;
+        __syncthreads();
+        if (row < N && sub == 0 && lane == 0) {
+            float s = 0.0f;
+            for (int g = 0; g < G; ++g) s += part[warp + g];
+            alpha[row] = s / float(K);
+        }
+        __syncthreads();   // part[] is rewritten by the next group
     }
 }
 
@@ -153,17 +189,29 @@ void launch_pack_rows(const float *X, int64_t N, int K, int64_t ldx, const float
     const int nchunks = (K + 31) / 32;
     const int64_t full_wave = int64_t(dev.sm_count) * 64;
     int G = 1;
-    while (G < kPackWarps && N * G < full_wave && nchunks >= 2 * G * kPackUnroll) G *= 2;
+    while (G < kPackWarps && N * G < full_wave && nchunks >= 2 * G * 8) G *= 2;
     const int rows_per_block = kPackWarps / G;
-    const unsigned grid = unsigned((N + rows_per_block - 1) / rows_per_block);
+    const int64_t groups = (N + rows_per_block - 1) / rows_per_block;
+    const int64_t resident = int64_t(dev.sm_count) * kPackBlocksPerSM;
+    const dim3 grid(unsigned(groups < resident ? groups : resident)), block(kPackThreads), one(1, 1, 1);
     uint32_t *b32 = reinterpret_cast<uint32_t *>(bits);
-    if (scale)
-        launch_kernel(pack_rows_kernel<true>, dim3(grid), dim3(kPackThreads), 0, stream, pdl,
-                      dim3(1, 1, 1), X, N, K, ldx, scale, shift, b32, int64_t(words) * 2, alpha, G);
-    else
-        launch_kernel(pack_rows_kernel<false>, dim3(grid), dim3(kPackThreads), 0, stream, pdl,
-                      dim3(1, 1, 1), X, N, K, ldx, static_cast<const float *>(nullptr),
-                      static_cast<const float *>(nullptr), b32, int64_t(words) * 2, alpha, G);
+    const int64_t ld32 = int64_t(words) * 2;
+    const float *no = nullptr;
+    if (G == 1) {
+        if (scale)
+            launch_kernel(pack_rows_kernel<true>, grid, block, 0, stream, pdl, one, X, N, K, ldx,
+                          scale, shift, b32, ld32, alpha);
+        else
+            launch_kernel(pack_rows_kernel<false>, grid, block, 0, stream, pdl, one, X, N, K, ldx,
+                          no, no, b32, ld32, alpha);
+    } else {
+        if (scale)
+            launch_kernel(pack_rows_split_kernel<true>, grid, block, 0, stream, pdl, one, X, N, K,
+                          ldx, scale, shift, b32, ld32, alpha, G);
+        else
+            launch_kernel(pack_rows_split_kernel<false>, grid, block, 0, stream, pdl, one, X, N, K,
+                          ldx, no, no, b32, ld32, alpha, G);
+    }
 }
 
 void launch_pack_weights2(const WeightPack &a, const WeightPack &b, cudaStream_t stream) {

@@ -2,6 +2,9 @@
 // the +-1 inner products of packed node rows with packed weight columns,
 //   dot[i,j] = K - 2 popcount(a_i XOR b_j),  Z[i,j] = alpha_i beta_j dot[i,j].
 //
+// Products with K >= 128, F >= 32 and at least one 128-row tile per SM run on
+// the tensor cores (xnor_gemm_tc.cu); the CUDA-core path below takes the rest.
+//
 // CUDA-core path: a 128 x (16*TN) output tile per 256-thread block, the two
 // packed operand tiles staged in shared memory 8 words (512 signs) at a time
 // with register double buffering; each thread accumulates TM x TN mismatch
@@ -187,6 +190,10 @@ void launch_deg(const GemmArgs &g, const DeviceInfo &dev, cudaStream_t s, bool p
 
 void launch_xnor_gemm(const GemmArgs &g, const DeviceInfo &dev, cudaStream_t stream, bool pdl) {
     if (g.N == 0) return;
+    if (xnor_gemm_tc_supported(g.N, g.K, g.F, dev)) {
+        launch_xnor_gemm_tc(g, dev, stream, pdl);
+        return;
+    }
     if (g.rowptr != nullptr) launch_deg<true>(g, dev, stream, pdl);
     else launch_deg<false>(g, dev, stream, pdl);
 }

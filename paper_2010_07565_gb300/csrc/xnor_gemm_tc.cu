@@ -1,0 +1,353 @@
+// Step 4 of the Bi-GCN layer forward (Wang et al., CVPR 2021, Eqs. 11-12) on
+// the fifth-generation tensor cores (tcgen05) of sm_103a.
+//
+// Eq. 11's inner product of two sign vectors is a dense contraction of +-1
+// values, and FP8 E4M3 represents +-1 exactly (+1 = 0x38, -1 = 0xB8): each
+// CTA expands its packed bits into FP8 bytes in shared memory and lets
+// tcgen05.mma (kind::f8f6f4, fp32 accumulators in tensor memory) sum the
+// products. Every product is +-1 and every partial sum an integer of
+// magnitude <= K < 2^24, so the fp32 accumulator holds the dot exactly:
+// dot = K - 2 popc(a XOR b), the same integer the XNOR/popcount form gives.
+// Elements of A at k >= K are written as 0.0, so padding adds nothing.
+//
+// CTA tile: 128 rows (UMMA M) x NT output columns (UMMA N = 64, 128 or 256),
+// k-blocks of 128 signs (one 128-byte row of a 128B-swizzled K-major
+// operand). Two shared-memory stages: while the tensor core works on one,
+// the CTA's 256 threads expand the next -- each thread owns one 16-sign chunk
+// position of several rows, issues all its packed-word loads for a k-block at
+// once (and the next k-block's while the MMAs are issued), and turns every
+// four signs into four E4M3 bytes with one multiply and three logic ops.
+// A stage is reused only after the tcgen05.commit of the MMAs that read it
+// has arrived on its mbarrier.
+// Every mbarrier wait is bounded; a wait that runs out is counted in
+// g_tc_timeouts (see bigcn_device_timeouts), the CTA skips its epilogue,
+// frees its tensor memory and returns.
+//
+// Epilogue: warp w reads tensor-memory lanes 32w..32w+31 (its rows) with
+// tcgen05.ld, converts the exact fp32 dots to integers and writes
+//   Z = (alpha_i * beta_j) * dot     or, degree-scaled,
+//   Z = (alpha_i / sqrt(dhat_i)) * (beta_j * dot).
+#include "launch.cuh"
+
+namespace bigcn {
+
+__device__ unsigned int g_tc_timeouts;
+
+namespace {
+
+constexpr int kTcThreads = 256;
+constexpr int kTcM = 128;
+constexpr int kTcKBytes = 128;
+constexpr int kTcStages = 2;
+constexpr uint32_t kWaitLimit = 1u << 20;
+
+__device__ __forceinline__ uint32_t smem_addr(const void *p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+// Four signs (bits 0..3 of n) as four FP8 E4M3 bytes, +1 for a set bit:
+// n * (1 + 2^7 + 2^14 + 2^21) moves bit i of n to bit 8i (the other partial
+// products never land on a multiple of 8 below 32), and flipping the sign bit
+// of -1.0 (0xB8) there gives +1.0 (0x38).
+__device__ __forceinline__ uint32_t signs4_to_e4m3(uint32_t n) {
+    const uint32_t spread = (n * 0x00204081u) & 0x01010101u;
+    return 0xB8B8B8B8u ^ (spread << 7);
+}
+
+// Byte offset of 16-byte chunk c of row r in a 128B-swizzled K-major tile.
+__device__ __forceinline__ uint32_t sw128_offset(int r, int c) {
+    return uint32_t((r >> 3) * 1024 + (r & 7) * 128 + ((c ^ (r & 7)) << 4));
+}
+
+// Shared-memory matrix descriptor: K-major, 128B swizzle, 8-row groups 1024 B
+// apart (stride byte offset), descriptor version 1.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+    uint64_t d = uint64_t((saddr >> 4) & 0x3FFFu);
+    d |= uint64_t(1) << 16;                     // leading byte offset (unused here)
+    d |= uint64_t(1024 >> 4) << 32;             // stride byte offset
+    d |= uint64_t(1) << 46;                     // version
+    d |= uint64_t(2) << 61;                     // swizzle: 128B
+    return d;
+}
+
+// Instruction descriptor: E4M3 x E4M3 -> F32, both K-major, M = 128, N = n.
+__host__ __device__ constexpr uint32_t e4m3_idesc(int n) {
+    return (1u << 4) | (uint32_t(n >> 3) << 17) | (uint32_t(kTcM >> 4) << 24);
+}
+
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+    for (uint32_t it = 0; it < kWaitLimit; ++it) {
+        uint32_t done;
+        asm volatile(
+            "{\n.reg .pred p;\n"
+            "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+            "selp.u32 %0, 1, 0, p;\n}"
+            : "=r"(done)
+            : "r"(bar), "r"(parity)
+            : "memory");
+        if (done) return true;
+    }
+    return false;
+}
+
+__device__ __forceinline__ void mma_e4m3(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
+                                         uint32_t accumulate) {
+    asm volatile(
+        "{\n.reg .pred p;\n"
+        "setp.ne.b32 p, %4, 0;\n"
+        "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n}" ::"r"(d_tmem),
+        "l"(a), "l"(b), "r"(idesc), "r"(accumulate));
+}
+
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]),
+          "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]),
+          "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+template <int NT, bool kDeg>
+__global__ void __launch_bounds__(kTcThreads)
+xnor_gemm_tc_kernel(const uint64_t *__restrict__ A, const float *__restrict__ alpha, int64_t N,
+                    const uint64_t *__restrict__ B, const float *__restrict__ beta, int F, int K,
+                    int words, float *__restrict__ Z, int64_t ldz, int32_t *__restrict__ dots,
+                    const int64_t *__restrict__ rowptr) {
+    constexpr int kStageA = kTcM * kTcKBytes;
+    constexpr int kStageB = NT * kTcKBytes;
+    constexpr int kStage = kStageA + kStageB;
+    constexpr int kRowsPerPass = kTcThreads / 8;         // 32: thread t owns chunk t & 7
+    constexpr int kAChunks = kTcM / kRowsPerPass;         // 4 rows of A per thread
+    constexpr int kBChunks = NT / kRowsPerPass;           // 2, 4 or 8 rows of B per thread
+    extern __shared__ unsigned char smem_raw[];
+    __shared__ __align__(8) uint64_t bars[kTcStages];
+    __shared__ uint32_t tmem_base;
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int64_t m0 = int64_t(blockIdx.x) * kTcM;
+    const int n0 = blockIdx.y * NT;
+    const uint32_t raw = smem_addr(smem_raw);
+    const uint32_t tile0 = (raw + 1023u) & ~1023u;          // 1024-byte aligned stages
+    unsigned char *tiles = smem_raw + (tile0 - raw);
+
+    if (warp == 0) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         smem_addr(&tmem_base)),
+                     "r"(NT));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    if (tid == 0) {
+        for (int s = 0; s < kTcStages; ++s)
+            asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_addr(&bars[s])));
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const uint32_t tmem = tmem_base;
+    grid_dependency_wait();     // the packed operands come from earlier kernels
+
+    // Thread t expands chunk c = t & 7 (16 signs) of rows (t >> 3) + 32 q.
+    const int c = tid & 7, r0 = tid >> 3;
+    const int KB = (K + kTcKBytes - 1) / kTcKBytes;
+    uint64_t wa[kAChunks], wb[kBChunks];
+    auto load_words = [&](int kb) {
+        const int k0 = kb * kTcKBytes + c * 16;
+#pragma unroll
+        for (int q = 0; q < kAChunks; ++q) {
+            const int64_t row = m0 + r0 + kRowsPerPass * q;
+            wa[q] = (row < N && k0 < K) ? __ldg(A + row * words + (k0 >> 6)) : 0ull;
+        }
+#pragma unroll
+        for (int q = 0; q < kBChunks; ++q) {
+            const int col = n0 + r0 + kRowsPerPass * q;
+            wb[q] = (col < F && k0 < K) ? __ldg(B + int64_t(col) * words + (k0 >> 6)) : 0ull;
+        }
+    };
+    // 16 signs from bit `sh` of w as E4M3 bytes, zero past `valid` signs.
+    auto expand = [&](uint64_t w, int sh, int valid) {
+        const uint32_t bits = uint32_t(w >> sh);
+        uint4 v = make_uint4(signs4_to_e4m3(bits & 15u), signs4_to_e4m3((bits >> 4) & 15u),
+                             signs4_to_e4m3((bits >> 8) & 15u), signs4_to_e4m3((bits >> 12) & 15u));
+        if (valid < 16) {
+            uint32_t *e = reinterpret_cast<uint32_t *>(&v);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const int keep = valid - 4 * q;
+                if (keep <= 0) e[q] = 0u;
+                else if (keep < 4) e[q] &= (1u << (8 * keep)) - 1u;
+            }
+        }
+        return v;
+    };
+
+    constexpr uint32_t idesc = e4m3_idesc(NT);
+    bool ok = true;
+    int committed = -1;          // last k-block whose MMAs were committed
+    load_words(0);
+    for (int kb = 0; kb < KB; ++kb) {
+        const int s = kb & 1;
+        if (kb >= kTcStages) {
+            const bool done = mbar_wait(smem_addr(&bars[s]), uint32_t((kb - kTcStages) >> 1) & 1u);
+            if (!__syncthreads_and(done)) {
+                ok = false;
+                break;
+            }
+        }
+        unsigned char *sa = tiles + s * kStage;
+        unsigned char *sb = sa + kStageA;
+        const int k0 = kb * kTcKBytes + c * 16;
+        const int sh = k0 & 63;
+        const int valid = min(max(K - k0, 0), 16);
+#pragma unroll
+        for (int q = 0; q < kAChunks; ++q) {
+            const int r = r0 + kRowsPerPass * q;
+            const bool live = m0 + r < N && valid > 0;
+            *reinterpret_cast<uint4 *>(sa + sw128_offset(r, c)) =
+                live ? expand(wa[q], sh, valid) : make_uint4(0u, 0u, 0u, 0u);
+        }
+#pragma unroll
+        for (int q = 0; q < kBChunks; ++q) {
+            const int r = r0 + kRowsPerPass * q;
+            *reinterpret_cast<uint4 *>(sb + sw128_offset(r, c)) = expand(wb[q], sh, 16);
+        }
+        if (kb + 1 < KB) load_words(kb + 1);      // in flight across the barrier and MMAs
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        __syncthreads();
+        if (tid == 0) {
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            const uint32_t a0 = smem_addr(sa), b0 = smem_addr(sb);
+#pragma unroll
+            for (int k = 0; k < kTcKBytes / 32; ++k)
+                mma_e4m3(tmem, sw128_desc(a0 + 32u * k), sw128_desc(b0 + 32u * k), idesc,
+                         (kb > 0 || k > 0) ? 1u : 0u);
+            asm volatile(
+                "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                    smem_addr(&bars[s]))
+                : "memory");
+        }
+        committed = kb;
+    }
+    // Every MMA issued is done once the last commit has arrived (waited for
+    // even after a failed wait, so that no MMA is in flight at deallocation).
+    bool done = true;
+    if (committed >= 0)
+        done = mbar_wait(smem_addr(&bars[committed & 1]), uint32_t(committed >> 1) & 1u);
+    ok = __syncthreads_and(ok && done) != 0;
+    if (!ok && tid == 0) atomicAdd(&g_tc_timeouts, 1u);
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+
+    // Epilogue: warp w reads tensor-memory lanes 32 (w % 4) .. (its rows),
+    // warps w and w + 4 take alternate 16-column slices.
+    // Rows of Z / dots take 16-byte stores when their starts are 16-byte aligned.
+    const bool vec_z = (ldz & 3) == 0 && (reinterpret_cast<uintptr_t>(Z) & 15) == 0;
+    const bool vec_d = (F & 3) == 0 && (reinterpret_cast<uintptr_t>(dots) & 15) == 0;
+    if (ok) {
+        const int quad = warp & 3;
+        const int64_t row = m0 + 32 * quad + lane;
+        float ai = 0.0f;
+        if (row < N) {
+            ai = __ldg(alpha + row);
+            if (kDeg) ai *= inv_sqrt_degree(__ldg(rowptr + row + 1) - __ldg(rowptr + row));
+        }
+        const uint32_t taddr = tmem + (uint32_t(32 * quad) << 16);
+#pragma unroll 1
+        for (int c0 = 16 * (warp >> 2); c0 < NT; c0 += 32) {
+            uint32_t acc[16];
+            tmem_ld16(taddr + uint32_t(c0), acc);
+            if (row >= N) continue;
+            const int col0 = n0 + c0;
+            float z[16];
+            int d[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+                const int col = col0 + j < F ? col0 + j : F - 1;
+                d[j] = __float2int_rn(__uint_as_float(acc[j]));
+                const float bj = __ldg(beta + col);
+                z[j] = kDeg ? ai * (bj * float(d[j])) : (ai * bj) * float(d[j]);
+            }
+            float *zr = Z + row * ldz + col0;
+            int32_t *dr = dots != nullptr ? dots + row * F + col0 : nullptr;
+            if (vec_z && col0 + 16 <= F) {
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+                    reinterpret_cast<float4 *>(zr)[q] =
+                        make_float4(z[4 * q], z[4 * q + 1], z[4 * q + 2], z[4 * q + 3]);
+            } else {
+#pragma unroll
+                for (int j = 0; j < 16; ++j)
+                    if (col0 + j < F) zr[j] = z[j];
+            }
+            if (dr != nullptr) {
+                if (vec_d && col0 + 16 <= F) {
+#pragma unroll
+                    for (int q = 0; q < 4; ++q)
+                        reinterpret_cast<int4 *>(dr)[q] =
+                            make_int4(d[4 * q], d[4 * q + 1], d[4 * q + 2], d[4 * q + 3]);
+                } else {
+#pragma unroll
+                    for (int j = 0; j < 16; ++j)
+                        if (col0 + j < F) dr[j] = d[j];
+                }
+            }
+        }
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    if (warp == 0)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(NT));
+}
+
+template <int NT>
+size_t tc_smem() {
+    return 1024 + size_t(kTcStages) * (kTcM * kTcKBytes + NT * kTcKBytes);
+}
+
+template <int NT, bool kDeg>
+void launch_nt(const GemmArgs &g, cudaStream_t s, bool pdl) {
+    const size_t smem = tc_smem<NT>();
+    cudaFuncSetAttribute(xnor_gemm_tc_kernel<NT, kDeg>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         int(smem));
+    const dim3 grid(unsigned((g.N + kTcM - 1) / kTcM), unsigned((g.F + NT - 1) / NT));
+    launch_kernel(xnor_gemm_tc_kernel<NT, kDeg>, grid, dim3(kTcThreads), smem, s, pdl,
+                  dim3(1, 1, 1), g.A, g.alpha, g.N, g.B, g.beta, g.F, g.K, g.words, g.Z, g.ldz,
+                  g.dots, g.rowptr);
+}
+
+template <bool kDeg>
+void launch_deg(const GemmArgs &g, cudaStream_t s, bool pdl) {
+    if (g.F <= 64) launch_nt<64, kDeg>(g, s, pdl);
+    else if (g.F <= 128) launch_nt<128, kDeg>(g, s, pdl);
+    else launch_nt<256, kDeg>(g, s, pdl);
+}
+
+}  // namespace
+
+bool xnor_gemm_tc_supported(int64_t N, int K, int F, const DeviceInfo &dev) {
+    // Enough 128-row tiles to give every SM one, and shared memory for two stages.
+    return K >= 128 && F >= 32 && (N + kTcM - 1) / kTcM >= dev.sm_count &&
+           size_t(dev.max_smem_optin) >= tc_smem<256>();
+}
+
+void launch_xnor_gemm_tc(const GemmArgs &g, const DeviceInfo &, cudaStream_t stream, bool pdl) {
+    if (g.N == 0) return;
+    if (g.rowptr != nullptr) launch_deg<true>(g, stream, pdl);
+    else launch_deg<false>(g, stream, pdl);
+}
+
+}  // namespace bigcn
+
+extern "C" int32_t bigcn_device_timeouts(void) {
+    unsigned int n = 0;
+    const unsigned int zero = 0;
+    if (cudaDeviceSynchronize() != cudaSuccess ||
+        cudaMemcpyFromSymbol(&n, bigcn::g_tc_timeouts, sizeof(n)) != cudaSuccess ||
+        cudaMemcpyToSymbol(bigcn::g_tc_timeouts, &zero, sizeof(zero)) != cudaSuccess) {
+        cudaGetLastError();
+        return -1;
+    }
+    return int32_t(n);
+}

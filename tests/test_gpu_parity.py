@@ -392,3 +392,44 @@ def test_forward_2layer_heavy_rows(cuda_device, Fh, Fo):
     assert_close(H1, ref1["H"], "H1 with heavy rows")
     ref2 = oracle.layer_forward(H1.cpu().numpy(), W2, rowptr, colidx)
     assert_close(out, ref2["H"], "logits with heavy rows")
+
+
+# ------------------------------------------- tensor-core path of step 4 ------
+TC_CASES = [(128, 32, 128), (129, 33, 129), (300, 64, 200), (1000, 128, 1000),
+            (257, 256, 8192), (77, 257, 300), (512, 100, 3703), (1, 40, 602), (384, 41, 64 * 40)]
+
+
+@pytest.mark.parametrize("N,F,K", TC_CASES)
+def test_xnor_gemm_tensor_core_path(cuda_device, N, F, K):
+    """K >= 128 and F >= 32 take the tcgen05 FP8 path: dots must still be exact."""
+    g = rng(N + 7 * F + 13 * K)
+    SF, SB = random_signs(g, N, K), random_signs(g, F, K)
+    if N >= 2 and F >= 2:
+        SF[0] = SB[0]            # dot = +K
+        SF[1] = -SB[1]           # dot = -K
+    alpha = g.uniform(0.1, 2.0, N).astype(np.float32)
+    beta = g.uniform(0.001, 0.1, F).astype(np.float32)
+    Z, dots = B.xnor_gemm(to_dev(oracle.pack(SF)), to_dev(alpha), to_dev(oracle.pack(SB)),
+                          to_dev(beta), K, with_dots=True)
+    ref_dot = oracle.binary_dot(SF, SB)
+    got = dots.cpu().numpy()
+    assert np.array_equal(got, ref_dot), f"{int((got != ref_dot).sum())} dots differ"
+    assert_close(Z, oracle.zeta(ref_dot, alpha.astype(np.float64), beta.astype(np.float64)), "Z")
+    assert B.device_timeouts() == 0
+
+
+def test_xnor_gemm_tensor_core_degree_scaled(cuda_device):
+    N, F, K = 700, 128, 602
+    g = rng(99)
+    SF, SB = random_signs(g, N, K), random_signs(g, F, K)
+    alpha = g.uniform(0.1, 2.0, N).astype(np.float32)
+    beta = g.uniform(0.001, 0.1, F).astype(np.float32)
+    rowptr, _ = inputs.random_graph(N, 6.0, seed=3, hub_degree=200)
+    Z = torch.empty((N, F), device=cuda_device)
+    B.bigcn_xnor_gemm_degscaled(to_dev(oracle.pack(SF)), to_dev(alpha), to_dev(oracle.pack(SB)),
+                                to_dev(beta), K, to_dev(rowptr), Z)
+    dinv = 1.0 / np.sqrt(oracle.degree(rowptr))
+    ref = oracle.zeta(oracle.binary_dot(SF, SB), alpha.astype(np.float64),
+                      beta.astype(np.float64)) * dinv[:, None]
+    assert_close(Z, ref, "Z'")
+    assert B.device_timeouts() == 0
