@@ -164,7 +164,7 @@ extern "C" bigcn_status bigcn_forward_2layer(
         launch_front(fr, dev, s, true);
         mark();
     } else {
-        launch_pack_rows(X, N, K, ldx, scale, shift, bits1, words1, alpha1, dev, s, true);
+        launch_pack_rows(X, N, K, ldx, scale, shift, bits1, words1, alpha1, dev, s, true, false);
         mark();
         GemmArgs g1{bits1, alpha1, N, wbits1, beta1, Fh, K, words1, Z1, Fh, nullptr, rowptr};
         launch_xnor_gemm(g1, dev, s, true);
@@ -182,7 +182,8 @@ extern "C" bigcn_status bigcn_forward_2layer(
         SpmmArgs a1{rowptr, colidx, N, nnz, Z1, Fh, Fh, H1w, ldh, true, false};
         launch_spmm_norm(a1, dev, s, true);
         mark();
-        launch_pack_rows(H1w, N, Fh, ldh, nullptr, nullptr, bits2, words2, alpha2, dev, s, true);
+        launch_pack_rows(H1w, N, Fh, ldh, nullptr, nullptr, bits2, words2, alpha2, dev, s, true,
+                         true);
         mark();
         GemmArgs g2{bits2, alpha2, N, wbits2, beta2, Fo, Fh, words2, Z2, ldz2, nullptr, rowptr};
         launch_xnor_gemm(g2, dev, s, true);

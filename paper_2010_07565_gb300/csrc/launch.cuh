@@ -12,10 +12,13 @@
 namespace bigcn {
 
 // Steps 1+2: centre, sign-pack rows, per-node scale (Sec. 6.2, Eqs. 7-8).
-// `pdl`: launch with programmatic serialization (see grid_dependency_wait).
+// `pdl`: launch with programmatic serialization (see grid_dependency_wait);
+// `x_upstream`: X is written by an earlier kernel of the chain (the kernel
+// then waits before reading it; otherwise it waits only before it exits).
 void launch_pack_rows(const float *X, int64_t N, int K, int64_t ldx, const float *scale,
                       const float *shift, uint64_t *bits, int words, float *alpha,
-                      const DeviceInfo &dev, cudaStream_t stream, bool pdl = false);
+                      const DeviceInfo &dev, cudaStream_t stream, bool pdl = false,
+                      bool x_upstream = true);
 
 // Step 3: sign-pack weight columns, per-column scale (Eqs. 3-4).
 void launch_pack_weights(const float *Wt, int K, int F, int64_t ldw, uint64_t *bits,

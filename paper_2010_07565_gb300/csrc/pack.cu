@@ -76,12 +76,12 @@ __device__ __forceinline__ float pack_row_chunks(const float *__restrict__ x, in
 
 // Whole rows per warp: every warp walks rows on its own (persistent grid,
 // no block barrier), which keeps the kernel small enough for full occupancy.
-template <bool kAffine>
+template <bool kAffine, bool kUpstream>
 __global__ void __launch_bounds__(kPackThreads)
 pack_rows_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
                  const float *__restrict__ scale, const float *__restrict__ shift,
                  uint32_t *__restrict__ bits32, int64_t ld32, float *__restrict__ alpha) {
-    grid_dependency_wait();     // X may be the output of the previous kernel
+    if (kUpstream) grid_dependency_wait();      // X is the previous kernel's output
     const int lane = threadIdx.x & 31;
     const int64_t nwarps = int64_t(gridDim.x) * kPackWarps;
     for (int64_t row = int64_t(blockIdx.x) * kPackWarps + (threadIdx.x >> 5); row < N;
@@ -90,18 +90,21 @@ pack_rows_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
             pack_row_chunks<kAffine>(X + row * ldx, K, scale, shift, bits32 + row * ld32, ld32, 0, 1);
         if (lane == 0) alpha[row] = l1 / float(K);
     }
+    // Otherwise wait only now: finishing after the predecessor keeps the
+    // chain's completion order for the kernels that follow.
+    if (!kUpstream) grid_dependency_wait();
 }
 
 // Rows shared by G > 1 warps (few, long rows): block b takes row groups
 // b, b + gridDim.x, ...; the G partial sums meet in shared memory.
 template <bool kAffine>
-__global__ void __launch_bounds__(kPackThreads)
+__global__ void __launch_bounds__(kPackThreads, 6)
 pack_rows_split_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
                        const float *__restrict__ scale, const float *__restrict__ shift,
                        uint32_t *__restrict__ bits32, int64_t ld32, float *__restrict__ alpha,
-                       int G) {
+                       int G, bool x_upstream) {
     __shared__ float part[kPackWarps];
-    grid_dependency_wait();
+    if (x_upstream) grid_dependency_wait();
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int sub = warp & (G - 1);
     const int rows_per_block = kPackWarps / G;
@@ -119,6 +122,7 @@ pack_rows_split_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ld
         }
         __syncthreads();   // part[] is rewritten by the next group
     }
+    if (!x_upstream) grid_dependency_wait();
 }
 
 constexpr int kWCols = 32;
@@ -182,7 +186,7 @@ pack_weights_kernel(WeightPack a, WeightPack b) {
 
 void launch_pack_rows(const float *X, int64_t N, int K, int64_t ldx, const float *scale,
                       const float *shift, uint64_t *bits, int words, float *alpha,
-                      const DeviceInfo &dev, cudaStream_t stream, bool pdl) {
+                      const DeviceInfo &dev, cudaStream_t stream, bool pdl, bool x_upstream) {
     if (N == 0) return;
     // Split rows over up to 8 warps while the grid is short of one full wave
     // of warps, as long as every warp keeps at least one 8-chunk batch.
@@ -198,19 +202,21 @@ void launch_pack_rows(const float *X, int64_t N, int K, int64_t ldx, const float
     const int64_t ld32 = int64_t(words) * 2;
     const float *no = nullptr;
     if (G == 1) {
-        if (scale)
-            launch_kernel(pack_rows_kernel<true>, grid, block, 0, stream, pdl, one, X, N, K, ldx,
-                          scale, shift, b32, ld32, alpha);
-        else
-            launch_kernel(pack_rows_kernel<false>, grid, block, 0, stream, pdl, one, X, N, K, ldx,
-                          no, no, b32, ld32, alpha);
+        auto run = [&](auto kernel, const float *sc, const float *sh) {
+            launch_kernel(kernel, grid, block, 0, stream, pdl, one, X, N, K, ldx, sc, sh, b32, ld32,
+                          alpha);
+        };
+        if (scale && x_upstream) run(pack_rows_kernel<true, true>, scale, shift);
+        else if (scale) run(pack_rows_kernel<true, false>, scale, shift);
+        else if (x_upstream) run(pack_rows_kernel<false, true>, no, no);
+        else run(pack_rows_kernel<false, false>, no, no);
     } else {
         if (scale)
             launch_kernel(pack_rows_split_kernel<true>, grid, block, 0, stream, pdl, one, X, N, K,
-                          ldx, scale, shift, b32, ld32, alpha, G);
+                          ldx, scale, shift, b32, ld32, alpha, G, x_upstream);
         else
             launch_kernel(pack_rows_split_kernel<false>, grid, block, 0, stream, pdl, one, X, N, K,
-                          ldx, no, no, b32, ld32, alpha, G);
+                          ldx, no, no, b32, ld32, alpha, G, x_upstream);
     }
 }
 
