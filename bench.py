@@ -124,7 +124,9 @@ def kernel_bitops(w, name):
             "L2.xnor_gemm": float(N) * Fh * Fo}.get(name, 0.0)
 
 
-KERNEL_FILES = {"pack_weights(W1,W2)": "pack.cu", "L1.pack_rows": "pack.cu",
+KERNEL_FILES = {"pack_rows": "pack.cu", "pack_weights": "pack.cu", "xnor_gemm": "xnor_gemm_tc.cu",
+                "spmm": "spmm.cu",
+                "pack_weights(W1,W2)": "pack.cu", "L1.pack_rows": "pack.cu",
                 "L1.pack_rows+L1.xnor_gemm": "front.cu",
                 "L2.pack_rows": "pack.cu", "L1.xnor_gemm": "xnor_gemm.cu",
                 "L2.xnor_gemm": "xnor_gemm.cu", "L1.spmm": "spmm.cu", "L2.spmm": "spmm.cu",
