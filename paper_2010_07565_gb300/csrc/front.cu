@@ -15,12 +15,13 @@
 // block's HBM-bound phase A with another's POPC-bound phase B.
 //
 // The packed weight columns and beta come from the weight-packing kernel
-// that runs first; the kernel is used when both packed tiles fit in shared
-// memory and rows are at most 2048 features (front_supported): a warp streams
-// whole rows one batch after another, so with long rows and few rows per SM
-// the separate row-packing kernel, which shares long rows between warps,
-// keeps more bytes in flight.
+// that runs first. This whole-row kernel is used when there are enough rows
+// to give every warp its own, both packed tiles fit in shared memory and rows
+// are at most 2048 features; with fewer rows the split front below shares
+// each row between several warps, as the row-packing kernel does, so that
+// more of the GPU's warps keep loads in flight (front_supported picks).
 #include "launch.cuh"
+#include "pack_row.cuh"
 
 namespace bigcn {
 namespace {
@@ -158,9 +159,130 @@ int front_rows(int64_t N, const DeviceInfo &dev) {
     return 16;
 }
 
+// ---------------------------------------------------------------------------
+// Split front, for layers with few rows (fewer than one warp per row would
+// leave most of the GPU idle, e.g. a few thousand long rows): each block
+// takes R = 8 / G rows at a time, G warps per row (the row-packing kernel's
+// split, same chunk order and the same alpha summation), and writes the
+// packed rows to shared memory. The block then computes their products: the
+// 32 G threads of a row take P lanes per output column (P a power of two,
+// words w = t mod P, t mod P + P, ... for lane t of the column), add their
+// mismatch counts with shuffles and write Z' as above. The packed weight
+// columns are staged in shared memory once per block, after the dependency
+// wait, which comes only after the block's first rows have been streamed.
+
+size_t split_smem(int F, int words) {
+    return (size_t(F) + size_t(kFrontWarps)) * size_t(words | 1) * 8;
+}
+
+// Warps per row: the row-packing kernel's policy (split while the grid is
+// short of one wave of warps and every warp keeps an 8-chunk batch).
+int split_warps(int64_t N, int K, const DeviceInfo &dev) {
+    const int nchunks = (K + 31) / 32;
+    const int64_t full_wave = int64_t(dev.sm_count) * 64;
+    int G = 1;
+    while (G < kFrontWarps && N * G < full_wave && nchunks >= 2 * G * 8) G *= 2;
+    return G;
+}
+
+template <bool kAffine>
+__global__ void __launch_bounds__(kFrontThreads, 3)
+front_split_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
+                   const float *__restrict__ scale, const float *__restrict__ shift,
+                   const uint64_t *__restrict__ wbits, const float *__restrict__ beta, int F,
+                   int words, const int64_t *__restrict__ rowptr, float *__restrict__ Z,
+                   int64_t ldz, int G, int P) {
+    extern __shared__ __align__(16) unsigned char smem[];
+    __shared__ float part[kFrontWarps];
+    const int pitch = words | 1;
+    uint64_t *Ws = reinterpret_cast<uint64_t *>(smem);      // F x pitch packed columns
+    uint64_t *As = Ws + size_t(F) * pitch;                   // R x pitch packed rows
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int R = kFrontWarps / G;
+    const int T = 32 * G;                    // threads per row in the product
+    const int rr = tid / T, tt = tid % T, sub = tt % P;
+    const int cstep = T / P;                 // columns per pass
+    const int passes = (F + cstep - 1) / cstep;
+    bool staged = false;
+    for (int64_t group = blockIdx.x; group * R < N; group += gridDim.x) {
+        const int64_t row = group * R + warp / G;
+        uint32_t *a32 = reinterpret_cast<uint32_t *>(As + size_t(warp / G) * pitch);
+        const float l1 = (row < N) ? pack_row_chunks<kAffine>(X + row * ldx, K, scale, shift, a32,
+                                                              2 * words, warp % G, G)
+                                   : 0.0f;
+        if (lane == 0) part[warp] = l1;
+        if (!staged) {
+            grid_dependency_wait();     // the packed weight columns come from the previous kernel
+            const int n = F * words;
+            for (int q0 = tid; q0 < n; q0 += 8 * kFrontThreads) {
+                uint64_t v[8];
+#pragma unroll
+                for (int u = 0; u < 8; ++u) {
+                    const int q = q0 + u * kFrontThreads;
+                    if (q < n) v[u] = __ldg(wbits + q);
+                }
+#pragma unroll
+                for (int u = 0; u < 8; ++u) {
+                    const int q = q0 + u * kFrontThreads;
+                    if (q < n) Ws[(q / words) * pitch + (q % words)] = v[u];
+                }
+            }
+            staged = true;
+        }
+        __syncthreads();
+        const int64_t row2 = group * R + rr;
+        if (row2 < N) {                      // uniform over each warp (T is a multiple of 32)
+            float t = 0.0f;
+            for (int g = 0; g < G; ++g) t += part[rr * G + g];
+            const float ai = (t / float(K)) *
+                             inv_sqrt_degree(__ldg(rowptr + row2 + 1) - __ldg(rowptr + row2));
+            const uint64_t *a = As + size_t(rr) * pitch;
+            for (int j = 0; j < passes; ++j) {
+                const int c = tt / P + j * cstep;
+                int mism = 0;
+                if (c < F)
+                    for (int w = sub; w < words; w += P) mism += __popcll(a[w] ^ Ws[c * pitch + w]);
+                for (int o = 1; o < P; o <<= 1) mism += __shfl_xor_sync(kFullMask, mism, o);
+                if (sub == 0 && c < F)
+                    Z[row2 * ldz + c] = ai * (__ldg(beta + c) * float(K - 2 * mism));
+            }
+        }
+        __syncthreads();                     // As and part are rewritten by the next rows
+    }
+    if (!staged) grid_dependency_wait();
+}
+
+bool split_supported(int64_t N, int K, int F, const DeviceInfo &dev) {
+    return F >= 1 && F <= 128 && split_warps(N, K, dev) > 1 &&
+           split_smem(F, (K + 63) / 64) <= kFrontMaxSmem / 2;
+}
+
+void launch_split(const FrontArgs &a, const DeviceInfo &dev, cudaStream_t s, bool pdl) {
+    const int G = split_warps(a.N, a.K, dev);
+    int fp = 1;
+    while (fp < a.F) fp *= 2;
+    int P = 32 * G / fp;
+    if (P < 1) P = 1;
+    if (P > 32) P = 32;
+    const size_t smem = split_smem(a.F, a.words);
+    auto kernel = a.scale != nullptr ? front_split_kernel<true> : front_split_kernel<false>;
+    cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, kFrontThreads, smem) !=
+            cudaSuccess ||
+        per_sm < 1)
+        per_sm = 1;
+    const int64_t groups = (a.N + kFrontWarps / G - 1) / (kFrontWarps / G);
+    const int64_t resident = int64_t(per_sm) * dev.sm_count;
+    launch_kernel(kernel, dim3(unsigned(groups < resident ? groups : resident)),
+                  dim3(kFrontThreads), smem, s, pdl, dim3(1, 1, 1), a.X, a.N, a.K, a.ldx, a.scale,
+                  a.shift, a.wbits, a.beta, a.F, a.words, a.rowptr, a.Z, a.ldz, G, P);
+}
+
 }  // namespace
 
 bool front_supported(int64_t N, int K, int F, const DeviceInfo &dev) {
+    if (split_supported(N, K, F, dev)) return true;
     if (F < 1 || F > 128 || K < 1 || K > kFrontMaxK) return false;
     const size_t smem = front_smem(front_rows(N, dev), F, (K + 63) / 64);
     return smem <= kFrontMaxSmem && smem <= size_t(dev.max_smem_optin);
@@ -168,6 +290,10 @@ bool front_supported(int64_t N, int K, int F, const DeviceInfo &dev) {
 
 void launch_front(const FrontArgs &a, const DeviceInfo &dev, cudaStream_t s, bool pdl) {
     if (a.N == 0) return;
+    if (split_supported(a.N, a.K, a.F, dev)) {
+        launch_split(a, dev, s, pdl);
+        return;
+    }
     const int BM = front_rows(a.N, dev);
     const size_t smem = front_smem(BM, a.F, a.words);
     if (BM == 64) launch_ri<4>(a, BM, smem, s, pdl);

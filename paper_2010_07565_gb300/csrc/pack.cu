@@ -27,6 +27,7 @@
 #include <cooperative_groups.h>
 
 #include "launch.cuh"
+#include "pack_row.cuh"
 
 namespace bigcn {
 namespace {
@@ -35,44 +36,7 @@ namespace cg = cooperative_groups;
 
 constexpr int kPackThreads = 256;
 constexpr int kPackWarps = kPackThreads / 32;
-constexpr int kPackUnroll = 8;
 constexpr int kPackBlocksPerSM = 8;   // resident blocks the persistent grids assume
-
-// Packs chunks sub, sub + G, ... of row `row` (lane l of chunk c owns
-// feature 32c + l) and returns this warp's sum of |y| (all lanes).
-template <bool kAffine>
-__device__ __forceinline__ float pack_row_chunks(const float *__restrict__ x, int K,
-                                                 const float *__restrict__ scale,
-                                                 const float *__restrict__ shift,
-                                                 uint32_t *__restrict__ out, int64_t ld32, int sub,
-                                                 int G) {
-    const int lane = threadIdx.x & 31;
-    const int nchunks = (K + 31) >> 5;          // 32-bit half-words that carry signs
-    float l1 = 0.0f;
-    for (int m0 = sub; m0 < nchunks; m0 += G * kPackUnroll) {
-        float v[kPackUnroll];
-#pragma unroll
-        for (int u = 0; u < kPackUnroll; ++u) {
-            const int k = (m0 + u * G) * 32 + lane;
-            v[u] = (k < K) ? __ldcs(x + k) : 0.0f;
-        }
-#pragma unroll
-        for (int u = 0; u < kPackUnroll; ++u) {
-            const int c = m0 + u * G;
-            const int k = c * 32 + lane;
-            const bool in = k < K;
-            float y = v[u];
-            if (kAffine && in) y = __fmaf_rn(y, __ldg(scale + k), __ldg(shift + k));
-            const unsigned m = __ballot_sync(kFullMask, in && y >= 0.0f);
-            if (c < nchunks && lane == 0) out[c] = m;
-            l1 += in ? fabsf(y) : 0.0f;
-        }
-    }
-    // Pad half-words past the last one that carries signs are zero.
-    if (sub == 0)
-        for (int64_t q = nchunks + lane; q < ld32; q += 32) out[q] = 0u;
-    return warp_sum(l1);
-}
 
 // Whole rows per warp: every warp walks rows on its own (persistent grid,
 // no block barrier), which keeps the kernel small enough for full occupancy.
@@ -98,7 +62,7 @@ pack_rows_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
 // Rows shared by G > 1 warps (few, long rows): block b takes row groups
 // b, b + gridDim.x, ...; the G partial sums meet in shared memory.
 template <bool kAffine>
-__global__ void __launch_bounds__(kPackThreads, 6)
+__global__ void __launch_bounds__(kPackThreads, 5)
 pack_rows_split_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
                        const float *__restrict__ scale, const float *__restrict__ shift,
                        uint32_t *__restrict__ bits32, int64_t ld32, float *__restrict__ alpha,

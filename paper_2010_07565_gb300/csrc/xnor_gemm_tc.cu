@@ -27,6 +27,7 @@
 // tcgen05.ld, converts the exact fp32 dots to integers and writes
 //   Z = (alpha_i * beta_j) * dot     or, degree-scaled,
 //   Z = (alpha_i / sqrt(dhat_i)) * (beta_j * dot).
+#include "async.cuh"
 #include "launch.cuh"
 
 namespace bigcn {
@@ -39,11 +40,6 @@ constexpr int kTcThreads = 256;
 constexpr int kTcM = 128;
 constexpr int kTcKBytes = 128;
 constexpr int kTcStages = 2;
-constexpr uint32_t kWaitLimit = 1u << 20;
-
-__device__ __forceinline__ uint32_t smem_addr(const void *p) {
-    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
 
 // Four signs (bits 0..3 of n) as four FP8 E4M3 bytes, +1 for a set bit:
 // n * (1 + 2^7 + 2^14 + 2^21) moves bit i of n to bit 8i (the other partial
@@ -73,21 +69,6 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
 // Instruction descriptor: E4M3 x E4M3 -> F32, both K-major, M = 128, N = n.
 __host__ __device__ constexpr uint32_t e4m3_idesc(int n) {
     return (1u << 4) | (uint32_t(n >> 3) << 17) | (uint32_t(kTcM >> 4) << 24);
-}
-
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
-    for (uint32_t it = 0; it < kWaitLimit; ++it) {
-        uint32_t done;
-        asm volatile(
-            "{\n.reg .pred p;\n"
-            "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
-            "selp.u32 %0, 1, 0, p;\n}"
-            : "=r"(done)
-            : "r"(bar), "r"(parity)
-            : "memory");
-        if (done) return true;
-    }
-    return false;
 }
 
 __device__ __forceinline__ void mma_e4m3(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
@@ -140,9 +121,8 @@ xnor_gemm_tc_kernel(const uint64_t *__restrict__ A, const float *__restrict__ al
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
     }
     if (tid == 0) {
-        for (int s = 0; s < kTcStages; ++s)
-            asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_addr(&bars[s])));
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        for (int s = 0; s < kTcStages; ++s) mbar_init(smem_addr(&bars[s]), 1);
+        mbar_fence_init();
     }
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();

@@ -314,6 +314,42 @@ def test_forward_2layer_matches_oracle(cuda_device, N, K, Fh, Fo, deg, hub):
     assert torch.equal(out, out2)
 
 
+# The layer-1 front streams whole rows of X into shared memory with bulk
+# copies of each row's 16-byte-aligned interior; these cases move the row
+# starts off that alignment (odd row strides, a base 4 bytes past a 16-byte
+# boundary), make rows too short to have an interior, and give every CTA
+# many more rows than its ring has stages.
+@pytest.mark.parametrize("N,K,ldx,offset,Fh,centred", [
+    (333, 1, 1, 0, 8, True),          # one feature: no interior at all
+    (333, 3, 5, 1, 8, False),         # rows shorter than 16 bytes, odd stride
+    (200, 9, 9, 1, 33, True),         # interior of at most one 16-byte unit
+    (700, 3703, 3703, 0, 64, True),   # Citeseer-shaped rows (stride 14812 bytes)
+    (700, 3703, 3705, 3, 64, True),   # same rows, odd stride, base 12 bytes past
+    (5000, 1433, 1437, 1, 16, True),  # many rows per CTA: the stage ring wraps
+    (64, 20000, 20001, 1, 128, True), # rows of 80 KB: two stages
+])
+def test_forward_2layer_front_unaligned_rows(cuda_device, N, K, ldx, offset, Fh, centred):
+    Fo = 5
+    case = inputs.layer_case(N, K, Fh, seed=N + K + ldx, mean_degree=3.0, centred=centred)
+    W2 = inputs.weights(Fh, Fo, seed=K + 5)
+    d = {k: to_dev(v) for k, v in case.items()}
+    buf = torch.full((N * ldx + offset + 8,), float("nan"), device=cuda_device)
+    X = buf[offset:offset + N * ldx].view(N, ldx)[:, :K]
+    X.copy_(d["X"])
+    ws = torch.empty(B.bigcn_forward_2layer_workspace_bytes(N, K, Fh, Fo), dtype=torch.uint8,
+                     device=cuda_device)
+    H1 = torch.full((N, Fh), float("nan"), device=cuda_device)
+    out = torch.full((N, Fo), float("nan"), device=cuda_device)
+    B.bigcn_forward_2layer(X, d["s"], d["t"], d["W"], to_dev(W2), d["rowptr"], d["colidx"],
+                           ws, out, H1=H1)
+    ref1 = oracle.layer_forward(case["X"], case["W"], case["rowptr"], case["colidx"],
+                                case["s"], case["t"])
+    assert_close(H1, ref1["H"], "H1")
+    ref2 = oracle.layer_forward(H1.cpu().numpy(), W2, case["rowptr"], case["colidx"])
+    assert_close(out, ref2["H"], "logits")
+    assert B.device_timeouts() == 0
+
+
 def test_forward_2layer_records_one_event_per_kernel_boundary(cuda_device):
     N, K, Fh, Fo = 500, 300, 64, 7
     case = inputs.layer_case(N, K, Fh, seed=3)
@@ -321,7 +357,8 @@ def test_forward_2layer_records_one_event_per_kernel_boundary(cuda_device):
     W2 = to_dev(inputs.weights(Fh, Fo, seed=4))
     n = B.bigcn_forward_2layer_launches(N, K, Fh, Fo)
     assert n == 4 and B.bigcn_forward_2layer_launches(N, K, 30, 7) == 6
-    assert B.bigcn_forward_2layer_launches(N, 3000, 64, 7) == 5
+    assert B.bigcn_forward_2layer_launches(N, 3000, 64, 7) == 4
+    assert B.bigcn_forward_2layer_launches(N, 3000, 200, 7) == 7
     assert B.bigcn_forward_2layer_launches(N, 8192, 256, 7) == 7
     events = [torch.cuda.Event(enable_timing=True) for _ in range(n + 1)]
     for e in events:
