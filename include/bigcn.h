@@ -169,13 +169,11 @@ bigcn_status bigcn_spmm_prescaled(const int64_t *rowptr, const int32_t *colidx,
  * as FP8 +-1, exact fp32 integer sums) when K >= 128, F >= 32 and N is at
  * least 128 rows per SM, and on the CUDA cores (XOR + popcount) otherwise;
  * the dots are identical either way.
- * Its kernels, and the layer-1 front of bigcn_forward_2layer (which stages
- * rows of X in shared memory with bulk async copies), wait on shared-memory
- * barriers with a bounded number of tries. bigcn_device_timeouts
- * synchronizes the current device, returns how many such waits ran out
- * since its last call (0 in correct operation; a CTA or warp whose wait ran
- * out leaves its outputs unwritten) and resets the count; -1 on a CUDA
- * error.
+ * Its kernels wait on shared-memory barriers with a bounded number of
+ * tries. bigcn_device_timeouts synchronizes the current device, returns how
+ * many such waits ran out since its last call (0 in correct operation; a
+ * CTA whose wait ran out writes no output) and resets the count; -1 on a
+ * CUDA error.
  */
 int32_t bigcn_device_timeouts(void);
 
