@@ -11,9 +11,11 @@
 // Partial sums are combined across groups with xor shuffles and group 0
 // writes H_i scaled by 1/sqrt(dhat_i).
 //
-// Heavy rows (more than kHeavyDegree neighbours, e.g. the hubs of a
-// power-law graph) would make one warp the critical path of the whole
-// launch. The first `heavy_blocks` blocks of every launch therefore scan the
+// Heavy rows (the hubs of a power-law graph) would make one warp the
+// critical path of the whole launch: a warp walks its row U * 32 / L
+// neighbours per round trip. A row is heavy when it has more than
+// max(32, 4 * that width, 4 * the mean degree) neighbours, i.e. when its walk
+// would take several times longer than a typical row's. The first `heavy_blocks` blocks of every launch therefore scan the
 // row pointers, skip light rows, and give each heavy row to all 8 warps of
 // the block: warp w gathers the w-th eighth of the row's list, the eight
 // partial rows meet in shared memory and warp 0 adds them in warp order
@@ -30,7 +32,6 @@ namespace {
 
 constexpr int kSpmmThreads = 256;
 constexpr int kSpmmWarps = kSpmmThreads / 32;
-constexpr int64_t kHeavyDegree = 2048;
 
 template <int VEC> struct Vec;
 template <> struct Vec<1> {
@@ -73,6 +74,7 @@ struct SpmmParams {
     float *H;
     int64_t ldh;
     int heavy_blocks;        // leading blocks that take the heavy rows
+    int64_t heavy_degree;    // rows with more neighbours are heavy
     bool vec_store;          // H rows start VEC-aligned: whole vectors may be stored
 };
 
@@ -182,7 +184,7 @@ __device__ __forceinline__ void light_rows(const SpmmParams &p, const Epi &epi, 
     const int64_t i = int64_t(blockIdx.x - p.heavy_blocks) * kSpmmWarps + warp;
     if (i >= p.N) return;
     const RowSpan sp = row_span(p.rowptr, p.nnz, i);
-    if (p.heavy_blocks > 0 && sp.total - 1 > kHeavyDegree) return;   // a heavy block's row
+    if (p.heavy_blocks > 0 && sp.total - 1 > p.heavy_degree) return;   // a heavy block's row
     float acc[NV][VEC];
 #pragma unroll
     for (int v = 0; v < NV; ++v)
@@ -203,7 +205,7 @@ __device__ __forceinline__ void heavy_rows(const SpmmParams &p, const Epi &epi, 
          base += int64_t(p.heavy_blocks) * kSpmmThreads) {
         const int64_t r = base + threadIdx.x;
         bool heavy = false;
-        if (r < p.N) heavy = row_span(p.rowptr, p.nnz, r).total - 1 > kHeavyDegree;
+        if (r < p.N) heavy = row_span(p.rowptr, p.nnz, r).total - 1 > p.heavy_degree;
         const unsigned m = __ballot_sync(kFullMask, heavy);
         if (lane == 0) mask[warp] = m;
         __syncthreads();
@@ -374,13 +376,21 @@ int heavy_block_count(int64_t N, const DeviceInfo &dev) {
     return int(chunks < cap ? chunks : cap);
 }
 
+// The heavy-row threshold for a walk of `per_iter` neighbours per round trip.
+int64_t heavy_degree(int64_t N, int64_t nnz, int per_iter) {
+    const int64_t mean = N > 0 ? nnz / N : 0;
+    int64_t h = 4 * int64_t(per_iter);
+    if (4 * mean > h) h = 4 * mean;
+    return h > 32 ? h : 32;
+}
+
 template <int VEC, int L, int NV, bool kPre>
 void launch_cfg(const SpmmArgs &a, const DeviceInfo &dev, int Fload, cudaStream_t s, bool pdl) {
     constexpr int SLAB = L * NV * VEC;
     constexpr int U = NV == 1 ? 4 : 2;
     const bool vec_store = a.ldh % VEC == 0 && aligned_to(a.H, size_t(VEC) * 4);
     SpmmParams p{a.rowptr, a.colidx, a.N, a.nnz, a.Z, a.ldz, Fload, a.F, a.H, a.ldh,
-                 heavy_block_count(a.N, dev), vec_store};
+                 heavy_block_count(a.N, dev), heavy_degree(a.N, a.nnz, (32 / L) * U), vec_store};
     dim3 grid(unsigned(p.heavy_blocks + (a.N + kSpmmWarps - 1) / kSpmmWarps),
               unsigned((a.F + SLAB - 1) / SLAB));
     launch_kernel(spmm_norm_kernel<VEC, L, NV, U, kPre>, grid, dim3(kSpmmThreads), 0, s, pdl,
@@ -429,8 +439,10 @@ void launch_spmm_pack_gemm(const SpmmPackGemmArgs &a, const DeviceInfo &dev, cud
                            bool pdl) {
     if (a.N == 0) return;
     const int nvec = a.Fh / 4;
+    int L = 4;
+    while (L < 32 && L < nvec) L *= 2;
     SpmmParams p{a.rowptr, a.colidx, a.N, a.nnz, a.Z1, a.Fh, a.Fh, a.Fh, nullptr, 0,
-                 heavy_block_count(a.N, dev), false};
+                 heavy_block_count(a.N, dev), heavy_degree(a.N, a.nnz, (32 / L) * 4), false};
     FusedLayer2 f{a.H1, a.ldh, nullptr, nullptr, a.Fo, (a.Fh + 63) / 64, a.Z2, a.ldz2};
     const dim3 grid(unsigned(p.heavy_blocks + (a.N + kSpmmWarps - 1) / kSpmmWarps));
     const dim3 one(1, 1, 1), block(kSpmmThreads);

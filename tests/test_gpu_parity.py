@@ -377,7 +377,8 @@ def test_forward_2layer_records_one_event_per_kernel_boundary(cuda_device):
 
 def hub_graph(N, hubs, seed, mean_degree=4.0):
     """Random graph plus hub rows: (node, degree) pairs joined to random others.
-    Degrees above 2048 take the kernels' whole-block path."""
+    Rows far above the mean degree (here 2049 to 8190 neighbours) take the
+    kernels' whole-block path."""
     g = rng(seed)
     rowptr, colidx = inputs.random_graph(N, mean_degree, seed=seed)
     rows = np.repeat(np.arange(N), np.diff(rowptr))
