@@ -54,7 +54,6 @@ front_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
     const int64_t m0 = int64_t(blockIdx.x) * BM;
 
     // Phase A: centre + sign + pack + |y| sums, rows warp, warp + 8, ...
-    const int nchunks = (K + 31) >> 5;
     const int nhalf = 2 * words;
     for (int r = warp; r < BM; r += kFrontWarps) {
         const int64_t row = m0 + r;
@@ -65,27 +64,10 @@ front_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
             continue;
         }
         const float *x = X + row * ldx;
-        float l1 = 0.0f;
-        for (int c0 = 0; c0 < nchunks; c0 += kFrontUnroll) {
-            float v[kFrontUnroll];
-#pragma unroll
-            for (int u = 0; u < kFrontUnroll; ++u) {
-                const int k = (c0 + u) * 32 + lane;
-                v[u] = (k < K) ? __ldcs(x + k) : 0.0f;
-            }
-#pragma unroll
-            for (int u = 0; u < kFrontUnroll; ++u) {
-                const int k = (c0 + u) * 32 + lane;
-                const bool in = k < K;
-                float y = v[u];
-                if (scale != nullptr && in) y = __fmaf_rn(y, __ldg(scale + k), __ldg(shift + k));
-                const unsigned m = __ballot_sync(kFullMask, in && y >= 0.0f);
-                if (lane == 0 && c0 + u < nchunks) a32[c0 + u] = m;
-                l1 += in ? fabsf(y) : 0.0f;
-            }
-        }
-        for (int q = nchunks + lane; q < nhalf; q += 32) a32[q] = 0u;
-        l1 = warp_sum(l1);
+        const float l1 =
+            scale != nullptr
+                ? pack_share<1, kFrontUnroll, Affine::kGlobal>(x, K, scale, shift, nullptr, a32, nhalf, 0)
+                : pack_share<1, kFrontUnroll, Affine::kNone>(x, K, nullptr, nullptr, nullptr, a32, nhalf, 0);
         if (lane == 0) sAlpha[r] = l1 / float(K);
     }
 
@@ -161,18 +143,26 @@ int front_rows(int64_t N, const DeviceInfo &dev) {
 
 // ---------------------------------------------------------------------------
 // Split front, for layers with few rows (fewer than one warp per row would
-// leave most of the GPU idle, e.g. a few thousand long rows): each block
-// takes R = 8 / G rows at a time, G warps per row (the row-packing kernel's
-// split, same chunk order and the same alpha summation), and writes the
-// packed rows to shared memory. The block then computes their products: the
-// 32 G threads of a row take P lanes per output column (P a power of two,
-// words w = t mod P, t mod P + P, ... for lane t of the column), add their
-// mismatch counts with shuffles and write Z' as above. The packed weight
-// columns are staged in shared memory once per block, after the dependency
-// wait, which comes only after the block's first rows have been streamed.
+// leave most of the GPU idle, e.g. a few thousand long rows): each 16-warp
+// block takes R = 16 / G rows at a time, G warps per row (the row-packing
+// kernel's split, the same chunk order and the same alpha summation), and
+// writes the packed rows to shared memory. The block then computes their
+// products: the 32 G threads of a row take P lanes per output column (P a
+// power of two, words w = t mod P, t mod P + P, ... for lane t of the
+// column), add their mismatch counts with shuffles and write Z' as above.
+// The centring affine is staged in shared memory as (scale, shift) pairs
+// when the block starts (it is the call's input); the packed weight columns
+// are staged once per block after the dependency wait, which comes only
+// after the block's first rows have been streamed.
 
-size_t split_smem(int F, int words) {
-    return (size_t(F) + size_t(kFrontWarps)) * size_t(words | 1) * 8;
+// Shared memory: F x pitch packed columns, 16 x pitch packed rows, and the
+// centring affine as K (scale, shift) pairs.
+constexpr int kSplitThreads = 512;
+constexpr int kSplitWarps = kSplitThreads / 32;
+
+size_t split_smem(int F, int K, int words, bool affine) {
+    return (size_t(F) + size_t(kSplitWarps)) * size_t(words | 1) * 8 +
+           (affine ? size_t(K) * 8 : 0);
 }
 
 // Warps per row: the row-packing kernel's policy (split while the grid is
@@ -185,45 +175,62 @@ int split_warps(int64_t N, int K, const DeviceInfo &dev) {
     return G;
 }
 
-template <bool kAffine>
-__global__ void __launch_bounds__(kFrontThreads, 3)
+template <int G, bool kAffine>
+__global__ void __launch_bounds__(kSplitThreads, 3)
 front_split_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
                    const float *__restrict__ scale, const float *__restrict__ shift,
                    const uint64_t *__restrict__ wbits, const float *__restrict__ beta, int F,
                    int words, const int64_t *__restrict__ rowptr, float *__restrict__ Z,
-                   int64_t ldz, int G, int P) {
+                   int64_t ldz, int P) {
     extern __shared__ __align__(16) unsigned char smem[];
-    __shared__ float part[kFrontWarps];
+    __shared__ float part[kSplitWarps];
+    constexpr int R = kSplitWarps / G;       // rows per group
+    constexpr int T = 32 * G;                // threads per row in the product
+    constexpr Affine kA = kAffine ? Affine::kShared : Affine::kNone;
     const int pitch = words | 1;
     uint64_t *Ws = reinterpret_cast<uint64_t *>(smem);      // F x pitch packed columns
     uint64_t *As = Ws + size_t(F) * pitch;                   // R x pitch packed rows
+    float2 *sST = reinterpret_cast<float2 *>(As + size_t(kSplitWarps) * pitch);
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int R = kFrontWarps / G;
-    const int T = 32 * G;                    // threads per row in the product
     const int rr = tid / T, tt = tid % T, sub = tt % P;
     const int cstep = T / P;                 // columns per pass
     const int passes = (F + cstep - 1) / cstep;
+    if (kAffine) {
+        for (int k0 = tid; k0 < K; k0 += 4 * kSplitThreads) {
+            float2 v[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int k = k0 + u * kSplitThreads;
+                if (k < K) v[u] = make_float2(__ldg(scale + k), __ldg(shift + k));
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+                if (k0 + u * kSplitThreads < K) sST[k0 + u * kSplitThreads] = v[u];
+        }
+        __syncthreads();
+    }
     bool staged = false;
     for (int64_t group = blockIdx.x; group * R < N; group += gridDim.x) {
         const int64_t row = group * R + warp / G;
         uint32_t *a32 = reinterpret_cast<uint32_t *>(As + size_t(warp / G) * pitch);
-        const float l1 = (row < N) ? pack_row_chunks<kAffine>(X + row * ldx, K, scale, shift, a32,
-                                                              2 * words, warp % G, G)
+        const float l1 = (row < N) ? pack_share<G, kFrontUnroll, kA>(X + row * ldx, K, nullptr,
+                                                                     nullptr, sST, a32,
+                                                                     2 * words, warp % G)
                                    : 0.0f;
         if (lane == 0) part[warp] = l1;
         if (!staged) {
             grid_dependency_wait();     // the packed weight columns come from the previous kernel
             const int n = F * words;
-            for (int q0 = tid; q0 < n; q0 += 8 * kFrontThreads) {
-                uint64_t v[8];
+            for (int q0 = tid; q0 < n; q0 += 4 * kSplitThreads) {
+                uint64_t v[4];
 #pragma unroll
-                for (int u = 0; u < 8; ++u) {
-                    const int q = q0 + u * kFrontThreads;
+                for (int u = 0; u < 4; ++u) {
+                    const int q = q0 + u * kSplitThreads;
                     if (q < n) v[u] = __ldg(wbits + q);
                 }
 #pragma unroll
-                for (int u = 0; u < 8; ++u) {
-                    const int q = q0 + u * kFrontThreads;
+                for (int u = 0; u < 4; ++u) {
+                    const int q = q0 + u * kSplitThreads;
                     if (q < n) Ws[(q / words) * pitch + (q % words)] = v[u];
                 }
             }
@@ -233,6 +240,7 @@ front_split_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
         const int64_t row2 = group * R + rr;
         if (row2 < N) {                      // uniform over each warp (T is a multiple of 32)
             float t = 0.0f;
+#pragma unroll
             for (int g = 0; g < G; ++g) t += part[rr * G + g];
             const float ai = (t / float(K)) *
                              inv_sqrt_degree(__ldg(rowptr + row2 + 1) - __ldg(rowptr + row2));
@@ -254,7 +262,7 @@ front_split_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
 
 bool split_supported(int64_t N, int K, int F, const DeviceInfo &dev) {
     return F >= 1 && F <= 128 && split_warps(N, K, dev) > 1 &&
-           split_smem(F, (K + 63) / 64) <= kFrontMaxSmem / 2;
+           split_smem(F, K, (K + 63) / 64, true) <= kFrontMaxSmem / 2;
 }
 
 void launch_split(const FrontArgs &a, const DeviceInfo &dev, cudaStream_t s, bool pdl) {
@@ -264,19 +272,25 @@ void launch_split(const FrontArgs &a, const DeviceInfo &dev, cudaStream_t s, boo
     int P = 32 * G / fp;
     if (P < 1) P = 1;
     if (P > 32) P = 32;
-    const size_t smem = split_smem(a.F, a.words);
-    auto kernel = a.scale != nullptr ? front_split_kernel<true> : front_split_kernel<false>;
+    const bool affine = a.scale != nullptr;
+    const size_t smem = split_smem(a.F, a.K, a.words, affine);
+    void (*kernel)(const float *, int64_t, int, int64_t, const float *, const float *,
+                   const uint64_t *, const float *, int, int, const int64_t *, float *, int64_t,
+                   int);
+    if (G == 2) kernel = affine ? front_split_kernel<2, true> : front_split_kernel<2, false>;
+    else if (G == 4) kernel = affine ? front_split_kernel<4, true> : front_split_kernel<4, false>;
+    else kernel = affine ? front_split_kernel<8, true> : front_split_kernel<8, false>;
     cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
     int per_sm = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, kFrontThreads, smem) !=
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, kSplitThreads, smem) !=
             cudaSuccess ||
         per_sm < 1)
         per_sm = 1;
-    const int64_t groups = (a.N + kFrontWarps / G - 1) / (kFrontWarps / G);
+    const int64_t groups = (a.N + kSplitWarps / G - 1) / (kSplitWarps / G);
     const int64_t resident = int64_t(per_sm) * dev.sm_count;
     launch_kernel(kernel, dim3(unsigned(groups < resident ? groups : resident)),
-                  dim3(kFrontThreads), smem, s, pdl, dim3(1, 1, 1), a.X, a.N, a.K, a.ldx, a.scale,
-                  a.shift, a.wbits, a.beta, a.F, a.words, a.rowptr, a.Z, a.ldz, G, P);
+                  dim3(kSplitThreads), smem, s, pdl, dim3(1, 1, 1), a.X, a.N, a.K, a.ldx, a.scale,
+                  a.shift, a.wbits, a.beta, a.F, a.words, a.rowptr, a.Z, a.ldz, P);
 }
 
 }  // namespace

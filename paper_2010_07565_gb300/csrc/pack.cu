@@ -37,21 +37,23 @@ namespace cg = cooperative_groups;
 constexpr int kPackThreads = 256;
 constexpr int kPackWarps = kPackThreads / 32;
 constexpr int kPackBlocksPerSM = 8;   // resident blocks the persistent grids assume
+constexpr int kPackUnroll = 8;
 
 // Whole rows per warp: every warp walks rows on its own (persistent grid,
 // no block barrier), which keeps the kernel small enough for full occupancy.
 template <bool kAffine, bool kUpstream>
-__global__ void __launch_bounds__(kPackThreads)
+__global__ void __launch_bounds__(kPackThreads, kPackBlocksPerSM)
 pack_rows_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
                  const float *__restrict__ scale, const float *__restrict__ shift,
                  uint32_t *__restrict__ bits32, int64_t ld32, float *__restrict__ alpha) {
     if (kUpstream) grid_dependency_wait();      // X is the previous kernel's output
+    constexpr Affine kA = kAffine ? Affine::kGlobalLate : Affine::kNone;
     const int lane = threadIdx.x & 31;
     const int64_t nwarps = int64_t(gridDim.x) * kPackWarps;
     for (int64_t row = int64_t(blockIdx.x) * kPackWarps + (threadIdx.x >> 5); row < N;
          row += nwarps) {
-        const float l1 =
-            pack_row_chunks<kAffine>(X + row * ldx, K, scale, shift, bits32 + row * ld32, ld32, 0, 1);
+        const float l1 = pack_share<1, kPackUnroll, kA>(X + row * ldx, K, scale, shift, nullptr,
+                                                        bits32 + row * ld32, ld32, 0);
         if (lane == 0) alpha[row] = l1 / float(K);
     }
     // Otherwise wait only now: finishing after the predecessor keeps the
@@ -61,21 +63,23 @@ pack_rows_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
 
 // Rows shared by G > 1 warps (few, long rows): block b takes row groups
 // b, b + gridDim.x, ...; the G partial sums meet in shared memory.
-template <bool kAffine>
+template <int G, bool kAffine>
 __global__ void __launch_bounds__(kPackThreads, 5)
 pack_rows_split_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
                        const float *__restrict__ scale, const float *__restrict__ shift,
                        uint32_t *__restrict__ bits32, int64_t ld32, float *__restrict__ alpha,
-                       int G, bool x_upstream) {
+                       bool x_upstream) {
     __shared__ float part[kPackWarps];
     if (x_upstream) grid_dependency_wait();
+    constexpr Affine kA = kAffine ? Affine::kGlobal : Affine::kNone;
+    constexpr int kRows = kPackWarps / G;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int sub = warp & (G - 1);
-    const int rows_per_block = kPackWarps / G;
-    for (int64_t group = blockIdx.x; group * rows_per_block < N; group += gridDim.x) {
-        const int64_t row = group * rows_per_block + warp / G;
-        const float l1 = (row < N) ? pack_row_chunks<kAffine>(X + row * ldx, K, scale, shift,
-                                                              bits32 + row * ld32, ld32, sub, G)
+    const int sub = warp % G;
+    for (int64_t group = blockIdx.x; group * kRows < N; group += gridDim.x) {
+        const int64_t row = group * kRows + warp / G;
+        const float l1 = (row < N) ? pack_share<G, kPackUnroll, kA>(X + row * ldx, K, scale, shift,
+                                                                    nullptr, bits32 + row * ld32,
+                                                                    ld32, sub)
                                    : 0.0f;
         if (lane == 0) part[warp] = l1;
         __syncthreads();
@@ -175,12 +179,20 @@ void launch_pack_rows(const float *X, int64_t N, int K, int64_t ldx, const float
         else if (x_upstream) run(pack_rows_kernel<false, true>, no, no);
         else run(pack_rows_kernel<false, false>, no, no);
     } else {
-        if (scale)
-            launch_kernel(pack_rows_split_kernel<true>, grid, block, 0, stream, pdl, one, X, N, K,
-                          ldx, scale, shift, b32, ld32, alpha, G, x_upstream);
-        else
-            launch_kernel(pack_rows_split_kernel<false>, grid, block, 0, stream, pdl, one, X, N, K,
-                          ldx, no, no, b32, ld32, alpha, G, x_upstream);
+        auto run = [&](auto kernel, const float *sc, const float *sh) {
+            launch_kernel(kernel, grid, block, 0, stream, pdl, one, X, N, K, ldx, sc, sh, b32, ld32,
+                          alpha, x_upstream);
+        };
+        if (G == 2) {
+            if (scale) run(pack_rows_split_kernel<2, true>, scale, shift);
+            else run(pack_rows_split_kernel<2, false>, no, no);
+        } else if (G == 4) {
+            if (scale) run(pack_rows_split_kernel<4, true>, scale, shift);
+            else run(pack_rows_split_kernel<4, false>, no, no);
+        } else {
+            if (scale) run(pack_rows_split_kernel<8, true>, scale, shift);
+            else run(pack_rows_split_kernel<8, false>, no, no);
+        }
     }
 }
 
