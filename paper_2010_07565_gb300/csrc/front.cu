@@ -172,6 +172,10 @@ int split_warps(int64_t N, int K, const DeviceInfo &dev) {
     const int64_t full_wave = int64_t(dev.sm_count) * 64;
     int G = 1;
     while (G < kFrontWarps && N * G < full_wave && nchunks >= 2 * G * 8) G *= 2;
+    // Each warp that shares a row adds a product pass: stop splitting once
+    // half a wave of warps is busy (measured: two warps per row beat four on
+    // a few thousand rows of 3703 features).
+    while (G > 2 && N * (G / 2) >= full_wave / 2) G /= 2;
     return G;
 }
 

@@ -29,6 +29,7 @@
 //   Z = (alpha_i / sqrt(dhat_i)) * (beta_j * dot).
 #include "async.cuh"
 #include "launch.cuh"
+#include "tc.cuh"
 
 namespace bigcn {
 
@@ -37,59 +38,8 @@ __device__ unsigned int g_tc_timeouts;
 namespace {
 
 constexpr int kTcThreads = 256;
-constexpr int kTcM = 128;
 constexpr int kTcKBytes = 128;
 constexpr int kTcStages = 2;
-
-// Four signs (bits 0..3 of n) as four FP8 E4M3 bytes, +1 for a set bit:
-// n * (1 + 2^7 + 2^14 + 2^21) moves bit i of n to bit 8i (the other partial
-// products never land on a multiple of 8 below 32), and flipping the sign bit
-// of -1.0 (0xB8) there gives +1.0 (0x38).
-__device__ __forceinline__ uint32_t signs4_to_e4m3(uint32_t n) {
-    const uint32_t spread = (n * 0x00204081u) & 0x01010101u;
-    return 0xB8B8B8B8u ^ (spread << 7);
-}
-
-// Byte offset of 16-byte chunk c of row r in a 128B-swizzled K-major tile.
-__device__ __forceinline__ uint32_t sw128_offset(int r, int c) {
-    return uint32_t((r >> 3) * 1024 + (r & 7) * 128 + ((c ^ (r & 7)) << 4));
-}
-
-// Shared-memory matrix descriptor: K-major, 128B swizzle, 8-row groups 1024 B
-// apart (stride byte offset), descriptor version 1.
-__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
-    uint64_t d = uint64_t((saddr >> 4) & 0x3FFFu);
-    d |= uint64_t(1) << 16;                     // leading byte offset (unused here)
-    d |= uint64_t(1024 >> 4) << 32;             // stride byte offset
-    d |= uint64_t(1) << 46;                     // version
-    d |= uint64_t(2) << 61;                     // swizzle: 128B
-    return d;
-}
-
-// Instruction descriptor: E4M3 x E4M3 -> F32, both K-major, M = 128, N = n.
-__host__ __device__ constexpr uint32_t e4m3_idesc(int n) {
-    return (1u << 4) | (uint32_t(n >> 3) << 17) | (uint32_t(kTcM >> 4) << 24);
-}
-
-__device__ __forceinline__ void mma_e4m3(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
-                                         uint32_t accumulate) {
-    asm volatile(
-        "{\n.reg .pred p;\n"
-        "setp.ne.b32 p, %4, 0;\n"
-        "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n}" ::"r"(d_tmem),
-        "l"(a), "l"(b), "r"(idesc), "r"(accumulate));
-}
-
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]),
-          "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]),
-          "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-        : "r"(taddr));
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-}
 
 template <int NT, bool kDeg>
 __global__ void __launch_bounds__(kTcThreads)
@@ -97,18 +47,18 @@ xnor_gemm_tc_kernel(const uint64_t *__restrict__ A, const float *__restrict__ al
                     const uint64_t *__restrict__ B, const float *__restrict__ beta, int F, int K,
                     int words, float *__restrict__ Z, int64_t ldz, int32_t *__restrict__ dots,
                     const int64_t *__restrict__ rowptr) {
-    constexpr int kStageA = kTcM * kTcKBytes;
+    constexpr int kStageA = kUmmaM * kTcKBytes;
     constexpr int kStageB = NT * kTcKBytes;
     constexpr int kStage = kStageA + kStageB;
     constexpr int kRowsPerPass = kTcThreads / 8;         // 32: thread t owns chunk t & 7
-    constexpr int kAChunks = kTcM / kRowsPerPass;         // 4 rows of A per thread
+    constexpr int kAChunks = kUmmaM / kRowsPerPass;         // 4 rows of A per thread
     constexpr int kBChunks = NT / kRowsPerPass;           // 2, 4 or 8 rows of B per thread
     extern __shared__ unsigned char smem_raw[];
     __shared__ __align__(8) uint64_t bars[kTcStages];
     __shared__ uint32_t tmem_base;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int64_t m0 = int64_t(blockIdx.x) * kTcM;
+    const int64_t m0 = int64_t(blockIdx.x) * kUmmaM;
     const int n0 = blockIdx.y * NT;
     const uint32_t raw = smem_addr(smem_raw);
     const uint32_t tile0 = (raw + 1023u) & ~1023u;          // 1024-byte aligned stages
@@ -283,7 +233,7 @@ xnor_gemm_tc_kernel(const uint64_t *__restrict__ A, const float *__restrict__ al
 
 template <int NT>
 size_t tc_smem() {
-    return 1024 + size_t(kTcStages) * (kTcM * kTcKBytes + NT * kTcKBytes);
+    return 1024 + size_t(kTcStages) * (kUmmaM * kTcKBytes + NT * kTcKBytes);
 }
 
 template <int NT, bool kDeg>
@@ -291,7 +241,7 @@ void launch_nt(const GemmArgs &g, cudaStream_t s, bool pdl) {
     const size_t smem = tc_smem<NT>();
     cudaFuncSetAttribute(xnor_gemm_tc_kernel<NT, kDeg>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          int(smem));
-    const dim3 grid(unsigned((g.N + kTcM - 1) / kTcM), unsigned((g.F + NT - 1) / NT));
+    const dim3 grid(unsigned((g.N + kUmmaM - 1) / kUmmaM), unsigned((g.F + NT - 1) / NT));
     launch_kernel(xnor_gemm_tc_kernel<NT, kDeg>, grid, dim3(kTcThreads), smem, s, pdl,
                   dim3(1, 1, 1), g.A, g.alpha, g.N, g.B, g.beta, g.F, g.K, g.words, g.Z, g.ldz,
                   g.dots, g.rowptr);
@@ -308,7 +258,7 @@ void launch_deg(const GemmArgs &g, cudaStream_t s, bool pdl) {
 
 bool xnor_gemm_tc_supported(int64_t N, int K, int F, const DeviceInfo &dev) {
     // Enough 128-row tiles to give every SM one, and shared memory for two stages.
-    return K >= 128 && F >= 32 && (N + kTcM - 1) / kTcM >= dev.sm_count &&
+    return K >= 128 && F >= 32 && (N + kUmmaM - 1) / kUmmaM >= dev.sm_count &&
            size_t(dev.max_smem_optin) >= tc_smem<256>();
 }
 
