@@ -449,10 +449,10 @@ SWEEP_KERNELS = ("pack_rows", "pack_weights", "xnor_gemm", "spmm")
 
 
 def run_sweep(args, rank, world, local_rank):
-    """One Bi-GCN layer on a C5 sweep point (2^20 nodes, K, F): the four step
-    kernels the layer runs (bigcn_pack_rows, bigcn_pack_weights,
-    bigcn_xnor_gemm_degscaled, bigcn_spmm_prescaled), each timed with events
-    on its stream. The features (up to 34 GB) are drawn on the device by
+    """One Bi-GCN layer on a C5 sweep point (2^20 nodes, K, F): one
+    bigcn_layer_forward_timed call per step, with an event before each of the
+    layer's four kernels (pack rows, pack weights, XNOR product, aggregation)
+    and after the last. The features (up to 34 GB) are drawn on the device by
     torch's seeded generator; the other inputs come from the usual seeds.
     The inputs are larger than L2, so no flush is needed between steps."""
     import torch
@@ -471,24 +471,14 @@ def run_sweep(args, rank, world, local_rank):
     rp, ci = inputs.graph(w)
     rowptr, colidx = torch.from_numpy(rp).to(dev), torch.from_numpy(ci).to(dev)
     nnz = int(ci.shape[0])
-    words = B.words_for(K)
-    bits = torch.empty((N, words), dtype=torch.int64, device=dev)
-    alpha = torch.empty(N, device=dev)
-    wbits = torch.empty((F, words), dtype=torch.int64, device=dev)
-    beta = torch.empty(F, device=dev)
-    Z, H = torch.empty((N, F), device=dev), torch.empty((N, F), device=dev)
+    ws = torch.empty(B.bigcn_layer_workspace_bytes(N, K, F), dtype=torch.uint8, device=dev)
+    H = torch.empty((N, F), device=dev)
     ev = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
+    for e in ev:            # torch creates the CUDA event at its first record
+        e.record()
 
     def step():
-        ev[0].record()
-        B.bigcn_pack_rows(X, None, None, bits, alpha)
-        ev[1].record()
-        B.bigcn_pack_weights(Wt, wbits, beta)
-        ev[2].record()
-        B.bigcn_xnor_gemm_degscaled(bits, alpha, wbits, beta, K, rowptr, Z)
-        ev[3].record()
-        B.bigcn_spmm_prescaled(rowptr, colidx, Z, H)
-        ev[4].record()
+        B.bigcn_layer_forward_timed(X, None, None, Wt, rowptr, colidx, ws, H, ev)
 
     for _ in range(args.warmup):
         step()
@@ -509,10 +499,13 @@ def run_sweep(args, rank, world, local_rank):
     peaks, peak_kind = load_peaks()
     hbm = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
     mean_us = [1e3 * statistics.fmean(t) for t in per_kernel]
+    words = (K + 63) // 64
+    # The layer keeps Z factored (uint16 dots + a row scale) when K <= 32767.
+    z_bytes = 2.0 * N * ((F + 3) // 4 * 4) + 4.0 * N if K <= 32767 else 4.0 * N * F
     work = {"pack_rows": (4.0 * N * K + 8.0 * N * words + 4.0 * N, "bytes", "hbm"),
             "pack_weights": (4.0 * K * F + 8.0 * F * words + 4.0 * F, "bytes", "hbm"),
             "xnor_gemm": (float(N) * K * F, "bit-ops", "tensor"),
-            "spmm": (8.0 * (N + 1) + 4.0 * nnz + 8.0 * N * F, "bytes", "hbm")}
+            "spmm": (8.0 * (N + 1) + 4.0 * nnz + z_bytes + 4.0 * N * F, "bytes", "hbm")}
     k_dom = max(range(4), key=lambda k: mean_us[k])
     name = SWEEP_KERNELS[k_dom]
     amount, unit, bound = work[name]
@@ -532,8 +525,8 @@ def run_sweep(args, rank, world, local_rank):
         "data": "synthetic",
         "config": {"workload": w.description, "name": w.name, "N": N, "K": K, "F": F, "nnz": nnz,
                    "l2": "inputs larger than L2 (no flush)",
-                   "launch": "bigcn_pack_rows, bigcn_pack_weights, bigcn_xnor_gemm_degscaled, "
-                             "bigcn_spmm_prescaled (the kernels of bigcn_layer_forward)"},
+                   "launch": "bigcn_layer_forward_timed: pack rows, pack weights, XNOR "
+                             "product, aggregation (4 kernels, an event between each)"},
         "components": {
             "per_kernel_us": {n: round(t, 3) for n, t in zip(SWEEP_KERNELS, mean_us)},
             "pack_rows_gbs": work["pack_rows"][0] / (mean_us[0] * 1e-6) / 1e9,

@@ -185,9 +185,13 @@ size_t bigcn_layer_workspace_bytes(int64_t N, int32_t K, int32_t F);
  * One binarized graph-convolution layer, H = A~ zeta (Eq. 13), with zeta from
  * the centred (scale/shift, as in bigcn_pack_rows) and binarized X and the
  * binarized W (Eqs. 3-12). The result equals the composition of the four
- * calls above within fp32 rounding; it runs exactly bigcn_pack_rows,
+ * calls above within fp32 rounding; it runs the kernels of bigcn_pack_rows,
  * bigcn_pack_weights, bigcn_xnor_gemm_degscaled and bigcn_spmm_prescaled on
- * `stream`. No activation follows (Sec. 4.1.2).
+ * `stream`, except that when K <= 32767 the product keeps Z' factored in the
+ * workspace -- the integer dots (as uint16 with a bias of 32768) and each
+ * row's alpha_i / sqrt(dhat_i) -- and the aggregation applies the row factor
+ * per neighbour and beta_j per column, gathering half the bytes. No
+ * activation follows (Sec. 4.1.2).
  *
  * X N x K (ldx), Wt K x F (ldw), CSR as in bigcn_spmm_norm, H N x F (ldh).
  * workspace  device memory of at least bigcn_layer_workspace_bytes(N, K, F)
@@ -201,6 +205,22 @@ bigcn_status bigcn_layer_forward(const float *X, int64_t N, int32_t K, int64_t l
                                  const int64_t *rowptr, const int32_t *colidx,
                                  int64_t nnz, void *workspace, size_t ws_bytes,
                                  float *H, int64_t ldh, void *stream);
+
+/*
+ * bigcn_layer_forward with timing events: event q of the n_events given
+ * (cudaEvent_t as void*, nullable array) is recorded on `stream` before the
+ * layer's kernel q (pack rows, pack weights, XNOR product, aggregation) and
+ * event 4 after the last (as external events while the stream is being
+ * captured); entries beyond 5 are not touched. Everything else is
+ * bigcn_layer_forward's.
+ */
+bigcn_status bigcn_layer_forward_timed(const float *X, int64_t N, int32_t K, int64_t ldx,
+                                       const float *scale, const float *shift,
+                                       const float *Wt, int32_t F, int64_t ldw,
+                                       const int64_t *rowptr, const int32_t *colidx,
+                                       int64_t nnz, void *workspace, size_t ws_bytes,
+                                       float *H, int64_t ldh, void *const *events,
+                                       int32_t n_events, void *stream);
 
 /*
  * The two-layer Bi-GCN of Sec. 6.2 in one call: a hidden layer of width Fh on

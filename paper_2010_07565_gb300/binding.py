@@ -48,6 +48,8 @@ SIGNATURES = {
     "bigcn_layer_workspace_bytes": ([_i64, _i32, _i32], _sz),
     "bigcn_layer_forward": ([_p, _i64, _i32, _i64, _p, _p, _p, _i32, _i64, _p, _p, _i64, _p,
                              _sz, _p, _i64, _p], ctypes.c_int),
+    "bigcn_layer_forward_timed": ([_p, _i64, _i32, _i64, _p, _p, _p, _i32, _i64, _p, _p, _i64,
+                                   _p, _sz, _p, _i64, _p, _i32, _p], ctypes.c_int),
     "bigcn_forward_2layer_workspace_bytes": ([_i64, _i32, _i32, _i32], _sz),
     "bigcn_forward_2layer_launches": ([_i64, _i32, _i32, _i32], _i32),
     "bigcn_forward_2layer": ([_p, _i64, _i32, _i64, _p, _p, _p, _i32, _i64, _p, _i32, _i64, _p,
@@ -194,6 +196,21 @@ def bigcn_layer_forward(X, scale, shift, Wt, rowptr, colidx, workspace, H, strea
         _ptr(X), N, K, _ld(X), _ptr(scale), _ptr(shift), _ptr(Wt), F, _ld(Wt), _ptr(rowptr),
         _ptr(colidx) if colidx.numel() else None, colidx.numel(), _ptr(workspace),
         workspace.numel() * workspace.element_size(), _ptr(H), _ld(H), _stream(stream)))
+
+
+def bigcn_layer_forward_timed(X, scale, shift, Wt, rowptr, colidx, workspace, H, events,
+                              stream=None):
+    """bigcn_layer_forward recording ``events`` (torch.cuda.Event objects
+    created with enable_timing=True and recorded once, so that the CUDA event
+    exists) before each of its four kernels and after the last."""
+    N, K = X.shape
+    F = Wt.shape[1]
+    ev = (ctypes.c_void_p * len(events))(*[e.cuda_event for e in events])
+    _check("bigcn_layer_forward_timed", lib().bigcn_layer_forward_timed(
+        _ptr(X), N, K, _ld(X), _ptr(scale), _ptr(shift), _ptr(Wt), F, _ld(Wt), _ptr(rowptr),
+        _ptr(colidx) if colidx.numel() else None, colidx.numel(), _ptr(workspace),
+        workspace.numel() * workspace.element_size(), _ptr(H), _ld(H), ev, len(events),
+        _stream(stream)))
 
 
 def bigcn_forward_2layer_workspace_bytes(N: int, K: int, Fh: int, Fo: int) -> int:

@@ -97,6 +97,41 @@ void launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
     cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
 }
 
+// Records caller-supplied timing events between the kernels of an entry
+// point: mark() records the next event of the array (if any is left) on the
+// stream. Inside a stream capture an event must be recorded as an external
+// node to be timed later; outside a capture a plain record does that.
+class EventMarks {
+  public:
+    EventMarks(void *const *events, int32_t n, cudaStream_t s) : events_(events), n_(n), s_(s) {
+        if (n_ > 0 && cudaStreamIsCapturing(s_, &capture_) != cudaSuccess) {
+            cudaGetLastError();
+            ok_ = false;
+        }
+    }
+    bool ok() const { return ok_; }
+    bool failed() const { return failed_; }
+    void mark() {
+        if (recorded_ < n_) {
+            cudaEvent_t ev = static_cast<cudaEvent_t>(events_[recorded_]);
+            const cudaError_t r = capture_ == cudaStreamCaptureStatusActive
+                                      ? cudaEventRecordWithFlags(ev, s_, cudaEventRecordExternal)
+                                      : cudaEventRecord(ev, s_);
+            if (r != cudaSuccess) failed_ = true;
+        }
+        ++recorded_;
+    }
+
+  private:
+    void *const *events_;
+    int32_t n_;
+    cudaStream_t s_;
+    cudaStreamCaptureStatus capture_ = cudaStreamCaptureStatusNone;
+    int32_t recorded_ = 0;
+    bool ok_ = true;
+    bool failed_ = false;
+};
+
 // 1 / sqrt(1 + row length): the D^-1/2 factor of A + I (Sec. 3.1, Eq. 1),
 // with IEEE-rounded sqrt and division.
 __device__ __forceinline__ float inv_sqrt_degree(int64_t row_len) {

@@ -134,25 +134,9 @@ extern "C" bigcn_status bigcn_forward_2layer(
     const int64_t ldz2 = (Fo + 3) / 4 * 4;
     const bool fused = spmm_pack_gemm_supported(Fh, Fo);
     cudaStream_t s = as_stream(stream);
-    // Inside a stream capture an event must be recorded as an external node
-    // to be timed later; outside a capture a plain record does that.
-    cudaStreamCaptureStatus capture = cudaStreamCaptureStatusNone;
-    if (n_events > 0 && cudaStreamIsCapturing(s, &capture) != cudaSuccess) {
-        cudaGetLastError();
-        return BIGCN_ERR_CUDA;
-    }
-    int recorded = 0;
-    bool event_failed = false;
-    auto mark = [&]() {
-        if (recorded < n_events) {
-            cudaEvent_t ev = static_cast<cudaEvent_t>(events[recorded]);
-            const cudaError_t r = capture == cudaStreamCaptureStatusActive
-                                      ? cudaEventRecordWithFlags(ev, s, cudaEventRecordExternal)
-                                      : cudaEventRecord(ev, s);
-            if (r != cudaSuccess) event_failed = true;
-        }
-        ++recorded;
-    };
+    EventMarks marks(events, n_events, s);
+    if (!marks.ok()) return BIGCN_ERR_CUDA;
+    auto mark = [&]() { marks.mark(); };
 
     mark();
     WeightPack p1{W1, K, Fh, ldw1, wbits1, words1, beta1, 0};
@@ -193,5 +177,5 @@ extern "C" bigcn_status bigcn_forward_2layer(
     launch_spmm_norm(a2, dev, s, true);
     mark();
     const bigcn_status ls = launch_status();
-    return event_failed ? BIGCN_ERR_CUDA : ls;
+    return marks.failed() ? BIGCN_ERR_CUDA : ls;
 }

@@ -53,6 +53,13 @@ struct GemmArgs {
     int64_t ldz;
     int32_t *dots;           // nullable N x F raw dots (row stride F)
     const int64_t *rowptr;   // nullable: scale row i by 1/sqrt(1 + deg_i)
+    // Compressed output (nullable; replaces Z): dots + 32768 as uint16 (row
+    // stride ldd16 = F rounded up to 4, padding columns hold 32768, i.e. 0),
+    // and each row's scale alpha_i (times 1/sqrt(1 + deg_i) with rowptr) in
+    // rowscale; Z[i,j] is then rowscale_i * beta_j * dot[i,j]. Needs K <= 32767.
+    uint16_t *dots16 = nullptr;
+    int64_t ldd16 = 0;
+    float *rowscale = nullptr;
 };
 
 // Step 4 on the tensor cores (xnor_gemm_tc.cu): +-1 signs as FP8 E4M3,
@@ -79,6 +86,13 @@ struct SpmmArgs {
     int64_t ldh;
     bool prescaled;          // Z rows already carry their 1/sqrt(dhat_j)
     bool z_pad4;             // Z's columns F .. round_up(F, 4) are readable and finite
+    // Compressed input (nullable; replaces Z): rows of dots + 32768 as uint16
+    // (row stride ldz, a multiple of 4; padding columns hold 32768), with
+    // Z[j,f] = rowscale_j * colscale_f * dot[j,f] and rowscale_j already
+    // including 1/sqrt(dhat_j).
+    const uint16_t *D16 = nullptr;
+    const float *rowscale = nullptr;
+    const float *colscale = nullptr;
 };
 
 // Step 5: H = D^-1/2 (A + I) D^-1/2 Z (Eqs. 1, 13).

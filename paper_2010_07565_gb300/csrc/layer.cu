@@ -7,7 +7,11 @@
 //   -> xnor_gemm whose epilogue also multiplies row j by 1/sqrt(dhat_j)
 //   -> spmm over the pre-scaled rows, which multiplies by 1/sqrt(dhat_i).
 // Folding the source-side degree factor into the product's epilogue saves the
-// aggregation one random read of the CSR row pointers per edge.
+// aggregation one random read of the CSR row pointers per edge. When the dots
+// fit 16 bits (K <= 32767) the product leaves Z factored: the integer dots as
+// biased uint16 and the row scale s_j = alpha_j / sqrt(dhat_j), and the
+// aggregation applies s_j per neighbour and beta_f per column, so each
+// gathered row is half the bytes.
 #include <mutex>
 
 #include "launch.cuh"
@@ -40,20 +44,36 @@ constexpr size_t kAlign = 256;
 size_t round_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 // Workspace carve-up of the fused layer; every piece 256-byte aligned.
+// Largest K whose dots (|dot| <= K) the compressed uint16 form holds.
+constexpr int32_t kMaxDots16K = 32767;
+
+// Workspace carve-up of the fused layer; every piece 256-byte aligned. Z is
+// either fp32 (N x F) or compressed: uint16 dots (N x round_up(F, 4)) and a
+// row scale (N).
 struct LayerWorkspace {
-    size_t a_bits, alpha, b_bits, beta, z, total;
+    size_t a_bits, alpha, b_bits, beta, z, rowscale, total;
+    bool compressed;
 };
 
 bool layer_workspace(int64_t N, int32_t K, int32_t F, LayerWorkspace *w) {
     if (N < 0 || K < 1 || F < 1) return false;
     const int64_t words = bigcn_words(K);
-    if (N > kMaxElems / (words > F ? words : F)) return false;
+    const int64_t F4 = (int64_t(F) + 3) / 4 * 4;
+    if (N > kMaxElems / (words > F4 ? words : F4)) return false;
+    w->compressed = K <= kMaxDots16K;
     size_t off = 0;
     w->a_bits = off; off = round_up(off + size_t(N) * size_t(words) * 8);
     w->alpha = off;  off = round_up(off + size_t(N) * 4);
     w->b_bits = off; off = round_up(off + size_t(F) * size_t(words) * 8);
     w->beta = off;   off = round_up(off + size_t(F) * 4);
-    w->z = off;      off = round_up(off + size_t(N) * size_t(F) * 4);
+    w->z = off;
+    if (w->compressed) {
+        off = round_up(off + size_t(N) * size_t(F4) * 2);
+        w->rowscale = off; off = round_up(off + size_t(N) * 4);
+    } else {
+        off = round_up(off + size_t(N) * size_t(F) * 4);
+        w->rowscale = off;
+    }
     w->total = off;
     return true;
 }
@@ -99,12 +119,15 @@ extern "C" size_t bigcn_layer_workspace_bytes(int64_t N, int32_t K, int32_t F) {
     return layer_workspace(N, K, F, &w) ? w.total : 0;
 }
 
-extern "C" bigcn_status bigcn_layer_forward(const float *X, int64_t N, int32_t K, int64_t ldx,
-                                            const float *scale, const float *shift,
-                                            const float *Wt, int32_t F, int64_t ldw,
-                                            const int64_t *rowptr, const int32_t *colidx,
-                                            int64_t nnz, void *workspace, size_t ws_bytes,
-                                            float *H, int64_t ldh, void *stream) {
+extern "C" bigcn_status bigcn_layer_forward_timed(const float *X, int64_t N, int32_t K,
+                                                  int64_t ldx, const float *scale,
+                                                  const float *shift, const float *Wt, int32_t F,
+                                                  int64_t ldw, const int64_t *rowptr,
+                                                  const int32_t *colidx, int64_t nnz,
+                                                  void *workspace, size_t ws_bytes, float *H,
+                                                  int64_t ldh, void *const *events,
+                                                  int32_t n_events, void *stream) {
+    if (n_events < 0 || (n_events > 0 && !events)) return BIGCN_ERR_INVALID_ARG;
     LayerWorkspace w;
     if (N < 0 || N > int64_t(INT32_MAX) || K < 1 || F < 1 || ldx < K || ldw < F || ldh < F ||
         nnz < 0)
@@ -144,14 +167,46 @@ extern "C" bigcn_status bigcn_layer_forward(const float *X, int64_t N, int32_t K
     float *Zs = reinterpret_cast<float *>(ws + w.z);
     const int words = bigcn_words(K);
     cudaStream_t s = as_stream(stream);
+    EventMarks marks(events, n_events, s);
+    if (!marks.ok()) return BIGCN_ERR_CUDA;
 
+    marks.mark();
     launch_pack_rows(X, N, K, ldx, scale, shift, a_bits, words, alpha, dev, s);
+    marks.mark();
     launch_pack_weights(Wt, K, F, ldw, b_bits, words, beta, s);
+    marks.mark();
     GemmArgs g{a_bits, alpha, N, b_bits, beta, F, K, words, Zs, F, nullptr, rowptr};
-    launch_xnor_gemm(g, dev, s);
     SpmmArgs a{rowptr, colidx, N, nnz, Zs, F, F, H, ldh, true, false};
+    if (w.compressed) {
+        uint16_t *D16 = reinterpret_cast<uint16_t *>(ws + w.z);
+        float *rowscale = reinterpret_cast<float *>(ws + w.rowscale);
+        const int64_t F4 = (int64_t(F) + 3) / 4 * 4;
+        g.Z = nullptr;
+        g.dots16 = D16;
+        g.ldd16 = F4;
+        g.rowscale = rowscale;
+        a.Z = nullptr;
+        a.ldz = F4;
+        a.D16 = D16;
+        a.rowscale = rowscale;
+        a.colscale = beta;
+    }
+    launch_xnor_gemm(g, dev, s);
+    marks.mark();
     launch_spmm_norm(a, dev, s);
-    return launch_status();
+    marks.mark();
+    const bigcn_status ls = launch_status();
+    return marks.failed() ? BIGCN_ERR_CUDA : ls;
+}
+
+extern "C" bigcn_status bigcn_layer_forward(const float *X, int64_t N, int32_t K, int64_t ldx,
+                                            const float *scale, const float *shift,
+                                            const float *Wt, int32_t F, int64_t ldw,
+                                            const int64_t *rowptr, const int32_t *colidx,
+                                            int64_t nnz, void *workspace, size_t ws_bytes,
+                                            float *H, int64_t ldh, void *stream) {
+    return bigcn_layer_forward_timed(X, N, K, ldx, scale, shift, Wt, F, ldw, rowptr, colidx, nnz,
+                                     workspace, ws_bytes, H, ldh, nullptr, 0, stream);
 }
 
 // ---------------------------------------------------------------------------

@@ -5,7 +5,8 @@
 // groups of L lanes; each group gathers a different neighbour's row of Z,
 // lane by lane in VEC-wide vectors (NV per lane), so rows narrower than a
 // warp still keep all 32 lanes busy, and U such gathers are issued before any
-// is consumed (U = 4, or 2 when each lane holds two vectors). Neighbour indices (and, unless Z is pre-scaled, their
+// is consumed (U = 4, or 2 when each lane holds two vectors; twice that for
+// compressed rows spread over all 32 lanes). Neighbour indices (and, unless Z is pre-scaled, their
 // 1/sqrt(dhat_j)) are fetched 32 at a time, one per lane, then broadcast with
 // shuffles. The self-loop that A + I adds is entry 0 of every row's list.
 // Partial sums are combined across groups with xor shuffles and group 0
@@ -20,6 +21,16 @@
 // the block: warp w gathers the w-th eighth of the row's list, the eight
 // partial rows meet in shared memory and warp 0 adds them in warp order
 // (deterministic) before the same epilogue. Light warps skip heavy rows.
+//
+// Rows of Z come in one of three forms (template S): fp32 rows weighted by
+// 1/sqrt(dhat_j) per neighbour (kDinv), fp32 rows that already carry it
+// (kPre), or compressed rows (kDots16) of integer dots stored as uint16 with
+// a bias of 32768, weighted per neighbour by the row scale s_j = alpha_j /
+// sqrt(dhat_j) and, in the epilogue, per column by beta_f:
+//   H_if = (1/sqrt(dhat_i)) * beta_f * sum_j s_j * dot_jf.
+// A compressed row is half the bytes of an fp32 row, and a dot is
+// turned back into a float exactly by placing its 16 bits under the exponent
+// of 2^23 (one byte permute) and subtracting 2^23 + 32768.
 //
 // A grid y dimension splits wide rows into column slabs of L * NV * VEC
 // features. Bounds: the row range is clamped to [0, nnz] and column indices
@@ -62,12 +73,14 @@ template <> struct Vec<4> {
     }
 };
 
+enum : int { kDinv = 0, kPre = 1, kDots16 = 2 };
+
 struct SpmmParams {
     const int64_t *rowptr;
     const int32_t *colidx;
     int64_t N;
     int64_t nnz;
-    const float *Z;
+    const void *Z;           // float rows, or uint16 rows for kDots16
     int64_t ldz;
     int Fload;               // features gathered per row (a multiple of VEC, <= ldz)
     int F;                   // features stored per row (<= Fload)
@@ -76,6 +89,43 @@ struct SpmmParams {
     int heavy_blocks;        // leading blocks that take the heavy rows
     int64_t heavy_degree;    // rows with more neighbours are heavy
     bool vec_store;          // H rows start VEC-aligned: whole vectors may be stored
+    const float *rowscale;   // kDots16: s_j
+    const float *colscale;   // kDots16: beta_f
+};
+
+// How a lane loads VEC consecutive entries of a row of Z and adds them,
+// weighted, into its accumulators.
+template <int VEC, int S>
+struct RowSrc {
+    using T = typename Vec<VEC>::T;
+    static __device__ __forceinline__ T load(const void *Z, int64_t row, int64_t ldz, int f) {
+        return __ldg(reinterpret_cast<const T *>(static_cast<const float *>(Z) + row * ldz + f));
+    }
+    static __device__ __forceinline__ void fma(float *acc, const T &v, float w) {
+        Vec<VEC>::fma(acc, v, w);
+    }
+};
+
+// A dot stored as uint16 with a bias of 32768, back to an exact float.
+__device__ __forceinline__ float dot16_lo(uint32_t w) {
+    return __int_as_float(int(__byte_perm(w, 0x4B000000u, 0x7410))) - 8421376.0f;
+}
+__device__ __forceinline__ float dot16_hi(uint32_t w) {
+    return __int_as_float(int(__byte_perm(w, 0x4B000000u, 0x7432))) - 8421376.0f;
+}
+
+template <>
+struct RowSrc<4, kDots16> {
+    using T = uint2;
+    static __device__ __forceinline__ T load(const void *Z, int64_t row, int64_t ldz, int f) {
+        return __ldg(reinterpret_cast<const uint2 *>(static_cast<const uint16_t *>(Z) + row * ldz + f));
+    }
+    static __device__ __forceinline__ void fma(float *acc, const T &v, float w) {
+        acc[0] = fmaf(w, dot16_lo(v.x), acc[0]);
+        acc[1] = fmaf(w, dot16_hi(v.x), acc[1]);
+        acc[2] = fmaf(w, dot16_lo(v.y), acc[2]);
+        acc[3] = fmaf(w, dot16_hi(v.y), acc[3]);
+    }
 };
 
 // Row i's neighbour list: CSR entries [b, b + total - 1) plus the self-loop.
@@ -94,11 +144,12 @@ __device__ __forceinline__ RowSpan row_span(const int64_t *__restrict__ rowptr, 
 }
 
 // Adds, into acc, the Z rows of entries [q0, q1) of row i's list (entry 0 is
-// the self-loop), weighted by 1/sqrt(dhat_j) unless Z is pre-scaled.
-template <int VEC, int L, int NV, int U, bool kPre>
+// the self-loop), weighted by 1/sqrt(dhat_j) (kDinv), 1 (kPre) or s_j (kDots16).
+template <int VEC, int L, int NV, int U, int S>
 __device__ __forceinline__ void gather(const SpmmParams &p, int64_t i, int64_t b, int64_t q0,
                                        int64_t q1, int f0, float (&acc)[NV][VEC]) {
-    using V = typename Vec<VEC>::T;
+    using Src = RowSrc<VEC, S>;
+    using V = typename Src::T;
     constexpr int P = 32 / L;
     const int lane = threadIdx.x & 31;
     const int g = lane / L, sl = lane % L;
@@ -110,8 +161,10 @@ __device__ __forceinline__ void gather(const SpmmParams &p, int64_t i, int64_t b
             j = (q == 0) ? int(i) : __ldg(p.colidx + b + q - 1);
             if (j < 0 || j >= p.N) j = -1;
             if (j >= 0)
-                wj = kPre ? 1.0f
-                          : inv_sqrt_degree(__ldg(p.rowptr + j + 1) - __ldg(p.rowptr + j));
+                wj = S == kPre ? 1.0f
+                               : S == kDots16
+                                     ? __ldg(p.rowscale + j)
+                                     : inv_sqrt_degree(__ldg(p.rowptr + j + 1) - __ldg(p.rowptr + j));
         }
         const int cnt = int(min(q1 - base, int64_t(32)));
         for (int t0 = 0; t0 < cnt; t0 += P * U) {
@@ -124,18 +177,18 @@ __device__ __forceinline__ void gather(const SpmmParams &p, int64_t i, int64_t b
                 w[u] = __shfl_sync(kFullMask, wj, src & 31);
                 const bool live = src < cnt && jj >= 0;
                 if (!live) w[u] = 0.0f;
-                const float *zr = p.Z + int64_t(live ? jj : 0) * p.ldz;
+                const int64_t zrow = live ? jj : 0;
 #pragma unroll
                 for (int v = 0; v < NV; ++v) {
                     const int f = f0 + (v * L + sl) * VEC;
-                    if (live && f < p.Fload) val[u][v] = __ldg(reinterpret_cast<const V *>(zr + f));
+                    if (live && f < p.Fload) val[u][v] = Src::load(p.Z, zrow, p.ldz, f);
                     else val[u][v] = V{};
                 }
             }
 #pragma unroll
             for (int u = 0; u < U; ++u)
 #pragma unroll
-                for (int v = 0; v < NV; ++v) Vec<VEC>::fma(acc[v], val[u][v], w[u]);
+                for (int v = 0; v < NV; ++v) Src::fma(acc[v], val[u][v], w[u]);
         }
     }
 }
@@ -150,8 +203,9 @@ __device__ __forceinline__ void reduce_groups(float (&acc)[NV][VEC]) {
             for (int c = 0; c < VEC; ++c) acc[v][c] += __shfl_xor_sync(kFullMask, acc[v][c], o);
 }
 
-// Epilogue of the plain aggregation: H_i = dinv_i * acc (lanes of group 0).
-template <int VEC, int L, int NV>
+// Epilogue of the plain aggregation: H_i = dinv_i * acc, or for compressed
+// rows H_if = dinv_i * (beta_f * acc_f) (lanes of group 0).
+template <int VEC, int L, int NV, int S>
 struct StoreRow {
     __device__ __forceinline__ void prologue() const {}
     __device__ __forceinline__ void operator()(const SpmmParams &p, int64_t i, float dinv,
@@ -165,7 +219,12 @@ struct StoreRow {
             const int f = f0 + (v * L + sl) * VEC;
             float o[VEC];
 #pragma unroll
-            for (int c = 0; c < VEC; ++c) o[c] = acc[v][c] * dinv;
+            for (int c = 0; c < VEC; ++c) {
+                if (S == kDots16)
+                    o[c] = f + c < p.F ? dinv * (__ldg(p.colscale + f + c) * acc[v][c]) : 0.0f;
+                else
+                    o[c] = acc[v][c] * dinv;
+            }
             float *h = p.H + i * p.ldh + f;
             if (p.vec_store && f + VEC <= p.F) {
                 *reinterpret_cast<V *>(h) = Vec<VEC>::make(o);
@@ -178,7 +237,7 @@ struct StoreRow {
     }
 };
 
-template <int VEC, int L, int NV, int U, bool kPre, class Epi>
+template <int VEC, int L, int NV, int U, int S, class Epi>
 __device__ __forceinline__ void light_rows(const SpmmParams &p, const Epi &epi, int f0) {
     const int warp = threadIdx.x >> 5;
     const int64_t i = int64_t(blockIdx.x - p.heavy_blocks) * kSpmmWarps + warp;
@@ -190,12 +249,12 @@ __device__ __forceinline__ void light_rows(const SpmmParams &p, const Epi &epi, 
     for (int v = 0; v < NV; ++v)
 #pragma unroll
         for (int c = 0; c < VEC; ++c) acc[v][c] = 0.0f;
-    gather<VEC, L, NV, U, kPre>(p, i, sp.b, 0, sp.total, f0, acc);
+    gather<VEC, L, NV, U, S>(p, i, sp.b, 0, sp.total, f0, acc);
     reduce_groups<VEC, L, NV>(acc);
     epi(p, i, sp.dinv, f0, acc);
 }
 
-template <int VEC, int L, int NV, int U, bool kPre, class Epi>
+template <int VEC, int L, int NV, int U, int S, class Epi>
 __device__ __forceinline__ void heavy_rows(const SpmmParams &p, const Epi &epi, int f0,
                                            float *part, unsigned *mask) {
     constexpr int SLAB = L * NV * VEC;
@@ -223,7 +282,7 @@ __device__ __forceinline__ void heavy_rows(const SpmmParams &p, const Epi &epi, 
                     for (int c = 0; c < VEC; ++c) acc[v][c] = 0.0f;
                 const int64_t q0 = sp.total * warp / kSpmmWarps;
                 const int64_t q1 = sp.total * (warp + 1) / kSpmmWarps;
-                gather<VEC, L, NV, U, kPre>(p, i, sp.b, q0, q1, f0, acc);
+                gather<VEC, L, NV, U, S>(p, i, sp.b, q0, q1, f0, acc);
                 reduce_groups<VEC, L, NV>(acc);
                 if (g == 0) {
 #pragma unroll
@@ -253,19 +312,19 @@ __device__ __forceinline__ void heavy_rows(const SpmmParams &p, const Epi &epi, 
     }
 }
 
-template <int VEC, int L, int NV, int U, bool kPre>
-__global__ void __launch_bounds__(kSpmmThreads, 3)
+template <int VEC, int L, int NV, int U, int S>
+__global__ void __launch_bounds__(kSpmmThreads, 4)
 spmm_norm_kernel(SpmmParams p) {
     constexpr int SLAB = L * NV * VEC;
     __shared__ float part[kSpmmWarps * SLAB];
     __shared__ unsigned mask[kSpmmWarps];
     grid_dependency_wait();     // Z is the output of the previous kernel
     const int f0 = blockIdx.y * SLAB;
-    StoreRow<VEC, L, NV> epi;
+    StoreRow<VEC, L, NV, S> epi;
     if (int(blockIdx.x) < p.heavy_blocks)
-        heavy_rows<VEC, L, NV, U, kPre>(p, epi, f0, part, mask);
+        heavy_rows<VEC, L, NV, U, S>(p, epi, f0, part, mask);
     else
-        light_rows<VEC, L, NV, U, kPre>(p, epi, f0);
+        light_rows<VEC, L, NV, U, S>(p, epi, f0);
 }
 
 // ---------------------------------------------------------------------------
@@ -364,9 +423,9 @@ spmm_pack_gemm_kernel(SpmmParams p, FusedLayer2 f, const uint64_t *__restrict__ 
     f.sBeta = sBeta;
     PackGemmRow<L> epi{f};
     if (int(blockIdx.x) < p.heavy_blocks)
-        heavy_rows<4, L, 1, 4, true>(p, epi, 0, part, mask);
+        heavy_rows<4, L, 1, 4, kPre>(p, epi, 0, part, mask);
     else
-        light_rows<4, L, 1, 4, true>(p, epi, 0);
+        light_rows<4, L, 1, 4, kPre>(p, epi, 0);
 }
 
 // Leading blocks that look for heavy rows: up to two per SM, one per 256 rows.
@@ -384,51 +443,62 @@ int64_t heavy_degree(int64_t N, int64_t nnz, int per_iter) {
     return h > 32 ? h : 32;
 }
 
-template <int VEC, int L, int NV, bool kPre>
+template <int VEC, int L, int NV, int S>
 void launch_cfg(const SpmmArgs &a, const DeviceInfo &dev, int Fload, cudaStream_t s, bool pdl) {
     constexpr int SLAB = L * NV * VEC;
-    constexpr int U = NV == 1 ? 4 : 2;
+    // Rows in flight per group. A compressed row costs half the registers, so
+    // where a warp holds only a few rows at a time (one row across all 32
+    // lanes) it takes twice as many.
+    constexpr int U = (S == kDots16 && L == 32 ? 2 : 1) * (NV == 1 ? 4 : 2);
     const bool vec_store = a.ldh % VEC == 0 && aligned_to(a.H, size_t(VEC) * 4);
-    SpmmParams p{a.rowptr, a.colidx, a.N, a.nnz, a.Z, a.ldz, Fload, a.F, a.H, a.ldh,
-                 heavy_block_count(a.N, dev), heavy_degree(a.N, a.nnz, (32 / L) * U), vec_store};
+    const void *Z = S == kDots16 ? static_cast<const void *>(a.D16) : a.Z;
+    SpmmParams p{a.rowptr, a.colidx, a.N, a.nnz, Z, a.ldz, Fload, a.F, a.H, a.ldh,
+                 heavy_block_count(a.N, dev), heavy_degree(a.N, a.nnz, (32 / L) * U), vec_store,
+                 a.rowscale, a.colscale};
     dim3 grid(unsigned(p.heavy_blocks + (a.N + kSpmmWarps - 1) / kSpmmWarps),
               unsigned((a.F + SLAB - 1) / SLAB));
-    launch_kernel(spmm_norm_kernel<VEC, L, NV, U, kPre>, grid, dim3(kSpmmThreads), 0, s, pdl,
+    launch_kernel(spmm_norm_kernel<VEC, L, NV, U, S>, grid, dim3(kSpmmThreads), 0, s, pdl,
                   dim3(1, 1, 1), p);
 }
 
 // Lanes per neighbour L = the power of two >= the row's vector count (at
 // least 4, at most 32); NV = 2 vectors per lane once a row exceeds 32.
-template <int VEC, bool kPre>
+template <int VEC, int S>
 void launch_vec(const SpmmArgs &a, const DeviceInfo &dev, int Fload, cudaStream_t s, bool pdl) {
     const int nvec = Fload / VEC;
-    if (nvec <= 4) launch_cfg<VEC, 4, 1, kPre>(a, dev, Fload, s, pdl);
-    else if (nvec <= 8) launch_cfg<VEC, 8, 1, kPre>(a, dev, Fload, s, pdl);
-    else if (nvec <= 16) launch_cfg<VEC, 16, 1, kPre>(a, dev, Fload, s, pdl);
-    else if (nvec <= 32) launch_cfg<VEC, 32, 1, kPre>(a, dev, Fload, s, pdl);
-    else launch_cfg<VEC, 32, 2, kPre>(a, dev, Fload, s, pdl);
+    if (nvec <= 4) launch_cfg<VEC, 4, 1, S>(a, dev, Fload, s, pdl);
+    else if (nvec <= 8) launch_cfg<VEC, 8, 1, S>(a, dev, Fload, s, pdl);
+    else if (nvec <= 16) launch_cfg<VEC, 16, 1, S>(a, dev, Fload, s, pdl);
+    else if (nvec <= 32) launch_cfg<VEC, 32, 1, S>(a, dev, Fload, s, pdl);
+    else launch_cfg<VEC, 32, 2, S>(a, dev, Fload, s, pdl);
 }
 
-template <bool kPre>
-void launch_pre(const SpmmArgs &a, const DeviceInfo &dev, cudaStream_t s, bool pdl) {
+template <int S>
+void launch_src(const SpmmArgs &a, const DeviceInfo &dev, cudaStream_t s, bool pdl) {
     auto al = [](const void *p, int n) { return aligned_to(p, size_t(n) * 4); };
     // Gathers may read whole vectors past F when the padding up to a multiple
     // of 4 lies inside the row stride and is declared readable (a.z_pad4).
     const int F4 = (a.F + 3) / 4 * 4;
     if (a.ldz % 4 == 0 && al(a.Z, 4) && (a.F % 4 == 0 || (a.z_pad4 && F4 <= a.ldz)))
-        launch_vec<4, kPre>(a, dev, F4, s, pdl);
+        launch_vec<4, S>(a, dev, F4, s, pdl);
     else if (a.F % 2 == 0 && a.ldz % 2 == 0 && a.ldh % 2 == 0 && al(a.Z, 2) && al(a.H, 2))
-        launch_vec<2, kPre>(a, dev, a.F, s, pdl);
+        launch_vec<2, S>(a, dev, a.F, s, pdl);
     else
-        launch_vec<1, kPre>(a, dev, a.F, s, pdl);
+        launch_vec<1, S>(a, dev, a.F, s, pdl);
 }
 
 }  // namespace
 
 void launch_spmm_norm(const SpmmArgs &a, const DeviceInfo &dev, cudaStream_t stream, bool pdl) {
     if (a.N == 0) return;
-    if (a.prescaled) launch_pre<true>(a, dev, stream, pdl);
-    else launch_pre<false>(a, dev, stream, pdl);
+    if (a.D16 != nullptr) {
+        // Compressed rows: four dots (8 bytes) per vector; the row stride is a
+        // multiple of 4 and its padding columns hold a zero dot.
+        launch_vec<4, kDots16>(a, dev, (a.F + 3) / 4 * 4, stream, pdl);
+        return;
+    }
+    if (a.prescaled) launch_src<kPre>(a, dev, stream, pdl);
+    else launch_src<kDinv>(a, dev, stream, pdl);
 }
 
 bool spmm_pack_gemm_supported(int Fh, int Fo) {
@@ -442,7 +512,8 @@ void launch_spmm_pack_gemm(const SpmmPackGemmArgs &a, const DeviceInfo &dev, cud
     int L = 4;
     while (L < 32 && L < nvec) L *= 2;
     SpmmParams p{a.rowptr, a.colidx, a.N, a.nnz, a.Z1, a.Fh, a.Fh, a.Fh, nullptr, 0,
-                 heavy_block_count(a.N, dev), heavy_degree(a.N, a.nnz, (32 / L) * 4), false};
+                 heavy_block_count(a.N, dev), heavy_degree(a.N, a.nnz, (32 / L) * 4), false,
+                 nullptr, nullptr};
     FusedLayer2 f{a.H1, a.ldh, nullptr, nullptr, a.Fo, (a.Fh + 63) / 64, a.Z2, a.ldz2};
     const dim3 grid(unsigned(p.heavy_blocks + (a.N + kSpmmWarps - 1) / kSpmmWarps));
     const dim3 one(1, 1, 1), block(kSpmmThreads);

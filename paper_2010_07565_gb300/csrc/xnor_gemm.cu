@@ -42,7 +42,8 @@ __global__ void __launch_bounds__(kThreads)
 xnor_gemm_popc_kernel(const uint64_t *__restrict__ A, const float *__restrict__ alpha, int64_t N,
                       const uint64_t *__restrict__ B, const float *__restrict__ beta, int F,
                       int K, int words, float *__restrict__ Z, int64_t ldz,
-                      int32_t *__restrict__ dots, const int64_t *__restrict__ rowptr) {
+                      int32_t *__restrict__ dots, const int64_t *__restrict__ rowptr,
+                      uint16_t *__restrict__ dots16, int64_t ldd16, float *__restrict__ rowscale) {
     constexpr int BN = 16 * TN;
     constexpr int kALoads = kBM * kBKW / kThreads;                         // 4
     constexpr int kBLoads = (BN * kBKW + kThreads - 1) / kThreads;          // 1..2
@@ -142,6 +143,17 @@ xnor_gemm_popc_kernel(const uint64_t *__restrict__ A, const float *__restrict__ 
         if (row >= N) continue;
         float ai = __ldg(alpha + row);
         if (kDegreeScale) ai *= inv_sqrt_degree(__ldg(rowptr + row + 1) - __ldg(rowptr + row));
+        if (dots16 != nullptr) {            // compressed output: biased dots + row scale
+            if (n0 == 0 && tx == 0) rowscale[row] = ai;
+#pragma unroll
+            for (int j = 0; j < TN; ++j) {
+                const int col = n0 + tx + 16 * j;
+                if (col < ldd16)
+                    dots16[row * ldd16 + col] =
+                        uint16_t(col < F ? K - 2 * mism[i][j] + 32768 : 32768);
+            }
+            continue;
+        }
 #pragma unroll
         for (int j = 0; j < TN; ++j) {
             const int col = n0 + tx + 16 * j;
@@ -171,12 +183,12 @@ void launch_tn(const GemmArgs &g, const DeviceInfo &dev, cudaStream_t s, bool pd
     if (S == 1) {
         launch_kernel(xnor_gemm_popc_kernel<TN, kDeg, false>, dim3(gx, gy), dim3(kThreads), 0, s,
                       pdl, dim3(1, 1, 1), g.A, g.alpha, g.N, g.B, g.beta, g.F, g.K, g.words, g.Z,
-                      g.ldz, g.dots, g.rowptr);
+                      g.ldz, g.dots, g.rowptr, g.dots16, g.ldd16, g.rowscale);
         return;
     }
     launch_kernel(xnor_gemm_popc_kernel<TN, kDeg, true>, dim3(gx, gy, S), dim3(kThreads), 0, s,
                   pdl, dim3(1, 1, S), g.A, g.alpha, g.N, g.B, g.beta, g.F, g.K, g.words, g.Z,
-                  g.ldz, g.dots, g.rowptr);
+                  g.ldz, g.dots, g.rowptr, g.dots16, g.ldd16, g.rowscale);
 }
 
 template <bool kDeg>

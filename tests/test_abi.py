@@ -60,10 +60,15 @@ def test_words_and_status_strings(lib):
 def test_workspace_bytes(lib):
     assert lib.bigcn_layer_workspace_bytes(0, 0, 5) == 0
     assert lib.bigcn_layer_workspace_bytes(-1, 10, 5) == 0
-    n = lib.bigcn_layer_workspace_bytes(1000, 130, 64)
-    need = 1000 * 3 * 8 + 1000 * 4 + 64 * 3 * 8 + 64 * 4 + 1000 * 64 * 4
-    assert need <= n <= need + 5 * 256 and n % 256 == 0
-    assert lib.bigcn_layer_workspace_bytes(2000, 130, 64) > n
+    # K <= 32767: Z kept factored as uint16 dots (rows padded to 4) plus a row scale
+    n = lib.bigcn_layer_workspace_bytes(1000, 130, 62)
+    need = 1000 * 3 * 8 + 1000 * 4 + 62 * 3 * 8 + 62 * 4 + 1000 * 64 * 2 + 1000 * 4
+    assert need <= n <= need + 6 * 256 and n % 256 == 0
+    assert lib.bigcn_layer_workspace_bytes(2000, 130, 62) > n
+    # larger K: fp32 Z
+    n = lib.bigcn_layer_workspace_bytes(100, 40000, 5)
+    need = 100 * 625 * 8 + 100 * 4 + 5 * 625 * 8 + 5 * 4 + 100 * 5 * 4
+    assert need <= n <= need + 6 * 256 and n % 256 == 0
 
 
 def test_pack_rows_argument_checks(lib):

@@ -233,7 +233,10 @@ def test_layer_forward_equals_step_by_step(cuda_device):
     Z = B.xnor_gemm(bits, alpha, wbits, beta, 300)
     H_steps = B.spmm_norm(d["rowptr"], d["colidx"], Z).cpu().numpy()
     H_fused = B.layer_forward(d["X"], d["W"], d["rowptr"], d["colidx"], d["s"], d["t"])
-    assert_close(H_fused, H_steps.astype(np.float64), "fused vs steps", rtol=2e-6, atol=1e-7)
+    # The fused layer keeps Z factored (integer dots, row scale, column scale)
+    # and so adds the same fp32 terms in another order: equal to the steps
+    # within the parity tolerance, not bit for bit.
+    assert_close(H_fused, H_steps.astype(np.float64), "fused vs steps")
 
 
 def test_layer_forward_strided_and_workspace_reuse(cuda_device):
