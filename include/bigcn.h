@@ -237,8 +237,10 @@ bigcn_status bigcn_layer_forward_timed(const float *X, int64_t N, int32_t K, int
  * (Fh <= 128 and the packed tiles fit); and when Fh is a multiple of 4 and at
  * most 128 and Fo <= 64, layer 1's aggregation kernel also binarizes H1 and
  * computes layer 2's XNOR product while the row is in registers, so H1 never
- * goes through memory. The call launches 4 to 7 kernels
- * (bigcn_forward_2layer_launches).
+ * goes through memory. When K <= 32767, layer 1's Z' stays factored in the
+ * workspace (integer dots as biased uint16 and a row scale, as in
+ * bigcn_layer_forward), so its aggregation gathers half-size rows. The call
+ * launches 4 to 7 kernels (bigcn_forward_2layer_launches).
  *
  * X N x K (ldx), W1 K x Fh (ldw1), W2 Fh x Fo (ldw2), CSR as in
  * bigcn_spmm_norm, out N x Fo (ldo).

@@ -27,27 +27,39 @@ namespace {
 constexpr size_t kAlign = 256;
 size_t round_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
+// Largest K (or Fh) whose dots the compressed uint16 form holds.
+constexpr int32_t kMaxDots16K = 32767;
+
+// Workspace carve-up. Layer 1's Z' is fp32 (N x Fh) or, when K <= 32767,
+// compressed: uint16 dots (N x Fh4, Fh4 = Fh rounded up to 4) and a row
+// scale. Layer 2's Z' is fp32, pre-scaled, with rows padded to a multiple of
+// 4 (its rows are narrow: the extra row-scale read would cost more than the
+// bytes a compressed row saves).
 struct Forward2Workspace {
-    size_t bits1, alpha1, wbits1, beta1, z1, wbits2, beta2, z2, h1, bits2, alpha2, total;
+    size_t bits1, alpha1, wbits1, beta1, z1, s1, wbits2, beta2, z2, h1, bits2, alpha2, total;
+    bool c16;
 };
 
 bool forward2_workspace(int64_t N, int32_t K, int32_t Fh, int32_t Fo, Forward2Workspace *w) {
     if (N < 0 || K < 1 || Fh < 1 || Fo < 1) return false;
     const int64_t w1 = bigcn_words(K), w2 = bigcn_words(Fh);
+    const int64_t Fh4 = (int64_t(Fh) + 3) / 4 * 4, Fo4 = (int64_t(Fo) + 3) / 4 * 4;
     int64_t widest = w1;
-    if (Fh > widest) widest = Fh;
-    if (Fo > widest) widest = Fo;
+    if (Fh4 > widest) widest = Fh4;
+    if (Fo4 > widest) widest = Fo4;
     if (N > kMaxElems / widest) return false;
+    w->c16 = K <= kMaxDots16K;
     size_t off = 0;
     auto take = [&](size_t bytes) { size_t at = off; off = round_up(off + bytes); return at; };
     w->bits1 = take(size_t(N) * w1 * 8);
     w->alpha1 = take(size_t(N) * 4);
     w->wbits1 = take(size_t(Fh) * w1 * 8);
     w->beta1 = take(size_t(Fh) * 4);
-    w->z1 = take(size_t(N) * Fh * 4);
+    w->z1 = take(w->c16 ? size_t(N) * Fh4 * 2 : size_t(N) * Fh * 4);
+    w->s1 = take(size_t(N) * 4);
     w->wbits2 = take(size_t(Fo) * w2 * 8);
     w->beta2 = take(size_t(Fo) * 4);
-    w->z2 = take(size_t(N) * ((Fo + 3) / 4 * 4) * 4);
+    w->z2 = take(size_t(N) * Fo4 * 4);
     w->h1 = take(size_t(N) * Fh * 4);
     w->bits2 = take(size_t(N) * w2 * 8);
     w->alpha2 = take(size_t(N) * 4);
@@ -124,15 +136,16 @@ extern "C" bigcn_status bigcn_forward_2layer(
     float *alpha1 = static_cast<float *>(at(w.alpha1));
     uint64_t *wbits1 = static_cast<uint64_t *>(at(w.wbits1));
     float *beta1 = static_cast<float *>(at(w.beta1));
-    float *Z1 = static_cast<float *>(at(w.z1));
+    void *Z1 = at(w.z1);
+    float *s1 = static_cast<float *>(at(w.s1));
     uint64_t *wbits2 = static_cast<uint64_t *>(at(w.wbits2));
     float *beta2 = static_cast<float *>(at(w.beta2));
     float *Z2 = static_cast<float *>(at(w.z2));
     const int words1 = bigcn_words(K), words2 = bigcn_words(Fh);
-    // Z2' rows are padded to a multiple of 4 floats; the fused kernel writes
-    // the padding as zeros, which lets the layer-2 aggregation gather float4s.
-    const int64_t ldz2 = (Fo + 3) / 4 * 4;
+    const int64_t Fh4 = (Fh + 3) / 4 * 4, Fo4 = (Fo + 3) / 4 * 4;
     const bool fused = spmm_pack_gemm_supported(Fh, Fo);
+    uint16_t *D1 = w.c16 ? static_cast<uint16_t *>(Z1) : nullptr;
+    float *Z1f = w.c16 ? nullptr : static_cast<float *>(Z1);
     cudaStream_t s = as_stream(stream);
     EventMarks marks(events, n_events, s);
     if (!marks.ok()) return BIGCN_ERR_CUDA;
@@ -144,18 +157,29 @@ extern "C" bigcn_status bigcn_forward_2layer(
     launch_pack_weights2(p1, p2, s);
     mark();
     if (front_supported(N, K, Fh, dev)) {
-        FrontArgs fr{X, N, K, ldx, scale, shift, wbits1, beta1, Fh, words1, rowptr, Z1, Fh};
+        FrontArgs fr{X, N, K, ldx, scale, shift, wbits1, beta1, Fh, words1, rowptr, Z1f, Fh};
+        if (w.c16) {
+            fr.D16 = D1;
+            fr.ldd16 = Fh4;
+            fr.rowscale = s1;
+        }
         launch_front(fr, dev, s, true);
         mark();
     } else {
         launch_pack_rows(X, N, K, ldx, scale, shift, bits1, words1, alpha1, dev, s, true, false);
         mark();
-        GemmArgs g1{bits1, alpha1, N, wbits1, beta1, Fh, K, words1, Z1, Fh, nullptr, rowptr};
+        GemmArgs g1{bits1, alpha1, N, wbits1, beta1, Fh, K, words1, Z1f, Fh, nullptr, rowptr};
+        if (w.c16) {
+            g1.dots16 = D1;
+            g1.ldd16 = Fh4;
+            g1.rowscale = s1;
+        }
         launch_xnor_gemm(g1, dev, s, true);
         mark();
     }
     if (fused) {
-        SpmmPackGemmArgs f{rowptr, colidx, N, nnz, Z1, Fh, H1, ldh1, wbits2, beta2, Fo, Z2, ldz2};
+        SpmmPackGemmArgs f{rowptr, colidx, N, nnz, Z1f, D1, s1, beta1, Fh, H1, ldh1, wbits2,
+                           beta2, Fo, Z2, Fo4};
         launch_spmm_pack_gemm(f, dev, s, true);
         mark();
     } else {
@@ -163,17 +187,24 @@ extern "C" bigcn_status bigcn_forward_2layer(
         const int64_t ldh = H1 ? ldh1 : Fh;
         uint64_t *bits2 = static_cast<uint64_t *>(at(w.bits2));
         float *alpha2 = static_cast<float *>(at(w.alpha2));
-        SpmmArgs a1{rowptr, colidx, N, nnz, Z1, Fh, Fh, H1w, ldh, true, false};
+        SpmmArgs a1{rowptr, colidx, N, nnz, Z1f, w.c16 ? Fh4 : Fh, Fh, H1w, ldh, true, false};
+        if (w.c16) {
+            a1.D16 = D1;
+            a1.rowscale = s1;
+            a1.colscale = beta1;
+        }
         launch_spmm_norm(a1, dev, s, true);
         mark();
         launch_pack_rows(H1w, N, Fh, ldh, nullptr, nullptr, bits2, words2, alpha2, dev, s, true,
                          true);
         mark();
-        GemmArgs g2{bits2, alpha2, N, wbits2, beta2, Fo, Fh, words2, Z2, ldz2, nullptr, rowptr};
+        GemmArgs g2{bits2, alpha2, N, wbits2, beta2, Fo, Fh, words2, Z2, Fo4, nullptr, rowptr};
         launch_xnor_gemm(g2, dev, s, true);
         mark();
     }
-    SpmmArgs a2{rowptr, colidx, N, nnz, Z2, ldz2, Fo, out, ldo, true, fused};
+    // The fused kernel writes Z2's padding columns as zeros: whole 4-wide
+    // vectors may be gathered.
+    SpmmArgs a2{rowptr, colidx, N, nnz, Z2, Fo4, Fo, out, ldo, true, fused};
     launch_spmm_norm(a2, dev, s, true);
     mark();
     const bigcn_status ls = launch_status();

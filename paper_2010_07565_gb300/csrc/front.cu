@@ -14,6 +14,11 @@
 // memory (odd row pitch: conflict-free). Several blocks per SM overlap one
 // block's HBM-bound phase A with another's POPC-bound phase B.
 //
+// Either kernel can leave Z' factored instead (D16 non-null, K <= 32767):
+// the integer dots as uint16 with a bias of 32768 (rows padded to a multiple
+// of 4 with zero dots) and the row scale alpha_i / sqrt(dhat_i), for an
+// aggregation that gathers half-size rows and applies beta per column.
+//
 // The packed weight columns and beta come from the weight-packing kernel
 // that runs first. This whole-row kernel is used when there are enough rows
 // to give every warp its own, both packed tiles fit in shared memory and rows
@@ -42,7 +47,8 @@ __global__ void __launch_bounds__(kFrontThreads)
 front_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
              const float *__restrict__ scale, const float *__restrict__ shift,
              const uint64_t *__restrict__ wbits, const float *__restrict__ beta, int F, int words,
-             const int64_t *__restrict__ rowptr, float *__restrict__ Z, int64_t ldz) {
+             const int64_t *__restrict__ rowptr, float *__restrict__ Z, int64_t ldz,
+             uint16_t *__restrict__ D16, int64_t ldd16, float *__restrict__ rowscale) {
     constexpr int BM = 16 * RI;
     extern __shared__ __align__(16) unsigned char smem[];
     const int pitch = words + 1;
@@ -107,6 +113,17 @@ front_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
         if (row >= N) continue;
         const float ai = sAlpha[rg + 16 * i] *
                          inv_sqrt_degree(__ldg(rowptr + row + 1) - __ldg(rowptr + row));
+        if (D16 != nullptr) {               // compressed output: biased dots + row scale
+            if (cg == 0) rowscale[row] = ai;
+#pragma unroll
+            for (int j = 0; j < CJ; ++j) {
+                const int col = cg + 16 * j;
+                if (col < ldd16)
+                    D16[row * ldd16 + col] =
+                        uint16_t(col < F ? K - 2 * mism[i][j] + 32768 : 32768);
+            }
+            continue;
+        }
 #pragma unroll
         for (int j = 0; j < CJ; ++j) {
             const int col = cg + 16 * j;
@@ -122,7 +139,7 @@ void launch_ri_cj(const FrontArgs &a, int BM, size_t smem, cudaStream_t s, bool 
                          int(smem));
     launch_kernel(front_kernel<RI, CJ>, dim3(grid), dim3(kFrontThreads), smem, s, pdl,
                   dim3(1, 1, 1), a.X, a.N, a.K, a.ldx, a.scale, a.shift, a.wbits, a.beta, a.F,
-                  a.words, a.rowptr, a.Z, a.ldz);
+                  a.words, a.rowptr, a.Z, a.ldz, a.D16, a.ldd16, a.rowscale);
 }
 
 template <int RI>
@@ -185,7 +202,8 @@ front_split_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
                    const float *__restrict__ scale, const float *__restrict__ shift,
                    const uint64_t *__restrict__ wbits, const float *__restrict__ beta, int F,
                    int words, const int64_t *__restrict__ rowptr, float *__restrict__ Z,
-                   int64_t ldz, int P) {
+                   int64_t ldz, uint16_t *__restrict__ D16, int64_t ldd16,
+                   float *__restrict__ rowscale, int P) {
     extern __shared__ __align__(16) unsigned char smem[];
     __shared__ float part[kSplitWarps];
     constexpr int R = kSplitWarps / G;       // rows per group
@@ -198,7 +216,8 @@ front_split_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int rr = tid / T, tt = tid % T, sub = tt % P;
     const int cstep = T / P;                 // columns per pass
-    const int passes = (F + cstep - 1) / cstep;
+    const int Fw = D16 != nullptr ? int(ldd16) : F;   // columns written (with padding)
+    const int passes = (Fw + cstep - 1) / cstep;
     if (kAffine) {
         for (int k0 = tid; k0 < K; k0 += 4 * kSplitThreads) {
             float2 v[4];
@@ -248,6 +267,7 @@ front_split_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
             for (int g = 0; g < G; ++g) t += part[rr * G + g];
             const float ai = (t / float(K)) *
                              inv_sqrt_degree(__ldg(rowptr + row2 + 1) - __ldg(rowptr + row2));
+            if (D16 != nullptr && tt == 0) rowscale[row2] = ai;
             const uint64_t *a = As + size_t(rr) * pitch;
             for (int j = 0; j < passes; ++j) {
                 const int c = tt / P + j * cstep;
@@ -255,7 +275,10 @@ front_split_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
                 if (c < F)
                     for (int w = sub; w < words; w += P) mism += __popcll(a[w] ^ Ws[c * pitch + w]);
                 for (int o = 1; o < P; o <<= 1) mism += __shfl_xor_sync(kFullMask, mism, o);
-                if (sub == 0 && c < F)
+                if (sub != 0 || c >= Fw) continue;
+                if (D16 != nullptr)
+                    D16[row2 * ldd16 + c] = uint16_t(c < F ? K - 2 * mism + 32768 : 32768);
+                else
                     Z[row2 * ldz + c] = ai * (__ldg(beta + c) * float(K - 2 * mism));
             }
         }
@@ -280,7 +303,7 @@ void launch_split(const FrontArgs &a, const DeviceInfo &dev, cudaStream_t s, boo
     const size_t smem = split_smem(a.F, a.K, a.words, affine);
     void (*kernel)(const float *, int64_t, int, int64_t, const float *, const float *,
                    const uint64_t *, const float *, int, int, const int64_t *, float *, int64_t,
-                   int);
+                   uint16_t *, int64_t, float *, int);
     if (G == 2) kernel = affine ? front_split_kernel<2, true> : front_split_kernel<2, false>;
     else if (G == 4) kernel = affine ? front_split_kernel<4, true> : front_split_kernel<4, false>;
     else kernel = affine ? front_split_kernel<8, true> : front_split_kernel<8, false>;
@@ -294,7 +317,8 @@ void launch_split(const FrontArgs &a, const DeviceInfo &dev, cudaStream_t s, boo
     const int64_t resident = int64_t(per_sm) * dev.sm_count;
     launch_kernel(kernel, dim3(unsigned(groups < resident ? groups : resident)),
                   dim3(kSplitThreads), smem, s, pdl, dim3(1, 1, 1), a.X, a.N, a.K, a.ldx, a.scale,
-                  a.shift, a.wbits, a.beta, a.F, a.words, a.rowptr, a.Z, a.ldz, P);
+                  a.shift, a.wbits, a.beta, a.F, a.words, a.rowptr, a.Z, a.ldz, a.D16, a.ldd16,
+                  a.rowscale, P);
 }
 
 }  // namespace

@@ -113,6 +113,12 @@ struct FrontArgs {
     const int64_t *rowptr;   // rows are scaled by 1/sqrt(1 + deg)
     float *Z;                // N x F (row stride ldz)
     int64_t ldz;
+    // Compressed output (nullable; replaces Z), as in GemmArgs: dots + 32768
+    // as uint16 (row stride ldd16 = F rounded up to 4, padding = 32768) and
+    // the row scale alpha_i / sqrt(1 + deg_i). Needs K <= 32767.
+    uint16_t *D16 = nullptr;
+    int64_t ldd16 = 0;
+    float *rowscale = nullptr;
 };
 
 // Whether the fused pack + XNOR-GEMM kernel fits (F <= 128, packed tiles in
@@ -131,7 +137,13 @@ struct SpmmPackGemmArgs {
     const int32_t *colidx;
     int64_t N;
     int64_t nnz;
-    const float *Z1;         // N x Fh, rows pre-scaled by 1/sqrt(dhat), row stride Fh
+    // Layer 1's Z', either fp32 rows pre-scaled by 1/sqrt(dhat) (Z1, row
+    // stride Fh) or compressed (D1 non-null: uint16 dots + 32768, row stride
+    // Fh, with the row scale s1 and the column scale beta1).
+    const float *Z1;
+    const uint16_t *D1;
+    const float *s1;
+    const float *beta1;
     int Fh;
     float *H1;               // nullable N x Fh output (row stride ldh)
     int64_t ldh;

@@ -28,9 +28,11 @@
 // a bias of 32768, weighted per neighbour by the row scale s_j = alpha_j /
 // sqrt(dhat_j) and, in the epilogue, per column by beta_f:
 //   H_if = (1/sqrt(dhat_i)) * beta_f * sum_j s_j * dot_jf.
-// A compressed row is half the bytes of an fp32 row, and a dot is
-// turned back into a float exactly by placing its 16 bits under the exponent
-// of 2^23 (one byte permute) and subtracting 2^23 + 32768.
+// A compressed row is half the bytes of an fp32 row, and a dot is turned
+// back into a float exactly by placing its 16 bits under the exponent of
+// 2^23 (one byte permute) and subtracting 2^23 + 32768. (The row scale costs
+// one more random 4-byte read per neighbour, which pays off for wide rows:
+// the fused forward compresses layer 1's rows, not layer 2's narrow ones.)
 //
 // A grid y dimension splits wide rows into column slabs of L * NV * VEC
 // features. Bounds: the row range is clamped to [0, nnz] and column indices
@@ -330,15 +332,16 @@ spmm_norm_kernel(SpmmParams p) {
 // ---------------------------------------------------------------------------
 // Layer-1 aggregation fused with layer 2's binarization and product.
 //
-// Each row's H1_i = dinv_i * sum_j Z1'_j is computed exactly as above (VEC = 4,
-// one vector per lane, pre-scaled rows). Then, without writing H1 (unless
-// asked to), layer 2's steps run on the row while it is in registers: the
-// signs of its Fh <= 128 features become one or two 64-bit words (four
-// ballots, one per vector component, spread into place), the row scale
-// alpha2_i = mean |H1_i| is one warp reduction, and the XNOR popcount against
-// the (shared-memory) packed columns of W2 gives
-//   Z2'_ij = (alpha2_i * dinv_i) * (beta2_j * (Fh - 2 popc(h_i ^ w_j))),
-// the expression the product's degree-scaled epilogue evaluates. Columns of
+// Each row's H1_i is computed exactly as above (VEC = 4, one vector per
+// lane), from layer 1's Z' as pre-scaled fp32 rows or, compressed, as uint16
+// dots weighted by s1_j with beta1 applied per column. Then, without writing
+// H1 (unless asked to), layer 2's steps run on the row while it is in
+// registers: the signs of its Fh <= 128 features become one or two 64-bit
+// words (four ballots, one per vector component, spread into place), the row
+// scale alpha2_i = mean |H1_i| is one warp reduction, and the XNOR popcount
+// against the (shared-memory) packed columns of W2 gives the dots of Eq. 11.
+// The result is written as Z2'_ij = (alpha2_i * dinv_i) * (beta2_j * dot_ij),
+// the expression the product's degree-scaled epilogue evaluates; columns of
 // Z2' from Fo up to its row stride are written as zeros, so the layer-2
 // aggregation can gather whole 4-wide vectors.
 
@@ -356,14 +359,15 @@ struct FusedLayer2 {
     float *H1;
     int64_t ldh;
     const uint64_t *sW;       // shared: Fo x words2 packed columns of W2
-    const float *sBeta;       // shared: Fo
+    const float *sBeta1;      // shared: Fh (compressed input only)
+    const float *sBeta2;      // shared: Fo
     int Fo;
     int words2;
     float *Z2;
     int64_t ldz2;
 };
 
-template <int L>
+template <int L, int S>
 struct PackGemmRow {
     FusedLayer2 f;
     __device__ __forceinline__ void operator()(const SpmmParams &p, int64_t i, float dinv,
@@ -374,7 +378,12 @@ struct PackGemmRow {
         const int Fh = p.F;
         float h[4];
 #pragma unroll
-        for (int c = 0; c < 4; ++c) h[c] = acc[0][c] * dinv;
+        for (int c = 0; c < 4; ++c) {
+            if (S == kDots16)
+                h[c] = fb + c < Fh ? dinv * (f.sBeta1[fb + c] * acc[0][c]) : 0.0f;
+            else
+                h[c] = acc[0][c] * dinv;
+        }
         if (f.H1 != nullptr && g == 0) {
 #pragma unroll
             for (int c = 0; c < 4; ++c)
@@ -399,33 +408,38 @@ struct PackGemmRow {
             if (jo < f.Fo) {
                 int mism = __popcll(w0 ^ f.sW[jo * f.words2]);
                 if (f.words2 > 1) mism += __popcll(w1 ^ f.sW[jo * f.words2 + 1]);
-                z = a * (f.sBeta[jo] * float(Fh - 2 * mism));
+                z = a * (f.sBeta2[jo] * float(Fh - 2 * mism));
             }
             f.Z2[i * f.ldz2 + jo] = z;
         }
     }
 };
 
-template <int L>
+template <int L, int S>
 __global__ void __launch_bounds__(kSpmmThreads, 3)
 spmm_pack_gemm_kernel(SpmmParams p, FusedLayer2 f, const uint64_t *__restrict__ wbits2,
-                      const float *__restrict__ beta2) {
+                      const float *__restrict__ beta1, const float *__restrict__ beta2) {
     constexpr int SLAB = L * 4;
+    constexpr int U = S == kDots16 && L == 32 ? 8 : 4;
     __shared__ float part[kSpmmWarps * SLAB];
     __shared__ unsigned mask[kSpmmWarps];
     __shared__ uint64_t sW[kMaxFusedOut * 2];
-    __shared__ float sBeta[kMaxFusedOut];
-    grid_dependency_wait();     // Z1' and the packed W2 come from earlier kernels
+    __shared__ float sBeta1[128];
+    __shared__ float sBeta2[kMaxFusedOut];
+    grid_dependency_wait();     // layer 1's Z' and the packed W2 come from earlier kernels
     for (int q = threadIdx.x; q < f.Fo * f.words2; q += kSpmmThreads) sW[q] = __ldg(wbits2 + q);
-    for (int q = threadIdx.x; q < f.Fo; q += kSpmmThreads) sBeta[q] = __ldg(beta2 + q);
+    for (int q = threadIdx.x; q < f.Fo; q += kSpmmThreads) sBeta2[q] = __ldg(beta2 + q);
+    if (S == kDots16)
+        for (int q = threadIdx.x; q < p.F; q += kSpmmThreads) sBeta1[q] = __ldg(beta1 + q);
     __syncthreads();
     f.sW = sW;
-    f.sBeta = sBeta;
-    PackGemmRow<L> epi{f};
+    f.sBeta1 = sBeta1;
+    f.sBeta2 = sBeta2;
+    PackGemmRow<L, S> epi{f};
     if (int(blockIdx.x) < p.heavy_blocks)
-        heavy_rows<4, L, 1, 4, kPre>(p, epi, 0, part, mask);
+        heavy_rows<4, L, 1, U, S>(p, epi, 0, part, mask);
     else
-        light_rows<4, L, 1, 4, kPre>(p, epi, 0);
+        light_rows<4, L, 1, U, S>(p, epi, 0);
 }
 
 // Leading blocks that look for heavy rows: up to two per SM, one per 256 rows.
@@ -511,22 +525,29 @@ void launch_spmm_pack_gemm(const SpmmPackGemmArgs &a, const DeviceInfo &dev, cud
     const int nvec = a.Fh / 4;
     int L = 4;
     while (L < 32 && L < nvec) L *= 2;
-    SpmmParams p{a.rowptr, a.colidx, a.N, a.nnz, a.Z1, a.Fh, a.Fh, a.Fh, nullptr, 0,
-                 heavy_block_count(a.N, dev), heavy_degree(a.N, a.nnz, (32 / L) * 4), false,
-                 nullptr, nullptr};
-    FusedLayer2 f{a.H1, a.ldh, nullptr, nullptr, a.Fo, (a.Fh + 63) / 64, a.Z2, a.ldz2};
+    const bool c16 = a.D1 != nullptr;
+    const int U = c16 && L == 32 ? 8 : 4;
+    const void *Z1 = c16 ? static_cast<const void *>(a.D1) : static_cast<const void *>(a.Z1);
+    SpmmParams p{a.rowptr, a.colidx, a.N, a.nnz, Z1, a.Fh, a.Fh, a.Fh, nullptr, 0,
+                 heavy_block_count(a.N, dev), heavy_degree(a.N, a.nnz, (32 / L) * U), false,
+                 a.s1, nullptr};
+    FusedLayer2 f{a.H1, a.ldh, nullptr, nullptr, nullptr, a.Fo, (a.Fh + 63) / 64, a.Z2, a.ldz2};
     const dim3 grid(unsigned(p.heavy_blocks + (a.N + kSpmmWarps - 1) / kSpmmWarps));
     const dim3 one(1, 1, 1), block(kSpmmThreads);
-    if (nvec <= 4)
-        launch_kernel(spmm_pack_gemm_kernel<4>, grid, block, 0, s, pdl, one, p, f, a.wbits2, a.beta2);
-    else if (nvec <= 8)
-        launch_kernel(spmm_pack_gemm_kernel<8>, grid, block, 0, s, pdl, one, p, f, a.wbits2, a.beta2);
-    else if (nvec <= 16)
-        launch_kernel(spmm_pack_gemm_kernel<16>, grid, block, 0, s, pdl, one, p, f, a.wbits2,
-                      a.beta2);
-    else
-        launch_kernel(spmm_pack_gemm_kernel<32>, grid, block, 0, s, pdl, one, p, f, a.wbits2,
-                      a.beta2);
+    auto run = [&](auto kernel) {
+        launch_kernel(kernel, grid, block, 0, s, pdl, one, p, f, a.wbits2, a.beta1, a.beta2);
+    };
+    if (c16) {
+        if (L == 4) run(spmm_pack_gemm_kernel<4, kDots16>);
+        else if (L == 8) run(spmm_pack_gemm_kernel<8, kDots16>);
+        else if (L == 16) run(spmm_pack_gemm_kernel<16, kDots16>);
+        else run(spmm_pack_gemm_kernel<32, kDots16>);
+    } else {
+        if (L == 4) run(spmm_pack_gemm_kernel<4, kPre>);
+        else if (L == 8) run(spmm_pack_gemm_kernel<8, kPre>);
+        else if (L == 16) run(spmm_pack_gemm_kernel<16, kPre>);
+        else run(spmm_pack_gemm_kernel<32, kPre>);
+    }
 }
 
 }  // namespace bigcn

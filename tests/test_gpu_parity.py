@@ -353,6 +353,27 @@ def test_forward_2layer_front_unaligned_rows(cuda_device, N, K, ldx, offset, Fh,
     assert B.device_timeouts() == 0
 
 
+# Above K = 32767 the dots no longer fit 16 bits: layer 1's Z' stays fp32.
+@pytest.mark.parametrize("N,K,Fh,Fo", [(40, 33000, 16, 3), (300, 32767, 8, 5)])
+def test_forward_2layer_k_at_and_past_the_16_bit_limit(cuda_device, N, K, Fh, Fo):
+    case = inputs.layer_case(N, K, Fh, seed=N + K, mean_degree=3.0)
+    W2 = inputs.weights(Fh, Fo, seed=K)
+    d = {k: to_dev(v) for k, v in case.items()}
+    ws = torch.empty(B.bigcn_forward_2layer_workspace_bytes(N, K, Fh, Fo), dtype=torch.uint8,
+                     device=cuda_device)
+    H1 = torch.full((N, Fh), float("nan"), device=cuda_device)
+    out = torch.full((N, Fo), float("nan"), device=cuda_device)
+    B.bigcn_forward_2layer(d["X"], d["s"], d["t"], d["W"], to_dev(W2), d["rowptr"], d["colidx"],
+                           ws, out, H1=H1)
+    ref1 = oracle.layer_forward(case["X"], case["W"], case["rowptr"], case["colidx"],
+                                case["s"], case["t"])
+    assert_close(H1, ref1["H"], "H1")
+    ref2 = oracle.layer_forward(H1.cpu().numpy(), W2, case["rowptr"], case["colidx"])
+    assert_close(out, ref2["H"], "logits")
+    H = B.layer_forward(d["X"], d["W"], d["rowptr"], d["colidx"], d["s"], d["t"])
+    assert_close(H, ref1["H"], "one layer")
+
+
 def test_forward_2layer_records_one_event_per_kernel_boundary(cuda_device):
     N, K, Fh, Fo = 500, 300, 64, 7
     case = inputs.layer_case(N, K, Fh, seed=3)
