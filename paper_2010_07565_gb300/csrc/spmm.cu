@@ -17,7 +17,8 @@
 // neighbours per round trip. A row is heavy when it has more than
 // max(32, 4 * that width, 4 * the mean degree) neighbours, i.e. when its walk
 // would take several times longer than a typical row's. The first `heavy_blocks` blocks of every launch therefore scan the
-// row pointers, skip light rows, and give each heavy row to all 8 warps of
+// row pointers in chunks of 32 rows (so that the hubs of a small graph land
+// on many blocks), skip light rows, and give each heavy row to all 8 warps of
 // the block: warp w gathers the w-th eighth of the row's list, the eight
 // partial rows meet in shared memory and warp 0 adds them in warp order
 // (deterministic) before the same epilogue. Light warps skip heavy rows.
@@ -258,59 +259,55 @@ __device__ __forceinline__ void light_rows(const SpmmParams &p, const Epi &epi, 
 
 template <int VEC, int L, int NV, int U, int S, class Epi>
 __device__ __forceinline__ void heavy_rows(const SpmmParams &p, const Epi &epi, int f0,
-                                           float *part, unsigned *mask) {
+                                           float *part) {
     constexpr int SLAB = L * NV * VEC;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int g = lane / L, sl = lane % L;
-    for (int64_t base = int64_t(blockIdx.x) * kSpmmThreads; base < p.N;
-         base += int64_t(p.heavy_blocks) * kSpmmThreads) {
-        const int64_t r = base + threadIdx.x;
+    // Chunks of 32 rows: every warp takes the same ballot over the chunk's
+    // row lengths, so the loop below is uniform over the block.
+    for (int64_t base = int64_t(blockIdx.x) * 32; base < p.N;
+         base += int64_t(p.heavy_blocks) * 32) {
+        const int64_t r = base + lane;
         bool heavy = false;
         if (r < p.N) heavy = row_span(p.rowptr, p.nnz, r).total - 1 > p.heavy_degree;
-        const unsigned m = __ballot_sync(kFullMask, heavy);
-        if (lane == 0) mask[warp] = m;
-        __syncthreads();
-        for (int w = 0; w < kSpmmWarps; ++w) {
-            unsigned mm = mask[w];
-            while (mm != 0u) {
-                const int bit = __ffs(mm) - 1;
-                mm &= mm - 1u;
-                const int64_t i = base + w * 32 + bit;
-                const RowSpan sp = row_span(p.rowptr, p.nnz, i);
-                float acc[NV][VEC];
+        unsigned mm = __ballot_sync(kFullMask, heavy);
+        while (mm != 0u) {
+            const int bit = __ffs(mm) - 1;
+            mm &= mm - 1u;
+            const int64_t i = base + bit;
+            const RowSpan sp = row_span(p.rowptr, p.nnz, i);
+            float acc[NV][VEC];
+#pragma unroll
+            for (int v = 0; v < NV; ++v)
+#pragma unroll
+                for (int c = 0; c < VEC; ++c) acc[v][c] = 0.0f;
+            const int64_t q0 = sp.total * warp / kSpmmWarps;
+            const int64_t q1 = sp.total * (warp + 1) / kSpmmWarps;
+            gather<VEC, L, NV, U, S>(p, i, sp.b, q0, q1, f0, acc);
+            reduce_groups<VEC, L, NV>(acc);
+            if (g == 0) {
 #pragma unroll
                 for (int v = 0; v < NV; ++v)
 #pragma unroll
-                    for (int c = 0; c < VEC; ++c) acc[v][c] = 0.0f;
-                const int64_t q0 = sp.total * warp / kSpmmWarps;
-                const int64_t q1 = sp.total * (warp + 1) / kSpmmWarps;
-                gather<VEC, L, NV, U, S>(p, i, sp.b, q0, q1, f0, acc);
-                reduce_groups<VEC, L, NV>(acc);
-                if (g == 0) {
-#pragma unroll
-                    for (int v = 0; v < NV; ++v)
-#pragma unroll
-                        for (int c = 0; c < VEC; ++c)
-                            part[warp * SLAB + (v * L + sl) * VEC + c] = acc[v][c];
-                }
-                __syncthreads();
-                if (warp == 0) {
-#pragma unroll
-                    for (int v = 0; v < NV; ++v)
-#pragma unroll
-                        for (int c = 0; c < VEC; ++c) {
-                            float t = 0.0f;
-                            if (g == 0)
-                                for (int q = 0; q < kSpmmWarps; ++q)
-                                    t += part[q * SLAB + (v * L + sl) * VEC + c];
-                            acc[v][c] = t;
-                        }
-                    epi(p, i, sp.dinv, f0, acc);
-                }
-                __syncthreads();
+                    for (int c = 0; c < VEC; ++c)
+                        part[warp * SLAB + (v * L + sl) * VEC + c] = acc[v][c];
             }
+            __syncthreads();
+            if (warp == 0) {
+#pragma unroll
+                for (int v = 0; v < NV; ++v)
+#pragma unroll
+                    for (int c = 0; c < VEC; ++c) {
+                        float t = 0.0f;
+                        if (g == 0)
+                            for (int q = 0; q < kSpmmWarps; ++q)
+                                t += part[q * SLAB + (v * L + sl) * VEC + c];
+                        acc[v][c] = t;
+                    }
+                epi(p, i, sp.dinv, f0, acc);
+            }
+            __syncthreads();    // part[] is rewritten by the next heavy row
         }
-        __syncthreads();   // every warp has read this chunk's masks before they change
     }
 }
 
@@ -319,12 +316,11 @@ __global__ void __launch_bounds__(kSpmmThreads, 4)
 spmm_norm_kernel(SpmmParams p) {
     constexpr int SLAB = L * NV * VEC;
     __shared__ float part[kSpmmWarps * SLAB];
-    __shared__ unsigned mask[kSpmmWarps];
     grid_dependency_wait();     // Z is the output of the previous kernel
     const int f0 = blockIdx.y * SLAB;
     StoreRow<VEC, L, NV, S> epi;
     if (int(blockIdx.x) < p.heavy_blocks)
-        heavy_rows<VEC, L, NV, U, S>(p, epi, f0, part, mask);
+        heavy_rows<VEC, L, NV, U, S>(p, epi, f0, part);
     else
         light_rows<VEC, L, NV, U, S>(p, epi, f0);
 }
@@ -422,7 +418,6 @@ spmm_pack_gemm_kernel(SpmmParams p, FusedLayer2 f, const uint64_t *__restrict__ 
     constexpr int SLAB = L * 4;
     constexpr int U = S == kDots16 && L == 32 ? 8 : 4;
     __shared__ float part[kSpmmWarps * SLAB];
-    __shared__ unsigned mask[kSpmmWarps];
     __shared__ uint64_t sW[kMaxFusedOut * 2];
     __shared__ float sBeta1[128];
     __shared__ float sBeta2[kMaxFusedOut];
@@ -437,14 +432,14 @@ spmm_pack_gemm_kernel(SpmmParams p, FusedLayer2 f, const uint64_t *__restrict__ 
     f.sBeta2 = sBeta2;
     PackGemmRow<L, S> epi{f};
     if (int(blockIdx.x) < p.heavy_blocks)
-        heavy_rows<4, L, 1, U, S>(p, epi, 0, part, mask);
+        heavy_rows<4, L, 1, U, S>(p, epi, 0, part);
     else
         light_rows<4, L, 1, U, S>(p, epi, 0);
 }
 
-// Leading blocks that look for heavy rows: up to two per SM, one per 256 rows.
+// Leading blocks that look for heavy rows: up to two per SM, one per 32 rows.
 int heavy_block_count(int64_t N, const DeviceInfo &dev) {
-    const int64_t chunks = (N + kSpmmThreads - 1) / kSpmmThreads;
+    const int64_t chunks = (N + 31) / 32;
     const int64_t cap = 2 * int64_t(dev.sm_count);
     return int(chunks < cap ? chunks : cap);
 }
