@@ -100,18 +100,23 @@ def kernel_work(w, nnz, name):
     N, K, Fh, Fo = w.N, w.K, w.hidden, w.out
     W1, W2 = (K + 63) // 64, (Fh + 63) // 64
     csr = 8.0 * (N + 1) + 4.0 * nnz
+    Fh4, Fo4 = (Fh + 3) // 4 * 4, (Fo + 3) // 4 * 4
+    # Layer 1's Z' as the forward keeps it: uint16 dots + a row scale when
+    # K <= 32767, else fp32; layer 2's Z' is fp32 with rows padded to Fo4.
+    z1 = 2.0 * N * Fh4 + 4.0 * N if K <= 32767 else 4.0 * N * Fh
+    z2 = 4.0 * N * Fo4
     table = {
         "pack_weights(W1,W2)": (4.0 * K * Fh + 8.0 * Fh * W1 + 4.0 * Fh + 4.0 * Fh * Fo
                                 + 8.0 * Fo * W2 + 4.0 * Fo, "bytes", "hbm"),
         "L1.pack_rows": (4.0 * N * K + 8.0 * N * W1 + 4.0 * N + 8.0 * K, "bytes", "hbm"),
-        "L1.pack_rows+L1.xnor_gemm": (4.0 * N * K + 8.0 * K + 4.0 * N * Fh + 8.0 * (N + 1),
+        "L1.pack_rows+L1.xnor_gemm": (4.0 * N * K + 8.0 * K + z1 + 8.0 * (N + 1),
                                       "bytes", "hbm", float(N) * K * Fh),
         "L1.xnor_gemm": (float(N) * K * Fh, "bit-ops", "alu"),
-        "L1.spmm+L2.pack_rows+L2.xnor_gemm": (csr + 4.0 * N * Fh + 4.0 * N * Fo, "bytes", "hbm"),
-        "L1.spmm": (csr + 8.0 * N * Fh, "bytes", "hbm"),
+        "L1.spmm+L2.pack_rows+L2.xnor_gemm": (csr + z1 + z2, "bytes", "hbm"),
+        "L1.spmm": (csr + z1 + 4.0 * N * Fh, "bytes", "hbm"),
         "L2.pack_rows": (4.0 * N * Fh + 8.0 * N * W2 + 4.0 * N, "bytes", "hbm"),
         "L2.xnor_gemm": (float(N) * Fh * Fo, "bit-ops", "alu"),
-        "L2.spmm": (csr + 8.0 * N * Fo, "bytes", "hbm"),
+        "L2.spmm": (csr + z2 + 4.0 * N * Fo, "bytes", "hbm"),
     }
     return table[name][:3]
 
