@@ -31,7 +31,7 @@ size_t round_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 constexpr int32_t kMaxDots16K = 32767;
 
 // Workspace carve-up. Layer 1's Z' is fp32 (N x Fh) or, when K <= 32767,
-// compressed: uint16 dots (N x Fh4, Fh4 = Fh rounded up to 4) and a row
+// compressed: uint16 dots (N x Fh8, Fh8 = Fh rounded up to 8) and a row
 // scale. Layer 2's Z' is fp32, pre-scaled, with rows padded to a multiple of
 // 4 (its rows are narrow: the extra row-scale read would cost more than the
 // bytes a compressed row saves).
@@ -43,9 +43,9 @@ struct Forward2Workspace {
 bool forward2_workspace(int64_t N, int32_t K, int32_t Fh, int32_t Fo, Forward2Workspace *w) {
     if (N < 0 || K < 1 || Fh < 1 || Fo < 1) return false;
     const int64_t w1 = bigcn_words(K), w2 = bigcn_words(Fh);
-    const int64_t Fh4 = (int64_t(Fh) + 3) / 4 * 4, Fo4 = (int64_t(Fo) + 3) / 4 * 4;
+    const int64_t Fh8 = (int64_t(Fh) + 7) / 8 * 8, Fo4 = (int64_t(Fo) + 3) / 4 * 4;
     int64_t widest = w1;
-    if (Fh4 > widest) widest = Fh4;
+    if (Fh8 > widest) widest = Fh8;
     if (Fo4 > widest) widest = Fo4;
     if (N > kMaxElems / widest) return false;
     w->c16 = K <= kMaxDots16K;
@@ -55,7 +55,7 @@ bool forward2_workspace(int64_t N, int32_t K, int32_t Fh, int32_t Fo, Forward2Wo
     w->alpha1 = take(size_t(N) * 4);
     w->wbits1 = take(size_t(Fh) * w1 * 8);
     w->beta1 = take(size_t(Fh) * 4);
-    w->z1 = take(w->c16 ? size_t(N) * Fh4 * 2 : size_t(N) * Fh * 4);
+    w->z1 = take(w->c16 ? size_t(N) * Fh8 * 2 : size_t(N) * Fh * 4);
     w->s1 = take(size_t(N) * 4);
     w->wbits2 = take(size_t(Fo) * w2 * 8);
     w->beta2 = take(size_t(Fo) * 4);
@@ -142,7 +142,7 @@ extern "C" bigcn_status bigcn_forward_2layer(
     float *beta2 = static_cast<float *>(at(w.beta2));
     float *Z2 = static_cast<float *>(at(w.z2));
     const int words1 = bigcn_words(K), words2 = bigcn_words(Fh);
-    const int64_t Fh4 = (Fh + 3) / 4 * 4, Fo4 = (Fo + 3) / 4 * 4;
+    const int64_t Fh8 = (Fh + 7) / 8 * 8, Fo4 = (Fo + 3) / 4 * 4;
     const bool fused = spmm_pack_gemm_supported(Fh, Fo);
     uint16_t *D1 = w.c16 ? static_cast<uint16_t *>(Z1) : nullptr;
     float *Z1f = w.c16 ? nullptr : static_cast<float *>(Z1);
@@ -160,7 +160,7 @@ extern "C" bigcn_status bigcn_forward_2layer(
         FrontArgs fr{X, N, K, ldx, scale, shift, wbits1, beta1, Fh, words1, rowptr, Z1f, Fh};
         if (w.c16) {
             fr.D16 = D1;
-            fr.ldd16 = Fh4;
+            fr.ldd16 = Fh8;
             fr.rowscale = s1;
         }
         launch_front(fr, dev, s, true);
@@ -171,15 +171,15 @@ extern "C" bigcn_status bigcn_forward_2layer(
         GemmArgs g1{bits1, alpha1, N, wbits1, beta1, Fh, K, words1, Z1f, Fh, nullptr, rowptr};
         if (w.c16) {
             g1.dots16 = D1;
-            g1.ldd16 = Fh4;
+            g1.ldd16 = Fh8;
             g1.rowscale = s1;
         }
         launch_xnor_gemm(g1, dev, s, true);
         mark();
     }
     if (fused) {
-        SpmmPackGemmArgs f{rowptr, colidx, N, nnz, Z1f, D1, s1, beta1, Fh, H1, ldh1, wbits2,
-                           beta2, Fo, Z2, Fo4};
+        SpmmPackGemmArgs f{rowptr, colidx, N, nnz, Z1f, D1, Fh8, s1, beta1, Fh, H1, ldh1,
+                           wbits2, beta2, Fo, Z2, Fo4};
         launch_spmm_pack_gemm(f, dev, s, true);
         mark();
     } else {
@@ -187,7 +187,7 @@ extern "C" bigcn_status bigcn_forward_2layer(
         const int64_t ldh = H1 ? ldh1 : Fh;
         uint64_t *bits2 = static_cast<uint64_t *>(at(w.bits2));
         float *alpha2 = static_cast<float *>(at(w.alpha2));
-        SpmmArgs a1{rowptr, colidx, N, nnz, Z1f, w.c16 ? Fh4 : Fh, Fh, H1w, ldh, true, false};
+        SpmmArgs a1{rowptr, colidx, N, nnz, Z1f, w.c16 ? Fh8 : Fh, Fh, H1w, ldh, true, false};
         if (w.c16) {
             a1.D16 = D1;
             a1.rowscale = s1;

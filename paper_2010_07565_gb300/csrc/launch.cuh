@@ -54,7 +54,7 @@ struct GemmArgs {
     int32_t *dots;           // nullable N x F raw dots (row stride F)
     const int64_t *rowptr;   // nullable: scale row i by 1/sqrt(1 + deg_i)
     // Compressed output (nullable; replaces Z): dots + 32768 as uint16 (row
-    // stride ldd16 = F rounded up to 4, padding columns hold 32768, i.e. 0),
+    // stride ldd16, a multiple of 4 >= F, padding columns hold 32768, i.e. 0),
     // and each row's scale alpha_i (times 1/sqrt(1 + deg_i) with rowptr) in
     // rowscale; Z[i,j] is then rowscale_i * beta_j * dot[i,j]. Needs K <= 32767.
     uint16_t *dots16 = nullptr;
@@ -114,7 +114,7 @@ struct FrontArgs {
     float *Z;                // N x F (row stride ldz)
     int64_t ldz;
     // Compressed output (nullable; replaces Z), as in GemmArgs: dots + 32768
-    // as uint16 (row stride ldd16 = F rounded up to 4, padding = 32768) and
+    // as uint16 (row stride ldd16, a multiple of 4 >= F, padding = 32768) and
     // the row scale alpha_i / sqrt(1 + deg_i). Needs K <= 32767.
     uint16_t *D16 = nullptr;
     int64_t ldd16 = 0;
@@ -139,9 +139,11 @@ struct SpmmPackGemmArgs {
     int64_t nnz;
     // Layer 1's Z', either fp32 rows pre-scaled by 1/sqrt(dhat) (Z1, row
     // stride Fh) or compressed (D1 non-null: uint16 dots + 32768, row stride
-    // Fh, with the row scale s1 and the column scale beta1).
+    // ldz1 >= Fh rounded up to 4 with zero dots as padding, with the row
+    // scale s1 and the column scale beta1).
     const float *Z1;
     const uint16_t *D1;
+    int64_t ldz1;
     const float *s1;
     const float *beta1;
     int Fh;

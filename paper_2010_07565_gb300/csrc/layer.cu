@@ -48,8 +48,8 @@ size_t round_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 constexpr int32_t kMaxDots16K = 32767;
 
 // Workspace carve-up of the fused layer; every piece 256-byte aligned. Z is
-// either fp32 (N x F) or compressed: uint16 dots (N x round_up(F, 4)) and a
-// row scale (N).
+// either fp32 (N x F) or compressed: uint16 dots (N x round_up(F, 8), so that
+// the aggregation can load eight dots at a time) and a row scale (N).
 struct LayerWorkspace {
     size_t a_bits, alpha, b_bits, beta, z, rowscale, total;
     bool compressed;
@@ -58,8 +58,8 @@ struct LayerWorkspace {
 bool layer_workspace(int64_t N, int32_t K, int32_t F, LayerWorkspace *w) {
     if (N < 0 || K < 1 || F < 1) return false;
     const int64_t words = bigcn_words(K);
-    const int64_t F4 = (int64_t(F) + 3) / 4 * 4;
-    if (N > kMaxElems / (words > F4 ? words : F4)) return false;
+    const int64_t F8 = (int64_t(F) + 7) / 8 * 8;
+    if (N > kMaxElems / (words > F8 ? words : F8)) return false;
     w->compressed = K <= kMaxDots16K;
     size_t off = 0;
     w->a_bits = off; off = round_up(off + size_t(N) * size_t(words) * 8);
@@ -68,7 +68,7 @@ bool layer_workspace(int64_t N, int32_t K, int32_t F, LayerWorkspace *w) {
     w->beta = off;   off = round_up(off + size_t(F) * 4);
     w->z = off;
     if (w->compressed) {
-        off = round_up(off + size_t(N) * size_t(F4) * 2);
+        off = round_up(off + size_t(N) * size_t(F8) * 2);
         w->rowscale = off; off = round_up(off + size_t(N) * 4);
     } else {
         off = round_up(off + size_t(N) * size_t(F) * 4);
@@ -180,13 +180,13 @@ extern "C" bigcn_status bigcn_layer_forward_timed(const float *X, int64_t N, int
     if (w.compressed) {
         uint16_t *D16 = reinterpret_cast<uint16_t *>(ws + w.z);
         float *rowscale = reinterpret_cast<float *>(ws + w.rowscale);
-        const int64_t F4 = (int64_t(F) + 3) / 4 * 4;
+        const int64_t F8 = (int64_t(F) + 7) / 8 * 8;
         g.Z = nullptr;
         g.dots16 = D16;
-        g.ldd16 = F4;
+        g.ldd16 = F8;
         g.rowscale = rowscale;
         a.Z = nullptr;
-        a.ldz = F4;
+        a.ldz = F8;
         a.D16 = D16;
         a.rowscale = rowscale;
         a.colscale = beta;

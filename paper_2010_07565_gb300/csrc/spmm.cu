@@ -131,6 +131,26 @@ struct RowSrc<4, kDots16> {
     }
 };
 
+// Eight dots (16 bytes) per vector: half the lanes per row of the 4-wide form,
+// so a warp gathers twice the neighbours per load instruction.
+template <>
+struct RowSrc<8, kDots16> {
+    using T = uint4;
+    static __device__ __forceinline__ T load(const void *Z, int64_t row, int64_t ldz, int f) {
+        return __ldg(reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(Z) + row * ldz + f));
+    }
+    static __device__ __forceinline__ void fma(float *acc, const T &v, float w) {
+        acc[0] = fmaf(w, dot16_lo(v.x), acc[0]);
+        acc[1] = fmaf(w, dot16_hi(v.x), acc[1]);
+        acc[2] = fmaf(w, dot16_lo(v.y), acc[2]);
+        acc[3] = fmaf(w, dot16_hi(v.y), acc[3]);
+        acc[4] = fmaf(w, dot16_lo(v.z), acc[4]);
+        acc[5] = fmaf(w, dot16_hi(v.z), acc[5]);
+        acc[6] = fmaf(w, dot16_lo(v.w), acc[6]);
+        acc[7] = fmaf(w, dot16_hi(v.w), acc[7]);
+    }
+};
+
 // Row i's neighbour list: CSR entries [b, b + total - 1) plus the self-loop.
 struct RowSpan {
     int64_t b;
@@ -213,7 +233,6 @@ struct StoreRow {
     __device__ __forceinline__ void prologue() const {}
     __device__ __forceinline__ void operator()(const SpmmParams &p, int64_t i, float dinv,
                                                int f0, float (&acc)[NV][VEC]) const {
-        using V = typename Vec<VEC>::T;
         const int lane = threadIdx.x & 31;
         if (lane / L != 0) return;
         const int sl = lane % L;
@@ -230,7 +249,12 @@ struct StoreRow {
             }
             float *h = p.H + i * p.ldh + f;
             if (p.vec_store && f + VEC <= p.F) {
-                *reinterpret_cast<V *>(h) = Vec<VEC>::make(o);
+                if constexpr (VEC == 8) {
+                    reinterpret_cast<float4 *>(h)[0] = make_float4(o[0], o[1], o[2], o[3]);
+                    reinterpret_cast<float4 *>(h)[1] = make_float4(o[4], o[5], o[6], o[7]);
+                } else {
+                    *reinterpret_cast<typename Vec<VEC>::T *>(h) = Vec<VEC>::make(o);
+                }
             } else {
 #pragma unroll
                 for (int c = 0; c < VEC; ++c)
@@ -328,12 +352,13 @@ spmm_norm_kernel(SpmmParams p) {
 // ---------------------------------------------------------------------------
 // Layer-1 aggregation fused with layer 2's binarization and product.
 //
-// Each row's H1_i is computed exactly as above (VEC = 4, one vector per
-// lane), from layer 1's Z' as pre-scaled fp32 rows or, compressed, as uint16
-// dots weighted by s1_j with beta1 applied per column. Then, without writing
+// Each row's H1_i is computed exactly as above (one vector per lane), from
+// layer 1's Z' as pre-scaled fp32 rows (VEC = 4) or, compressed, as uint16
+// dots weighted by s1_j with beta1 applied per column (VEC = 8 when the row
+// stride is a multiple of 8, else 4). Then, without writing
 // H1 (unless asked to), layer 2's steps run on the row while it is in
 // registers: the signs of its Fh <= 128 features become one or two 64-bit
-// words (four ballots, one per vector component, spread into place), the row
+// words (VEC ballots, one per vector component, spread into place), the row
 // scale alpha2_i = mean |H1_i| is one warp reduction, and the XNOR popcount
 // against the (shared-memory) packed columns of W2 gives the dots of Eq. 11.
 // The result is written as Z2'_ij = (alpha2_i * dinv_i) * (beta2_j * dot_ij),
@@ -351,6 +376,15 @@ __device__ __forceinline__ uint64_t spread16by4(uint32_t x) {
     return v;
 }
 
+// Spreads 8 bits so that bit i lands on bit 8i of a 64-bit word.
+__device__ __forceinline__ uint64_t spread8by8(uint32_t x) {
+    uint64_t v = x & 0xFFu;
+    v = (v | (v << 28)) & 0x0000000F0000000Full;
+    v = (v | (v << 14)) & 0x0003000300030003ull;
+    v = (v | (v << 7)) & 0x0101010101010101ull;
+    return v;
+}
+
 struct FusedLayer2 {
     float *H1;
     int64_t ldh;
@@ -363,18 +397,18 @@ struct FusedLayer2 {
     int64_t ldz2;
 };
 
-template <int L, int S>
+template <int VEC, int L, int S>
 struct PackGemmRow {
     FusedLayer2 f;
     __device__ __forceinline__ void operator()(const SpmmParams &p, int64_t i, float dinv,
-                                               int, float (&acc)[1][4]) const {
+                                               int, float (&acc)[1][VEC]) const {
         const int lane = threadIdx.x & 31;
         const int g = lane / L, sl = lane % L;
-        const int fb = sl * 4;
+        const int fb = sl * VEC;
         const int Fh = p.F;
-        float h[4];
+        float h[VEC];
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
+        for (int c = 0; c < VEC; ++c) {
             if (S == kDots16)
                 h[c] = fb + c < Fh ? dinv * (f.sBeta1[fb + c] * acc[0][c]) : 0.0f;
             else
@@ -382,18 +416,24 @@ struct PackGemmRow {
         }
         if (f.H1 != nullptr && g == 0) {
 #pragma unroll
-            for (int c = 0; c < 4; ++c)
+            for (int c = 0; c < VEC; ++c)
                 if (fb + c < Fh) f.H1[i * f.ldh + fb + c] = h[c];
         }
         // Layer 2, Eqs. 7-8: signs of H1_i packed LSB-first, and its mean |.|.
+        // Ballot c holds component c of every lane's vector: feature VEC l + c.
         uint64_t w0 = 0, w1 = 0;
         float l1 = 0.0f;
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
+        for (int c = 0; c < VEC; ++c) {
             const bool in = g == 0 && fb + c < Fh;
             const unsigned m = __ballot_sync(kFullMask, in && h[c] >= 0.0f);
-            w0 |= spread16by4(m) << c;
-            w1 |= spread16by4(m >> 16) << c;
+            if (VEC == 4) {
+                w0 |= spread16by4(m) << c;
+                w1 |= spread16by4(m >> 16) << c;
+            } else {
+                w0 |= spread8by8(m) << c;
+                w1 |= spread8by8(m >> 8) << c;
+            }
             l1 += in ? fabsf(h[c]) : 0.0f;
         }
         l1 = warp_sum(l1);
@@ -411,12 +451,12 @@ struct PackGemmRow {
     }
 };
 
-template <int L, int S>
+template <int VEC, int L, int S>
 __global__ void __launch_bounds__(kSpmmThreads, 3)
 spmm_pack_gemm_kernel(SpmmParams p, FusedLayer2 f, const uint64_t *__restrict__ wbits2,
                       const float *__restrict__ beta1, const float *__restrict__ beta2) {
-    constexpr int SLAB = L * 4;
-    constexpr int U = S == kDots16 && L == 32 ? 8 : 4;
+    constexpr int SLAB = L * VEC;
+    constexpr int U = S == kDots16 && VEC == 4 && L == 32 ? 8 : 4;
     __shared__ float part[kSpmmWarps * SLAB];
     __shared__ uint64_t sW[kMaxFusedOut * 2];
     __shared__ float sBeta1[128];
@@ -430,11 +470,11 @@ spmm_pack_gemm_kernel(SpmmParams p, FusedLayer2 f, const uint64_t *__restrict__ 
     f.sW = sW;
     f.sBeta1 = sBeta1;
     f.sBeta2 = sBeta2;
-    PackGemmRow<L, S> epi{f};
+    PackGemmRow<VEC, L, S> epi{f};
     if (int(blockIdx.x) < p.heavy_blocks)
-        heavy_rows<4, L, 1, U, S>(p, epi, 0, part);
+        heavy_rows<VEC, L, 1, U, S>(p, epi, 0, part);
     else
-        light_rows<4, L, 1, U, S>(p, epi, 0);
+        light_rows<VEC, L, 1, U, S>(p, epi, 0);
 }
 
 // Leading blocks that look for heavy rows: up to two per SM, one per 32 rows.
@@ -452,14 +492,20 @@ int64_t heavy_degree(int64_t N, int64_t nnz, int per_iter) {
     return h > 32 ? h : 32;
 }
 
+// Eight dots per lane halve the gather instructions per neighbour but double
+// the per-row reduction and epilogue work: worth it from a mean degree of 8.
+bool wide_dots(int64_t N, int64_t nnz) { return N > 0 && nnz >= 8 * N; }
+
 template <int VEC, int L, int NV, int S>
 void launch_cfg(const SpmmArgs &a, const DeviceInfo &dev, int Fload, cudaStream_t s, bool pdl) {
     constexpr int SLAB = L * NV * VEC;
     // Rows in flight per group. A compressed row costs half the registers, so
     // where a warp holds only a few rows at a time (one row across all 32
     // lanes) it takes twice as many.
-    constexpr int U = (S == kDots16 && L == 32 ? 2 : 1) * (NV == 1 ? 4 : 2);
-    const bool vec_store = a.ldh % VEC == 0 && aligned_to(a.H, size_t(VEC) * 4);
+    constexpr int U = VEC == 8 ? (NV == 1 ? 4 : 2)
+                               : (S == kDots16 && L == 32 ? 2 : 1) * (NV == 1 ? 4 : 2);
+    constexpr int kStoreVec = VEC < 4 ? VEC : 4;    // 8-wide rows are stored as two float4
+    const bool vec_store = a.ldh % kStoreVec == 0 && aligned_to(a.H, size_t(kStoreVec) * 4);
     const void *Z = S == kDots16 ? static_cast<const void *>(a.D16) : a.Z;
     SpmmParams p{a.rowptr, a.colidx, a.N, a.nnz, Z, a.ldz, Fload, a.F, a.H, a.ldh,
                  heavy_block_count(a.N, dev), heavy_degree(a.N, a.nnz, (32 / L) * U), vec_store,
@@ -501,9 +547,13 @@ void launch_src(const SpmmArgs &a, const DeviceInfo &dev, cudaStream_t s, bool p
 void launch_spmm_norm(const SpmmArgs &a, const DeviceInfo &dev, cudaStream_t stream, bool pdl) {
     if (a.N == 0) return;
     if (a.D16 != nullptr) {
-        // Compressed rows: four dots (8 bytes) per vector; the row stride is a
-        // multiple of 4 and its padding columns hold a zero dot.
-        launch_vec<4, kDots16>(a, dev, (a.F + 3) / 4 * 4, stream, pdl);
+        // Compressed rows: eight dots (16 bytes) per vector when the row
+        // stride and base allow and rows are long, else four (8 bytes);
+        // padding columns up to the stride hold a zero dot.
+        if (a.ldz % 8 == 0 && aligned_to(a.D16, 16) && wide_dots(a.N, a.nnz))
+            launch_vec<8, kDots16>(a, dev, (a.F + 7) / 8 * 8, stream, pdl);
+        else
+            launch_vec<4, kDots16>(a, dev, (a.F + 3) / 4 * 4, stream, pdl);
         return;
     }
     if (a.prescaled) launch_src<kPre>(a, dev, stream, pdl);
@@ -517,13 +567,17 @@ bool spmm_pack_gemm_supported(int Fh, int Fo) {
 void launch_spmm_pack_gemm(const SpmmPackGemmArgs &a, const DeviceInfo &dev, cudaStream_t s,
                            bool pdl) {
     if (a.N == 0) return;
-    const int nvec = a.Fh / 4;
+    const bool c16 = a.D1 != nullptr;
+    // Compressed rows take eight dots per lane when their stride allows and
+    // the rows are long enough to repay it.
+    const int VEC = c16 && a.ldz1 % 8 == 0 && aligned_to(a.D1, 16) && wide_dots(a.N, a.nnz) ? 8 : 4;
+    const int Fload = (a.Fh + VEC - 1) / VEC * VEC;
+    const int nvec = Fload / VEC;
     int L = 4;
     while (L < 32 && L < nvec) L *= 2;
-    const bool c16 = a.D1 != nullptr;
-    const int U = c16 && L == 32 ? 8 : 4;
+    const int U = c16 && VEC == 4 && L == 32 ? 8 : 4;
     const void *Z1 = c16 ? static_cast<const void *>(a.D1) : static_cast<const void *>(a.Z1);
-    SpmmParams p{a.rowptr, a.colidx, a.N, a.nnz, Z1, a.Fh, a.Fh, a.Fh, nullptr, 0,
+    SpmmParams p{a.rowptr, a.colidx, a.N, a.nnz, Z1, c16 ? a.ldz1 : a.Fh, Fload, a.Fh, nullptr, 0,
                  heavy_block_count(a.N, dev), heavy_degree(a.N, a.nnz, (32 / L) * U), false,
                  a.s1, nullptr};
     FusedLayer2 f{a.H1, a.ldh, nullptr, nullptr, nullptr, a.Fo, (a.Fh + 63) / 64, a.Z2, a.ldz2};
@@ -532,16 +586,20 @@ void launch_spmm_pack_gemm(const SpmmPackGemmArgs &a, const DeviceInfo &dev, cud
     auto run = [&](auto kernel) {
         launch_kernel(kernel, grid, block, 0, s, pdl, one, p, f, a.wbits2, a.beta1, a.beta2);
     };
-    if (c16) {
-        if (L == 4) run(spmm_pack_gemm_kernel<4, kDots16>);
-        else if (L == 8) run(spmm_pack_gemm_kernel<8, kDots16>);
-        else if (L == 16) run(spmm_pack_gemm_kernel<16, kDots16>);
-        else run(spmm_pack_gemm_kernel<32, kDots16>);
+    if (c16 && VEC == 8) {
+        if (L == 4) run(spmm_pack_gemm_kernel<8, 4, kDots16>);
+        else if (L == 8) run(spmm_pack_gemm_kernel<8, 8, kDots16>);
+        else run(spmm_pack_gemm_kernel<8, 16, kDots16>);
+    } else if (c16) {
+        if (L == 4) run(spmm_pack_gemm_kernel<4, 4, kDots16>);
+        else if (L == 8) run(spmm_pack_gemm_kernel<4, 8, kDots16>);
+        else if (L == 16) run(spmm_pack_gemm_kernel<4, 16, kDots16>);
+        else run(spmm_pack_gemm_kernel<4, 32, kDots16>);
     } else {
-        if (L == 4) run(spmm_pack_gemm_kernel<4, kPre>);
-        else if (L == 8) run(spmm_pack_gemm_kernel<8, kPre>);
-        else if (L == 16) run(spmm_pack_gemm_kernel<16, kPre>);
-        else run(spmm_pack_gemm_kernel<32, kPre>);
+        if (L == 4) run(spmm_pack_gemm_kernel<4, 4, kPre>);
+        else if (L == 8) run(spmm_pack_gemm_kernel<4, 8, kPre>);
+        else if (L == 16) run(spmm_pack_gemm_kernel<4, 16, kPre>);
+        else run(spmm_pack_gemm_kernel<4, 32, kPre>);
     }
 }
 
