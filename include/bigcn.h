@@ -251,7 +251,10 @@ bigcn_status bigcn_layer_forward_timed(const float *X, int64_t N, int32_t K, int
  *            recorded on `stream` before kernel q and the last one after the
  *            last kernel (recorded with cudaEventRecordExternal), for timing
  *            each kernel; entries beyond launches + 1 are not touched.
- * out, H1 and the workspace must not overlap each other or any input.
+ * pred       nullable N int32: each node's predicted class, the argmax of its
+ *            logits row (lowest index on ties; computed in the last
+ *            aggregation's epilogue, or by one more kernel when Fo > 256).
+ * out, H1, pred and the workspace must not overlap each other or any input.
  */
 size_t bigcn_forward_2layer_workspace_bytes(int64_t N, int32_t K, int32_t Fh, int32_t Fo);
 
@@ -266,7 +269,8 @@ bigcn_status bigcn_forward_2layer(const float *X, int64_t N, int32_t K, int64_t 
                                   const int64_t *rowptr, const int32_t *colidx, int64_t nnz,
                                   void *workspace, size_t ws_bytes,
                                   float *H1, int64_t ldh1, float *out, int64_t ldo,
-                                  void *const *events, int32_t n_events, void *stream);
+                                  int32_t *pred, void *const *events, int32_t n_events,
+                                  void *stream);
 
 /* Bytes of the device scratch array behind bigcn_layer_forward_static. */
 #define BIGCN_STATIC_SCRATCH_BYTES ((size_t)32 << 20)

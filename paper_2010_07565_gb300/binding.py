@@ -53,7 +53,7 @@ SIGNATURES = {
     "bigcn_forward_2layer_workspace_bytes": ([_i64, _i32, _i32, _i32], _sz),
     "bigcn_forward_2layer_launches": ([_i64, _i32, _i32, _i32], _i32),
     "bigcn_forward_2layer": ([_p, _i64, _i32, _i64, _p, _p, _p, _i32, _i64, _p, _i32, _i64, _p,
-                              _p, _i64, _p, _sz, _p, _i64, _p, _i64, _p, _i32, _p],
+                              _p, _i64, _p, _sz, _p, _i64, _p, _i64, _p, _p, _i32, _p],
                              ctypes.c_int),
     "bigcn_layer_forward_static": ([_p, _i64, _i32, _i64, _p, _p, _p, _i32, _i64, _p, _p, _i64,
                                     _p, _i64, _p], ctypes.c_int),
@@ -225,11 +225,12 @@ def bigcn_forward_2layer_launches(N: int, K: int, Fh: int, Fo: int) -> int:
 
 
 def bigcn_forward_2layer(X, scale, shift, W1, W2, rowptr, colidx, workspace, out, H1=None,
-                         events=None, stream=None):
+                         events=None, stream=None, pred=None):
     """The two-layer forward of Sec. 6.2 (hidden layer on centred X, output
     layer on H1 raw). ``events``: torch.cuda.Event objects (created with
     enable_timing=True, external=True and recorded once) to be recorded
-    before each kernel and after the last."""
+    before each kernel and after the last. ``pred``: optional int32 tensor of
+    N that receives each row's argmax of the logits."""
     N, K = X.shape
     Fh, Fo = W1.shape[1], W2.shape[1]
     if W2.shape[0] != Fh:
@@ -243,7 +244,8 @@ def bigcn_forward_2layer(X, scale, shift, W1, W2, rowptr, colidx, workspace, out
         _ptr(X), N, K, _ld(X), _ptr(scale), _ptr(shift), _ptr(W1), Fh, _ld(W1), _ptr(W2), Fo,
         _ld(W2), _ptr(rowptr), _ptr(colidx) if colidx.numel() else None, colidx.numel(),
         _ptr(workspace), workspace.numel() * workspace.element_size(), _ptr(H1),
-        _ld(H1) if H1 is not None else 0, _ptr(out), _ld(out), ev, n_ev, _stream(stream)))
+        _ld(H1) if H1 is not None else 0, _ptr(out), _ld(out), _ptr(pred), ev, n_ev,
+        _stream(stream)))
 
 
 def bigcn_layer_forward_static(X, scale, shift, Wt, rowptr, colidx, H, stream=None):

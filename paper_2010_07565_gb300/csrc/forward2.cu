@@ -90,8 +90,8 @@ extern "C" bigcn_status bigcn_forward_2layer(
     const float *X, int64_t N, int32_t K, int64_t ldx, const float *scale, const float *shift,
     const float *W1, int32_t Fh, int64_t ldw1, const float *W2, int32_t Fo, int64_t ldw2,
     const int64_t *rowptr, const int32_t *colidx, int64_t nnz, void *workspace, size_t ws_bytes,
-    float *H1, int64_t ldh1, float *out, int64_t ldo, void *const *events, int32_t n_events,
-    void *stream) {
+    float *H1, int64_t ldh1, float *out, int64_t ldo, int32_t *pred, void *const *events,
+    int32_t n_events, void *stream) {
     Forward2Workspace w;
     if (N < 0 || N > int64_t(INT32_MAX) || K < 1 || Fh < 1 || Fo < 1 || ldx < K || ldw1 < Fh ||
         ldw2 < Fo || ldo < Fo || (H1 && ldh1 < Fh) || nnz < 0 || n_events < 0)
@@ -109,6 +109,7 @@ extern "C" bigcn_status bigcn_forward_2layer(
     if (ws_bytes < w.total) return BIGCN_ERR_INVALID_ARG;
     if (!aligned_to(X, 4) || !aligned_to(W1, 4) || !aligned_to(W2, 4) || !aligned_to(rowptr, 8) ||
         (colidx && !aligned_to(colidx, 4)) || !aligned_to(out, 4) || (H1 && !aligned_to(H1, 4)) ||
+        (pred && !aligned_to(pred, 4)) ||
         !aligned_to(workspace, kAlign) ||
         (scale && (!aligned_to(scale, 4) || !aligned_to(shift, 4))))
         return BIGCN_ERR_MISALIGNED;
@@ -116,13 +117,13 @@ extern "C" bigcn_status bigcn_forward_2layer(
     const size_t in_bytes[] = {span_bytes(N, K, ldx, 4), span_bytes(K, Fh, ldw1, 4),
                                span_bytes(Fh, Fo, ldw2, 4), size_t(N + 1) * 8, size_t(nnz) * 4,
                                size_t(K) * 4, size_t(K) * 4};
-    const void *outs[] = {workspace, out, H1};
+    const void *outs[] = {workspace, out, H1, pred};
     const size_t out_bytes[] = {w.total, span_bytes(N, Fo, ldo, 4),
-                                H1 ? span_bytes(N, Fh, ldh1, 4) : 0};
-    for (int o = 0; o < 3; ++o) {
+                                H1 ? span_bytes(N, Fh, ldh1, 4) : 0, pred ? size_t(N) * 4 : 0};
+    for (int o = 0; o < 4; ++o) {
         for (int q = 0; q < 7; ++q)
             if (overlaps(outs[o], out_bytes[o], in[q], in_bytes[q])) return BIGCN_ERR_INVALID_ARG;
-        for (int p = o + 1; p < 3; ++p)
+        for (int p = o + 1; p < 4; ++p)
             if (overlaps(outs[o], out_bytes[o], outs[p], out_bytes[p])) return BIGCN_ERR_INVALID_ARG;
     }
 
@@ -205,6 +206,7 @@ extern "C" bigcn_status bigcn_forward_2layer(
     // The fused kernel writes Z2's padding columns as zeros: whole 4-wide
     // vectors may be gathered.
     SpmmArgs a2{rowptr, colidx, N, nnz, Z2, Fo4, Fo, out, ldo, true, fused};
+    a2.pred = pred;
     launch_spmm_norm(a2, dev, s, true);
     mark();
     const bigcn_status ls = launch_status();

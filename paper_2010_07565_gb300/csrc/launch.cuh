@@ -93,9 +93,14 @@ struct SpmmArgs {
     const uint16_t *D16 = nullptr;
     const float *rowscale = nullptr;
     const float *colscale = nullptr;
+    // Nullable: receives each output row's argmax (lowest index on ties),
+    // in the aggregation's epilogue when a row fits one column slab, else
+    // by a separate kernel.
+    int32_t *pred = nullptr;
 };
 
-// Step 5: H = D^-1/2 (A + I) D^-1/2 Z (Eqs. 1, 13).
+// Step 5: H = D^-1/2 (A + I) D^-1/2 Z (Eqs. 1, 13); launches one kernel, or
+// two when an argmax is asked for rows wider than one column slab.
 void launch_spmm_norm(const SpmmArgs &args, const DeviceInfo &dev, cudaStream_t stream,
                       bool pdl = false);
 

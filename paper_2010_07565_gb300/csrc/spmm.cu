@@ -94,6 +94,7 @@ struct SpmmParams {
     bool vec_store;          // H rows start VEC-aligned: whole vectors may be stored
     const float *rowscale;   // kDots16: s_j
     const float *colscale;   // kDots16: beta_f
+    int32_t *pred;           // nullable: argmax of each output row (one column slab only)
 };
 
 // How a lane loads VEC consecutive entries of a row of Z and adds them,
@@ -236,6 +237,8 @@ struct StoreRow {
         const int lane = threadIdx.x & 31;
         if (lane / L != 0) return;
         const int sl = lane % L;
+        float bestv = 0.0f;
+        int best = -1;              // this lane's argmax candidate (lowest index on ties)
 #pragma unroll
         for (int v = 0; v < NV; ++v) {
             const int f = f0 + (v * L + sl) * VEC;
@@ -246,6 +249,14 @@ struct StoreRow {
                     o[c] = f + c < p.F ? dinv * (__ldg(p.colscale + f + c) * acc[v][c]) : 0.0f;
                 else
                     o[c] = acc[v][c] * dinv;
+            }
+            if (p.pred != nullptr) {
+#pragma unroll
+                for (int c = 0; c < VEC; ++c)
+                    if (f + c < p.F && (best < 0 || o[c] > bestv)) {
+                        bestv = o[c];
+                        best = f + c;
+                    }
             }
             float *h = p.H + i * p.ldh + f;
             if (p.vec_store && f + VEC <= p.F) {
@@ -261,8 +272,51 @@ struct StoreRow {
                     if (f + c < p.F) h[c] = o[c];
             }
         }
+        if (p.pred != nullptr) {    // the row's argmax over the L lanes of group 0
+            const unsigned gm = L == 32 ? kFullMask : (1u << L) - 1u;
+#pragma unroll
+            for (int o = L / 2; o > 0; o >>= 1) {
+                const float ov = __shfl_xor_sync(gm, bestv, o);
+                const int oi = __shfl_xor_sync(gm, best, o);
+                if (oi >= 0 && (best < 0 || ov > bestv || (ov == bestv && oi < best))) {
+                    bestv = ov;
+                    best = oi;
+                }
+            }
+            if (sl == 0) p.pred[i] = best;
+        }
     }
 };
+
+// Argmax of each row of H (F columns, row stride ldh; lowest index on ties),
+// one warp per row: for outputs too wide for the aggregation's epilogue.
+__global__ void __launch_bounds__(kSpmmThreads)
+argmax_rows_kernel(const float *__restrict__ H, int64_t N, int F, int64_t ldh,
+                   int32_t *__restrict__ pred) {
+    grid_dependency_wait();     // H is the previous kernel's output
+    const int lane = threadIdx.x & 31;
+    const int64_t i = int64_t(blockIdx.x) * kSpmmWarps + (threadIdx.x >> 5);
+    if (i >= N) return;
+    float bestv = 0.0f;
+    int best = -1;
+    for (int f = lane; f < F; f += 32) {
+        const float v = __ldg(H + i * ldh + f);
+        if (best < 0 || v > bestv) {
+            bestv = v;
+            best = f;
+        }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const float ov = __shfl_xor_sync(kFullMask, bestv, o);
+        const int oi = __shfl_xor_sync(kFullMask, best, o);
+        if (oi >= 0 && (best < 0 || ov > bestv || (ov == bestv && oi < best))) {
+            bestv = ov;
+            best = oi;
+        }
+    }
+    if (lane == 0) pred[i] = best;
+}
 
 template <int VEC, int L, int NV, int U, int S, class Epi>
 __device__ __forceinline__ void light_rows(const SpmmParams &p, const Epi &epi, int f0) {
@@ -507,13 +561,18 @@ void launch_cfg(const SpmmArgs &a, const DeviceInfo &dev, int Fload, cudaStream_
     constexpr int kStoreVec = VEC < 4 ? VEC : 4;    // 8-wide rows are stored as two float4
     const bool vec_store = a.ldh % kStoreVec == 0 && aligned_to(a.H, size_t(kStoreVec) * 4);
     const void *Z = S == kDots16 ? static_cast<const void *>(a.D16) : a.Z;
+    const bool one_slab = a.F <= SLAB;
     SpmmParams p{a.rowptr, a.colidx, a.N, a.nnz, Z, a.ldz, Fload, a.F, a.H, a.ldh,
                  heavy_block_count(a.N, dev), heavy_degree(a.N, a.nnz, (32 / L) * U), vec_store,
-                 a.rowscale, a.colscale};
+                 a.rowscale, a.colscale, one_slab ? a.pred : nullptr};
     dim3 grid(unsigned(p.heavy_blocks + (a.N + kSpmmWarps - 1) / kSpmmWarps),
               unsigned((a.F + SLAB - 1) / SLAB));
     launch_kernel(spmm_norm_kernel<VEC, L, NV, U, S>, grid, dim3(kSpmmThreads), 0, s, pdl,
                   dim3(1, 1, 1), p);
+    if (a.pred != nullptr && !one_slab)
+        launch_kernel(argmax_rows_kernel, dim3(unsigned((a.N + kSpmmWarps - 1) / kSpmmWarps)),
+                      dim3(kSpmmThreads), 0, s, pdl, dim3(1, 1, 1), static_cast<const float *>(a.H),
+                      a.N, a.F, a.ldh, a.pred);
 }
 
 // Lanes per neighbour L = the power of two >= the row's vector count (at
@@ -579,7 +638,7 @@ void launch_spmm_pack_gemm(const SpmmPackGemmArgs &a, const DeviceInfo &dev, cud
     const void *Z1 = c16 ? static_cast<const void *>(a.D1) : static_cast<const void *>(a.Z1);
     SpmmParams p{a.rowptr, a.colidx, a.N, a.nnz, Z1, c16 ? a.ldz1 : a.Fh, Fload, a.Fh, nullptr, 0,
                  heavy_block_count(a.N, dev), heavy_degree(a.N, a.nnz, (32 / L) * U), false,
-                 a.s1, nullptr};
+                 a.s1, nullptr, nullptr};
     FusedLayer2 f{a.H1, a.ldh, nullptr, nullptr, nullptr, a.Fo, (a.Fh + 63) / 64, a.Z2, a.ldz2};
     const dim3 grid(unsigned(p.heavy_blocks + (a.N + kSpmmWarps - 1) / kSpmmWarps));
     const dim3 one(1, 1, 1), block(kSpmmThreads);

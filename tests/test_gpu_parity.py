@@ -374,6 +374,40 @@ def test_forward_2layer_k_at_and_past_the_16_bit_limit(cuda_device, N, K, Fh, Fo
     assert_close(H, ref1["H"], "one layer")
 
 
+# Predicted classes: the argmax of each logits row, lowest index on ties
+# (numpy's rule), computed in the last aggregation's epilogue, or by a separate
+# kernel when the rows span more than one column slab (Fo > 256).
+@pytest.mark.parametrize("N,K,Fh,Fo,dup", [
+    (2708, 1433, 64, 7, False),     # Cora-shaped
+    (1000, 602, 128, 41, True),      # ties: W2 columns 3 and 7 equal 0 and 5
+    (300, 100, 64, 80, False),       # unfused layer 2, one slab
+    (257, 70, 32, 300, True),        # two slabs: the separate argmax kernel
+])
+def test_forward_2layer_predictions(cuda_device, N, K, Fh, Fo, dup):
+    case = inputs.layer_case(N, K, Fh, seed=N + Fo, mean_degree=4.0)
+    W2 = inputs.weights(Fh, Fo, seed=Fo)
+    if dup:
+        W2[:, 3], W2[:, 7] = W2[:, 0], W2[:, 5]
+    d = {k: to_dev(v) for k, v in case.items()}
+    ws = torch.empty(B.bigcn_forward_2layer_workspace_bytes(N, K, Fh, Fo), dtype=torch.uint8,
+                     device=cuda_device)
+    H1 = torch.empty((N, Fh), device=cuda_device)
+    out = torch.empty((N, Fo), device=cuda_device)
+    pred = torch.full((N,), -7, dtype=torch.int32, device=cuda_device)
+    B.bigcn_forward_2layer(d["X"], d["s"], d["t"], d["W"], to_dev(W2), d["rowptr"], d["colidx"],
+                           ws, out, H1=H1, pred=pred)
+    logits = out.cpu().numpy()
+    p = pred.cpu().numpy()
+    assert np.array_equal(p, np.argmax(logits, axis=1)), "argmax of the GPU's own logits"
+    if dup:
+        assert not np.any((p == 3) | (p == 7)), "a tie goes to the lower index"
+    ref2 = oracle.layer_forward(H1.cpu().numpy(), W2, case["rowptr"], case["colidx"])["H"]
+    top2 = np.sort(ref2, axis=1)[:, -2:]
+    clear = (top2[:, 1] - top2[:, 0]) > 2 * (1e-6 + 1e-4 * np.abs(top2[:, 1]))
+    assert np.array_equal(p[clear], np.argmax(ref2, axis=1)[clear]), "oracle argmax"
+    assert clear.mean() > 0.5
+
+
 def test_forward_2layer_records_one_event_per_kernel_boundary(cuda_device):
     N, K, Fh, Fo = 500, 300, 64, 7
     case = inputs.layer_case(N, K, Fh, seed=3)
