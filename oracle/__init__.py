@@ -12,6 +12,12 @@ order:
     step 4  zeta = alpha beta (F . B) (Eq. 11, Eq. 12)  oracle_binary_dot, oracle_zeta
     step 5  H = A~ zeta (Eq. 13, Eq. 1)                 oracle_aggregate
 
+and the layer's back-propagation (Algorithm 1, Eqs. bp-H, bp-W):
+
+    G = A~^T dH                      oracle_aggregate_t
+    dL/dW~ = H~^T G, dL/dH~ = G W~^T oracle_grad_wtilde, oracle_grad_htilde
+    dL/dH (clipped), dL/dW (STE)     oracle_grad_input, oracle_grad_weight
+
 Naming follows the layer's C interface: ``alpha`` is the per-node scale (the
 paper's beta, Eq. 7) and ``beta`` the per-weight-column scale (the paper's
 alpha, Eq. 4). Floating-point results are float64; the only fp32 arithmetic is
@@ -66,6 +72,16 @@ def lib() -> ctypes.CDLL:
             h.oracle_aggregate.argtypes = [_i64p, _i32p, _i64, _f64p, _i32, _vp, _i64,
                                            _f64p, _vp]
             h.oracle_aggregate.restype = ctypes.c_int
+            h.oracle_aggregate_t.argtypes = [_i64p, _i32p, _i64, _f64p, _i32, _f64p]
+            h.oracle_aggregate_t.restype = ctypes.c_int
+            h.oracle_grad_wtilde.argtypes = [_i8p, _f64p, _f64p, _i64, _i32, _i32, _f64p, _vp]
+            h.oracle_grad_wtilde.restype = None
+            h.oracle_grad_htilde.argtypes = [_f64p, _f64p, _i8p, _i64, _i32, _i32, _f64p, _vp]
+            h.oracle_grad_htilde.restype = None
+            h.oracle_grad_input.argtypes = [_f64p, _i64, _f64p]
+            h.oracle_grad_input.restype = None
+            h.oracle_grad_weight.argtypes = [_f64p, _i8p, _f64p, _f32p, _i32, _i32, _i64, _f64p]
+            h.oracle_grad_weight.restype = None
             _lib = h
     return _lib
 
@@ -222,3 +238,80 @@ def forward_2layer(X, s, t, W1, W2, rowptr, colidx) -> dict:
     H1 = l1["H"].astype(np.float32)
     l2 = layer_forward(H1, W2, rowptr, colidx)
     return dict(layer1=l1, layer2=l2, H1=H1, logits=l2["H"])
+
+
+# ------------------------------------------------------- back-propagation ----
+def aggregate_t(rowptr, colidx, dH) -> np.ndarray:
+    """Algorithm 1: G = A~^T dH, scattering each row's gradient to its
+    neighbours and itself (float64)."""
+    rowptr = _c(rowptr, np.int64)
+    colidx = _c(colidx, np.int32)
+    dH = _c(dH, np.float64)
+    N, F = dH.shape
+    assert rowptr.shape[0] == N + 1
+    G = np.empty((N, F), np.float64)
+    if colidx.size == 0:
+        colidx = np.zeros(1, np.int32)
+    if lib().oracle_aggregate_t(rowptr, colidx, N, dH, F, G) != 0:
+        raise ValueError("malformed CSR")
+    return G
+
+
+def grad_wtilde(SF, alpha, G, with_absterm=False):
+    """Algorithm 1: dL/dW~ = H~^T G with H~ = diag(alpha) SF (K x F)."""
+    SF = _c(SF, np.int8)
+    G = _c(G, np.float64)
+    N, K = SF.shape
+    F = G.shape[1]
+    out = np.empty((K, F), np.float64)
+    a = np.empty(F, np.float64) if with_absterm else None
+    lib().oracle_grad_wtilde(SF, _c(alpha, np.float64), G, N, K, F, out,
+                             None if a is None else a.ctypes.data)
+    return (out, a) if with_absterm else out
+
+
+def grad_htilde(G, beta, SB, with_absterm=False):
+    """Algorithm 1: dL/dH~ = G W~^T with W~[k,j] = beta_j SB[j,k] (N x K)."""
+    G = _c(G, np.float64)
+    SB = _c(SB, np.int8)
+    N, F = G.shape
+    K = SB.shape[1]
+    out = np.empty((N, K), np.float64)
+    a = np.empty(N, np.float64) if with_absterm else None
+    lib().oracle_grad_htilde(G, _c(beta, np.float64), SB, N, K, F, out,
+                             None if a is None else a.ctypes.data)
+    return (out, a) if with_absterm else out
+
+
+def grad_input(Ht) -> np.ndarray:
+    """Eq. bp-H: dL/dH = dL/dH~ where |dL/dH~| < 1, else 0."""
+    Ht = _c(Ht, np.float64)
+    out = np.empty(Ht.shape, np.float64)
+    lib().oracle_grad_input(Ht.reshape(-1), Ht.size, out.reshape(-1))
+    return out
+
+
+def grad_weight(Wg, SB, beta, Wt) -> np.ndarray:
+    """Eq. bp-W (d_in = K): the gradient of W through the column scale plus
+    the straight-through estimator 1(|W| < 1) of sign()."""
+    Wg = _c(Wg, np.float64)
+    Wt = _c(Wt, np.float32)
+    K, F = Wt.shape
+    out = np.empty((K, F), np.float64)
+    lib().oracle_grad_weight(Wg, _c(SB, np.int8), _c(beta, np.float64), Wt, K, F, F, out)
+    return out
+
+
+def layer_backward(X, Wt, rowptr, colidx, dH, s=None, t=None) -> dict:
+    """Algorithm 1 for one layer: from dL/dH^(l+1) (dH, N x F) to dL/dH^(l)
+    (Eq. bp-H, w.r.t. the layer's binarized input, i.e. the centred X for
+    layer 1) and dL/dW (Eq. bp-W), every intermediate kept."""
+    Y = centre(X, s, t)
+    SF = sign(Y)
+    alpha = row_scale(Y)
+    SB, beta = weight_binarize(Wt)
+    G = aggregate_t(rowptr, colidx, dH)
+    Wg, wg_abs = grad_wtilde(SF, alpha, G, with_absterm=True)
+    Ht, ht_abs = grad_htilde(G, beta, SB, with_absterm=True)
+    return dict(Y=Y, SF=SF, alpha=alpha, SB=SB, beta=beta, G=G, Wg=Wg, Wg_abs=wg_abs,
+                Ht=Ht, Ht_abs=ht_abs, dX=grad_input(Ht), dW=grad_weight(Wg, SB, beta, Wt))

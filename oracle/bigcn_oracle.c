@@ -12,6 +12,10 @@
  *                     mean absolute value over the d_in entries of the bucket
  *   binary product .. Eq. 11 / Eq. 12 (dot of +-1 vectors, then scaled)
  *   aggregation ..... Eq. 13 with the operator of Eq. 1, D^-1/2 (A+I) D^-1/2
+ *   back-propagation  Algorithm 1 (A~^T dH, H~^T G, G W~^T), Eq. bp-H (the
+ *                     gradient of the layer input, clipped to |.| < 1) and
+ *                     Eq. bp-W (the weight gradient through the column scale
+ *                     and the straight-through estimator of sign)
  *
  * The pins that tie these routines to the paper and to mathematics (brute
  * force on tiny inputs, the scale's least-squares optimality, dense-matrix
@@ -22,6 +26,7 @@
 
 #include <math.h>
 #include <stddef.h>
+#include <stdlib.h>
 
 void oracle_centre(const float *X, int64_t N, int32_t K, int64_t ldx,
                    const float *s, const float *t, float *Y) {
@@ -148,4 +153,88 @@ int oracle_aggregate(const int64_t *rowptr, const int32_t *colidx, int64_t N,
         }
     }
     return 0;
+}
+
+/* ---- Back-propagation (Algorithm 1, Eqs. bp-H, bp-W) ---- */
+
+int oracle_aggregate_t(const int64_t *rowptr, const int32_t *colidx, int64_t N,
+                       const double *dH, int32_t F, double *G) {
+    double *dhat;
+    int64_t i, e;
+    int32_t f;
+    if (rowptr[0] != 0) return -1;
+    for (i = 0; i < N; ++i)
+        if (rowptr[i + 1] < rowptr[i]) return -1;
+    for (e = 0; e < rowptr[N]; ++e)
+        if (colidx[e] < 0 || colidx[e] >= N) return -1;
+    dhat = (double *)malloc(sizeof(double) * (size_t)(N > 0 ? N : 1));
+    if (!dhat) return -1;
+    oracle_degree(rowptr, N, dhat);
+    for (i = 0; i < N * (int64_t)F; ++i) G[i] = 0.0;
+    for (i = 0; i < N; ++i) {
+        /* the self-loop of A + I, then the CSR entries of row i */
+        for (e = rowptr[i] - 1; e < rowptr[i + 1]; ++e) {
+            const int64_t jj = (e < rowptr[i]) ? i : (int64_t)colidx[e];
+            const double c = 1.0 / sqrt(dhat[i] * dhat[jj]);
+            for (f = 0; f < F; ++f) G[jj * F + f] += dH[i * F + f] * c;
+        }
+    }
+    free(dhat);
+    return 0;
+}
+
+void oracle_grad_wtilde(const int8_t *SF, const double *alpha, const double *G,
+                        int64_t N, int32_t K, int32_t F, double *out, double *absterm) {
+    int64_t i;
+    int32_t k, j;
+    for (k = 0; k < K; ++k)
+        for (j = 0; j < F; ++j) {
+            double acc = 0.0;
+            for (i = 0; i < N; ++i) acc += alpha[i] * (double)SF[i * K + k] * G[i * F + j];
+            out[(int64_t)k * F + j] = acc;
+        }
+    if (absterm)
+        for (j = 0; j < F; ++j) {
+            double a = 0.0;
+            for (i = 0; i < N; ++i) a += fabs(alpha[i] * G[i * F + j]);
+            absterm[j] = a;
+        }
+}
+
+void oracle_grad_htilde(const double *G, const double *beta, const int8_t *SB,
+                        int64_t N, int32_t K, int32_t F, double *out, double *absterm) {
+    int64_t i;
+    int32_t k, j;
+    for (i = 0; i < N; ++i) {
+        for (k = 0; k < K; ++k) {
+            double acc = 0.0;
+            for (j = 0; j < F; ++j) acc += G[i * F + j] * beta[j] * (double)SB[(int64_t)j * K + k];
+            out[i * K + k] = acc;
+        }
+        if (absterm) {
+            double a = 0.0;
+            for (j = 0; j < F; ++j) a += fabs(G[i * F + j] * beta[j]);
+            absterm[i] = a;
+        }
+    }
+}
+
+void oracle_grad_input(const double *Ht, int64_t n, double *out) {
+    int64_t q;
+    for (q = 0; q < n; ++q) out[q] = fabs(Ht[q]) < 1.0 ? Ht[q] : 0.0;
+}
+
+void oracle_grad_weight(const double *Wg, const int8_t *SB, const double *beta,
+                        const float *Wt, int32_t K, int32_t F, int64_t ldw, double *out) {
+    int32_t k, j, m;
+    for (j = 0; j < F; ++j) {
+        double c = 0.0;   /* sum_m dL/dW~[m,j] B[m,j] */
+        for (m = 0; m < K; ++m) c += Wg[(int64_t)m * F + j] * (double)SB[(int64_t)j * K + m];
+        for (k = 0; k < K; ++k) {
+            const double w = (double)Wt[(int64_t)k * ldw + j];
+            const double ste = fabs(w) < 1.0 ? 1.0 : 0.0;
+            out[(int64_t)k * F + j] = (double)SB[(int64_t)j * K + k] * c / (double)K +
+                                      beta[j] * Wg[(int64_t)k * F + j] * ste;
+        }
+    }
 }

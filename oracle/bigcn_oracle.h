@@ -1,7 +1,7 @@
 /*
  * bigcn_oracle.h -- plain CPU oracle of the Bi-GCN binarized graph-convolution
- * layer forward (Wang et al., "Bi-GCN: Binary Graph Convolutional Network",
- * CVPR 2021, arXiv:2010.07565).
+ * layer, forward and back-propagation (Wang et al., "Bi-GCN: Binary Graph
+ * Convolutional Network", CVPR 2021, arXiv:2010.07565).
  *
  * TEST INFRASTRUCTURE. Only the test suite, the smoke check and the
  * benchmark's CPU-baseline leg load this library. It shares no source, header,
@@ -73,6 +73,40 @@ void oracle_degree(const int64_t *rowptr, int64_t N, double *dhat);
 int oracle_aggregate(const int64_t *rowptr, const int32_t *colidx, int64_t N,
                      const double *zeta, int32_t F, const int64_t *rows,
                      int64_t nrows, double *H, double *absterm);
+
+/* ---- Back-propagation of one layer (Algorithm 1, Eqs. bp-H and bp-W). ----
+ * G = dL/dzeta, Ht = dL/dH~, Wt~ = dL/dW~ below are all double. The layer's
+ * binarized operands are H~ = diag(alpha) SF (N x K) and W~[k,j] =
+ * beta_j SB[j,k] (K x F). */
+
+/* Algorithm 1, first line: G = A~^T dH with A~ = D^-1/2 (A + I) D^-1/2,
+ * applied as written: row i's incoming gradient is scattered to every j in
+ * N(i) u {i} as dH[i,:] / sqrt(dhat_i dhat_j). Returns 0, or -1 for a
+ * malformed CSR. */
+int oracle_aggregate_t(const int64_t *rowptr, const int32_t *colidx, int64_t N,
+                       const double *dH, int32_t F, double *G);
+
+/* Algorithm 1: dL/dW~ = H~^T G, i.e. out[k,j] = sum_i alpha_i SF[i,k] G[i,j]
+ * (K x F). absterm[j] (nullable) = sum_i |alpha_i G[i,j]|, the scale of any
+ * evaluation order's rounding error (the same for every k). */
+void oracle_grad_wtilde(const int8_t *SF, const double *alpha, const double *G,
+                        int64_t N, int32_t K, int32_t F, double *out, double *absterm);
+
+/* Algorithm 1: dL/dH~ = G W~^T (the printed "G . W~" is read with the
+ * transpose the shapes require): out[i,k] = sum_j G[i,j] beta_j SB[j,k]
+ * (N x K). absterm[i] (nullable) = sum_j |G[i,j] beta_j|. */
+void oracle_grad_htilde(const double *G, const double *beta, const int8_t *SB,
+                        int64_t N, int32_t K, int32_t F, double *out, double *absterm);
+
+/* Eq. bp-H: dL/dH[i,k] = dL/dH~[i,k] * 1(|dL/dH~[i,k]| < 1), over n values. */
+void oracle_grad_input(const double *Ht, int64_t n, double *out);
+
+/* Eq. bp-W with d_in = K: out[k,j] = (1/K) SB[j,k] sum_m Wg[m,j] SB[j,m]
+ * + beta_j Wg[k,j] 1(|W[k,j]| < 1), Wg = dL/dW~ (K x F), W = Wt (K x F,
+ * row stride ldw), the straight-through estimator of sign() being
+ * 1(|r| < 1). */
+void oracle_grad_weight(const double *Wg, const int8_t *SB, const double *beta,
+                        const float *Wt, int32_t K, int32_t F, int64_t ldw, double *out);
 
 #ifdef __cplusplus
 }
