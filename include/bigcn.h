@@ -272,6 +272,35 @@ bigcn_status bigcn_forward_2layer(const float *X, int64_t N, int32_t K, int64_t 
                                   int32_t *pred, void *const *events, int32_t n_events,
                                   void *stream);
 
+/*
+ * Back-propagation of one layer (Algorithm 1 with Eqs. bp-H and bp-W), from
+ * the gradient dH = dL/dH^(l+1) of the layer's output (N x F, row stride ldg)
+ * to
+ *   dX = dL/dH^(l) (nullable; N x K, row stride lddx): Algorithm 1's
+ *        dL/dH~ = G W~^T clipped by Eq. bp-H (entries with |.| >= 1 are 0),
+ *        the gradient of the layer's binarized input (for layer 1, the
+ *        centred features);
+ *   dW = dL/dW (K x F, row stride lddw): Eq. bp-W with d_in = K and the
+ *        straight-through estimator 1(|W| < 1) of sign(),
+ * where G = A~^T dH, dL/dW~ = H~^T G, H~ = diag(alpha) sign(Y) and W~ =
+ * sign(W) diag(beta) are those of the forward with the same X, scale/shift
+ * and Wt (the signs and scales are recomputed from them). A~^T is applied as
+ * A~: the CSR must be symmetric, as everywhere in this interface.
+ * workspace  >= bigcn_layer_backward_workspace_bytes(N, K, F) bytes of device
+ *            memory, 256-byte aligned, overlapping no argument.
+ * dX and dW must not overlap each other or any input. The sums over the N
+ * rows (dW) are evaluated in a fixed order (chunks of rows added in order).
+ */
+size_t bigcn_layer_backward_workspace_bytes(int64_t N, int32_t K, int32_t F);
+
+bigcn_status bigcn_layer_backward(const float *X, int64_t N, int32_t K, int64_t ldx,
+                                  const float *scale, const float *shift,
+                                  const float *Wt, int32_t F, int64_t ldw,
+                                  const int64_t *rowptr, const int32_t *colidx, int64_t nnz,
+                                  const float *dH, int64_t ldg, float *dX, int64_t lddx,
+                                  float *dW, int64_t lddw, void *workspace, size_t ws_bytes,
+                                  void *stream);
+
 /* Bytes of the device scratch array behind bigcn_layer_forward_static. */
 #define BIGCN_STATIC_SCRATCH_BYTES ((size_t)32 << 20)
 

@@ -50,6 +50,9 @@ SIGNATURES = {
                              _sz, _p, _i64, _p], ctypes.c_int),
     "bigcn_layer_forward_timed": ([_p, _i64, _i32, _i64, _p, _p, _p, _i32, _i64, _p, _p, _i64,
                                    _p, _sz, _p, _i64, _p, _i32, _p], ctypes.c_int),
+    "bigcn_layer_backward_workspace_bytes": ([_i64, _i32, _i32], _sz),
+    "bigcn_layer_backward": ([_p, _i64, _i32, _i64, _p, _p, _p, _i32, _i64, _p, _p, _i64, _p,
+                              _i64, _p, _i64, _p, _i64, _p, _sz, _p], ctypes.c_int),
     "bigcn_forward_2layer_workspace_bytes": ([_i64, _i32, _i32, _i32], _sz),
     "bigcn_forward_2layer_launches": ([_i64, _i32, _i32, _i32], _i32),
     "bigcn_forward_2layer": ([_p, _i64, _i32, _i64, _p, _p, _p, _i32, _i64, _p, _i32, _i64, _p,
@@ -211,6 +214,23 @@ def bigcn_layer_forward_timed(X, scale, shift, Wt, rowptr, colidx, workspace, H,
         _ptr(colidx) if colidx.numel() else None, colidx.numel(), _ptr(workspace),
         workspace.numel() * workspace.element_size(), _ptr(H), _ld(H), ev, len(events),
         _stream(stream)))
+
+
+def bigcn_layer_backward_workspace_bytes(N: int, K: int, F: int) -> int:
+    return int(lib().bigcn_layer_backward_workspace_bytes(N, K, F))
+
+
+def bigcn_layer_backward(X, scale, shift, Wt, rowptr, colidx, dH, workspace, dW, dX=None,
+                         stream=None):
+    """Algorithm 1 for one layer: dW (K x F, Eq. bp-W) and optionally dX
+    (N x K, Eq. bp-H) from dH = dL/dH^(l+1) (N x F)."""
+    N, K = X.shape
+    F = Wt.shape[1]
+    _check("bigcn_layer_backward", lib().bigcn_layer_backward(
+        _ptr(X), N, K, _ld(X), _ptr(scale), _ptr(shift), _ptr(Wt), F, _ld(Wt), _ptr(rowptr),
+        _ptr(colidx) if colidx.numel() else None, colidx.numel(), _ptr(dH), _ld(dH), _ptr(dX),
+        _ld(dX) if dX is not None else 0, _ptr(dW), _ld(dW), _ptr(workspace),
+        workspace.numel() * workspace.element_size(), _stream(stream)))
 
 
 def bigcn_forward_2layer_workspace_bytes(N: int, K: int, Fh: int, Fo: int) -> int:

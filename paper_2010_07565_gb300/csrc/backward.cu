@@ -1,0 +1,308 @@
+// Back-propagation of one Bi-GCN layer (Wang et al., CVPR 2021, Algorithm 1,
+// Eqs. bp-H and bp-W), from dL/dH^(l+1) (dH, N x F) to the gradient of the
+// layer's binarized input and of its weights:
+//
+//   G      = A~^T dH                 = A~ dH (the CSR is symmetric)
+//   dW~    = H~^T G,  H~ = diag(alpha) sign(Y)          (K x F)
+//   dH~    = G W~^T,  W~[k,j] = beta_j sign(W_kj)       (N x K)
+//   dL/dH  = dH~ * 1(|dH~| < 1)                          Eq. bp-H
+//   dL/dW  = (1/K) B_kj sum_m dW~_mj B_mj
+//            + beta_j dW~_kj 1(|W_kj| < 1)               Eq. bp-W
+//
+// (alpha: per-node scale, the paper's beta; beta: per-column scale, the
+// paper's alpha; B = sign(W).) The signs come packed from the forward's own
+// kernels (the rows re-packed from X with the same centring, the columns
+// from W). Both products multiply a +-1 matrix by an fp32 one; they run on
+// the CUDA cores in fp32 (the tensor cores' bf16 / tf32 inputs would round
+// G): 64 x 64 output tiles, each thread a 4 x 4 register block that adds
+// +-v for the signs of one packed word.
+//
+// dW~ sums over all N rows: the rows are split into S chunks (grid z) whose
+// partial sums are added, chunk by chunk in order, by a second kernel, so
+// the result does not depend on scheduling.
+#include "launch.cuh"
+
+namespace bigcn {
+namespace {
+
+constexpr int kBwThreads = 256;
+constexpr int kTile = 64;        // output tile edge
+constexpr int kRowsPerStage = 32;
+
+// +1.0f where bit b of w is set, else -1.0f.
+__device__ __forceinline__ float pm1(uint64_t w, int b) {
+    return ((w >> b) & 1ull) ? 1.0f : -1.0f;
+}
+
+// Partial dW~ over the rows [chunk start, chunk end): tile (kt, jt) of the
+// K x F output, thread (tk, tj) owning k = 64 kt + 4 tk + 0..3 and
+// j = 64 jt + 4 tj + 0..3.
+__global__ void __launch_bounds__(kBwThreads)
+grad_wtilde_kernel(const uint64_t *__restrict__ bits, int words, const float *__restrict__ alpha,
+                   const float *__restrict__ G, int64_t ldg, int64_t N, int K, int F,
+                   int64_t chunk, float *__restrict__ partial) {
+    __shared__ __align__(16) float sV[kRowsPerStage][kTile];    // alpha_i G[i, j-tile]
+    __shared__ uint64_t sB[kRowsPerStage];                      // row i's word of the k-tile
+    const int tid = threadIdx.x, tk = tid / 16, tj = tid % 16;
+    const int kt = blockIdx.x, jt = blockIdx.y;
+    const int64_t r0 = int64_t(blockIdx.z) * chunk;
+    const int64_t r1 = r0 + chunk < N ? r0 + chunk : N;
+    float acc[4][4] = {};
+    for (int64_t base = r0; base < r1; base += kRowsPerStage) {
+        __syncthreads();
+        for (int q = tid; q < kRowsPerStage * kTile; q += kBwThreads) {
+            const int r = q / kTile, c = q % kTile;
+            const int64_t i = base + r;
+            const int j = jt * kTile + c;
+            sV[r][c] = (i < r1 && j < F) ? __ldg(alpha + i) * __ldg(G + i * ldg + j) : 0.0f;
+        }
+        for (int r = tid; r < kRowsPerStage; r += kBwThreads) {
+            const int64_t i = base + r;
+            sB[r] = i < r1 ? __ldg(bits + i * words + kt) : 0ull;
+        }
+        __syncthreads();
+        const int n = int(r1 - base < kRowsPerStage ? r1 - base : kRowsPerStage);
+        for (int r = 0; r < n; ++r) {
+            const uint64_t w = sB[r];
+            const float4 v = *reinterpret_cast<const float4 *>(&sV[r][4 * tj]);
+#pragma unroll
+            for (int a = 0; a < 4; ++a) {
+                const float s = pm1(w, 4 * tk + a);
+                acc[a][0] = fmaf(s, v.x, acc[a][0]);
+                acc[a][1] = fmaf(s, v.y, acc[a][1]);
+                acc[a][2] = fmaf(s, v.z, acc[a][2]);
+                acc[a][3] = fmaf(s, v.w, acc[a][3]);
+            }
+        }
+    }
+    float *out = partial + int64_t(blockIdx.z) * K * F;
+#pragma unroll
+    for (int a = 0; a < 4; ++a) {
+        const int k = kt * kTile + 4 * tk + a;
+        if (k >= K) continue;
+#pragma unroll
+        for (int b = 0; b < 4; ++b) {
+            const int j = jt * kTile + 4 * tj + b;
+            if (j < F) out[int64_t(k) * F + j] = acc[a][b];
+        }
+    }
+}
+
+// dW~ = the S partial sums added in chunk order.
+__global__ void __launch_bounds__(kBwThreads)
+sum_partials_kernel(const float *__restrict__ partial, int S, int64_t n, float *__restrict__ out) {
+    for (int64_t q = int64_t(blockIdx.x) * kBwThreads + threadIdx.x; q < n;
+         q += int64_t(gridDim.x) * kBwThreads) {
+        float t = 0.0f;
+        for (int s = 0; s < S; ++s) t += __ldg(partial + int64_t(s) * n + q);
+        out[q] = t;
+    }
+}
+
+// dL/dH (Eq. bp-H) for tile (it, kt) of the N x K output: thread (ti, tk)
+// owns rows 64 it + 4 ti + 0..3 and k = 64 kt + 4 tk + 0..3; the sum over j
+// walks the F columns of G (times beta_j) and the signs of W's column j.
+__global__ void __launch_bounds__(kBwThreads)
+grad_input_kernel(const float *__restrict__ G, int64_t ldg, const float *__restrict__ beta,
+                  const uint64_t *__restrict__ wbits, int words, int64_t N, int K, int F,
+                  float *__restrict__ dX, int64_t lddx) {
+    __shared__ __align__(16) float sG[kRowsPerStage][kTile];    // beta_j G[i, j], [j][row]
+    __shared__ uint64_t sW[kRowsPerStage];                      // column j's word of the k-tile
+    const int tid = threadIdx.x, ti = tid / 16, tk = tid % 16;
+    const int64_t i0 = int64_t(blockIdx.x) * kTile;
+    const int kt = blockIdx.y;
+    float acc[4][4] = {};
+    for (int j0 = 0; j0 < F; j0 += kRowsPerStage) {
+        __syncthreads();
+        for (int q = tid; q < kRowsPerStage * kTile; q += kBwThreads) {
+            const int jj = q / kTile, r = q % kTile;
+            const int64_t i = i0 + r;
+            const int j = j0 + jj;
+            sG[jj][r] = (i < N && j < F) ? __ldg(beta + j) * __ldg(G + i * ldg + j) : 0.0f;
+        }
+        for (int jj = tid; jj < kRowsPerStage; jj += kBwThreads) {
+            const int j = j0 + jj;
+            sW[jj] = j < F ? __ldg(wbits + int64_t(j) * words + kt) : 0ull;
+        }
+        __syncthreads();
+        const int n = F - j0 < kRowsPerStage ? F - j0 : kRowsPerStage;
+        for (int jj = 0; jj < n; ++jj) {
+            const uint64_t w = sW[jj];
+            const float4 g = *reinterpret_cast<const float4 *>(&sG[jj][4 * ti]);
+            float s[4];
+#pragma unroll
+            for (int b = 0; b < 4; ++b) s[b] = pm1(w, 4 * tk + b);
+#pragma unroll
+            for (int b = 0; b < 4; ++b) {
+                acc[0][b] = fmaf(g.x, s[b], acc[0][b]);
+                acc[1][b] = fmaf(g.y, s[b], acc[1][b]);
+                acc[2][b] = fmaf(g.z, s[b], acc[2][b]);
+                acc[3][b] = fmaf(g.w, s[b], acc[3][b]);
+            }
+        }
+    }
+#pragma unroll
+    for (int a = 0; a < 4; ++a) {
+        const int64_t i = i0 + 4 * ti + a;
+        if (i >= N) continue;
+#pragma unroll
+        for (int b = 0; b < 4; ++b) {
+            const int k = kt * kTile + 4 * tk + b;
+            if (k < K) dX[i * lddx + k] = fabsf(acc[a][b]) < 1.0f ? acc[a][b] : 0.0f;
+        }
+    }
+}
+
+// Eq. bp-W, one warp per column j: c_j = sum_k dW~_kj B_kj (lane-strided,
+// then a fixed shuffle tree), then every entry of the column.
+__global__ void __launch_bounds__(kBwThreads)
+grad_weight_kernel(const float *__restrict__ Wg, const uint64_t *__restrict__ wbits, int words,
+                   const float *__restrict__ beta, const float *__restrict__ Wt, int64_t ldw,
+                   int K, int F, float *__restrict__ dW, int64_t lddw) {
+    const int lane = threadIdx.x & 31;
+    const int j = blockIdx.x * (kBwThreads / 32) + (threadIdx.x >> 5);
+    if (j >= F) return;
+    const uint64_t *wb = wbits + int64_t(j) * words;
+    float c = 0.0f;
+    for (int k = lane; k < K; k += 32) c = fmaf(__ldg(Wg + int64_t(k) * F + j), pm1(__ldg(wb + k / 64), k % 64), c);
+    c = warp_sum(c);
+    const float bj = __ldg(beta + j), cK = c / float(K);
+    for (int k = lane; k < K; k += 32) {
+        const float w = __ldg(Wt + int64_t(k) * ldw + j);
+        const float ste = fabsf(w) < 1.0f ? 1.0f : 0.0f;
+        dW[int64_t(k) * lddw + j] =
+            pm1(__ldg(wb + k / 64), k % 64) * cK + bj * __ldg(Wg + int64_t(k) * F + j) * ste;
+    }
+}
+
+constexpr size_t kAlign = 256;
+size_t round_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+
+// Most row chunks the dW~ reduction may use for a K x F output: enough for
+// about two blocks per SM on up to 256 SMs, at most 64.
+int64_t max_chunks(int K, int F) {
+    const int64_t tiles = int64_t((K + kTile - 1) / kTile) * ((F + kTile - 1) / kTile);
+    const int64_t s = (512 + tiles - 1) / tiles;
+    return s < 64 ? s : 64;
+}
+
+// Row chunks of the dW~ reduction: about two blocks per SM in all.
+int wtilde_chunks(int64_t N, int K, int F, const DeviceInfo &dev) {
+    const int64_t tiles = int64_t((K + kTile - 1) / kTile) * ((F + kTile - 1) / kTile);
+    int64_t S = (2 * int64_t(dev.sm_count) + tiles - 1) / tiles;
+    const int64_t max_s = (N + kRowsPerStage - 1) / kRowsPerStage;
+    if (S > max_s) S = max_s;
+    if (S > max_chunks(K, F)) S = max_chunks(K, F);
+    return int(S < 1 ? 1 : S);
+}
+
+struct BackwardWorkspace {
+    size_t bits, alpha, wbits, beta, g, wg, partial, total;
+};
+
+bool backward_workspace(int64_t N, int32_t K, int32_t F, BackwardWorkspace *w) {
+    if (N < 0 || K < 1 || F < 1) return false;
+    const int64_t words = bigcn_words(K);
+    if (N > kMaxElems / (words > F ? words : F)) return false;
+    size_t off = 0;
+    auto take = [&](size_t bytes) { size_t at = off; off = round_up(off + bytes); return at; };
+    w->bits = take(size_t(N) * words * 8);
+    w->alpha = take(size_t(N) * 4);
+    w->wbits = take(size_t(F) * words * 8);
+    w->beta = take(size_t(F) * 4);
+    w->g = take(size_t(N) * F * 4);
+    w->wg = take(size_t(K) * F * 4);
+    w->partial = take(size_t(max_chunks(K, F)) * K * F * 4);
+    w->total = off;
+    return true;
+}
+
+}  // namespace
+}  // namespace bigcn
+
+using namespace bigcn;
+
+extern "C" size_t bigcn_layer_backward_workspace_bytes(int64_t N, int32_t K, int32_t F) {
+    BackwardWorkspace w;
+    return backward_workspace(N, K, F, &w) ? w.total : 0;
+}
+
+extern "C" bigcn_status bigcn_layer_backward(
+    const float *X, int64_t N, int32_t K, int64_t ldx, const float *scale, const float *shift,
+    const float *Wt, int32_t F, int64_t ldw, const int64_t *rowptr, const int32_t *colidx,
+    int64_t nnz, const float *dH, int64_t ldg, float *dX, int64_t lddx, float *dW, int64_t lddw,
+    void *workspace, size_t ws_bytes, void *stream) {
+    BackwardWorkspace w;
+    if (N < 0 || N > int64_t(INT32_MAX) || K < 1 || F < 1 || ldx < K || ldw < F || ldg < F ||
+        (dX && lddx < K) || lddw < F || nnz < 0)
+        return BIGCN_ERR_INVALID_ARG;
+    if ((scale == nullptr) != (shift == nullptr)) return BIGCN_ERR_INVALID_ARG;
+    if (!backward_workspace(N, K, F, &w)) return BIGCN_ERR_INVALID_ARG;
+    if (N > 0 && (N > kMaxElems / ldx || N > kMaxElems / ldg || (dX && N > kMaxElems / lddx)))
+        return BIGCN_ERR_INVALID_ARG;
+    if (int64_t(K) > kMaxElems / ldw || int64_t(K) > kMaxElems / lddw) return BIGCN_ERR_INVALID_ARG;
+    if (!Wt || !dW) return BIGCN_ERR_INVALID_ARG;
+    if (N > 0 && (!X || !rowptr || !dH || !workspace || (nnz > 0 && !colidx)))
+        return BIGCN_ERR_INVALID_ARG;
+    if (N > 0 && ws_bytes < w.total) return BIGCN_ERR_INVALID_ARG;
+    if ((X && !aligned_to(X, 4)) || !aligned_to(Wt, 4) || (rowptr && !aligned_to(rowptr, 8)) ||
+        (colidx && !aligned_to(colidx, 4)) || (dH && !aligned_to(dH, 4)) ||
+        (dX && !aligned_to(dX, 4)) || !aligned_to(dW, 4) ||
+        (workspace && !aligned_to(workspace, kAlign)) ||
+        (scale && (!aligned_to(scale, 4) || !aligned_to(shift, 4))))
+        return BIGCN_ERR_MISALIGNED;
+    const size_t dwb = span_bytes(K, F, lddw, 4), dxb = dX ? span_bytes(N, K, lddx, 4) : 0;
+    const void *in[] = {X, Wt, rowptr, colidx, dH, scale, shift};
+    const size_t in_bytes[] = {span_bytes(N, K, ldx, 4), span_bytes(K, F, ldw, 4),
+                               size_t(N + 1) * 8, size_t(nnz) * 4, span_bytes(N, F, ldg, 4),
+                               size_t(K) * 4, size_t(K) * 4};
+    const void *outs[] = {dW, dX, N > 0 ? workspace : nullptr};
+    const size_t out_bytes[] = {dwb, dxb, N > 0 ? w.total : 0};
+    for (int o = 0; o < 3; ++o) {
+        for (int q = 0; q < 7; ++q)
+            if (overlaps(outs[o], out_bytes[o], in[q], in_bytes[q])) return BIGCN_ERR_INVALID_ARG;
+        for (int p = o + 1; p < 3; ++p)
+            if (overlaps(outs[o], out_bytes[o], outs[p], out_bytes[p])) return BIGCN_ERR_INVALID_ARG;
+    }
+    DeviceInfo dev;
+    bigcn_status st = current_device(&dev);
+    if (st != BIGCN_OK) return st;
+    cudaStream_t s = as_stream(stream);
+    if (N == 0) {       // no rows: dW~ = 0, so dW = 0
+        if (cudaMemset2DAsync(dW, size_t(lddw) * 4, 0, size_t(F) * 4, size_t(K), s) != cudaSuccess) {
+            cudaGetLastError();
+            return BIGCN_ERR_CUDA;
+        }
+        return BIGCN_OK;
+    }
+
+    char *ws = static_cast<char *>(workspace);
+    uint64_t *bits = reinterpret_cast<uint64_t *>(ws + w.bits);
+    float *alpha = reinterpret_cast<float *>(ws + w.alpha);
+    uint64_t *wbits = reinterpret_cast<uint64_t *>(ws + w.wbits);
+    float *beta = reinterpret_cast<float *>(ws + w.beta);
+    float *G = reinterpret_cast<float *>(ws + w.g);
+    float *Wg = reinterpret_cast<float *>(ws + w.wg);
+    float *partial = reinterpret_cast<float *>(ws + w.partial);
+    const int words = bigcn_words(K);
+
+    launch_pack_rows(X, N, K, ldx, scale, shift, bits, words, alpha, dev, s);
+    launch_pack_weights(Wt, K, F, ldw, wbits, words, beta, s);
+    SpmmArgs a{rowptr, colidx, N, nnz, dH, ldg, F, G, F, false, false};
+    launch_spmm_norm(a, dev, s);                                   // G = A~ dH
+    const int S = wtilde_chunks(N, K, F, dev);
+    const int64_t chunk = (N + S - 1) / S;
+    const dim3 gw(unsigned((K + kTile - 1) / kTile), unsigned((F + kTile - 1) / kTile), unsigned(S));
+    grad_wtilde_kernel<<<gw, kBwThreads, 0, s>>>(bits, words, alpha, G, F, N, K, F, chunk, partial);
+    const int64_t kf = int64_t(K) * F;
+    sum_partials_kernel<<<unsigned((kf + kBwThreads - 1) / kBwThreads < 4096
+                                       ? (kf + kBwThreads - 1) / kBwThreads : 4096),
+                          kBwThreads, 0, s>>>(partial, S, kf, Wg);
+    if (dX) {
+        const dim3 gi(unsigned((N + kTile - 1) / kTile), unsigned((K + kTile - 1) / kTile));
+        grad_input_kernel<<<gi, kBwThreads, 0, s>>>(G, F, beta, wbits, words, N, K, F, dX, lddx);
+    }
+    grad_weight_kernel<<<unsigned((F + kBwThreads / 32 - 1) / (kBwThreads / 32)), kBwThreads, 0,
+                         s>>>(Wg, wbits, words, beta, Wt, ldw, K, F, dW, lddw);
+    return launch_status();
+}
