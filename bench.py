@@ -549,6 +549,83 @@ def run_sweep(args, rank, world, local_rank):
     return 0
 
 
+def run_backward(args, rank, world, local_rank):
+    """Back-propagation of layer 1 of a 2-layer workload (C1..C4): one
+    bigcn_layer_backward call per step (Algorithm 1 with Eqs. bp-H and bp-W:
+    pack rows and weights, A~ dH, dL/dW~, dL/dH~ clipped, dL/dW), from a
+    seeded upstream gradient dH = dL/dH1 (N x hidden, N(0, 1)); inputs resident
+    on the device, L2 flushed before every step outside the timed events."""
+    import torch
+
+    from paper_2010_07565_gb300 import binding as B
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    w, data = build_workload(args.workload)
+    N, K, F = w.N, w.K, w.hidden
+    d = {k: torch.from_numpy(np.ascontiguousarray(v)).to(dev)
+         for k, v in data.items() if k in ("X", "s", "t", "W1", "rowptr", "colidx")}
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(4000 + w.index)
+    dH = torch.randn((N, F), device=dev, generator=gen)
+    ws = torch.empty(B.bigcn_layer_backward_workspace_bytes(N, K, F), dtype=torch.uint8,
+                     device=dev)
+    dW = torch.empty((K, F), device=dev)
+    dX = torch.empty((N, K), device=dev)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    flush_half = flush[: flush.numel() // 2]
+
+    def step():
+        B.bigcn_layer_backward(d["X"], d["s"], d["t"], d["W1"], d["rowptr"], d["colidx"], dH,
+                               ws, dW, dX=dX)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    times = []
+    with ClockSampler(local_rank) as clocks:
+        for _ in range(args.steps):
+            flush.zero_()
+            flush_half.sum()
+            e0.record()
+            step()
+            e1.record()
+            e1.synchronize()
+            times.append(e0.elapsed_time(e1))
+    total_ms = float(sum(times))
+    max_ms, units = aggregate_over_ranks(total_ms, float(N) * args.steps, world)
+    if rank != 0:
+        return 0
+    peaks, peak_kind = load_peaks()
+    mean_ms = max_ms / args.steps
+    # The two +-1 x fp32 products dominate: N K F fused multiply-adds each,
+    # on the CUDA cores. fp32 FMA peak from the unit counts: 152 SMs x 128
+    # lanes x 2 flops x 2070 MHz.
+    flops = 2.0 * 2.0 * N * K * F
+    fma_peak = 152 * 128 * 2 * 2.070e9 / 1e12
+    line = {
+        "metric": "Bi-GCN layer backward nodes/s (Algorithm 1, Eqs. bp-H, bp-W)",
+        "value": units / (max_ms * 1e-3), "unit": "nodes/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": mean_ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32+b1",
+        "data": "synthetic",
+        "config": {"workload": w.description + " -- layer 1 backward", "name": w.name, "N": N,
+                   "K": K, "F": F, "nnz": int(data["colidx"].shape[0]),
+                   "l2": "flushed before every step outside the timed events",
+                   "launch": "bigcn_layer_backward (7 kernels)"},
+        "roofline": {"kernel": "whole backward", "bound": "alu",
+                     "achieved": flops / (mean_ms * 1e-3) / 1e12,
+                     "peak": fma_peak, "unit": "TFLOP/s (fp32 FMA, the two +-1 x fp32 products)",
+                     "frac": flops / (mean_ms * 1e-3) / 1e12 / fma_peak, "traffic": None,
+                     "peak_source": "derived: 152 SMs x 128 FMA/clk x 2 x 2070 MHz"},
+        "cpu_baseline": None, "e2e": None, "gpu_launches": 7 * args.steps,
+        "clocks": clocks.summary(),
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def run_forward_only(args):
     """R plain forwards of the workload on cuda:0, nothing timed or printed."""
     import torch
@@ -575,6 +652,8 @@ def main(argv=None):
                     help="C1..C4, or a one-layer sweep point such as C5_K4096_F256")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--backward", action="store_true",
+                    help="time layer 1's back-propagation (bigcn_layer_backward) instead")
     ap.add_argument("--forward-only", type=int, default=0, metavar="R",
                     help="run R plain forwards (no graph, no timing, no output) and exit: "
                          "a fixed launch sequence for profilers")
@@ -588,6 +667,8 @@ def main(argv=None):
         return run_forward_only(args)
     if args.workload.startswith("C5_"):
         return run_sweep(args, rank, world, local_rank)
+    if args.backward:
+        return run_backward(args, rank, world, local_rank)
     if world > 1:
         import torch
         import torch.distributed as dist
