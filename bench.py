@@ -403,6 +403,12 @@ def run_gpu(args, rank, world, local_rank):
     gemm1 = by_name.get("L1.xnor_gemm") or by_name["L1.pack_rows+L1.xnor_gemm"]
     agg1 = by_name.get("L1.spmm+L2.pack_rows+L2.xnor_gemm") or by_name["L1.spmm"]
     spmm_gbs = kernel_work(w, nnz, agg1["name"])[0] / (agg1["mean_us"] * 1e-6) / 1e9
+    # Bytes the layer-1 aggregation gathers: one row of Z1' (and its row scale
+    # when factored) per CSR entry and self-loop, plus the CSR itself -- what
+    # a graph without reuse moves, served from L2 where rows repeat.
+    row1 = 2 * ((w.hidden + 7) // 8 * 8) + 4 if w.K <= 32767 else 4 * w.hidden
+    gather1 = float(nnz + w.N) * row1 + 8.0 * (w.N + 1) + 4.0 * nnz
+    gather_gbs = gather1 / (agg1["mean_us"] * 1e-6) / 1e9
 
     cpu_baseline = None
     if world == 1 and not args.no_cpu_baseline:
@@ -425,6 +431,11 @@ def run_gpu(args, rank, world, local_rank):
         "components": {
             "xnor_gemm_bitops_per_s": kernel_bitops(w, gemm1["name"]) / (gemm1["mean_us"] * 1e-6),
             "spmm_gbs": spmm_gbs, "spmm_pct_of_hbm_peak": 100.0 * spmm_gbs / hbm,
+            "l1_aggregation_gather_gbs": gather_gbs,
+            "l1_aggregation_gather_frac_of_hbm": gather_gbs / hbm,
+            "l1_aggregation_gather_note": "every neighbour row (and row scale) of Z1' the "
+                                          "layer-1 aggregation reads, per second; rows that "
+                                          "repeat are served from L2, so this can exceed HBM",
             "per_kernel_us": {r["name"]: round(r["mean_us"], 3) for r in kernels},
             "per_kernel_note": "from a second pass of the same graph with an event node "
                                "between kernels (each node adds a few us)"},
