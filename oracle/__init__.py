@@ -12,6 +12,11 @@ order:
     step 4  zeta = alpha beta (F . B) (Eq. 11, Eq. 12)  oracle_binary_dot, oracle_zeta
     step 5  H = A~ zeta (Eq. 13, Eq. 1)                 oracle_aggregate
 
+the ablation variants of step 4 (Sec. 6.3, one operand kept real):
+
+    zeta = Y W~   (weights binarized only)              oracle_real_binary_product
+    zeta = H~ W   (features binarized only)             oracle_binary_real_product
+
 and the layer's back-propagation (Algorithm 1, Eqs. bp-H, bp-W):
 
     G = A~^T dH                      oracle_aggregate_t
@@ -80,6 +85,12 @@ def lib() -> ctypes.CDLL:
             h.oracle_grad_htilde.restype = None
             h.oracle_grad_input.argtypes = [_f64p, _i64, _f64p]
             h.oracle_grad_input.restype = None
+            h.oracle_real_binary_product.argtypes = [_f32p, _i64, _i32, _i8p, _f64p, _i32,
+                                                     _f64p, _vp]
+            h.oracle_real_binary_product.restype = None
+            h.oracle_binary_real_product.argtypes = [_i8p, _f64p, _i64, _i32, _f32p, _i32,
+                                                     _i64, _f64p, _vp]
+            h.oracle_binary_real_product.restype = None
             h.oracle_grad_weight.argtypes = [_f64p, _i8p, _f64p, _f32p, _i32, _i32, _i64, _f64p]
             h.oracle_grad_weight.restype = None
             _lib = h
@@ -238,6 +249,72 @@ def forward_2layer(X, s, t, W1, W2, rowptr, colidx) -> dict:
     H1 = l1["H"].astype(np.float32)
     l2 = layer_forward(H1, W2, rowptr, colidx)
     return dict(layer1=l1, layer2=l2, H1=H1, logits=l2["H"])
+
+
+# ------------------------------------------------------ ablation variants ----
+BINARIZE = ("both", "weights", "features")
+
+
+def real_binary_product(Y, SB, beta, with_absterm=False):
+    """Weights binarized, features real: zeta = Y W~, W~[k,j] = beta_j SB[j,k]
+    (the "binarize weights only" row of Sec. 6.3's transductive table)."""
+    Y = _c(Y, np.float32)
+    SB = _c(SB, np.int8)
+    N, K = Y.shape
+    F = SB.shape[0]
+    assert SB.shape[1] == K
+    z = np.empty((N, F), np.float64)
+    a = np.empty((N, F), np.float64) if with_absterm else None
+    lib().oracle_real_binary_product(Y, N, K, SB, _c(beta, np.float64), F, z,
+                                     None if a is None else a.ctypes.data)
+    return (z, a) if with_absterm else z
+
+
+def binary_real_product(SF, alpha, Wt, with_absterm=False):
+    """Features binarized, weights real: zeta = H~ W, H~[i,k] = alpha_i SF[i,k]
+    (the "binarize features only" row of Sec. 6.3's transductive table)."""
+    SF = _c(SF, np.int8)
+    Wt = _c(Wt, np.float32)
+    N, K = SF.shape
+    F = Wt.shape[1]
+    assert Wt.shape[0] == K
+    z = np.empty((N, F), np.float64)
+    a = np.empty((N, F), np.float64) if with_absterm else None
+    lib().oracle_binary_real_product(SF, _c(alpha, np.float64), N, K, Wt, F, F, z,
+                                     None if a is None else a.ctypes.data)
+    return (z, a) if with_absterm else z
+
+
+def layer_forward_ablation(X, Wt, rowptr, colidx, binarize, s=None, t=None, rows=None) -> dict:
+    """One graph-convolution layer with the operands of Eq. 11 binarized as
+    ``binarize`` says: "both" (Bi-GCN, Eqs. 10-13), "weights" (features kept
+    real) or "features" (weights kept real), then Eq. 13's aggregation.
+
+    Besides H and the aggregation's own |terms|, returns ``scale``: A~ applied
+    to the product's |terms|, the error scale of any evaluation order of the
+    whole layer (A~ has no negative entries).
+    """
+    if binarize == "both":
+        r = layer_forward(X, Wt, rowptr, colidx, s, t, rows)
+        za = np.abs(r["alpha"])[:, None] * np.abs(r["beta"])[None, :] * Wt.shape[0]
+        r["scale"] = aggregate(rowptr, colidx, za, rows=rows)
+        return r
+    assert binarize in ("weights", "features")
+    Y = centre(X, s, t)
+    out = dict(Y=Y)
+    if binarize == "weights":
+        SB, beta = weight_binarize(Wt)
+        z, za = real_binary_product(Y, SB, beta, with_absterm=True)
+        out.update(SB=SB, beta=beta, wbits=pack(SB))
+    else:
+        SF = sign(Y)
+        alpha = row_scale(Y)
+        z, za = binary_real_product(SF, alpha, Wt, with_absterm=True)
+        out.update(SF=SF, alpha=alpha, bits=pack(SF))
+    H, absterm = aggregate(rowptr, colidx, z, rows=rows, with_absterm=True)
+    out.update(zeta=z, zeta_abs=za, H=H, absterm=absterm,
+               scale=aggregate(rowptr, colidx, za, rows=rows))
+    return out
 
 
 # ------------------------------------------------------- back-propagation ----

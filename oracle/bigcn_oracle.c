@@ -238,3 +238,44 @@ void oracle_grad_weight(const double *Wg, const int8_t *SB, const double *beta,
         }
     }
 }
+
+void oracle_real_binary_product(const float *Y, int64_t N, int32_t K, const int8_t *SB,
+                                const double *beta, int32_t F, double *zeta, double *absterm) {
+    int64_t i;
+    int32_t j, k;
+    for (i = 0; i < N; ++i) {
+        const float *y = Y + i * (int64_t)K;
+        for (j = 0; j < F; ++j) {
+            const int8_t *b = SB + (int64_t)j * K;
+            double acc = 0.0, mag = 0.0;
+            for (k = 0; k < K; ++k) {
+                const double w = beta[j] * (double)b[k];   /* W~[k,j] */
+                acc += (double)y[k] * w;
+                mag += fabs((double)y[k] * w);
+            }
+            zeta[i * (int64_t)F + j] = acc;
+            if (absterm != NULL) absterm[i * (int64_t)F + j] = mag;
+        }
+    }
+}
+
+void oracle_binary_real_product(const int8_t *SF, const double *alpha, int64_t N, int32_t K,
+                                const float *Wt, int32_t F, int64_t ldw, double *zeta,
+                                double *absterm) {
+    int64_t i;
+    int32_t j, k;
+    for (i = 0; i < N; ++i) {
+        const int8_t *f = SF + i * (int64_t)K;
+        for (j = 0; j < F; ++j) {
+            double acc = 0.0, mag = 0.0;
+            for (k = 0; k < K; ++k) {
+                const double h = alpha[i] * (double)f[k];   /* H~[i,k] */
+                const double w = (double)Wt[(int64_t)k * ldw + j];
+                acc += h * w;
+                mag += fabs(h * w);
+            }
+            zeta[i * (int64_t)F + j] = acc;
+            if (absterm != NULL) absterm[i * (int64_t)F + j] = mag;
+        }
+    }
+}

@@ -108,6 +108,24 @@ void oracle_grad_input(const double *Ht, int64_t n, double *out);
 void oracle_grad_weight(const double *Wg, const int8_t *SB, const double *beta,
                         const float *Wt, int32_t K, int32_t F, int64_t ldw, double *out);
 
+/* ---- Ablation variants of the product (Sec. 6.3, the transductive table's
+ * "binarize features only" and "binarize weights only" rows): one operand of
+ * Eq. 11 keeps its real values, the other is binarized as in Bi-GCN. ---- */
+
+/* Weights binarized, features real: zeta = Y W~ with W~[k,j] = beta_j SB[j,k]:
+ * zeta[i,j] = sum_k Y[i,k] beta_j SB[j,k] (N x F, double). absterm[i,j]
+ * (nullable) = sum_k |Y[i,k]| beta_j, the scale of any evaluation order's
+ * rounding error. */
+void oracle_real_binary_product(const float *Y, int64_t N, int32_t K, const int8_t *SB,
+                                const double *beta, int32_t F, double *zeta, double *absterm);
+
+/* Features binarized, weights real: zeta = H~ W with H~[i,k] = alpha_i SF[i,k]
+ * and W = Wt (K x F, row stride ldw): zeta[i,j] = sum_k alpha_i SF[i,k] W[k,j]
+ * (N x F, double). absterm[i,j] (nullable) = sum_k alpha_i |W[k,j]|. */
+void oracle_binary_real_product(const int8_t *SF, const double *alpha, int64_t N, int32_t K,
+                                const float *Wt, int32_t F, int64_t ldw, double *zeta,
+                                double *absterm);
+
 #ifdef __cplusplus
 }
 #endif
