@@ -169,8 +169,9 @@ bigcn_status bigcn_spmm_prescaled(const int64_t *rowptr, const int32_t *colidx,
  * as FP8 +-1, exact fp32 integer sums) when K >= 128, F >= 32 and N is at
  * least 128 rows per SM, and on the CUDA cores (XOR + popcount) otherwise;
  * the dots are identical either way.
- * Its kernels wait on shared-memory barriers with a bounded number of
- * tries. bigcn_device_timeouts synchronizes the current device, returns how
+ * Its kernels, and those of the ablation products below, wait on
+ * shared-memory barriers with a bounded number of tries.
+ * bigcn_device_timeouts synchronizes the current device, returns how
  * many such waits ran out since its last call (0 in correct operation; a
  * CTA whose wait ran out writes no output) and resets the count; -1 on a
  * CUDA error.
@@ -271,6 +272,80 @@ bigcn_status bigcn_forward_2layer(const float *X, int64_t N, int32_t K, int64_t 
                                   float *H1, int64_t ldh1, float *out, int64_t ldo,
                                   int32_t *pred, void *const *events, int32_t n_events,
                                   void *stream);
+
+/*
+ * Ablation variants of the layer (Sec. 6.3, the transductive table's rows
+ * "binarize weights only" and "binarize features only"): one operand of the
+ * product of Eq. 11 keeps its real fp32 values, the other is binarized as in
+ * Bi-GCN (sign and mean-|.| scale, Eqs. 3-4 / 7-8).
+ *
+ * Both products run on the tensor cores: the real operand is split into
+ * three bf16 parts whose sum equals it to within 2^-24 of its magnitude
+ * (each part the bf16 rounding of what the earlier parts leave), the signs
+ * are exact in bf16, and the three products are accumulated in fp32. The
+ * result is therefore that of an fp32 evaluation of the sum in some order.
+ * Sums over K may be split between the CTAs of a cluster and added in a
+ * fixed order, so results are deterministic.
+ */
+typedef enum bigcn_binarize {
+    BIGCN_BINARIZE_BOTH = 0,      /* Bi-GCN: zeta = H~ W~ (Eqs. 11-12) */
+    BIGCN_BINARIZE_WEIGHTS = 1,   /* features real:  zeta = Y W~ */
+    BIGCN_BINARIZE_FEATURES = 2   /* weights real:   zeta = H~ W */
+} bigcn_binarize;
+
+/*
+ * zeta = Y W~ with Y[i,k] = fmaf(X[i,k], scale[k], shift[k]) (the centring of
+ * bigcn_pack_rows; scale == shift == NULL: Y = X) and W~[k,j] =
+ * beta[j] * (bit k of column j ? +1 : -1):
+ *
+ *   Z[i,j] = beta[j] * sum_k Y[i,k] * sign_jk.
+ *
+ * X N x K (row stride ldx >= K), b_bits/beta from bigcn_pack_weights (F x
+ * words, words = bigcn_words(K)), Z N x F (row stride ldz >= F). Z must not
+ * overlap an input. Pointers 4-byte aligned (b_bits 8).
+ */
+bigcn_status bigcn_real_binary_gemm(const float *X, int64_t N, int32_t K, int64_t ldx,
+                                    const float *scale, const float *shift,
+                                    const uint64_t *b_bits, const float *beta, int32_t F,
+                                    int32_t words, float *Z, int64_t ldz, void *stream);
+
+/* Bytes of device workspace bigcn_binary_real_gemm needs (the bf16 parts of
+ * W); 0 on invalid sizes. */
+size_t bigcn_binary_real_gemm_workspace_bytes(int32_t K, int32_t F);
+
+/*
+ * zeta = H~ W with H~[i,k] = alpha[i] * (bit k of row i ? +1 : -1):
+ *
+ *   Z[i,j] = alpha[i] * sum_k sign_ik * W[k,j].
+ *
+ * a_bits/alpha from bigcn_pack_rows (N x words), Wt K x F (row stride
+ * ldw >= F), Z N x F (row stride ldz >= F). workspace >=
+ * bigcn_binary_real_gemm_workspace_bytes(K, F) bytes, 256-byte aligned;
+ * neither it nor Z may overlap an input or each other.
+ */
+bigcn_status bigcn_binary_real_gemm(const uint64_t *a_bits, const float *alpha, int64_t N,
+                                    int32_t K, int32_t words, const float *Wt, int32_t F,
+                                    int64_t ldw, void *workspace, size_t ws_bytes, float *Z,
+                                    int64_t ldz, void *stream);
+
+/* Bytes of device workspace bigcn_layer_forward_ablation needs; 0 on invalid
+ * sizes or an unknown `binarize`. */
+size_t bigcn_layer_ablation_workspace_bytes(int32_t binarize, int64_t N, int32_t K, int32_t F);
+
+/*
+ * One graph-convolution layer H = A~ zeta (Eq. 13) with zeta binarized as
+ * `binarize` (a bigcn_binarize) says. BIGCN_BINARIZE_BOTH is
+ * bigcn_layer_forward. The others run bigcn_pack_weights (resp.
+ * bigcn_pack_rows) and the product above with each row j multiplied by
+ * 1/sqrt(dhat_j), then bigcn_spmm_prescaled. Arguments, layouts and errors
+ * are bigcn_layer_forward's, with this call's workspace size.
+ */
+bigcn_status bigcn_layer_forward_ablation(int32_t binarize, const float *X, int64_t N,
+                                          int32_t K, int64_t ldx, const float *scale,
+                                          const float *shift, const float *Wt, int32_t F,
+                                          int64_t ldw, const int64_t *rowptr,
+                                          const int32_t *colidx, int64_t nnz, void *workspace,
+                                          size_t ws_bytes, float *H, int64_t ldh, void *stream);
 
 /*
  * Back-propagation of one layer (Algorithm 1 with Eqs. bp-H and bp-W), from

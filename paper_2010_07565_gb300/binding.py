@@ -58,6 +58,14 @@ SIGNATURES = {
     "bigcn_forward_2layer": ([_p, _i64, _i32, _i64, _p, _p, _p, _i32, _i64, _p, _i32, _i64, _p,
                               _p, _i64, _p, _sz, _p, _i64, _p, _i64, _p, _p, _i32, _p],
                              ctypes.c_int),
+    "bigcn_real_binary_gemm": ([_p, _i64, _i32, _i64, _p, _p, _p, _p, _i32, _i32, _p, _i64,
+                                _p], ctypes.c_int),
+    "bigcn_binary_real_gemm_workspace_bytes": ([_i32, _i32], _sz),
+    "bigcn_binary_real_gemm": ([_p, _p, _i64, _i32, _i32, _p, _i32, _i64, _p, _sz, _p, _i64,
+                                _p], ctypes.c_int),
+    "bigcn_layer_ablation_workspace_bytes": ([_i32, _i64, _i32, _i32], _sz),
+    "bigcn_layer_forward_ablation": ([_i32, _p, _i64, _i32, _i64, _p, _p, _p, _i32, _i64, _p,
+                                      _p, _i64, _p, _sz, _p, _i64, _p], ctypes.c_int),
     "bigcn_layer_forward_static": ([_p, _i64, _i32, _i64, _p, _p, _p, _i32, _i64, _p, _p, _i64,
                                     _p, _i64, _p], ctypes.c_int),
 }
@@ -214,6 +222,51 @@ def bigcn_layer_forward_timed(X, scale, shift, Wt, rowptr, colidx, workspace, H,
         _ptr(colidx) if colidx.numel() else None, colidx.numel(), _ptr(workspace),
         workspace.numel() * workspace.element_size(), _ptr(H), _ld(H), ev, len(events),
         _stream(stream)))
+
+
+# Which operands of Eq. 11 are binarized (enum bigcn_binarize).
+BINARIZE = {"both": 0, "weights": 1, "features": 2}
+
+
+def bigcn_real_binary_gemm(X, scale, shift, b_bits, beta, Z, stream=None):
+    """Weights binarized, features real: Z = Y W~ (Y = X centred by
+    scale/shift)."""
+    N, K = X.shape
+    F = beta.shape[0]
+    _check("bigcn_real_binary_gemm", lib().bigcn_real_binary_gemm(
+        _ptr(X), N, K, _ld(X), _ptr(scale), _ptr(shift), _ptr(b_bits), _ptr(beta), F,
+        _ld(b_bits), _ptr(Z), _ld(Z), _stream(stream)))
+
+
+def bigcn_binary_real_gemm_workspace_bytes(K: int, F: int) -> int:
+    return int(lib().bigcn_binary_real_gemm_workspace_bytes(K, F))
+
+
+def bigcn_binary_real_gemm(a_bits, alpha, K, Wt, workspace, Z, stream=None):
+    """Features binarized, weights real: Z = H~ W (H~ = diag(alpha) signs)."""
+    N = alpha.shape[0]
+    F = Wt.shape[1]
+    _check("bigcn_binary_real_gemm", lib().bigcn_binary_real_gemm(
+        _ptr(a_bits), _ptr(alpha), N, K, _ld(a_bits), _ptr(Wt), F, _ld(Wt), _ptr(workspace),
+        workspace.numel() * workspace.element_size(), _ptr(Z), _ld(Z), _stream(stream)))
+
+
+def bigcn_layer_ablation_workspace_bytes(binarize, N: int, K: int, F: int) -> int:
+    return int(lib().bigcn_layer_ablation_workspace_bytes(BINARIZE.get(binarize, binarize),
+                                                          N, K, F))
+
+
+def bigcn_layer_forward_ablation(binarize, X, scale, shift, Wt, rowptr, colidx, workspace, H,
+                                 stream=None):
+    """One layer with the operands of Eq. 11 binarized as ``binarize`` says
+    ("both", "weights", "features" or the enum's value)."""
+    N, K = X.shape
+    F = Wt.shape[1]
+    _check("bigcn_layer_forward_ablation", lib().bigcn_layer_forward_ablation(
+        BINARIZE.get(binarize, binarize), _ptr(X), N, K, _ld(X), _ptr(scale), _ptr(shift),
+        _ptr(Wt), F, _ld(Wt), _ptr(rowptr), _ptr(colidx) if colidx.numel() else None,
+        colidx.numel(), _ptr(workspace), workspace.numel() * workspace.element_size(), _ptr(H),
+        _ld(H), _stream(stream)))
 
 
 def bigcn_layer_backward_workspace_bytes(N: int, K: int, F: int) -> int:

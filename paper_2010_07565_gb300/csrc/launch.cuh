@@ -168,4 +168,49 @@ bool spmm_pack_gemm_supported(int Fh, int Fo);
 void launch_spmm_pack_gemm(const SpmmPackGemmArgs &args, const DeviceInfo &dev,
                            cudaStream_t stream, bool pdl = false);
 
+// Ablation products of step 4 (ablation.cu): one operand real, the other
+// binarized, on the tensor cores with the real operand as three bf16 parts.
+struct RealBinaryArgs {      // weights binarized: Z = Y W~
+    const float *X;          // N x K (row stride ldx), centred by scale/shift
+    int64_t ldx;
+    const float *scale;      // nullable (identity)
+    const float *shift;
+    const uint64_t *b_bits;  // F x words
+    const float *beta;       // F
+    int64_t N;
+    int K;
+    int F;
+    int words;
+    float *Z;                // N x F (row stride ldz)
+    int64_t ldz;
+    const int64_t *rowptr;   // nullable: scale row i by 1/sqrt(1 + deg_i)
+};
+void launch_real_binary_gemm(const RealBinaryArgs &args, const DeviceInfo &dev,
+                             cudaStream_t stream, bool pdl = false);
+
+struct BinaryRealArgs {      // features binarized: Z = H~ W
+    const uint64_t *a_bits;  // N x words
+    const float *alpha;      // N
+    const uint16_t *wparts;  // 3 x F x (words * 64) bf16 parts of W (launch_split_weights)
+    int64_t N;
+    int K;
+    int F;
+    int words;
+    float *Z;                // N x F (row stride ldz)
+    int64_t ldz;
+    const int64_t *rowptr;   // nullable: scale row i by 1/sqrt(1 + deg_i)
+};
+void launch_binary_real_gemm(const BinaryRealArgs &args, const DeviceInfo &dev,
+                             cudaStream_t stream, bool pdl = false);
+
+// Bytes of the bf16 parts of a K x F weight matrix, and the kernel that
+// writes them (parts[p][j][k], zero for k >= K up to bigcn_words(K) * 64).
+size_t weight_parts_bytes(int K, int F);
+void launch_split_weights(const float *Wt, int K, int F, int64_t ldw, uint16_t *wparts,
+                          cudaStream_t stream);
+
+// Waits of the ablation products that ran out since the last call (and
+// resets the count); ~0u on a CUDA error.
+uint32_t take_mix_timeouts();
+
 }  // namespace bigcn

@@ -299,5 +299,7 @@ extern "C" int32_t bigcn_device_timeouts(void) {
         cudaGetLastError();
         return -1;
     }
-    return int32_t(n);
+    const uint32_t mix = bigcn::take_mix_timeouts();
+    if (mix == ~0u) return -1;
+    return int32_t(n + mix);
 }
