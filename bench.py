@@ -637,6 +637,139 @@ def run_backward(args, rank, world, local_rank):
     return 0
 
 
+def run_ablation(args, rank, world, local_rank):
+    """Layer 1 of a workload with one operand of Eq. 11 kept real (Sec. 6.3's
+    ablation rows): ``--ablation weights`` binarizes only the weights (zeta =
+    Y W~, the centred features real), ``--ablation features`` only the
+    features (zeta = H~ W). Each step is one bigcn_layer_forward_ablation
+    call (pack, product with the degree scale, aggregation); the product is
+    also timed alone through its own entry point. C1..C4 use the workload's
+    seeded inputs with L2 flushed before every step (outside the events); a
+    C5 point draws its features on the device and needs no flush."""
+    import torch
+
+    from paper_2010_07565_gb300 import binding as B
+    from paper_2010_07565_gb300 import inputs
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    mode = args.ablation
+    w = inputs.get_workload(args.workload)
+    N, K, F = w.N, w.K, w.hidden
+    if w.name.startswith("C5_"):
+        gen = torch.Generator(device=dev)
+        gen.manual_seed(1000 + w.index)
+        X = torch.randn((N, K), device=dev, generator=gen)
+        s = t = None
+        Wt = torch.from_numpy(inputs.weights(K, F, 3000 + w.index)).to(dev)
+        rp, ci = inputs.graph(w)
+        flush_needed = False
+    else:
+        w, data = build_workload(args.workload)
+        X = torch.from_numpy(data["X"]).to(dev)
+        s, t = torch.from_numpy(data["s"]).to(dev), torch.from_numpy(data["t"]).to(dev)
+        Wt = torch.from_numpy(data["W1"]).to(dev)
+        rp, ci = data["rowptr"], data["colidx"]
+        flush_needed = True
+    rowptr, colidx = torch.from_numpy(rp).to(dev), torch.from_numpy(ci).to(dev)
+    nnz = int(ci.shape[0])
+    words = (K + 63) // 64
+    ws = torch.empty(B.bigcn_layer_ablation_workspace_bytes(mode, N, K, F), dtype=torch.uint8,
+                     device=dev)
+    H = torch.empty((N, F), device=dev)
+    Z = torch.empty((N, F), device=dev)
+    # Packed operand of the product-alone timing, made once by the library.
+    if mode == "weights":
+        bits = torch.empty((F, words), dtype=torch.int64, device=dev)
+        scl = torch.empty(F, device=dev)
+        B.bigcn_pack_weights(Wt, bits, scl)
+
+        def product():
+            B.bigcn_real_binary_gemm(X, s, t, bits, scl, Z)
+        pbytes = 4.0 * N * K + 8.0 * F * words + 4.0 * F + 8.0 * K + 4.0 * N * F
+    else:
+        bits = torch.empty((N, words), dtype=torch.int64, device=dev)
+        scl = torch.empty(N, device=dev)
+        B.bigcn_pack_rows(X, s, t, bits, scl)
+        pws = torch.empty(B.bigcn_binary_real_gemm_workspace_bytes(K, F), dtype=torch.uint8,
+                          device=dev)
+
+        def product():
+            B.bigcn_binary_real_gemm(bits, scl, K, Wt, pws, Z)
+        pbytes = 8.0 * N * words + 4.0 * N + 4.0 * K * F + 4.0 * N * F
+
+    def layer():
+        B.bigcn_layer_forward_ablation(mode, X, s, t, Wt, rowptr, colidx, ws, H)
+
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    flush_half = flush[: flush.numel() // 2]
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+    def timed(fn, steps):
+        out = []
+        for _ in range(steps):
+            if flush_needed:
+                flush.zero_()
+                flush_half.sum()
+            e0.record()
+            fn()
+            e1.record()
+            e1.synchronize()
+            out.append(e0.elapsed_time(e1))
+        return out
+
+    for _ in range(args.warmup):
+        layer()
+        product()
+    torch.cuda.synchronize()
+    with ClockSampler(local_rank) as clocks:
+        layer_ms = timed(layer, args.steps)
+        prod_ms = timed(product, args.steps)
+    assert B.device_timeouts() == 0
+    total_ms = float(sum(layer_ms))
+    max_ms, units = aggregate_over_ranks(total_ms, float(N) * args.steps, world)
+    if rank != 0:
+        return 0
+    peaks, peak_kind = load_peaks()
+    hbm = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+    bf16 = float(peaks.get("bf16_tflops", 1900.0))
+    prod_s = statistics.fmean(prod_ms) * 1e-3
+    flops = 2.0 * N * K * F
+    # The product is fp32-accurate on the tensor cores with three bf16 MMAs per
+    # real multiply-add, so its tensor ceiling is the bf16 peak / 3.
+    t_hbm, t_tc = pbytes / (hbm * 1e9), flops / (bf16 / 3.0 * 1e12)
+    if t_hbm >= t_tc:
+        roof = {"bound": "hbm", "achieved": pbytes / prod_s / 1e9, "peak": hbm, "unit": "GB/s",
+                "peak_source": f"{peak_kind} MEASURED_PEAKS.json hbm_gbs"}
+    else:
+        roof = {"bound": "tensor", "achieved": flops / prod_s / 1e12, "peak": bf16 / 3.0,
+                "unit": "TFLOP/s (2 N K F; fp32-accurate = 3 bf16 MMAs per multiply-add)",
+                "peak_source": f"{peak_kind} MEASURED_PEAKS.json bf16_tflops / 3"}
+    roof.update({"kernel": f"product ({'Y W~' if mode == 'weights' else 'H~ W'})",
+                 "frac": roof["achieved"] / roof["peak"], "traffic": None,
+                 "other_bound_frac": (t_tc if roof["bound"] == "hbm" else t_hbm) / prod_s})
+    line = {
+        "metric": f"Bi-GCN ablation layer fwd nodes/s ({mode} binarized only)",
+        "value": units / (max_ms * 1e-3), "unit": "nodes/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": max_ms / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f32 (3 x bf16 parts) x b1", "data": "synthetic",
+        "config": {"workload": w.description + f" -- layer 1, {mode} binarized only",
+                   "name": w.name, "N": N, "K": K, "F": F, "nnz": nnz,
+                   "l2": "flushed before every step outside the timed events" if flush_needed
+                         else "inputs larger than L2 (no flush)",
+                   "launch": "bigcn_layer_forward_ablation (pack, product, aggregation)"},
+        "components": {"product_us": 1e3 * statistics.fmean(prod_ms),
+                       "product_algorithmic_bytes": pbytes, "product_flops": flops,
+                       "layer_us": 1e3 * statistics.fmean(layer_ms)},
+        "roofline": roof, "cpu_baseline": None, "e2e": None,
+        "gpu_launches": (3 if mode == "weights" else 4) * args.steps,
+        "clocks": clocks.summary(),
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def run_forward_only(args):
     """R plain forwards of the workload on cuda:0, nothing timed or printed."""
     import torch
@@ -665,6 +798,9 @@ def main(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--backward", action="store_true",
                     help="time layer 1's back-propagation (bigcn_layer_backward) instead")
+    ap.add_argument("--ablation", choices=["weights", "features"], default=None,
+                    help="time layer 1 with only the weights (or only the features) "
+                         "binarized (bigcn_layer_forward_ablation) instead")
     ap.add_argument("--forward-only", type=int, default=0, metavar="R",
                     help="run R plain forwards (no graph, no timing, no output) and exit: "
                          "a fixed launch sequence for profilers")
@@ -676,6 +812,8 @@ def main(argv=None):
         return run_reference(args, rank, world)
     if args.forward_only > 0:
         return run_forward_only(args)
+    if args.ablation is not None:
+        return run_ablation(args, rank, world, local_rank)
     if args.workload.startswith("C5_"):
         return run_sweep(args, rank, world, local_rank)
     if args.backward:

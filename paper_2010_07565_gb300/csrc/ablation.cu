@@ -45,7 +45,10 @@ namespace {
 
 __device__ unsigned int g_mix_timeouts;
 
-constexpr int kMixThreads = 256;
+constexpr int kProducerWarps = 16;
+constexpr int kProducers = 32 * kProducerWarps;     // threads that build the operand tiles
+constexpr int kMmaWarp = kProducerWarps;            // the warp that issues the MMAs
+constexpr int kMixThreads = kProducers + 32;
 constexpr int kMixK = 64;        // elements per k-block
 constexpr int kParts = 3;        // bf16 parts of the real operand
 constexpr int kMaxSplit = 8;     // CTAs of a cluster sharing one tile's k-blocks
@@ -65,6 +68,13 @@ __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b
         "l"(a), "l"(b), "r"(idesc), "r"(accumulate));
 }
 
+__device__ __forceinline__ void commit_to(uint64_t *bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+            smem_addr(bar))
+        : "memory");
+}
+
 // Eight signs (bits 0..7 of `byte`) as eight bf16 values, +1 (0x3F80) for a
 // set bit and -1 (0xBF80) otherwise, element e in the e-th 16-bit half.
 __device__ __forceinline__ uint4 signs8_to_bf16(uint32_t byte) {
@@ -77,16 +87,23 @@ __device__ __forceinline__ uint4 signs8_to_bf16(uint32_t byte) {
     return make_uint4(u[0], u[1], u[2], u[3]);
 }
 
-// The three bf16 parts of v, as 16-bit patterns.
-__device__ __forceinline__ void split3(float v, uint32_t &hi, uint32_t &mid, uint32_t &lo) {
-    const __nv_bfloat16 h = __float2bfloat16_rn(v);
-    const float r1 = v - __bfloat162float(h);
-    const __nv_bfloat16 m = __float2bfloat16_rn(r1);
-    const float r2 = r1 - __bfloat162float(m);
-    const __nv_bfloat16 l = __float2bfloat16_rn(r2);
-    hi = __bfloat16_as_ushort(h);
-    mid = __bfloat16_as_ushort(m);
-    lo = __bfloat16_as_ushort(l);
+// Three bf16 parts of two values v0, v1, packed as pairs (v0 in the low half).
+// hi keeps the top 16 bits of v (a bf16 by truncation), so r = v - hi is
+// exact in fp32 (v's low 16 mantissa bits) with |r| < 2^-7 |v|; mid is r
+// truncated the same way, q = r - mid exact with |q| < 2^-14 |v|; lo is q
+// rounded to nearest bf16, so |v - (hi + mid + lo)| <= 2^-9 |q| < 2^-23 |v|.
+__device__ __forceinline__ void split3x2(float v0, float v1, uint32_t &hi, uint32_t &mid,
+                                         uint32_t &lo) {
+    const uint32_t u0 = __float_as_uint(v0), u1 = __float_as_uint(v1);
+    const float r0 = v0 - __uint_as_float(u0 & 0xFFFF0000u);
+    const float r1 = v1 - __uint_as_float(u1 & 0xFFFF0000u);
+    const uint32_t w0 = __float_as_uint(r0), w1 = __float_as_uint(r1);
+    const float q0 = r0 - __uint_as_float(w0 & 0xFFFF0000u);
+    const float q1 = r1 - __uint_as_float(w1 & 0xFFFF0000u);
+    hi = __byte_perm(u0, u1, 0x7632);
+    mid = __byte_perm(w0, w1, 0x7632);
+    const __nv_bfloat162 l = __floats2bfloat162_rn(q0, q1);
+    lo = *reinterpret_cast<const uint32_t *>(&l);
 }
 
 __device__ __forceinline__ uint32_t cluster_rank() {
@@ -121,6 +138,53 @@ __device__ __forceinline__ uint32_t ld_cluster_u32(uint32_t addr) {
     return v;
 }
 
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, uint32_t src_bytes) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src),
+                 "r"(src_bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ void cp_async8(uint32_t dst, const void *src, uint32_t src_bytes) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 8, %2;" ::"r"(dst), "l"(src),
+                 "r"(src_bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ void cp_async4(uint32_t dst, const void *src, uint32_t src_bytes) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(dst), "l"(src),
+                 "r"(src_bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ void cp_async_commit() {
+    asm volatile("cp.async.commit_group;" ::: "memory");
+}
+
+// Waits until at most N of this thread's most recent copy groups are pending.
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+// mbar_wait that also gives up as soon as another thread of the CTA has
+// raised *abort (after its own wait ran out); false if it gave up.
+__device__ __forceinline__ bool wait_or_abort(uint32_t bar, uint32_t parity,
+                                              const volatile uint32_t *abort) {
+    for (uint32_t it = 0; it < kWaitLimit; ++it) {
+        uint32_t done;
+        asm volatile(
+            "{\n.reg .pred p;\n"
+            "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+            "selp.u32 %0, 1, 0, p;\n}"
+            : "=r"(done)
+            : "r"(bar), "r"(parity)
+            : "memory");
+        if (done) return true;
+        if (*abort) return false;
+    }
+    return false;
+}
+
 struct MixParams {
     // A real (weights binarized): X, centring, packed weight columns.
     const float *X;
@@ -144,213 +208,125 @@ struct MixParams {
     int split;               // KS: CTAs of a cluster sharing a tile's k-blocks
 };
 
+// Shared-memory plan. Weights binarized (A real): kStages operand stages of
+// three 128-row part tiles plus the NT-row sign tile, then a ring of kRaw raw
+// fp32 k-blocks of X (128 rows x 64). Features binarized (B real): kHalves = 2
+// row tiles of 128 (256 node rows per CTA, so that each copy of W's parts
+// serves twice the rows): stages of the two sign tiles plus W's three NT-row
+// part tiles.
 template <int NT, bool kRealA>
 struct MixShape {
-    static constexpr int kTileA = kUmmaM * 128;           // bytes of one 128-row bf16 tile
+    static constexpr int kHalves = kRealA ? 1 : 2;
+    static constexpr int kRows = kUmmaM * kHalves;                 // node rows per CTA
+    static constexpr int kTileA = kUmmaM * 128;                    // one 128-row bf16 tile
     static constexpr int kTileB = NT * 128;
-    static constexpr int kStage = kRealA ? kParts * kTileA + kTileB : kTileA + kParts * kTileB;
-    static constexpr int kStages = (kStage <= 48 * 1024) ? 4 : (kStage <= 64 * 1024 ? 3 : 2);
-    static constexpr int kRedStride = NT + 4;              // floats per partial row
-    static constexpr size_t kSmem = 1024 + size_t(kStages) * kStage;
-    static_assert(size_t(kUmmaM) * kRedStride * 4 <= size_t(kStages) * kStage,
+    static constexpr int kStage =
+        kRealA ? kParts * kTileA + kTileB : kHalves * kTileA + kParts * kTileB;
+    static constexpr int kRawBlock = kUmmaM * kMixK * 4;           // 32 KB of X
+    static constexpr int kRaw = kRealA ? (NT <= 128 ? 3 : 2) : 0;
+    static constexpr int kStages = kRealA ? 2 : 4;
+    static constexpr int kRedStride = NT + 4;                      // floats per partial row
+    static constexpr size_t kBytes = size_t(kRaw) * kRawBlock + size_t(kStages) * kStage;
+    static constexpr size_t kSmem = 1024 + kBytes;
+    static_assert(kSmem <= 227 * 1024, "shared memory per CTA");
+    static_assert(size_t(kRows) * kRedStride * 4 <= size_t(kStages) * kStage,
                   "the partial tile reuses the stage buffers");
 };
 
-template <int NT, bool kRealA>
-__global__ void __launch_bounds__(kMixThreads)
-mixed_gemm_tc_kernel(const MixParams p) {
-    using S = MixShape<NT, kRealA>;
-    constexpr int kStages = S::kStages;
-    constexpr int kBRows = NT / 32;                        // B rows per thread
-    extern __shared__ unsigned char smem_raw[];
-    __shared__ __align__(8) uint64_t bars[kStages];
-    __shared__ uint32_t tmem_base;
-    __shared__ uint32_t s_ok;
+// Barriers and flags of one CTA: stage s is full once every producer thread
+// has arrived on full[s], and empty again once the MMAs that read it commit
+// to empty[s]; `done` receives the commit that follows the last MMA.
+template <int kStages>
+struct MixSync {
+    uint64_t full[kStages];
+    uint64_t empty[kStages];
+    uint64_t done;
+    uint32_t tmem_base;
+    uint32_t abort;
+    uint32_t ok;
+};
 
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int KS = p.split;
-    const int rank = KS > 1 ? int(cluster_rank()) : 0;
-    const int64_t m0 = int64_t(blockIdx.x / KS) * kUmmaM;
-    const int n0 = blockIdx.y * NT;
-    const uint32_t raw = smem_addr(smem_raw);
-    const uint32_t tile0 = (raw + 1023u) & ~1023u;
-    unsigned char *tiles = smem_raw + (tile0 - raw);
-
-    // This CTA's k-blocks.
-    const int KB = p.words;
-    const int per = (KB + KS - 1) / KS;
-    const int kb0 = min(KB, rank * per), kb1 = min(KB, kb0 + per);
-
-    if (warp == 0) {
+template <int kCols, int kStages>
+__device__ __forceinline__ uint32_t mix_setup(MixSync<kStages> &sy) {
+    const int tid = threadIdx.x;
+    if ((tid >> 5) == 0) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                         smem_addr(&tmem_base)),
-                     "r"(NT));
+                         smem_addr(&sy.tmem_base)),
+                     "r"(kCols));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
     }
     if (tid == 0) {
-        for (int s = 0; s < kStages; ++s) mbar_init(smem_addr(&bars[s]), 1);
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(smem_addr(&sy.full[s]), kProducers);
+            mbar_init(smem_addr(&sy.empty[s]), 1);
+        }
+        mbar_init(smem_addr(&sy.done), 1);
+        sy.abort = 0u;
         mbar_fence_init();
     }
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-    const uint32_t tmem = tmem_base;
-    grid_dependency_wait();     // packed operands and parts come from earlier kernels
+    return sy.tmem_base;
+}
 
-    // Thread t builds 16-byte chunk c = t & 7 (elements 8c .. 8c + 7 of the
-    // k-block) of rows r0 + 32 q of each tile.
-    const int c = tid & 7, r0 = tid >> 3;
-    const bool vec_x = kRealA && (p.ldx & 3) == 0 && (reinterpret_cast<uintptr_t>(p.X) & 15) == 0;
+template <int kCols>
+__device__ __forceinline__ void mix_teardown(uint32_t tmem) {
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    if ((threadIdx.x >> 5) == 0)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                     "r"(kCols));
+}
 
-    float xv[kRealA ? 4 : 1][8];       // A real: 4 rows x 8 elements
-    float sv[8], tv[8];                // centring of those elements
-    uint64_t wsign[kRealA ? kBRows : 4];   // packed words of the sign tile's rows
-    uint4 wpart[kRealA ? 1 : kBRows][kParts];
-
-    auto load = [&](int kb) {
-        const int k = kb * kMixK + 8 * c;
-        if constexpr (kRealA) {
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const int64_t row = m0 + r0 + 32 * q;
-                const float *x = p.X + row * p.ldx + k;
-                if (row < p.N && vec_x && k + 8 <= p.K) {
-                    const float4 a = __ldg(reinterpret_cast<const float4 *>(x));
-                    const float4 b = __ldg(reinterpret_cast<const float4 *>(x) + 1);
-                    xv[q][0] = a.x; xv[q][1] = a.y; xv[q][2] = a.z; xv[q][3] = a.w;
-                    xv[q][4] = b.x; xv[q][5] = b.y; xv[q][6] = b.z; xv[q][7] = b.w;
-                } else {
-#pragma unroll
-                    for (int e = 0; e < 8; ++e)
-                        xv[q][e] = (row < p.N && k + e < p.K) ? __ldg(x + e) : 0.0f;
-                }
-            }
-            if (p.scale != nullptr) {
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    const bool in = k + e < p.K;     // y = fmaf(0, 0, 0) = 0 past K
-                    sv[e] = in ? __ldg(p.scale + k + e) : 0.0f;
-                    tv[e] = in ? __ldg(p.shift + k + e) : 0.0f;
-                }
-            }
-#pragma unroll
-            for (int q = 0; q < kBRows; ++q) {
-                const int col = n0 + r0 + 32 * q;
-                wsign[q] = col < p.F ? __ldg(p.b_bits + int64_t(col) * p.words + kb) : 0ull;
-            }
-        } else {
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const int64_t row = m0 + r0 + 32 * q;
-                wsign[q] = row < p.N ? __ldg(p.a_bits + row * p.words + kb) : 0ull;
-            }
-            const int64_t kp = int64_t(p.words) * kMixK;
-#pragma unroll
-            for (int q = 0; q < kBRows; ++q) {
-                const int col = n0 + r0 + 32 * q;
-#pragma unroll
-                for (int part = 0; part < kParts; ++part)
-                    wpart[q][part] =
-                        col < p.F ? __ldg(reinterpret_cast<const uint4 *>(
-                                        p.wparts + (int64_t(part) * p.F + col) * kp + k))
-                                  : make_uint4(0u, 0u, 0u, 0u);
-            }
-        }
-    };
-
-    auto store = [&](unsigned char *sa, unsigned char *sb) {
-        if constexpr (kRealA) {
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                uint32_t h[4], m[4], l[4];
-#pragma unroll
-                for (int w = 0; w < 4; ++w) {
-                    uint32_t h0, m0_, l0, h1, m1, l1;
-                    float y0 = xv[q][2 * w], y1 = xv[q][2 * w + 1];
-                    if (p.scale != nullptr) {
-                        y0 = __fmaf_rn(y0, sv[2 * w], tv[2 * w]);
-                        y1 = __fmaf_rn(y1, sv[2 * w + 1], tv[2 * w + 1]);
-                    }
-                    split3(y0, h0, m0_, l0);
-                    split3(y1, h1, m1, l1);
-                    h[w] = h0 | (h1 << 16);
-                    m[w] = m0_ | (m1 << 16);
-                    l[w] = l0 | (l1 << 16);
-                }
-                const uint32_t off = sw128_offset(r0 + 32 * q, c);
-                *reinterpret_cast<uint4 *>(sa + off) = make_uint4(h[0], h[1], h[2], h[3]);
-                *reinterpret_cast<uint4 *>(sa + S::kTileA + off) = make_uint4(m[0], m[1], m[2], m[3]);
-                *reinterpret_cast<uint4 *>(sa + 2 * S::kTileA + off) =
-                    make_uint4(l[0], l[1], l[2], l[3]);
-            }
-#pragma unroll
-            for (int q = 0; q < kBRows; ++q)
-                *reinterpret_cast<uint4 *>(sb + sw128_offset(r0 + 32 * q, c)) =
-                    signs8_to_bf16(uint32_t(wsign[q] >> (8 * c)) & 0xFFu);
-        } else {
-#pragma unroll
-            for (int q = 0; q < 4; ++q)
-                *reinterpret_cast<uint4 *>(sa + sw128_offset(r0 + 32 * q, c)) =
-                    signs8_to_bf16(uint32_t(wsign[q] >> (8 * c)) & 0xFFu);
-#pragma unroll
-            for (int q = 0; q < kBRows; ++q) {
-                const uint32_t off = sw128_offset(r0 + 32 * q, c);
-#pragma unroll
-                for (int part = 0; part < kParts; ++part)
-                    *reinterpret_cast<uint4 *>(sb + part * S::kTileB + off) = wpart[q][part];
-            }
-        }
-    };
-
-    constexpr uint32_t idesc = bf16_idesc(NT);
-    bool ok = true;
-    int committed = -1;          // last local k-block whose MMAs were committed
-    if (kb0 < kb1) load(kb0);
-    for (int kb = kb0; kb < kb1; ++kb) {
-        const int it = kb - kb0;
+// The MMA warp: for each k-block, wait until its stage is full, issue the
+// MMAs (lane 0) and commit them to the stage's `empty` barrier; finally commit
+// to `done`, which then tracks every MMA issued.
+template <int kStages, typename Issue>
+__device__ __forceinline__ void mma_loop(MixSync<kStages> &sy, int nkb, Issue issue) {
+    const int lane = threadIdx.x & 31;
+    bool any = false;
+#pragma unroll 1
+    for (int it = 0; it < nkb; ++it) {
         const int s = it % kStages;
-        if (it >= kStages) {
-            const bool done = mbar_wait(smem_addr(&bars[s]), uint32_t(it / kStages - 1) & 1u);
-            if (!__syncthreads_and(done)) {
-                ok = false;
-                break;
-            }
+        if (!wait_or_abort(smem_addr(&sy.full[s]), uint32_t(it / kStages) & 1u, &sy.abort)) {
+            sy.abort = 1u;
+            break;
         }
-        unsigned char *sa = tiles + s * S::kStage;
-        unsigned char *sb = sa + (kRealA ? kParts * S::kTileA : S::kTileA);
-        store(sa, sb);
-        if (kb + 1 < kb1) load(kb + 1);      // in flight across the barrier and MMAs
-        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-        __syncthreads();
-        if (tid == 0) {
-            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-            const uint32_t a0 = smem_addr(sa), b0 = smem_addr(sb);
-#pragma unroll
-            for (int k = 0; k < kMixK / 16; ++k)
-#pragma unroll
-                for (int part = 0; part < kParts; ++part) {
-                    const uint32_t a = a0 + (kRealA ? part * S::kTileA : 0) + 32u * k;
-                    const uint32_t b = b0 + (kRealA ? 0 : part * S::kTileB) + 32u * k;
-                    mma_bf16(tmem, sw128_desc(a), sw128_desc(b), idesc,
-                             (it > 0 || k > 0 || part > 0) ? 1u : 0u);
-                }
-            asm volatile(
-                "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-                    smem_addr(&bars[s]))
-                : "memory");
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        if (lane == 0) {
+            issue(it, s);
+            commit_to(&sy.empty[s]);
         }
-        committed = it;
+        any = true;
+        __syncwarp();
     }
-    bool done = true;
-    if (committed >= 0)
-        done = mbar_wait(smem_addr(&bars[committed % kStages]),
-                         uint32_t(committed / kStages) & 1u);
-    ok = __syncthreads_and(ok && done) != 0;
-    if (!ok && tid == 0) atomicAdd(&g_mix_timeouts, 1u);
-    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    if (lane == 0) {
+        if (any) commit_to(&sy.done);
+        else mbar_arrive(smem_addr(&sy.done));
+    }
+    __syncwarp();
+}
 
-    const int quad = warp & 3;
-    const uint32_t taddr = tmem + (uint32_t(32 * quad) << 16);
+// After the main loop: move the accumulators out of tensor memory and store
+// Z (KS == 1), or add the KS partials of the cluster in rank order first.
+// Accumulator h (h < kHalves) holds rows 128 h .. 128 h + 127 in tensor-memory
+// columns h NT .. h NT + NT - 1. The producer warps read it: warp w may read
+// lanes 32 (w % 4) ..; group g = w / 4 takes a share of the columns.
+template <int NT, bool kRealA, int kStages>
+__device__ __forceinline__ void mix_epilogue(const MixParams &p, unsigned char *tiles,
+                                             uint32_t tmem, int64_t m0, int n0, int rank,
+                                             bool ok, bool has_acc, MixSync<kStages> &sy) {
+    using S = MixShape<NT, kRealA>;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int KS = p.split;
+    const bool reader = warp < kProducerWarps;
+    const int quad = warp & 3, group = (warp >> 2) & 3;
+    const int half = S::kHalves == 2 ? (group & 1) : 0;
+    const int cfirst = S::kHalves == 2 ? 16 * (group >> 1) : 16 * group;
+    const int cstep = S::kHalves == 2 ? 32 : 64;
+    const int rl = 128 * half + 32 * quad + lane;                 // row within the CTA
+    const uint32_t taddr = tmem + (uint32_t(32 * quad) << 16) + uint32_t(half * NT);
     auto row_scale = [&](int64_t row) {
         float rs = kRealA ? 1.0f : __ldg(p.alpha + row);
         if (p.rowptr != nullptr) {
@@ -365,40 +341,40 @@ mixed_gemm_tc_kernel(const MixParams p) {
     const bool vec_z = (p.ldz & 3) == 0 && (reinterpret_cast<uintptr_t>(p.Z) & 15) == 0;
 
     if (KS == 1) {
-        if (ok) {
-            const int64_t row = m0 + 32 * quad + lane;
-            const float rs = row < p.N ? row_scale(row) : 0.0f;
+        if (!ok || !reader) return;
+        const int64_t row = m0 + rl;
+        const float rs = row < p.N ? row_scale(row) : 0.0f;
 #pragma unroll 1
-            for (int c0 = 16 * (warp >> 2); c0 < NT; c0 += 32) {
-                uint32_t acc[16];
-                tmem_ld16(taddr + uint32_t(c0), acc);
-                if (row >= p.N) continue;
-                const int col0 = n0 + c0;
-                float z[16];
+        for (int c0 = cfirst; c0 < NT; c0 += cstep) {
+            uint32_t acc[16];
+            tmem_ld16(taddr + uint32_t(c0), acc);
+            if (row >= p.N) continue;
+            const int col0 = n0 + c0;
+            float z[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j)
+                z[j] = scaled(rs, min(col0 + j, p.F - 1), __uint_as_float(acc[j]));
+            float *zr = p.Z + row * p.ldz + col0;
+            if (vec_z && col0 + 16 <= p.F) {
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+                    reinterpret_cast<float4 *>(zr)[q] =
+                        make_float4(z[4 * q], z[4 * q + 1], z[4 * q + 2], z[4 * q + 3]);
+            } else {
 #pragma unroll
                 for (int j = 0; j < 16; ++j)
-                    z[j] = scaled(rs, min(col0 + j, p.F - 1), __uint_as_float(acc[j]));
-                float *zr = p.Z + row * p.ldz + col0;
-                if (vec_z && col0 + 16 <= p.F) {
-#pragma unroll
-                    for (int q = 0; q < 4; ++q)
-                        reinterpret_cast<float4 *>(zr)[q] =
-                            make_float4(z[4 * q], z[4 * q + 1], z[4 * q + 2], z[4 * q + 3]);
-                } else {
-#pragma unroll
-                    for (int j = 0; j < 16; ++j)
-                        if (col0 + j < p.F) zr[j] = z[j];
-                }
+                    if (col0 + j < p.F) zr[j] = z[j];
             }
         }
-    } else {
-        // Partial tile -> this CTA's shared memory (all stages are idle now).
-        float *red = reinterpret_cast<float *>(tiles);
-        const int rl = 32 * quad + lane;
+        return;
+    }
+    // Partial tile -> this CTA's shared memory (every stage is idle now).
+    float *red = reinterpret_cast<float *>(tiles);
+    if (reader) {
 #pragma unroll 1
-        for (int c0 = 16 * (warp >> 2); c0 < NT; c0 += 32) {
+        for (int c0 = cfirst; c0 < NT; c0 += cstep) {
             uint32_t acc[16];
-            if (committed >= 0 && ok) tmem_ld16(taddr + uint32_t(c0), acc);
+            if (has_acc && ok) tmem_ld16(taddr + uint32_t(c0), acc);
             else {
 #pragma unroll
                 for (int j = 0; j < 16; ++j) acc[j] = 0u;
@@ -410,46 +386,340 @@ mixed_gemm_tc_kernel(const MixParams p) {
                                      __uint_as_float(acc[4 * q + 2]),
                                      __uint_as_float(acc[4 * q + 3]));
         }
-        if (tid == 0) s_ok = ok ? 1u : 0u;
-        cluster_sync();
-        uint32_t peer_ok = 1u;
-        if (tid < KS) peer_ok = ld_cluster_u32(map_to_rank(smem_addr(&s_ok), uint32_t(tid)));
-        const bool all_ok = __syncthreads_and(peer_ok != 0u) != 0;
-        if (all_ok) {
-            const int lo = (kUmmaM * rank) / KS, hi = (kUmmaM * (rank + 1)) / KS;
-            constexpr int kC4 = NT / 4;
-            const uint32_t red0 = smem_addr(red);
-            for (int idx = tid; idx < (hi - lo) * kC4; idx += kMixThreads) {
-                const int r = lo + idx / kC4, c4 = idx % kC4;
-                const int64_t row = m0 + r;
-                const int col0 = n0 + 4 * c4;
-                if (row >= p.N || col0 >= p.F) continue;
-                const uint32_t off = red0 + uint32_t(r * S::kRedStride + 4 * c4) * 4u;
-                float4 v = ld_cluster_f4(map_to_rank(off, 0));
-                for (int q = 1; q < KS; ++q) {
-                    const float4 w = ld_cluster_f4(map_to_rank(off, uint32_t(q)));
-                    v.x += w.x; v.y += w.y; v.z += w.z; v.w += w.w;
-                }
-                const float rs = row_scale(row);
-                const float a[4] = {v.x, v.y, v.z, v.w};
-                float *zr = p.Z + row * p.ldz + col0;
-                if (vec_z && col0 + 4 <= p.F) {
-                    *reinterpret_cast<float4 *>(zr) =
-                        make_float4(scaled(rs, col0, a[0]), scaled(rs, col0 + 1, a[1]),
-                                    scaled(rs, col0 + 2, a[2]), scaled(rs, col0 + 3, a[3]));
-                } else {
+    }
+    if (tid == 0) sy.ok = ok ? 1u : 0u;
+    cluster_sync();
+    uint32_t peer_ok = 1u;
+    if (tid < KS) peer_ok = ld_cluster_u32(map_to_rank(smem_addr(&sy.ok), uint32_t(tid)));
+    if (__syncthreads_and(peer_ok != 0u)) {
+        const int lo = (S::kRows * rank) / KS, hi = (S::kRows * (rank + 1)) / KS;
+        constexpr int kC4 = NT / 4;
+        const uint32_t red0 = smem_addr(red);
+        for (int idx = tid; idx < (hi - lo) * kC4; idx += kMixThreads) {
+            const int r = lo + idx / kC4, c4 = idx % kC4;
+            const int64_t row = m0 + r;
+            const int col0 = n0 + 4 * c4;
+            if (row >= p.N || col0 >= p.F) continue;
+            const uint32_t off = red0 + uint32_t(r * S::kRedStride + 4 * c4) * 4u;
+            float4 v = ld_cluster_f4(map_to_rank(off, 0));
+            for (int q = 1; q < KS; ++q) {
+                const float4 w = ld_cluster_f4(map_to_rank(off, uint32_t(q)));
+                v.x += w.x; v.y += w.y; v.z += w.z; v.w += w.w;
+            }
+            const float rs = row_scale(row);
+            const float a[4] = {v.x, v.y, v.z, v.w};
+            float *zr = p.Z + row * p.ldz + col0;
+            if (vec_z && col0 + 4 <= p.F) {
+                *reinterpret_cast<float4 *>(zr) =
+                    make_float4(scaled(rs, col0, a[0]), scaled(rs, col0 + 1, a[1]),
+                                scaled(rs, col0 + 2, a[2]), scaled(rs, col0 + 3, a[3]));
+            } else {
 #pragma unroll
-                    for (int e = 0; e < 4; ++e)
-                        if (col0 + e < p.F) zr[e] = scaled(rs, col0 + e, a[e]);
-                }
+                for (int e = 0; e < 4; ++e)
+                    if (col0 + e < p.F) zr[e] = scaled(rs, col0 + e, a[e]);
             }
         }
-        cluster_sync();          // peers have finished reading this CTA's partials
     }
-    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-    __syncthreads();
-    if (warp == 0)
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(NT));
+    cluster_sync();          // peers have finished reading this CTA's partials
+}
+
+// Common end of both kernels: wait for the last MMA (`done`), count a wait
+// that ran out, then the epilogue and the release of tensor memory.
+template <int NT, bool kRealA, int kStages>
+__device__ __forceinline__ void mix_finish(const MixParams &p, unsigned char *tiles, uint32_t tmem,
+                                           int64_t m0, int n0, int rank, bool has_acc,
+                                           MixSync<kStages> &sy) {
+    cp_async_wait<0>();            // no copy of this thread is left in flight
+    const bool done = mbar_wait(smem_addr(&sy.done), 0u);
+    const bool ok = __syncthreads_and(done && sy.abort == 0u) != 0;
+    if (!ok && threadIdx.x == 0) atomicAdd(&g_mix_timeouts, 1u);
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    mix_epilogue<NT, kRealA, kStages>(p, tiles, tmem, m0, n0, rank, ok, has_acc, sy);
+    mix_teardown<MixShape<NT, kRealA>::kHalves * NT>(tmem);
+}
+
+// ---- weights binarized: Z = Y W~ (A = centred X, real; B = signs of W) ----
+//
+// Producer thread t owns 16-byte chunk c = t & 7 (elements 8c .. 8c + 7 of a
+// k-block) of rows r0 + 64 q (r0 = t >> 3, q < 2) of the A tiles and of rows
+// r0 + 64 q (q < NT / 64) of the sign tile. It copies its own 64 elements of
+// X for k-block kb + kRaw - 1 into the raw ring with cp.async (zero-filled
+// past N and K) while it converts k-block kb, so kRaw - 1 k-blocks of X are in
+// flight per thread; it reads back only what it copied itself, so the wait on
+// its own copy group suffices. Odd rows take their two 16-byte halves in the
+// other order, which spreads each copy and read instruction over all banks.
+template <int NT>
+__global__ void __launch_bounds__(kMixThreads, 1)
+real_binary_tc_kernel(const MixParams p) {
+    using S = MixShape<NT, true>;
+    constexpr int kStages = S::kStages, kRaw = S::kRaw;
+    constexpr int kARows = kUmmaM / 64, kBRows = NT / 64;
+    extern __shared__ unsigned char smem_raw[];
+    __shared__ __align__(8) MixSync<kStages> sy;
+
+    const int tid = threadIdx.x, warp = tid >> 5;
+    const int KS = p.split;
+    const int rank = KS > 1 ? int(cluster_rank()) : 0;
+    const int64_t m0 = int64_t(blockIdx.x / KS) * kUmmaM;
+    const int n0 = blockIdx.y * NT;
+    const uint32_t raw_addr = smem_addr(smem_raw);
+    const uint32_t base = (raw_addr + 1023u) & ~1023u;
+    unsigned char *tiles = smem_raw + (base - raw_addr);          // stages, then the raw ring
+    unsigned char *ring = tiles + kStages * S::kStage;
+    const uint32_t ring_addr = base + kStages * S::kStage;
+
+    const int KB = p.words;
+    const int per = (KB + KS - 1) / KS;
+    const int kb0 = min(KB, rank * per), kb1 = min(KB, kb0 + per);
+
+    const uint32_t tmem = mix_setup<NT, kStages>(sy);
+    grid_dependency_wait();     // the packed weights come from an earlier kernel
+
+    if (warp == kMmaWarp) {
+        constexpr uint32_t idesc = bf16_idesc(NT);
+        mma_loop<kStages>(sy, kb1 - kb0, [&](int it, int s) {
+            const uint32_t a0 = base + s * S::kStage, b0 = a0 + kParts * S::kTileA;
+#pragma unroll
+            for (int k = 0; k < kMixK / 16; ++k)
+#pragma unroll
+                for (int part = 0; part < kParts; ++part)
+                    mma_bf16(tmem, sw128_desc(a0 + part * S::kTileA + 32u * k),
+                             sw128_desc(b0 + 32u * k), idesc,
+                             (it > 0 || k > 0 || part > 0) ? 1u : 0u);
+        });
+    } else {
+        const int c = tid & 7, r0 = tid >> 3;
+        const int odd = r0 & 1;
+        // Widest copy every row start allows: 16, 8 or 4 bytes.
+        const uintptr_t xa = reinterpret_cast<uintptr_t>(p.X);
+        const int width = ((p.ldx & 3) == 0 && (xa & 15) == 0) ? 16
+                          : ((p.ldx & 1) == 0 && (xa & 7) == 0) ? 8 : 4;
+
+        auto issue = [&](int kb) {      // this thread's 64 elements of X for k-block kb
+            const uint32_t slot = ring_addr + uint32_t(((kb - kb0) % kRaw) * S::kRawBlock);
+#pragma unroll
+            for (int q = 0; q < kARows; ++q) {
+                const int r = r0 + 64 * q;
+                const int64_t row = m0 + r;
+                const int k = kb * kMixK + 8 * c;
+                const uint32_t dst = slot + uint32_t(r * kMixK + 8 * c) * 4u;
+                const float *src = p.X + (row < p.N ? row : 0) * p.ldx;
+                if (width == 16) {
+#pragma unroll
+                    for (int h = 0; h < 2; ++h) {
+                        const int hh = h ^ odd;
+                        const int kk = k + 4 * hh;
+                        const int n = row < p.N ? min(max(p.K - kk, 0), 4) : 0;
+                        cp_async16(dst + 16u * hh, n > 0 ? src + kk : p.X, uint32_t(4 * n));
+                    }
+                } else if (width == 8) {
+#pragma unroll
+                    for (int h = 0; h < 4; ++h) {
+                        const int hh = h ^ (2 * odd);
+                        const int kk = k + 2 * hh;
+                        const int n = row < p.N ? min(max(p.K - kk, 0), 2) : 0;
+                        cp_async8(dst + 8u * hh, n > 0 ? src + kk : p.X, uint32_t(4 * n));
+                    }
+                } else {
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        const bool in = row < p.N && k + e < p.K;
+                        cp_async4(dst + 4u * e, in ? src + k + e : p.X, in ? 4u : 0u);
+                    }
+                }
+            }
+        };
+        uint64_t wsign[kBRows];
+        float sv[8], tv[8];
+        auto load_small = [&](int kb) {     // sign words and centring of k-block kb
+#pragma unroll
+            for (int q = 0; q < kBRows; ++q) {
+                const int col = n0 + r0 + 64 * q;
+                wsign[q] = col < p.F ? __ldg(p.b_bits + int64_t(col) * p.words + kb) : 0ull;
+            }
+            if (p.scale != nullptr) {
+                const int k = kb * kMixK + 8 * c;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    const bool in = k + e < p.K;      // y = fmaf(0, 0, 0) = 0 past K
+                    sv[e] = in ? __ldg(p.scale + k + e) : 0.0f;
+                    tv[e] = in ? __ldg(p.shift + k + e) : 0.0f;
+                }
+            }
+        };
+
+#pragma unroll 1
+        for (int d = 0; d < kRaw - 1; ++d) {
+            if (kb0 + d < kb1) issue(kb0 + d);
+            cp_async_commit();
+        }
+        if (kb0 < kb1) load_small(kb0);
+#pragma unroll 1
+        for (int kb = kb0; kb < kb1; ++kb) {
+            const int it = kb - kb0;
+            const int s = it % kStages;
+            if (kb + kRaw - 1 < kb1) issue(kb + kRaw - 1);
+            cp_async_commit();
+            if (it >= kStages &&
+                !wait_or_abort(smem_addr(&sy.empty[s]), uint32_t(it / kStages - 1) & 1u,
+                               &sy.abort)) {
+                sy.abort = 1u;
+                break;
+            }
+            cp_async_wait<kRaw - 1>();     // this thread's copy of k-block kb has landed
+            unsigned char *sa = tiles + s * S::kStage;
+            unsigned char *sb = sa + kParts * S::kTileA;
+            const unsigned char *slot = ring + (it % kRaw) * S::kRawBlock;
+#pragma unroll
+            for (int q = 0; q < kARows; ++q) {
+                const int r = r0 + 64 * q;
+                const float4 *xr =
+                    reinterpret_cast<const float4 *>(slot + (r * kMixK + 8 * c) * 4);
+                const float4 xa = xr[odd], xb = xr[odd ^ 1];
+                const float4 x0 = odd ? xb : xa, x1 = odd ? xa : xb;
+                float y[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+                if (p.scale != nullptr) {
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) y[e] = __fmaf_rn(y[e], sv[e], tv[e]);
+                }
+                uint32_t h[4], m[4], l[4];
+#pragma unroll
+                for (int w = 0; w < 4; ++w) split3x2(y[2 * w], y[2 * w + 1], h[w], m[w], l[w]);
+                const uint32_t off = sw128_offset(r, c);
+                *reinterpret_cast<uint4 *>(sa + off) = make_uint4(h[0], h[1], h[2], h[3]);
+                *reinterpret_cast<uint4 *>(sa + S::kTileA + off) =
+                    make_uint4(m[0], m[1], m[2], m[3]);
+                *reinterpret_cast<uint4 *>(sa + 2 * S::kTileA + off) =
+                    make_uint4(l[0], l[1], l[2], l[3]);
+            }
+#pragma unroll
+            for (int q = 0; q < kBRows; ++q)
+                *reinterpret_cast<uint4 *>(sb + sw128_offset(r0 + 64 * q, c)) =
+                    signs8_to_bf16(uint32_t(wsign[q] >> (8 * c)) & 0xFFu);
+            if (kb + 1 < kb1) load_small(kb + 1);
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            mbar_arrive(smem_addr(&sy.full[s]));
+        }
+    }
+    mix_finish<NT, true, kStages>(p, tiles, tmem, m0, n0, rank, kb1 > kb0, sy);
+}
+
+// ---- features binarized: Z = H~ W (A = signs of the node rows; B = W real) ----
+//
+// 256 node rows per CTA (two 128-row accumulators sharing each B tile). W's
+// bf16 parts (already split, K-contiguous per column) are copied with
+// cp.async straight into their 128B-swizzled places, two k-blocks ahead: the
+// copies for k-block kb + 2 go into the stage of kb - 2 once its MMAs have
+// completed. The sign tiles are expanded from the packed words (loaded one
+// k-block ahead) by the same threads.
+template <int NT>
+__global__ void __launch_bounds__(kMixThreads, 1)
+binary_real_tc_kernel(const MixParams p) {
+    using S = MixShape<NT, false>;
+    constexpr int kStages = S::kStages;
+    constexpr int kAhead = kStages - 2;
+    constexpr int kARows = S::kRows / 64;                  // sign rows per thread
+    constexpr int kBRows = NT / 64;
+    extern __shared__ unsigned char smem_raw[];
+    __shared__ __align__(8) MixSync<kStages> sy;
+
+    const int tid = threadIdx.x, warp = tid >> 5;
+    const int KS = p.split;
+    const int rank = KS > 1 ? int(cluster_rank()) : 0;
+    const int64_t m0 = int64_t(blockIdx.x / KS) * S::kRows;
+    const int n0 = blockIdx.y * NT;
+    const uint32_t raw_addr = smem_addr(smem_raw);
+    const uint32_t base = (raw_addr + 1023u) & ~1023u;
+    unsigned char *tiles = smem_raw + (base - raw_addr);
+
+    const int KB = p.words;
+    const int per = (KB + KS - 1) / KS;
+    const int kb0 = min(KB, rank * per), kb1 = min(KB, kb0 + per);
+
+    const uint32_t tmem = mix_setup<S::kHalves * NT, kStages>(sy);
+    grid_dependency_wait();     // packed rows and W's parts come from earlier kernels
+
+    if (warp == kMmaWarp) {
+        constexpr uint32_t idesc = bf16_idesc(NT);
+        mma_loop<kStages>(sy, kb1 - kb0, [&](int it, int s) {
+            const uint32_t a0 = base + s * S::kStage, b0 = a0 + S::kHalves * S::kTileA;
+#pragma unroll
+            for (int k = 0; k < kMixK / 16; ++k)
+#pragma unroll
+                for (int h = 0; h < S::kHalves; ++h)
+#pragma unroll
+                    for (int part = 0; part < kParts; ++part)
+                        mma_bf16(tmem + uint32_t(h * NT),
+                                 sw128_desc(a0 + h * S::kTileA + 32u * k),
+                                 sw128_desc(b0 + part * S::kTileB + 32u * k), idesc,
+                                 (it > 0 || k > 0 || part > 0) ? 1u : 0u);
+        });
+    } else {
+        const int c = tid & 7, r0 = tid >> 3;
+        const int64_t kp = int64_t(p.words) * kMixK;
+        auto issue = [&](int kb) {          // W's parts of k-block kb into its stage
+            const uint32_t sb = base + uint32_t(((kb - kb0) % kStages) * S::kStage +
+                                                S::kHalves * S::kTileA);
+#pragma unroll
+            for (int q = 0; q < kBRows; ++q) {
+                const int r = r0 + 64 * q;
+                const int col = n0 + r;
+                const uint32_t off = sw128_offset(r, c);
+#pragma unroll
+                for (int part = 0; part < kParts; ++part) {
+                    const uint16_t *src = p.wparts +
+                                          (int64_t(part) * p.F + (col < p.F ? col : 0)) * kp +
+                                          int64_t(kb) * kMixK + 8 * c;
+                    cp_async16(sb + part * S::kTileB + off, src, col < p.F ? 16u : 0u);
+                }
+            }
+        };
+        uint64_t wsign[kARows];
+        auto load_signs = [&](int kb) {
+#pragma unroll
+            for (int q = 0; q < kARows; ++q) {
+                const int64_t row = m0 + r0 + 64 * q;
+                wsign[q] = row < p.N ? __ldg(p.a_bits + row * p.words + kb) : 0ull;
+            }
+        };
+
+#pragma unroll 1
+        for (int d = 0; d < kAhead; ++d) {
+            if (kb0 + d < kb1) issue(kb0 + d);
+            cp_async_commit();
+        }
+        if (kb0 < kb1) load_signs(kb0);
+#pragma unroll 1
+        for (int kb = kb0; kb < kb1; ++kb) {
+            const int it = kb - kb0;
+            const int s = it % kStages;
+            // The stage of k-block kb + kAhead last held k-block kb - 2: its
+            // MMAs (committed to that stage's `empty`) must be complete; those
+            // of k-block kb - 4, which last used stage s, are then too.
+            if (it >= 2) {
+                const int prev = it - 2;
+                if (!wait_or_abort(smem_addr(&sy.empty[prev % kStages]),
+                                   uint32_t(prev / kStages) & 1u, &sy.abort)) {
+                    sy.abort = 1u;
+                    break;
+                }
+            }
+            if (kb + kAhead < kb1) issue(kb + kAhead);
+            cp_async_commit();
+            unsigned char *sa = tiles + s * S::kStage;
+#pragma unroll
+            for (int q = 0; q < kARows; ++q) {
+                const int r = r0 + 64 * q;             // row within the CTA's 256
+                *reinterpret_cast<uint4 *>(sa + (r >> 7) * S::kTileA + sw128_offset(r & 127, c)) =
+                    signs8_to_bf16(uint32_t(wsign[q] >> (8 * c)) & 0xFFu);
+            }
+            if (kb + 1 < kb1) load_signs(kb + 1);
+            cp_async_wait<kAhead>();       // this thread's part copies of k-block kb have landed
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            mbar_arrive(smem_addr(&sy.full[s]));
+        }
+    }
+    mix_finish<NT, false, kStages>(p, tiles, tmem, m0, n0, rank, kb1 > kb0, sy);
 }
 
 // W (K x F, row stride ldw) -> wparts[p][j][k], the three bf16 parts of
@@ -463,20 +733,12 @@ split_weights_kernel(const float *__restrict__ Wt, int K, int F, int64_t ldw, in
     if (idx >= chunks * F) return;
     const int j = int(idx % F);
     const int64_t k0 = (idx / F) * 8;
+    float v[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) v[e] = k0 + e < K ? __ldg(Wt + (k0 + e) * ldw + j) : 0.0f;
     uint32_t h[4], m[4], l[4];
 #pragma unroll
-    for (int w = 0; w < 4; ++w) {
-        uint32_t hh[2], mm[2], ll[2];
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-            const int64_t k = k0 + 2 * w + e;
-            const float v = k < K ? __ldg(Wt + k * ldw + j) : 0.0f;
-            split3(v, hh[e], mm[e], ll[e]);
-        }
-        h[w] = hh[0] | (hh[1] << 16);
-        m[w] = mm[0] | (mm[1] << 16);
-        l[w] = ll[0] | (ll[1] << 16);
-    }
+    for (int w = 0; w < 4; ++w) split3x2(v[2 * w], v[2 * w + 1], h[w], m[w], l[w]);
     uint4 *dst = reinterpret_cast<uint4 *>(wparts + int64_t(j) * kp + k0);
     const int64_t part = int64_t(F) * kp / 8;     // uint4s per part
     dst[0] = make_uint4(h[0], h[1], h[2], h[3]);
@@ -487,17 +749,19 @@ split_weights_kernel(const float *__restrict__ Wt, int K, int F, int64_t ldw, in
 template <int NT, bool kRealA>
 void launch_mix(MixParams p, const DeviceInfo &dev, cudaStream_t stream, bool pdl) {
     using S = MixShape<NT, kRealA>;
-    const int64_t tiles = (p.N + kUmmaM - 1) / kUmmaM;
+    void (*kernel)(const MixParams);
+    if constexpr (kRealA) kernel = real_binary_tc_kernel<NT>;
+    else kernel = binary_real_tc_kernel<NT>;
+    const int64_t tiles = (p.N + S::kRows - 1) / S::kRows;
     const int ctiles = (p.F + NT - 1) / NT;
     // Split the k-blocks over a cluster while the tiles leave SMs idle.
     int ks = 1;
     while (ks < kMaxSplit && ks < p.words && tiles * ctiles * (ks + 1) <= dev.sm_count) ++ks;
     p.split = ks;
-    cudaFuncSetAttribute(mixed_gemm_tc_kernel<NT, kRealA>,
-                         cudaFuncAttributeMaxDynamicSharedMemorySize, int(S::kSmem));
+    cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(S::kSmem));
     const dim3 grid(unsigned(tiles * ks), unsigned(ctiles));
-    launch_kernel(mixed_gemm_tc_kernel<NT, kRealA>, grid, dim3(kMixThreads), S::kSmem, stream, pdl,
-                  dim3(unsigned(ks), 1, 1), p);
+    launch_kernel(kernel, grid, dim3(kMixThreads), S::kSmem, stream, pdl, dim3(unsigned(ks), 1, 1),
+                  p);
 }
 
 }  // namespace
@@ -549,8 +813,7 @@ void launch_binary_real_gemm(const BinaryRealArgs &g, const DeviceInfo &dev, cud
     p.Z = g.Z;
     p.ldz = g.ldz;
     p.rowptr = g.rowptr;
-    if (g.F <= 64) launch_mix<64, false>(p, dev, stream, pdl);
-    else launch_mix<128, false>(p, dev, stream, pdl);
+    launch_mix<64, false>(p, dev, stream, pdl);
 }
 
 uint32_t take_mix_timeouts() {

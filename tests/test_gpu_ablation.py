@@ -77,8 +77,9 @@ def test_real_binary_gemm(cuda_device, N, K, F, centred):
     assert B.device_timeouts() == 0
 
 
-def test_real_binary_gemm_padded_strides(cuda_device):
-    N, K, F, ldx, ldz = 900, 150, 40, 157, 45
+@pytest.mark.parametrize("ldx", [157, 158, 160])   # rows 4-, 8- and 16-byte aligned
+def test_real_binary_gemm_padded_strides(cuda_device, ldx):
+    N, K, F, ldz = 900, 150, 40, 45
     X = features(N, K, 11)
     s, t = inputs.bn_stats(X)
     Wt = inputs.weights(K, F, seed=12)
