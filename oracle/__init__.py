@@ -17,6 +17,11 @@ the ablation variants of step 4 (Sec. 6.3, one operand kept real):
     zeta = Y W~   (weights binarized only)              oracle_real_binary_product
     zeta = H~ W   (features binarized only)             oracle_binary_real_product
 
+the inductive aggregators (Sec. 6.3, Table 3, GraphSAGE's definitions):
+
+    H_i = mean over N(i) u {i} of zeta_j            oracle_aggregate_mean
+    H_i = zself_i + mean over N(i) of zneigh_j      oracle_aggregate_sage
+
 and the layer's back-propagation (Algorithm 1, Eqs. bp-H, bp-W):
 
     G = A~^T dH                      oracle_aggregate_t
@@ -91,6 +96,12 @@ def lib() -> ctypes.CDLL:
             h.oracle_binary_real_product.argtypes = [_i8p, _f64p, _i64, _i32, _f32p, _i32,
                                                      _i64, _f64p, _vp]
             h.oracle_binary_real_product.restype = None
+            h.oracle_aggregate_mean.argtypes = [_i64p, _i32p, _i64, _f64p, _i32, _vp, _i64,
+                                                _f64p, _vp]
+            h.oracle_aggregate_mean.restype = ctypes.c_int
+            h.oracle_aggregate_sage.argtypes = [_i64p, _i32p, _i64, _f64p, _f64p, _i32, _vp,
+                                                _i64, _f64p, _vp]
+            h.oracle_aggregate_sage.restype = ctypes.c_int
             h.oracle_grad_weight.argtypes = [_f64p, _i8p, _f64p, _f32p, _i32, _i32, _i64, _f64p]
             h.oracle_grad_weight.restype = None
             _lib = h
@@ -314,6 +325,77 @@ def layer_forward_ablation(X, Wt, rowptr, colidx, binarize, s=None, t=None, rows
     H, absterm = aggregate(rowptr, colidx, z, rows=rows, with_absterm=True)
     out.update(zeta=z, zeta_abs=za, H=H, absterm=absterm,
                scale=aggregate(rowptr, colidx, za, rows=rows))
+    return out
+
+
+# ---------------------------------------------------- inductive aggregators ----
+AGGREGATORS = ("gcn", "mean", "sage")
+
+
+def _rows_arg(rows, N):
+    if rows is None:
+        return None, N, None
+    r = _c(rows, np.int64)
+    return r, r.shape[0], r.ctypes.data
+
+
+def aggregate_mean(rowptr, colidx, zeta_, rows=None, with_absterm=False):
+    """Inductive GCN's mean aggregator: H_i = mean of zeta over N(i) u {i}."""
+    rowptr, colidx, z = _c(rowptr, np.int64), _c(colidx, np.int32), _c(zeta_, np.float64)
+    N, F = z.shape
+    keep, nrows, rp = _rows_arg(rows, N)
+    H = np.empty((nrows, F), np.float64)
+    A = np.empty((nrows, F), np.float64) if with_absterm else None
+    if colidx.size == 0:
+        colidx = np.zeros(1, np.int32)
+    if lib().oracle_aggregate_mean(rowptr, colidx, N, z, F, rp, nrows, H,
+                                   None if A is None else A.ctypes.data) != 0:
+        raise ValueError("malformed CSR or row index")
+    return (H, A) if with_absterm else H
+
+
+def aggregate_sage(rowptr, colidx, zself, zneigh, rows=None, with_absterm=False):
+    """GraphSAGE's mean aggregator with concatenation on the products:
+    H_i = zself_i + mean over N(i) of zneigh (0 without neighbours)."""
+    rowptr, colidx = _c(rowptr, np.int64), _c(colidx, np.int32)
+    zs, zn = _c(zself, np.float64), _c(zneigh, np.float64)
+    assert zs.shape == zn.shape
+    N, F = zs.shape
+    keep, nrows, rp = _rows_arg(rows, N)
+    H = np.empty((nrows, F), np.float64)
+    A = np.empty((nrows, F), np.float64) if with_absterm else None
+    if colidx.size == 0:
+        colidx = np.zeros(1, np.int32)
+    if lib().oracle_aggregate_sage(rowptr, colidx, N, zs, zn, F, rp, nrows, H,
+                                   None if A is None else A.ctypes.data) != 0:
+        raise ValueError("malformed CSR or row index")
+    return (H, A) if with_absterm else H
+
+
+def layer_forward_inductive(X, Wt, rowptr, colidx, aggregator, s=None, t=None, W_neigh=None,
+                            rows=None) -> dict:
+    """One binarized layer of an inductive GNN (Sec. 6.3, Table 3): the
+    product of Eqs. 10-12 on every node's own features, then the aggregator:
+    "gcn" (Eq. 13), "mean" (inductive GCN) or "sage" (GraphSAGE-mean, with a
+    second weight matrix W_neigh binarized column by column like Wt)."""
+    Y = centre(X, s, t)
+    SF = sign(Y)
+    alpha = row_scale(Y)
+    SB, beta = weight_binarize(Wt)
+    z = zeta(binary_dot(SF, SB), alpha, beta)
+    out = dict(Y=Y, SF=SF, alpha=alpha, SB=SB, beta=beta, zeta=z)
+    if aggregator == "gcn":
+        H, a = aggregate(rowptr, colidx, z, rows=rows, with_absterm=True)
+    elif aggregator == "mean":
+        H, a = aggregate_mean(rowptr, colidx, z, rows=rows, with_absterm=True)
+    elif aggregator == "sage":
+        SBn, beta_n = weight_binarize(W_neigh)
+        zn = zeta(binary_dot(SF, SBn), alpha, beta_n)
+        out.update(SBn=SBn, beta_n=beta_n, zeta_n=zn)
+        H, a = aggregate_sage(rowptr, colidx, z, zn, rows=rows, with_absterm=True)
+    else:
+        raise ValueError(aggregator)
+    out.update(H=H, absterm=a)
     return out
 
 

@@ -279,3 +279,82 @@ void oracle_binary_real_product(const int8_t *SF, const double *alpha, int64_t N
         }
     }
 }
+
+/* 0 if the CSR is well formed (rowptr monotone from 0, indices in [0, N)). */
+static int csr_check(const int64_t *rowptr, const int32_t *colidx, int64_t N) {
+    int64_t i, e;
+    if (rowptr[0] != 0)
+        return -1;
+    for (i = 0; i < N; ++i)
+        if (rowptr[i + 1] < rowptr[i])
+            return -1;
+    for (e = 0; e < rowptr[N]; ++e)
+        if (colidx[e] < 0 || (int64_t)colidx[e] >= N)
+            return -1;
+    return 0;
+}
+
+/* h += w * z, a += |w * z| over F entries. */
+static void add_weighted(double *h, double *a, const double *z, int32_t F, double w) {
+    int32_t f;
+    for (f = 0; f < F; ++f) {
+        double term = w * z[f];
+        h[f] += term;
+        if (a != NULL)
+            a[f] += fabs(term);
+    }
+}
+
+int oracle_aggregate_mean(const int64_t *rowptr, const int32_t *colidx, int64_t N,
+                          const double *zeta, int32_t F, const int64_t *rows,
+                          int64_t nrows, double *H, double *absterm) {
+    int64_t r, e, count = (rows != NULL) ? nrows : N;
+    int32_t f;
+    if (csr_check(rowptr, colidx, N) != 0)
+        return -1;
+    for (r = 0; r < count; ++r) {
+        int64_t i = (rows != NULL) ? rows[r] : r;
+        double *h = H + r * (int64_t)F;
+        double *a = (absterm != NULL) ? absterm + r * (int64_t)F : NULL;
+        double w;
+        if (i < 0 || i >= N)
+            return -1;
+        w = 1.0 / (1.0 + (double)(rowptr[i + 1] - rowptr[i]));   /* 1 / dhat_i */
+        for (f = 0; f < F; ++f) {
+            h[f] = 0.0;
+            if (a != NULL)
+                a[f] = 0.0;
+        }
+        add_weighted(h, a, zeta + i * (int64_t)F, F, w);          /* the node itself */
+        for (e = rowptr[i]; e < rowptr[i + 1]; ++e)               /* its neighbours */
+            add_weighted(h, a, zeta + (int64_t)colidx[e] * F, F, w);
+    }
+    return 0;
+}
+
+int oracle_aggregate_sage(const int64_t *rowptr, const int32_t *colidx, int64_t N,
+                          const double *zself, const double *zneigh, int32_t F,
+                          const int64_t *rows, int64_t nrows, double *H, double *absterm) {
+    int64_t r, e, count = (rows != NULL) ? nrows : N;
+    int32_t f;
+    if (csr_check(rowptr, colidx, N) != 0)
+        return -1;
+    for (r = 0; r < count; ++r) {
+        int64_t i = (rows != NULL) ? rows[r] : r;
+        double *h = H + r * (int64_t)F;
+        double *a = (absterm != NULL) ? absterm + r * (int64_t)F : NULL;
+        int64_t deg;
+        if (i < 0 || i >= N)
+            return -1;
+        deg = rowptr[i + 1] - rowptr[i];
+        for (f = 0; f < F; ++f) {
+            h[f] = 0.0;
+            if (a != NULL)
+                a[f] = 0.0;
+        }
+        add_weighted(h, a, zself + i * (int64_t)F, F, 1.0);       /* W_self h_i */
+        for (e = rowptr[i]; e < rowptr[i + 1]; ++e)               /* W_neigh mean_j h_j */
+            add_weighted(h, a, zneigh + (int64_t)colidx[e] * F, F, 1.0 / (double)deg);
+    }
+    return 0;
+}

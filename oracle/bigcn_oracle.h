@@ -126,6 +126,26 @@ void oracle_binary_real_product(const int8_t *SF, const double *alpha, int64_t N
                                 const float *Wt, int32_t F, int64_t ldw, double *zeta,
                                 double *absterm);
 
+/* ---- Inductive aggregators (Sec. 6.3's inductive models, Table 3, which
+ * take GraphSAGE's definitions: the binarized feature extraction of every
+ * node's own features first, then the aggregation of the products). ---- */
+
+/* The "GCN" (mean) aggregator of inductive GCN: H[r,:] = (1/dhat_i) sum over
+ * j in N(i) u {i} of zeta[j,:], dhat_i = 1 + |N(i)|, for each requested row
+ * i = rows[r] (rows == NULL: all rows). absterm as in oracle_aggregate.
+ * Returns 0, or -1 for a malformed CSR or row index. */
+int oracle_aggregate_mean(const int64_t *rowptr, const int32_t *colidx, int64_t N,
+                          const double *zeta, int32_t F, const int64_t *rows,
+                          int64_t nrows, double *H, double *absterm);
+
+/* GraphSAGE's mean aggregator with concatenation, W [h_i || mean_j h_j] =
+ * W_self h_i + W_neigh mean_j h_j, applied to the products:
+ * H[r,:] = zself[i,:] + (1/|N(i)|) sum over j in N(i) of zneigh[j,:]
+ * (the mean is 0 for a node without neighbours). Returns 0 or -1 as above. */
+int oracle_aggregate_sage(const int64_t *rowptr, const int32_t *colidx, int64_t N,
+                          const double *zself, const double *zneigh, int32_t F,
+                          const int64_t *rows, int64_t nrows, double *H, double *absterm);
+
 #ifdef __cplusplus
 }
 #endif

@@ -14,21 +14,28 @@ Counting rules (each pinned by the test suite against the printed tables):
   layer costs N d_in d_out / 64 + 2 N d_out + |E| d_out. |E| is the paper's
   undirected edge count, self-loops not counted.
 
+* GraphSAGE-style layers (Table 3's GraphSAGE rows) carry two weight
+  matrices per layer, W_self and W_neigh (the concatenation [h_i || mean_j h_j]
+  times a 2 d_in x d_out matrix): twice the parameters and twice the feature
+  extraction (each binarized product with its own 2 N d_out scalings), and one
+  aggregation of d_out-wide rows.
+
 Nothing here is on the compute path; the benchmark reports these figures as
 the paper's context next to measured numbers.
 """
 from __future__ import annotations
 
 
-def model_size_kib(dims, binary: bool) -> float:
-    """Sum over layers of the parameter storage, in KiB (Eq. 16's terms)."""
+def model_size_kib(dims, binary: bool, weights: int = 1) -> float:
+    """Sum over layers of the parameter storage, in KiB (Eq. 16's terms);
+    ``weights`` weight matrices per layer."""
     total_bits = 0
     for d_in, d_out in zip(dims[:-1], dims[1:]):
         if binary:
             total_bits += d_in * d_out + 32 * d_out
         else:
             total_bits += 32 * d_in * d_out
-    return total_bits / 8.0 / 1024.0
+    return weights * total_bits / 8.0 / 1024.0
 
 
 def data_size_mib(N: int, d: int, binary: bool) -> float:
@@ -37,15 +44,15 @@ def data_size_mib(N: int, d: int, binary: bool) -> float:
     return bits / 8.0 / 1024.0 / 1024.0
 
 
-def cycle_ops(N: int, edges: int, dims, binary: bool) -> float:
+def cycle_ops(N: int, edges: int, dims, binary: bool, weights: int = 1) -> float:
     """Cycle operations of a GCN / Bi-GCN forward (Eq. 18-19's numerators and
-    denominators summed over layers)."""
+    denominators summed over layers); ``weights`` products per layer."""
     total = 0.0
     for d_in, d_out in zip(dims[:-1], dims[1:]):
         if binary:
-            total += N * d_in * d_out / 64.0 + 2.0 * N * d_out + edges * d_out
+            total += weights * (N * d_in * d_out / 64.0 + 2.0 * N * d_out) + edges * d_out
         else:
-            total += float(N) * d_in * d_out + edges * d_out
+            total += weights * float(N) * d_in * d_out + edges * d_out
     return total
 
 

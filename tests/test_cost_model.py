@@ -27,11 +27,12 @@ def dims_of(row):
 def test_table_figures_reproduce_to_print_precision(row):
     d, dims = dims_of(row)
     dg = row["digits"]
-    assert round_sig(cm.model_size_kib(dims, row["binary"]), dg["ms"]) == pytest.approx(
+    nw = row.get("weights", 1)
+    assert round_sig(cm.model_size_kib(dims, row["binary"], nw), dg["ms"]) == pytest.approx(
         row["ms_kib"], rel=1e-12)
     assert round_sig(cm.data_size_mib(d["N"], d["features"], row["binary"]), dg["ds"]) == \
         pytest.approx(row["ds_mib"], rel=1e-12)
-    assert round_sig(cm.cycle_ops(d["N"], d["edges"], dims, row["binary"]), dg["co"]) == \
+    assert round_sig(cm.cycle_ops(d["N"], d["edges"], dims, row["binary"], nw), dg["co"]) == \
         pytest.approx(row["co"], rel=1e-12)
 
 
