@@ -348,6 +348,44 @@ bigcn_status bigcn_layer_forward_ablation(int32_t binarize, const float *X, int6
                                           size_t ws_bytes, float *H, int64_t ldh, void *stream);
 
 /*
+ * Binarized layers of inductive GNNs (Sec. 6.3, Table 3: Bi-inductiveGCN and
+ * Bi-GraphSAGE, which binarize every feature-extraction step of GraphSAGE's
+ * models). The product of Eqs. 10-12 is taken on every node's own features,
+ * then one of these aggregators combines the products:
+ */
+typedef enum bigcn_aggregator {
+    BIGCN_AGG_GCN = 0,    /* Eq. 1: D^-1/2 (A + I) D^-1/2 zeta (bigcn_layer_forward) */
+    BIGCN_AGG_MEAN = 1,   /* inductive GCN: H_i = mean of zeta_j over j in N(i) u {i} */
+    BIGCN_AGG_SAGE = 2    /* GraphSAGE-mean: H_i = zeta_i + mean over j in N(i) of
+                             zeta'_j, zeta' the product with a second weight matrix
+                             W_neigh (0 for a node without neighbours) */
+} bigcn_aggregator;
+
+/* Bytes of device workspace bigcn_inductive_layer_forward needs; 0 on invalid
+ * sizes or an unknown aggregator. */
+size_t bigcn_inductive_layer_workspace_bytes(int32_t aggregator, int64_t N, int32_t K,
+                                             int32_t F);
+
+/*
+ * One inductive layer. X, scale/shift, Wt (K x F, ldw), the CSR, workspace,
+ * H and the errors are those of bigcn_layer_forward. W_neigh (K x F, row
+ * stride ldwn >= F) is required for BIGCN_AGG_SAGE and ignored otherwise; its
+ * columns are binarized like Wt's (their own signs and mean-|.| scales).
+ * BIGCN_AGG_SAGE computes both products with one XNOR product over the
+ * concatenated columns [Wt | W_neigh] (each half padded to a multiple of 8
+ * columns) and keeps them factored like bigcn_layer_forward's when
+ * K <= 32767. The mean over N(i) uses the CSR's row lengths, so a malformed
+ * CSR (skipped indices) still divides by the listed degree.
+ */
+bigcn_status bigcn_inductive_layer_forward(int32_t aggregator, const float *X, int64_t N,
+                                           int32_t K, int64_t ldx, const float *scale,
+                                           const float *shift, const float *Wt, int32_t F,
+                                           int64_t ldw, const float *W_neigh, int64_t ldwn,
+                                           const int64_t *rowptr, const int32_t *colidx,
+                                           int64_t nnz, void *workspace, size_t ws_bytes,
+                                           float *H, int64_t ldh, void *stream);
+
+/*
  * Back-propagation of one layer (Algorithm 1 with Eqs. bp-H and bp-W), from
  * the gradient dH = dL/dH^(l+1) of the layer's output (N x F, row stride ldg)
  * to

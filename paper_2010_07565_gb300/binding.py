@@ -66,6 +66,9 @@ SIGNATURES = {
     "bigcn_layer_ablation_workspace_bytes": ([_i32, _i64, _i32, _i32], _sz),
     "bigcn_layer_forward_ablation": ([_i32, _p, _i64, _i32, _i64, _p, _p, _p, _i32, _i64, _p,
                                       _p, _i64, _p, _sz, _p, _i64, _p], ctypes.c_int),
+    "bigcn_inductive_layer_workspace_bytes": ([_i32, _i64, _i32, _i32], _sz),
+    "bigcn_inductive_layer_forward": ([_i32, _p, _i64, _i32, _i64, _p, _p, _p, _i32, _i64, _p,
+                                       _i64, _p, _p, _i64, _p, _sz, _p, _i64, _p], ctypes.c_int),
     "bigcn_layer_forward_static": ([_p, _i64, _i32, _i64, _p, _p, _p, _i32, _i64, _p, _p, _i64,
                                     _p, _i64, _p], ctypes.c_int),
 }
@@ -267,6 +270,28 @@ def bigcn_layer_forward_ablation(binarize, X, scale, shift, Wt, rowptr, colidx, 
         _ptr(Wt), F, _ld(Wt), _ptr(rowptr), _ptr(colidx) if colidx.numel() else None,
         colidx.numel(), _ptr(workspace), workspace.numel() * workspace.element_size(), _ptr(H),
         _ld(H), _stream(stream)))
+
+
+# Aggregators of the inductive layers (enum bigcn_aggregator).
+AGGREGATOR = {"gcn": 0, "mean": 1, "sage": 2}
+
+
+def bigcn_inductive_layer_workspace_bytes(aggregator, N: int, K: int, F: int) -> int:
+    return int(lib().bigcn_inductive_layer_workspace_bytes(
+        AGGREGATOR.get(aggregator, aggregator), N, K, F))
+
+
+def bigcn_inductive_layer_forward(aggregator, X, scale, shift, Wt, rowptr, colidx, workspace, H,
+                                  W_neigh=None, stream=None):
+    """One binarized inductive layer: the product, then the ``aggregator``
+    ("gcn", "mean", "sage"; "sage" takes W_neigh)."""
+    N, K = X.shape
+    F = Wt.shape[1]
+    _check("bigcn_inductive_layer_forward", lib().bigcn_inductive_layer_forward(
+        AGGREGATOR.get(aggregator, aggregator), _ptr(X), N, K, _ld(X), _ptr(scale), _ptr(shift),
+        _ptr(Wt), F, _ld(Wt), _ptr(W_neigh), _ld(W_neigh) if W_neigh is not None else 0,
+        _ptr(rowptr), _ptr(colidx) if colidx.numel() else None, colidx.numel(), _ptr(workspace),
+        workspace.numel() * workspace.element_size(), _ptr(H), _ld(H), _stream(stream)))
 
 
 def bigcn_layer_backward_workspace_bytes(N: int, K: int, F: int) -> int:

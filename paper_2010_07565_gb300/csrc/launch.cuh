@@ -74,6 +74,10 @@ void launch_xnor_gemm_tc(const GemmArgs &args, const DeviceInfo &dev, cudaStream
 void launch_xnor_gemm(const GemmArgs &args, const DeviceInfo &dev, cudaStream_t stream,
                       bool pdl = false);
 
+// Aggregators of step 5: Eq. 1's D^-1/2 (A + I) D^-1/2, the mean over
+// N(i) u {i} (inductive GCN), GraphSAGE's self + mean over N(i).
+enum : int { kAggGcn = 0, kAggMean = 1, kAggSage = 2 };
+
 struct SpmmArgs {
     const int64_t *rowptr;   // N + 1
     const int32_t *colidx;   // nnz
@@ -97,6 +101,14 @@ struct SpmmArgs {
     // in the aggregation's epilogue when a row fits one column slab, else
     // by a separate kernel.
     int32_t *pred = nullptr;
+    // Aggregator: kAggGcn (Eq. 1, the default), kAggMean (the mean over
+    // N(i) u {i}: pass prescaled rows carrying no degree factor, or dots with
+    // rowscale = alpha) or kAggSage (Zs[i] + the mean over N(i) of Z[j]: Z /
+    // D16 point at the neighbour half of each row, Zs at the self half with
+    // the same stride, colscale_s its column scales for dots).
+    int agg = kAggGcn;
+    const void *Zs = nullptr;
+    const float *colscale_s = nullptr;
 };
 
 // Step 5: H = D^-1/2 (A + I) D^-1/2 Z (Eqs. 1, 13); launches one kernel, or

@@ -95,6 +95,12 @@ struct SpmmParams {
     const float *rowscale;   // kDots16: s_j
     const float *colscale;   // kDots16: beta_f
     int32_t *pred;           // nullable: argmax of each output row (one column slab only)
+    // Aggregator (kAggGcn, kAggMean, kAggSage). kAggSage: Z (or the dots)
+    // holds the neighbour half of each row and Zs the self half (same row
+    // stride), with colscale_s the self half's column scales (kDots16).
+    int agg = 0;
+    const void *Zs = nullptr;
+    const float *colscale_s = nullptr;
 };
 
 // How a lane loads VEC consecutive entries of a row of Z and adds them,
@@ -152,19 +158,29 @@ struct RowSrc<8, kDots16> {
     }
 };
 
-// Row i's neighbour list: CSR entries [b, b + total - 1) plus the self-loop.
+// Row i's neighbour list: CSR entries [b, b + total - 1) plus the self-loop
+// (entry 0); `first` is the first entry the aggregator sums (1 when the self
+// row is added separately), `dinv` the factor applied to the sum: Eq. 1's
+// 1/sqrt(dhat_i), the mean's 1/dhat_i, or GraphSAGE's 1/|N(i)| (0 without
+// neighbours).
 struct RowSpan {
     int64_t b;
     int64_t total;
+    int64_t first;
     float dinv;
 };
 
 __device__ __forceinline__ RowSpan row_span(const int64_t *__restrict__ rowptr, int64_t nnz,
-                                            int64_t i) {
+                                            int64_t i, int agg = kAggGcn) {
     const int64_t rb = __ldg(rowptr + i), re = __ldg(rowptr + i + 1);
     const int64_t b = min(max(rb, int64_t(0)), nnz);
     const int64_t e = min(max(re, b), nnz);
-    return RowSpan{b, (e - b) + 1, inv_sqrt_degree(e - b)};
+    const int64_t deg = e - b;
+    const float norm = agg == kAggGcn    ? inv_sqrt_degree(deg)
+                       : agg == kAggMean ? 1.0f / (1.0f + float(deg))
+                       : deg > 0         ? 1.0f / float(deg)
+                                         : 0.0f;
+    return RowSpan{b, deg + 1, agg == kAggSage ? 1 : 0, norm};
 }
 
 // Adds, into acc, the Z rows of entries [q0, q1) of row i's list (entry 0 is
@@ -229,7 +245,7 @@ __device__ __forceinline__ void reduce_groups(float (&acc)[NV][VEC]) {
 
 // Epilogue of the plain aggregation: H_i = dinv_i * acc, or for compressed
 // rows H_if = dinv_i * (beta_f * acc_f) (lanes of group 0).
-template <int VEC, int L, int NV, int S>
+template <int VEC, int L, int NV, int S, int AGG = kAggGcn>
 struct StoreRow {
     __device__ __forceinline__ void prologue() const {}
     __device__ __forceinline__ void operator()(const SpmmParams &p, int64_t i, float dinv,
@@ -249,6 +265,19 @@ struct StoreRow {
                     o[c] = f + c < p.F ? dinv * (__ldg(p.colscale + f + c) * acc[v][c]) : 0.0f;
                 else
                     o[c] = acc[v][c] * dinv;
+            }
+            if constexpr (AGG == kAggSage) {   // GraphSAGE: the node's own (self-half) product
+                const float si = S == kDots16 ? __ldg(p.rowscale + i) : 0.0f;
+#pragma unroll
+                for (int c = 0; c < VEC; ++c) {
+                    if (f + c >= p.F) continue;
+                    if (S == kDots16) {
+                        const uint32_t d = __ldg(static_cast<const uint16_t *>(p.Zs) + i * p.ldz + f + c);
+                        o[c] += si * (__ldg(p.colscale_s + f + c) * (float(d) - 32768.0f));
+                    } else {
+                        o[c] += __ldg(static_cast<const float *>(p.Zs) + i * p.ldz + f + c);
+                    }
+                }
             }
             if (p.pred != nullptr) {
 #pragma unroll
@@ -318,24 +347,24 @@ argmax_rows_kernel(const float *__restrict__ H, int64_t N, int F, int64_t ldh,
     if (lane == 0) pred[i] = best;
 }
 
-template <int VEC, int L, int NV, int U, int S, class Epi>
+template <int VEC, int L, int NV, int U, int S, class Epi, int AGG = kAggGcn>
 __device__ __forceinline__ void light_rows(const SpmmParams &p, const Epi &epi, int f0) {
     const int warp = threadIdx.x >> 5;
     const int64_t i = int64_t(blockIdx.x - p.heavy_blocks) * kSpmmWarps + warp;
     if (i >= p.N) return;
-    const RowSpan sp = row_span(p.rowptr, p.nnz, i);
+    const RowSpan sp = row_span(p.rowptr, p.nnz, i, AGG);
     if (p.heavy_blocks > 0 && sp.total - 1 > p.heavy_degree) return;   // a heavy block's row
     float acc[NV][VEC];
 #pragma unroll
     for (int v = 0; v < NV; ++v)
 #pragma unroll
         for (int c = 0; c < VEC; ++c) acc[v][c] = 0.0f;
-    gather<VEC, L, NV, U, S>(p, i, sp.b, 0, sp.total, f0, acc);
+    gather<VEC, L, NV, U, S>(p, i, sp.b, sp.first, sp.total, f0, acc);
     reduce_groups<VEC, L, NV>(acc);
     epi(p, i, sp.dinv, f0, acc);
 }
 
-template <int VEC, int L, int NV, int U, int S, class Epi>
+template <int VEC, int L, int NV, int U, int S, class Epi, int AGG = kAggGcn>
 __device__ __forceinline__ void heavy_rows(const SpmmParams &p, const Epi &epi, int f0,
                                            float *part) {
     constexpr int SLAB = L * NV * VEC;
@@ -353,14 +382,15 @@ __device__ __forceinline__ void heavy_rows(const SpmmParams &p, const Epi &epi, 
             const int bit = __ffs(mm) - 1;
             mm &= mm - 1u;
             const int64_t i = base + bit;
-            const RowSpan sp = row_span(p.rowptr, p.nnz, i);
+            const RowSpan sp = row_span(p.rowptr, p.nnz, i, AGG);
             float acc[NV][VEC];
 #pragma unroll
             for (int v = 0; v < NV; ++v)
 #pragma unroll
                 for (int c = 0; c < VEC; ++c) acc[v][c] = 0.0f;
-            const int64_t q0 = sp.total * warp / kSpmmWarps;
-            const int64_t q1 = sp.total * (warp + 1) / kSpmmWarps;
+            const int64_t span = sp.total - sp.first;
+            const int64_t q0 = sp.first + span * warp / kSpmmWarps;
+            const int64_t q1 = sp.first + span * (warp + 1) / kSpmmWarps;
             gather<VEC, L, NV, U, S>(p, i, sp.b, q0, q1, f0, acc);
             reduce_groups<VEC, L, NV>(acc);
             if (g == 0) {
@@ -389,18 +419,19 @@ __device__ __forceinline__ void heavy_rows(const SpmmParams &p, const Epi &epi, 
     }
 }
 
-template <int VEC, int L, int NV, int U, int S>
+template <int VEC, int L, int NV, int U, int S, int AGG>
 __global__ void __launch_bounds__(kSpmmThreads, 4)
 spmm_norm_kernel(SpmmParams p) {
     constexpr int SLAB = L * NV * VEC;
     __shared__ float part[kSpmmWarps * SLAB];
     grid_dependency_wait();     // Z is the output of the previous kernel
     const int f0 = blockIdx.y * SLAB;
-    StoreRow<VEC, L, NV, S> epi;
+    using Epi = StoreRow<VEC, L, NV, S, AGG>;
+    Epi epi;
     if (int(blockIdx.x) < p.heavy_blocks)
-        heavy_rows<VEC, L, NV, U, S>(p, epi, f0, part);
+        heavy_rows<VEC, L, NV, U, S, Epi, AGG>(p, epi, f0, part);
     else
-        light_rows<VEC, L, NV, U, S>(p, epi, f0);
+        light_rows<VEC, L, NV, U, S, Epi, AGG>(p, epi, f0);
 }
 
 // ---------------------------------------------------------------------------
@@ -550,7 +581,7 @@ int64_t heavy_degree(int64_t N, int64_t nnz, int per_iter) {
 // the per-row reduction and epilogue work: worth it from a mean degree of 8.
 bool wide_dots(int64_t N, int64_t nnz) { return N > 0 && nnz >= 8 * N; }
 
-template <int VEC, int L, int NV, int S>
+template <int VEC, int L, int NV, int S, int AGG>
 void launch_cfg(const SpmmArgs &a, const DeviceInfo &dev, int Fload, cudaStream_t s, bool pdl) {
     constexpr int SLAB = L * NV * VEC;
     // Rows in flight per group. A compressed row costs half the registers, so
@@ -564,10 +595,11 @@ void launch_cfg(const SpmmArgs &a, const DeviceInfo &dev, int Fload, cudaStream_
     const bool one_slab = a.F <= SLAB;
     SpmmParams p{a.rowptr, a.colidx, a.N, a.nnz, Z, a.ldz, Fload, a.F, a.H, a.ldh,
                  heavy_block_count(a.N, dev), heavy_degree(a.N, a.nnz, (32 / L) * U), vec_store,
-                 a.rowscale, a.colscale, one_slab ? a.pred : nullptr};
+                 a.rowscale, a.colscale, one_slab ? a.pred : nullptr, a.agg, a.Zs,
+                 a.colscale_s};
     dim3 grid(unsigned(p.heavy_blocks + (a.N + kSpmmWarps - 1) / kSpmmWarps),
               unsigned((a.F + SLAB - 1) / SLAB));
-    launch_kernel(spmm_norm_kernel<VEC, L, NV, U, S>, grid, dim3(kSpmmThreads), 0, s, pdl,
+    launch_kernel(spmm_norm_kernel<VEC, L, NV, U, S, AGG>, grid, dim3(kSpmmThreads), 0, s, pdl,
                   dim3(1, 1, 1), p);
     if (a.pred != nullptr && !one_slab)
         launch_kernel(argmax_rows_kernel, dim3(unsigned((a.N + kSpmmWarps - 1) / kSpmmWarps)),
@@ -577,34 +609,49 @@ void launch_cfg(const SpmmArgs &a, const DeviceInfo &dev, int Fload, cudaStream_
 
 // Lanes per neighbour L = the power of two >= the row's vector count (at
 // least 4, at most 32); NV = 2 vectors per lane once a row exceeds 32.
-template <int VEC, int S>
+template <int VEC, int S, int AGG = kAggGcn>
 void launch_vec(const SpmmArgs &a, const DeviceInfo &dev, int Fload, cudaStream_t s, bool pdl) {
     const int nvec = Fload / VEC;
-    if (nvec <= 4) launch_cfg<VEC, 4, 1, S>(a, dev, Fload, s, pdl);
-    else if (nvec <= 8) launch_cfg<VEC, 8, 1, S>(a, dev, Fload, s, pdl);
-    else if (nvec <= 16) launch_cfg<VEC, 16, 1, S>(a, dev, Fload, s, pdl);
-    else if (nvec <= 32) launch_cfg<VEC, 32, 1, S>(a, dev, Fload, s, pdl);
-    else launch_cfg<VEC, 32, 2, S>(a, dev, Fload, s, pdl);
+    if (nvec <= 4) launch_cfg<VEC, 4, 1, S, AGG>(a, dev, Fload, s, pdl);
+    else if (nvec <= 8) launch_cfg<VEC, 8, 1, S, AGG>(a, dev, Fload, s, pdl);
+    else if (nvec <= 16) launch_cfg<VEC, 16, 1, S, AGG>(a, dev, Fload, s, pdl);
+    else if (nvec <= 32) launch_cfg<VEC, 32, 1, S, AGG>(a, dev, Fload, s, pdl);
+    else launch_cfg<VEC, 32, 2, S, AGG>(a, dev, Fload, s, pdl);
 }
 
-template <int S>
+template <int S, int AGG = kAggGcn>
 void launch_src(const SpmmArgs &a, const DeviceInfo &dev, cudaStream_t s, bool pdl) {
     auto al = [](const void *p, int n) { return aligned_to(p, size_t(n) * 4); };
     // Gathers may read whole vectors past F when the padding up to a multiple
     // of 4 lies inside the row stride and is declared readable (a.z_pad4).
     const int F4 = (a.F + 3) / 4 * 4;
     if (a.ldz % 4 == 0 && al(a.Z, 4) && (a.F % 4 == 0 || (a.z_pad4 && F4 <= a.ldz)))
-        launch_vec<4, S>(a, dev, F4, s, pdl);
+        launch_vec<4, S, AGG>(a, dev, F4, s, pdl);
     else if (a.F % 2 == 0 && a.ldz % 2 == 0 && a.ldh % 2 == 0 && al(a.Z, 2) && al(a.H, 2))
-        launch_vec<2, S>(a, dev, a.F, s, pdl);
+        launch_vec<2, S, AGG>(a, dev, a.F, s, pdl);
     else
-        launch_vec<1, S>(a, dev, a.F, s, pdl);
+        launch_vec<1, S, AGG>(a, dev, a.F, s, pdl);
+}
+
+// Inductive aggregators: fp32 rows without a per-neighbour factor, or dots.
+template <int AGG>
+void launch_inductive(const SpmmArgs &a, const DeviceInfo &dev, cudaStream_t stream, bool pdl) {
+    if (a.D16 != nullptr) {
+        if (a.ldz % 8 == 0 && aligned_to(a.D16, 16) && wide_dots(a.N, a.nnz))
+            launch_vec<8, kDots16, AGG>(a, dev, (a.F + 7) / 8 * 8, stream, pdl);
+        else
+            launch_vec<4, kDots16, AGG>(a, dev, (a.F + 3) / 4 * 4, stream, pdl);
+        return;
+    }
+    launch_src<kPre, AGG>(a, dev, stream, pdl);
 }
 
 }  // namespace
 
 void launch_spmm_norm(const SpmmArgs &a, const DeviceInfo &dev, cudaStream_t stream, bool pdl) {
     if (a.N == 0) return;
+    if (a.agg == kAggMean) return launch_inductive<kAggMean>(a, dev, stream, pdl);
+    if (a.agg == kAggSage) return launch_inductive<kAggSage>(a, dev, stream, pdl);
     if (a.D16 != nullptr) {
         // Compressed rows: eight dots (16 bytes) per vector when the row
         // stride and base allow and rows are long, else four (8 bytes);
