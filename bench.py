@@ -770,6 +770,89 @@ def run_ablation(args, rank, world, local_rank):
     return 0
 
 
+def run_inductive(args, rank, world, local_rank):
+    """Layer 1 of a workload as a binarized inductive GNN layer (Sec. 6.3,
+    Table 3): ``--inductive mean`` (Bi-inductiveGCN's aggregator) or
+    ``--inductive sage`` (Bi-GraphSAGE: a second, seeded neighbour weight
+    matrix). One bigcn_inductive_layer_forward call per step; C1..C4 with L2
+    flushed before every step outside the timed events. The roofline is the
+    whole layer's algorithmic bytes (X read once, packed rows, the factored
+    product written and read once, the CSR, H written) against HBM."""
+    import torch
+
+    from paper_2010_07565_gb300 import binding as B
+    from paper_2010_07565_gb300 import inputs
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    agg = args.inductive
+    w, data = build_workload(args.workload)
+    N, K, F = w.N, w.K, w.hidden
+    d = {k: torch.from_numpy(np.ascontiguousarray(v)).to(dev)
+         for k, v in data.items() if k in ("X", "s", "t", "W1", "rowptr", "colidx")}
+    Wn = torch.from_numpy(inputs.weights(K, F, 3200 + w.index)).to(dev) if agg == "sage" else None
+    nnz = int(data["colidx"].shape[0])
+    ws = torch.empty(B.bigcn_inductive_layer_workspace_bytes(agg, N, K, F), dtype=torch.uint8,
+                     device=dev)
+    H = torch.empty((N, F), device=dev)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    flush_half = flush[: flush.numel() // 2]
+
+    def step():
+        B.bigcn_inductive_layer_forward(agg, d["X"], d["s"], d["t"], d["W1"], d["rowptr"],
+                                        d["colidx"], ws, H, W_neigh=Wn)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    times = []
+    with ClockSampler(local_rank) as clocks:
+        for _ in range(args.steps):
+            flush.zero_()
+            flush_half.sum()
+            e0.record()
+            step()
+            e1.record()
+            e1.synchronize()
+            times.append(e0.elapsed_time(e1))
+    assert B.device_timeouts() == 0
+    total_ms = float(sum(times))
+    max_ms, units = aggregate_over_ranks(total_ms, float(N) * args.steps, world)
+    if rank != 0:
+        return 0
+    peaks, peak_kind = load_peaks()
+    hbm = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+    words = (K + 63) // 64
+    Fz = 2 * ((F + 7) // 8 * 8) if agg == "sage" else (F + 7) // 8 * 8
+    zrow = 2.0 * Fz + 4.0 if K <= 32767 else 4.0 * Fz
+    layer_bytes = (4.0 * N * K + 2 * 8.0 * N * words + 2.0 * N * zrow + 8.0 * (N + 1) +
+                   4.0 * nnz + 4.0 * N * F)
+    mean_ms = max_ms / args.steps
+    achieved = layer_bytes / (mean_ms * 1e-3) / 1e9
+    line = {
+        "metric": f"Bi-GCN inductive layer fwd nodes/s ({agg} aggregator)",
+        "value": units / (max_ms * 1e-3), "unit": "nodes/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": mean_ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32+b1",
+        "data": "synthetic",
+        "config": {"workload": w.description + f" -- layer 1, {agg} aggregator", "name": w.name,
+                   "N": N, "K": K, "F": F, "nnz": nnz,
+                   "l2": "flushed before every step outside the timed events",
+                   "launch": "bigcn_inductive_layer_forward (pack rows, pack weights, XNOR "
+                             "product, aggregation" + (", plus the weight concatenation copies"
+                                                       if agg == "sage" else "") + ")"},
+        "roofline": {"kernel": "whole layer", "bound": "hbm", "achieved": achieved, "peak": hbm,
+                     "unit": "GB/s", "frac": achieved / hbm, "traffic": None,
+                     "peak_source": f"{peak_kind} MEASURED_PEAKS.json hbm_gbs",
+                     "algorithmic_bytes": layer_bytes},
+        "cpu_baseline": None, "e2e": None, "gpu_launches": 4 * args.steps,
+        "clocks": clocks.summary(),
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def run_forward_only(args):
     """R plain forwards of the workload on cuda:0, nothing timed or printed."""
     import torch
@@ -801,6 +884,9 @@ def main(argv=None):
     ap.add_argument("--ablation", choices=["weights", "features"], default=None,
                     help="time layer 1 with only the weights (or only the features) "
                          "binarized (bigcn_layer_forward_ablation) instead")
+    ap.add_argument("--inductive", choices=["gcn", "mean", "sage"], default=None,
+                    help="time layer 1 as a binarized inductive layer "
+                         "(bigcn_inductive_layer_forward) instead")
     ap.add_argument("--forward-only", type=int, default=0, metavar="R",
                     help="run R plain forwards (no graph, no timing, no output) and exit: "
                          "a fixed launch sequence for profilers")
@@ -814,6 +900,8 @@ def main(argv=None):
         return run_forward_only(args)
     if args.ablation is not None:
         return run_ablation(args, rank, world, local_rank)
+    if args.inductive is not None:
+        return run_inductive(args, rank, world, local_rank)
     if args.workload.startswith("C5_"):
         return run_sweep(args, rank, world, local_rank)
     if args.backward:

@@ -212,7 +212,9 @@ bigcn_status bigcn_layer_forward(const float *X, int64_t N, int32_t K, int64_t l
  * (cudaEvent_t as void*, nullable array) is recorded on `stream` before the
  * layer's kernel q (pack rows, pack weights, XNOR product, aggregation) and
  * event 4 after the last (as external events while the stream is being
- * captured); entries beyond 5 are not touched. Everything else is
+ * captured); entries beyond 5 are not touched. When the rows are few and
+ * long (fewer than a wave of warps), the rows are packed inside the product's
+ * kernel and the first interval is empty. Everything else is
  * bigcn_layer_forward's.
  */
 bigcn_status bigcn_layer_forward_timed(const float *X, int64_t N, int32_t K, int64_t ldx,

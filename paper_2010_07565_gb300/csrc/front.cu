@@ -111,8 +111,10 @@ front_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
     for (int i = 0; i < RI; ++i) {
         const int64_t row = m0 + rg + 16 * i;
         if (row >= N) continue;
-        const float ai = sAlpha[rg + 16 * i] *
-                         inv_sqrt_degree(__ldg(rowptr + row + 1) - __ldg(rowptr + row));
+        const float ai = rowptr == nullptr
+                             ? sAlpha[rg + 16 * i]
+                             : sAlpha[rg + 16 * i] *
+                                   inv_sqrt_degree(__ldg(rowptr + row + 1) - __ldg(rowptr + row));
         if (D16 != nullptr) {               // compressed output: biased dots + row scale
             if (cg == 0) rowscale[row] = ai;
 #pragma unroll
@@ -265,8 +267,11 @@ front_split_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
             float t = 0.0f;
 #pragma unroll
             for (int g = 0; g < G; ++g) t += part[rr * G + g];
-            const float ai = (t / float(K)) *
-                             inv_sqrt_degree(__ldg(rowptr + row2 + 1) - __ldg(rowptr + row2));
+            const float ai =
+                rowptr == nullptr
+                    ? t / float(K)
+                    : (t / float(K)) *
+                          inv_sqrt_degree(__ldg(rowptr + row2 + 1) - __ldg(rowptr + row2));
             if (D16 != nullptr && tt == 0) rowscale[row2] = ai;
             const uint64_t *a = As + size_t(rr) * pitch;
             for (int j = 0; j < passes; ++j) {
@@ -328,6 +333,10 @@ bool front_supported(int64_t N, int K, int F, const DeviceInfo &dev) {
     if (F < 1 || F > 128 || K < 1 || K > kFrontMaxK) return false;
     const size_t smem = front_smem(front_rows(N, dev), F, (K + 63) / 64);
     return smem <= kFrontMaxSmem && smem <= size_t(dev.max_smem_optin);
+}
+
+bool front_split_supported(int64_t N, int K, int F, const DeviceInfo &dev) {
+    return split_supported(N, K, F, dev);
 }
 
 void launch_front(const FrontArgs &a, const DeviceInfo &dev, cudaStream_t s, bool pdl) {

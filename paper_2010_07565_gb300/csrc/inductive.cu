@@ -13,12 +13,14 @@
 // taken after the product, as Bi-GCN aggregates after its product).
 //
 // Both run on the Bi-GCN kernels: pack rows (centre, sign, alpha), pack
-// weights, the XNOR product without a degree factor (its row scale is alpha_j
+// weights, the XNOR product without a degree factor (for few long rows the
+// split front kernel packs and multiplies in one pass) (its row scale is alpha_j
 // alone) and the aggregation in its mean / GraphSAGE mode. GraphSAGE's two
-// products are one product over the concatenated columns [W_self | W_neigh],
-// each half padded with zero columns to a multiple of 8 (a zero column packs
-// as +1 signs with beta = 0, so its products are exactly 0), so that both
-// halves of a product row start on a 16-byte boundary for the gathers.
+// products are one product over the packed columns of W_self and W_neigh
+// (packed by one launch into the two halves of one array), each half padded
+// to a multiple of 8 columns with beta = 0 (so the padding's products are
+// exactly 0), so that both halves of a product row start on a 16-byte
+// boundary for the gathers.
 #include "launch.cuh"
 
 using namespace bigcn;
@@ -29,10 +31,10 @@ constexpr size_t kIAlign = 256;
 size_t iround(size_t x) { return (x + kIAlign - 1) / kIAlign * kIAlign; }
 constexpr int32_t kMaxDots16K = 32767;
 
-// Workspace: [W_cat (sage)] A bits, alpha, B bits, beta, Z (factored or fp32),
-// row scale. Fz = product columns (F, or 2 Fp for GraphSAGE).
+// Workspace: A bits, alpha, B bits, beta, Z (factored or fp32), row scale.
+// Fz = product columns (F, or 2 Fp for GraphSAGE).
 struct InductiveWorkspace {
-    size_t wcat, a_bits, alpha, b_bits, beta, z, rowscale, total;
+    size_t a_bits, alpha, b_bits, beta, z, rowscale, total;
     int64_t Fp, Fz, ldz;
     bool compressed;
 };
@@ -49,7 +51,6 @@ bool inductive_workspace(int32_t agg, int64_t N, int32_t K, int32_t F, Inductive
     if (N > kMaxElems / (words > w->ldz ? words : w->ldz)) return false;
     if (int64_t(K) > kMaxElems / w->Fz) return false;
     size_t off = 0;
-    w->wcat = off;   if (sage) off = iround(off + size_t(K) * size_t(w->Fz) * 4);
     w->a_bits = off; off = iround(off + size_t(N) * size_t(words) * 8);
     w->alpha = off;  off = iround(off + size_t(N) * 4);
     w->b_bits = off; off = iround(off + size_t(w->Fz) * size_t(words) * 8);
@@ -120,24 +121,18 @@ extern "C" bigcn_status bigcn_inductive_layer_forward(
     const int Fz = int(w.Fz);
     cudaStream_t s = as_stream(stream);
 
-    // Weight columns: Wt alone, or [Wt | 0 | W_neigh | 0] (K x 2 Fp).
-    const float *Wp = Wt;
-    int64_t ldwp = ldw;
-    if (sage) {
-        float *wcat = reinterpret_cast<float *>(ws + w.wcat);
-        const size_t pitch = size_t(Fz) * 4;
-        if (F != w.Fp && cudaMemsetAsync(wcat, 0, size_t(K) * pitch, s) != cudaSuccess)
-            return BIGCN_ERR_CUDA;
-        if (cudaMemcpy2DAsync(wcat, pitch, Wt, size_t(ldw) * 4, size_t(F) * 4, size_t(K),
-                              cudaMemcpyDeviceToDevice, s) != cudaSuccess ||
-            cudaMemcpy2DAsync(wcat + w.Fp, pitch, W_neigh, size_t(ldwn) * 4, size_t(F) * 4,
-                              size_t(K), cudaMemcpyDeviceToDevice, s) != cudaSuccess)
-            return BIGCN_ERR_CUDA;
-        Wp = wcat;
-        ldwp = Fz;
-    }
-    launch_pack_rows(X, N, K, ldx, scale, shift, a_bits, words, alpha, dev, s);
-    launch_pack_weights(Wp, K, Fz, ldwp, b_bits, words, beta, s);
+    // Packed weight columns: Wt's, or Wt's in columns [0, F) and W_neigh's in
+    // [Fp, Fp + F), the padding columns with beta = 0 (their bits are never
+    // scaled by anything else).
+    if (sage && F != w.Fp && cudaMemsetAsync(beta, 0, size_t(Fz) * 4, s) != cudaSuccess)
+        return BIGCN_ERR_CUDA;
+    const bool fused = front_split_supported(N, K, Fz, dev);
+    if (!fused) launch_pack_rows(X, N, K, ldx, scale, shift, a_bits, words, alpha, dev, s);
+    const WeightPack wa{Wt, K, F, ldw, b_bits, words, beta, 0};
+    const WeightPack wb = sage ? WeightPack{W_neigh, K, F, ldwn, b_bits + w.Fp * words, words,
+                                            beta + w.Fp, 0}
+                               : WeightPack{nullptr, 1, 0, 0, nullptr, 0, nullptr, 0};
+    launch_pack_weights2(wa, wb, s);
     // The product without a degree factor: Z_ij = alpha_i beta_j dot_ij, kept
     // factored (uint16 dots, row scale alpha_i) when K allows.
     GemmArgs g{a_bits, alpha, N, b_bits, beta, Fz, K, words, nullptr, Fz, nullptr, nullptr};
@@ -164,7 +159,13 @@ extern "C" bigcn_status bigcn_inductive_layer_forward(
         // fp32 rows: the gathers read up to F rounded to 4, inside the padded half.
         a.z_pad4 = sage || F % 4 == 0;
     }
-    launch_xnor_gemm(g, dev, s);
+    if (fused) {         // few long rows: centring, packing and product in one kernel
+        FrontArgs fr{X, N, K, ldx, scale, shift, b_bits, beta, Fz, words, nullptr, g.Z, g.ldz,
+                     g.dots16, g.ldd16, g.rowscale};
+        launch_front(fr, dev, s);
+    } else {
+        launch_xnor_gemm(g, dev, s);
+    }
     launch_spmm_norm(a, dev, s);
     return launch_status();
 }

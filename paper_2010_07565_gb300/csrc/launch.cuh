@@ -127,7 +127,7 @@ struct FrontArgs {
     const float *beta;       // F
     int F;
     int words;
-    const int64_t *rowptr;   // rows are scaled by 1/sqrt(1 + deg)
+    const int64_t *rowptr;   // nullable: rows are scaled by 1/sqrt(1 + deg)
     float *Z;                // N x F (row stride ldz)
     int64_t ldz;
     // Compressed output (nullable; replaces Z), as in GemmArgs: dots + 32768
@@ -141,6 +141,10 @@ struct FrontArgs {
 // Whether the fused pack + XNOR-GEMM kernel fits (F <= 128, packed tiles in
 // shared memory).
 bool front_supported(int64_t N, int K, int F, const DeviceInfo &dev);
+
+// Whether the split form of that kernel applies (few rows, each shared by
+// several warps): then it is faster than packing and multiplying apart.
+bool front_split_supported(int64_t N, int K, int F, const DeviceInfo &dev);
 
 // Steps 1, 2 and 4 of one layer in one kernel (see front.cu).
 void launch_front(const FrontArgs &args, const DeviceInfo &dev, cudaStream_t stream,

@@ -5,7 +5,9 @@
 // bigcn_layer_forward enqueues, on one stream:
 //   pack_rows (centre + sign + alpha) -> pack_weights (sign + beta)
 //   -> xnor_gemm whose epilogue also multiplies row j by 1/sqrt(dhat_j)
-//   -> spmm over the pre-scaled rows, which multiplies by 1/sqrt(dhat_i).
+//   -> spmm over the pre-scaled rows, which multiplies by 1/sqrt(dhat_i);
+// for few long rows (fewer than a wave of warps) the split front kernel does
+// pack_rows' and xnor_gemm's work in one pass after pack_weights.
 // Folding the source-side degree factor into the product's epilogue saves the
 // aggregation one random read of the CSR row pointers per edge. When the dots
 // fit 16 bits (K <= 32767) the product leaves Z factored: the integer dots as
@@ -170,8 +172,11 @@ extern "C" bigcn_status bigcn_layer_forward_timed(const float *X, int64_t N, int
     EventMarks marks(events, n_events, s);
     if (!marks.ok()) return BIGCN_ERR_CUDA;
 
+    // Few long rows: centring, packing and the product in one kernel (the
+    // split front), after the weights are packed.
+    const bool fused = front_split_supported(N, K, F, dev);
     marks.mark();
-    launch_pack_rows(X, N, K, ldx, scale, shift, a_bits, words, alpha, dev, s);
+    if (!fused) launch_pack_rows(X, N, K, ldx, scale, shift, a_bits, words, alpha, dev, s);
     marks.mark();
     launch_pack_weights(Wt, K, F, ldw, b_bits, words, beta, s);
     marks.mark();
@@ -191,7 +196,13 @@ extern "C" bigcn_status bigcn_layer_forward_timed(const float *X, int64_t N, int
         a.rowscale = rowscale;
         a.colscale = beta;
     }
-    launch_xnor_gemm(g, dev, s);
+    if (fused) {
+        FrontArgs fr{X, N, K, ldx, scale, shift, b_bits, beta, F, words, rowptr, g.Z, g.ldz,
+                     g.dots16, g.ldd16, g.rowscale};
+        launch_front(fr, dev, s);
+    } else {
+        launch_xnor_gemm(g, dev, s);
+    }
     marks.mark();
     launch_spmm_norm(a, dev, s);
     marks.mark();
