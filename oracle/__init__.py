@@ -17,6 +17,11 @@ the ablation variants of step 4 (Sec. 6.3, one operand kept real):
     zeta = Y W~   (weights binarized only)              oracle_real_binary_product
     zeta = H~ W   (features binarized only)             oracle_binary_real_product
 
+sub-row bucketing (Sec. 4.1, buckets of B consecutive values):
+
+    per-bucket alpha, beta; zeta = sum_b alpha_ib beta_jb dot_b
+        oracle_row_scale_bucketed, oracle_weight_scale_bucketed, oracle_zeta_bucketed
+
 the inductive aggregators (Sec. 6.3, Table 3, GraphSAGE's definitions):
 
     H_i = mean over N(i) u {i} of zeta_j            oracle_aggregate_mean
@@ -102,6 +107,13 @@ def lib() -> ctypes.CDLL:
             h.oracle_aggregate_sage.argtypes = [_i64p, _i32p, _i64, _f64p, _f64p, _i32, _vp,
                                                 _i64, _f64p, _vp]
             h.oracle_aggregate_sage.restype = ctypes.c_int
+            h.oracle_row_scale_bucketed.argtypes = [_f32p, _i64, _i32, _i32, _f64p]
+            h.oracle_row_scale_bucketed.restype = None
+            h.oracle_weight_scale_bucketed.argtypes = [_f32p, _i32, _i32, _i64, _i32, _f64p]
+            h.oracle_weight_scale_bucketed.restype = None
+            h.oracle_zeta_bucketed.argtypes = [_i8p, _f64p, _i64, _i8p, _f64p, _i32, _i32, _i32,
+                                               _f64p, _vp]
+            h.oracle_zeta_bucketed.restype = None
             h.oracle_grad_weight.argtypes = [_f64p, _i8p, _f64p, _f32p, _i32, _i32, _i64, _f64p]
             h.oracle_grad_weight.restype = None
             _lib = h
@@ -326,6 +338,57 @@ def layer_forward_ablation(X, Wt, rowptr, colidx, binarize, s=None, t=None, rows
     out.update(zeta=z, zeta_abs=za, H=H, absterm=absterm,
                scale=aggregate(rowptr, colidx, za, rows=rows))
     return out
+
+
+# ------------------------------------------------------ sub-row bucketing ----
+def buckets(K: int, B: int) -> int:
+    return (K + B - 1) // B
+
+
+def row_scale_bucketed(Y, B):
+    """Eq. 7 per bucket of B consecutive features: alpha (N x nb)."""
+    Y = _c(Y, np.float32)
+    N, K = Y.shape
+    a = np.empty((N, buckets(K, B)), np.float64)
+    lib().oracle_row_scale_bucketed(Y, N, K, B, a)
+    return a
+
+
+def weight_scale_bucketed(Wt, B):
+    """Eq. 4 per bucket of B consecutive entries of each column: beta (F x nb)."""
+    Wt = _c(Wt, np.float32)
+    K, F = Wt.shape
+    b = np.empty((F, buckets(K, B)), np.float64)
+    lib().oracle_weight_scale_bucketed(Wt, K, F, F, B, b)
+    return b
+
+
+def zeta_bucketed(SF, alpha_b, SB, beta_b, B, with_absterm=False):
+    """Eqs. 11-12 with one scale pair per bucket: sum_b alpha_ib beta_jb dot_b."""
+    SF, SB = _c(SF, np.int8), _c(SB, np.int8)
+    N, K = SF.shape
+    F = SB.shape[0]
+    z = np.empty((N, F), np.float64)
+    a = np.empty((N, F), np.float64) if with_absterm else None
+    lib().oracle_zeta_bucketed(SF, _c(alpha_b, np.float64), N, SB, _c(beta_b, np.float64), F,
+                               K, B, z, None if a is None else a.ctypes.data)
+    return (z, a) if with_absterm else z
+
+
+def layer_forward_bucketed(X, Wt, rowptr, colidx, B, s=None, t=None, rows=None) -> dict:
+    """The Bi-GCN layer with buckets of B consecutive features (Sec. 4.1) in
+    place of whole rows / columns, then Eq. 13's aggregation. ``scale`` is
+    A~ applied to the product's |terms| (A~ has no negative entries)."""
+    Y = centre(X, s, t)
+    SF = sign(Y)
+    SB = sign(np.ascontiguousarray(np.asarray(Wt, np.float32).T))
+    alpha_b = row_scale_bucketed(Y, B)
+    beta_b = weight_scale_bucketed(Wt, B)
+    z, za = zeta_bucketed(SF, alpha_b, SB, beta_b, B, with_absterm=True)
+    H, absterm = aggregate(rowptr, colidx, z, rows=rows, with_absterm=True)
+    return dict(Y=Y, SF=SF, SB=SB, alpha_b=alpha_b, beta_b=beta_b, bits=pack(SF),
+                wbits=pack(SB), zeta=z, zeta_abs=za, H=H, absterm=absterm,
+                scale=aggregate(rowptr, colidx, za, rows=rows))
 
 
 # ---------------------------------------------------- inductive aggregators ----

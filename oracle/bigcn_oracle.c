@@ -358,3 +358,56 @@ int oracle_aggregate_sage(const int64_t *rowptr, const int32_t *colidx, int64_t 
     }
     return 0;
 }
+
+/* Number of buckets of B entries that cover K entries. */
+static int32_t bucket_count(int32_t K, int32_t B) { return (K + B - 1) / B; }
+
+void oracle_row_scale_bucketed(const float *Y, int64_t N, int32_t K, int32_t B, double *alpha) {
+    const int32_t nb = bucket_count(K, B);
+    int64_t i;
+    int32_t b, k;
+    for (i = 0; i < N; ++i)
+        for (b = 0; b < nb; ++b) {
+            const int32_t k0 = b * B, k1 = (k0 + B < K) ? k0 + B : K;
+            double sum = 0.0;
+            for (k = k0; k < k1; ++k) sum += fabs((double)Y[i * (int64_t)K + k]);
+            alpha[i * nb + b] = sum / (double)(k1 - k0);
+        }
+}
+
+void oracle_weight_scale_bucketed(const float *Wt, int32_t K, int32_t F, int64_t ldw, int32_t B,
+                                  double *beta) {
+    const int32_t nb = bucket_count(K, B);
+    int32_t j, b, k;
+    for (j = 0; j < F; ++j)
+        for (b = 0; b < nb; ++b) {
+            const int32_t k0 = b * B, k1 = (k0 + B < K) ? k0 + B : K;
+            double sum = 0.0;
+            for (k = k0; k < k1; ++k) sum += fabs((double)Wt[(int64_t)k * ldw + j]);
+            beta[(int64_t)j * nb + b] = sum / (double)(k1 - k0);
+        }
+}
+
+void oracle_zeta_bucketed(const int8_t *SF, const double *alpha, int64_t N, const int8_t *SB,
+                          const double *beta, int32_t F, int32_t K, int32_t B, double *zeta,
+                          double *absterm) {
+    const int32_t nb = bucket_count(K, B);
+    int64_t i;
+    int32_t j, b, k;
+    for (i = 0; i < N; ++i)
+        for (j = 0; j < F; ++j) {
+            double acc = 0.0, mag = 0.0;
+            for (b = 0; b < nb; ++b) {
+                const int32_t k0 = b * B, k1 = (k0 + B < K) ? k0 + B : K;
+                int32_t dot = 0;
+                double term;
+                for (k = k0; k < k1; ++k)
+                    dot += (int32_t)SF[i * (int64_t)K + k] * (int32_t)SB[(int64_t)j * K + k];
+                term = alpha[i * nb + b] * beta[(int64_t)j * nb + b] * (double)dot;
+                acc += term;
+                mag += fabs(term);
+            }
+            zeta[i * (int64_t)F + j] = acc;
+            if (absterm != NULL) absterm[i * (int64_t)F + j] = mag;
+        }
+}

@@ -146,6 +146,24 @@ int oracle_aggregate_sage(const int64_t *rowptr, const int32_t *colidx, int64_t 
                           const double *zself, const double *zneigh, int32_t F,
                           const int64_t *rows, int64_t nrows, double *H, double *absterm);
 
+/* ---- Sub-row bucketing (Sec. 4.1: buckets of B consecutive values, each
+ * scaled separately). Bucket b of a row (column) holds its entries k in
+ * [bB, min(K, (b + 1)B)); nb = ceil(K / B) buckets. ---- */
+
+/* alpha[i * nb + b] = mean over bucket b of |Y[i,k]| (Eq. 7 per bucket). */
+void oracle_row_scale_bucketed(const float *Y, int64_t N, int32_t K, int32_t B, double *alpha);
+
+/* beta[j * nb + b] = mean over bucket b of |Wt[k,j]| (Eq. 4 per bucket). */
+void oracle_weight_scale_bucketed(const float *Wt, int32_t K, int32_t F, int64_t ldw, int32_t B,
+                                  double *beta);
+
+/* zeta[i,j] = sum over buckets b of alpha[i,b] beta[j,b] sum_{k in b} SF[i,k] SB[j,k]
+ * (Eq. 11-12 with one scale pair per bucket). absterm[i,j] (nullable) = the
+ * sum over b of |alpha[i,b] beta[j,b] dot_b|. */
+void oracle_zeta_bucketed(const int8_t *SF, const double *alpha, int64_t N, const int8_t *SB,
+                          const double *beta, int32_t F, int32_t K, int32_t B, double *zeta,
+                          double *absterm);
+
 #ifdef __cplusplus
 }
 #endif
