@@ -350,6 +350,50 @@ bigcn_status bigcn_layer_forward_ablation(int32_t binarize, const float *X, int6
                                           size_t ws_bytes, float *H, int64_t ldh, void *stream);
 
 /*
+ * Sub-row bucketing (Sec. 4.1: the matrix split into buckets of B consecutive
+ * values, each scaled separately). Bucket b of a node row / weight column
+ * holds entries k in [bB, min(K, (b + 1)B)); nb = ceil(K / B). B must be a
+ * positive multiple of 64 (a bucket is whole packed words); B >= K is one
+ * bucket, i.e. Bi-GCN. The packed signs are bigcn_pack_rows' /
+ * bigcn_pack_weights'; the scales gain a bucket index:
+ *
+ *   alpha[i * nb + b] = mean over bucket b of |y_ik|   (N x nb)
+ *   beta[j * nb + b]  = mean over bucket b of |W_kj|   (F x nb)
+ *   Z[i,j] = sum over b of alpha_ib beta_jb (signs in b - 2 popc over b's words)
+ *
+ * Z is accumulated in fp32 bucket by bucket (exact integer counts per bucket).
+ */
+bigcn_status bigcn_pack_rows_bucketed(const float *X, int64_t N, int32_t K, int64_t ldx,
+                                      const float *scale, const float *shift, int32_t B,
+                                      uint64_t *bits, int32_t words, float *alpha, void *stream);
+
+bigcn_status bigcn_pack_weights_bucketed(const float *Wt, int32_t K, int32_t F, int64_t ldw,
+                                         int32_t B, uint64_t *bits, int32_t words, float *beta,
+                                         void *stream);
+
+/* words must equal bigcn_words(K). */
+bigcn_status bigcn_xnor_gemm_bucketed(const uint64_t *a_bits, const float *alpha, int64_t N,
+                                      const uint64_t *b_bits, const float *beta, int32_t F,
+                                      int32_t K, int32_t words, int32_t B, float *Z, int64_t ldz,
+                                      void *stream);
+
+/* Bytes of device workspace bigcn_layer_forward_bucketed needs; 0 on invalid sizes. */
+size_t bigcn_layer_bucketed_workspace_bytes(int64_t N, int32_t K, int32_t F, int32_t B);
+
+/*
+ * One layer H = A~ zeta (Eq. 13) with bucketed binarization: the three calls
+ * above (the product's rows multiplied by 1/sqrt(dhat_i)), then
+ * bigcn_spmm_prescaled. Arguments, layouts and errors are bigcn_layer_forward's
+ * plus B, with this call's workspace size.
+ */
+bigcn_status bigcn_layer_forward_bucketed(int32_t B, const float *X, int64_t N, int32_t K,
+                                          int64_t ldx, const float *scale, const float *shift,
+                                          const float *Wt, int32_t F, int64_t ldw,
+                                          const int64_t *rowptr, const int32_t *colidx,
+                                          int64_t nnz, void *workspace, size_t ws_bytes,
+                                          float *H, int64_t ldh, void *stream);
+
+/*
  * Binarized layers of inductive GNNs (Sec. 6.3, Table 3: Bi-inductiveGCN and
  * Bi-GraphSAGE, which binarize every feature-extraction step of GraphSAGE's
  * models). The product of Eqs. 10-12 is taken on every node's own features,

@@ -69,6 +69,14 @@ SIGNATURES = {
     "bigcn_inductive_layer_workspace_bytes": ([_i32, _i64, _i32, _i32], _sz),
     "bigcn_inductive_layer_forward": ([_i32, _p, _i64, _i32, _i64, _p, _p, _p, _i32, _i64, _p,
                                        _i64, _p, _p, _i64, _p, _sz, _p, _i64, _p], ctypes.c_int),
+    "bigcn_pack_rows_bucketed": ([_p, _i64, _i32, _i64, _p, _p, _i32, _p, _i32, _p, _p],
+                                 ctypes.c_int),
+    "bigcn_pack_weights_bucketed": ([_p, _i32, _i32, _i64, _i32, _p, _i32, _p, _p], ctypes.c_int),
+    "bigcn_xnor_gemm_bucketed": ([_p, _p, _i64, _p, _p, _i32, _i32, _i32, _i32, _p, _i64, _p],
+                                 ctypes.c_int),
+    "bigcn_layer_bucketed_workspace_bytes": ([_i64, _i32, _i32, _i32], _sz),
+    "bigcn_layer_forward_bucketed": ([_i32, _p, _i64, _i32, _i64, _p, _p, _p, _i32, _i64, _p,
+                                      _p, _i64, _p, _sz, _p, _i64, _p], ctypes.c_int),
     "bigcn_layer_forward_static": ([_p, _i64, _i32, _i64, _p, _p, _p, _i32, _i64, _p, _p, _i64,
                                     _p, _i64, _p], ctypes.c_int),
 }
@@ -270,6 +278,46 @@ def bigcn_layer_forward_ablation(binarize, X, scale, shift, Wt, rowptr, colidx, 
         _ptr(Wt), F, _ld(Wt), _ptr(rowptr), _ptr(colidx) if colidx.numel() else None,
         colidx.numel(), _ptr(workspace), workspace.numel() * workspace.element_size(), _ptr(H),
         _ld(H), _stream(stream)))
+
+
+def bigcn_pack_rows_bucketed(X, scale, shift, B, bits, alpha, stream=None):
+    """Sub-row bucketing (Sec. 4.1): packed signs and alpha (N x nb) per
+    bucket of B features (a multiple of 64)."""
+    N, K = X.shape
+    _check("bigcn_pack_rows_bucketed", lib().bigcn_pack_rows_bucketed(
+        _ptr(X), N, K, _ld(X), _ptr(scale), _ptr(shift), B, _ptr(bits), _ld(bits), _ptr(alpha),
+        _stream(stream)))
+
+
+def bigcn_pack_weights_bucketed(Wt, B, bits, beta, stream=None):
+    """Packed weight columns and beta (F x nb) per bucket of B entries."""
+    K, F = Wt.shape
+    _check("bigcn_pack_weights_bucketed", lib().bigcn_pack_weights_bucketed(
+        _ptr(Wt), K, F, _ld(Wt), B, _ptr(bits), _ld(bits), _ptr(beta), _stream(stream)))
+
+
+def bigcn_xnor_gemm_bucketed(a_bits, alpha, b_bits, beta, K, B, Z, stream=None):
+    """Z = sum over buckets of alpha_ib beta_jb dot_b."""
+    N = a_bits.shape[0]
+    F = b_bits.shape[0]
+    _check("bigcn_xnor_gemm_bucketed", lib().bigcn_xnor_gemm_bucketed(
+        _ptr(a_bits), _ptr(alpha), N, _ptr(b_bits), _ptr(beta), F, K, _ld(a_bits), B, _ptr(Z),
+        _ld(Z), _stream(stream)))
+
+
+def bigcn_layer_bucketed_workspace_bytes(N: int, K: int, F: int, B: int) -> int:
+    return int(lib().bigcn_layer_bucketed_workspace_bytes(N, K, F, B))
+
+
+def bigcn_layer_forward_bucketed(B, X, scale, shift, Wt, rowptr, colidx, workspace, H,
+                                 stream=None):
+    """One layer with bucketed binarization (buckets of B features)."""
+    N, K = X.shape
+    F = Wt.shape[1]
+    _check("bigcn_layer_forward_bucketed", lib().bigcn_layer_forward_bucketed(
+        B, _ptr(X), N, K, _ld(X), _ptr(scale), _ptr(shift), _ptr(Wt), F, _ld(Wt), _ptr(rowptr),
+        _ptr(colidx) if colidx.numel() else None, colidx.numel(), _ptr(workspace),
+        workspace.numel() * workspace.element_size(), _ptr(H), _ld(H), _stream(stream)))
 
 
 # Aggregators of the inductive layers (enum bigcn_aggregator).

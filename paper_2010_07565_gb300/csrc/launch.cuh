@@ -225,6 +225,29 @@ size_t weight_parts_bytes(int K, int F);
 void launch_split_weights(const float *Wt, int K, int F, int64_t ldw, uint16_t *wparts,
                           cudaStream_t stream);
 
+// Sub-row bucketing (bucket.cu): buckets of 64 bw signs, scales N x nb / F x nb.
+void launch_pack_rows_bucketed(const float *X, int64_t N, int K, int64_t ldx, const float *scale,
+                               const float *shift, int bw, uint64_t *bits, int words,
+                               float *alpha, const DeviceInfo &dev, cudaStream_t stream);
+void launch_pack_weights_bucketed(const float *Wt, int K, int F, int64_t ldw, int bw,
+                                  uint64_t *bits, int words, float *beta, cudaStream_t stream);
+struct BucketGemmArgs {
+    const uint64_t *A;       // N x words
+    const float *alpha;      // N x nb
+    int64_t N;
+    const uint64_t *B;       // F x words
+    const float *beta;       // F x nb
+    int F;
+    int K;
+    int words;               // ceil(K / 64)
+    int bw;                  // words per bucket
+    float *Z;                // N x F (row stride ldz)
+    int64_t ldz;
+    const int64_t *rowptr;   // nullable: scale row i by 1/sqrt(1 + deg_i)
+};
+void launch_xnor_gemm_bucketed(const BucketGemmArgs &args, const DeviceInfo &dev,
+                               cudaStream_t stream);
+
 // Waits of the ablation products that ran out since the last call (and
 // resets the count); ~0u on a CUDA error.
 uint32_t take_mix_timeouts();
