@@ -853,6 +853,98 @@ def run_inductive(args, rank, world, local_rank):
     return 0
 
 
+def run_bucketed(args, rank, world, local_rank):
+    """Layer 1 of a workload with sub-row bucketing (Sec. 4.1): buckets of
+    ``--bucket`` B features, each with its own scales. One
+    bigcn_layer_forward_bucketed call per step, L2 flushed before every step
+    outside the timed events; also the bucketed product alone, against the
+    POPC peak (its bit-ops) like the plain product."""
+    import torch
+
+    from paper_2010_07565_gb300 import binding as B
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    Bk = args.bucket
+    w, data = build_workload(args.workload)
+    N, K, F = w.N, w.K, w.hidden
+    d = {k: torch.from_numpy(np.ascontiguousarray(v)).to(dev)
+         for k, v in data.items() if k in ("X", "s", "t", "W1", "rowptr", "colidx")}
+    nnz = int(data["colidx"].shape[0])
+    ws = torch.empty(B.bigcn_layer_bucketed_workspace_bytes(N, K, F, Bk), dtype=torch.uint8,
+                     device=dev)
+    H = torch.empty((N, F), device=dev)
+    words, nb = (K + 63) // 64, (K + Bk - 1) // Bk
+    a_bits = torch.empty((N, words), dtype=torch.int64, device=dev)
+    alpha = torch.empty((N, nb), device=dev)
+    b_bits = torch.empty((F, words), dtype=torch.int64, device=dev)
+    beta = torch.empty((F, nb), device=dev)
+    Z = torch.empty((N, F), device=dev)
+    B.bigcn_pack_rows_bucketed(d["X"], d["s"], d["t"], Bk, a_bits, alpha)
+    B.bigcn_pack_weights_bucketed(d["W1"], Bk, b_bits, beta)
+
+    def layer():
+        B.bigcn_layer_forward_bucketed(Bk, d["X"], d["s"], d["t"], d["W1"], d["rowptr"],
+                                       d["colidx"], ws, H)
+
+    def product():
+        B.bigcn_xnor_gemm_bucketed(a_bits, alpha, b_bits, beta, K, Bk, Z)
+
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    flush_half = flush[: flush.numel() // 2]
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+    def timed(fn):
+        out = []
+        for _ in range(args.steps):
+            flush.zero_()
+            flush_half.sum()
+            e0.record()
+            fn()
+            e1.record()
+            e1.synchronize()
+            out.append(e0.elapsed_time(e1))
+        return out
+
+    for _ in range(args.warmup):
+        layer()
+        product()
+    torch.cuda.synchronize()
+    with ClockSampler(local_rank) as clocks:
+        layer_ms = timed(layer)
+        prod_ms = timed(product)
+    total_ms = float(sum(layer_ms))
+    max_ms, units = aggregate_over_ranks(total_ms, float(N) * args.steps, world)
+    if rank != 0:
+        return 0
+    prod_s = statistics.fmean(prod_ms) * 1e-3
+    bitops = float(N) * K * F
+    peak = POPC_PER_CLK_PER_SM * 32 * 152 * 2.070e9 / 1e12
+    achieved = bitops / prod_s / 1e12
+    line = {
+        "metric": f"Bi-GCN bucketed layer fwd nodes/s (buckets of {Bk} features)",
+        "value": units / (max_ms * 1e-3), "unit": "nodes/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": max_ms / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32+b1",
+        "data": "synthetic",
+        "config": {"workload": w.description + f" -- layer 1, buckets of {Bk}", "name": w.name,
+                   "N": N, "K": K, "F": F, "nnz": nnz, "bucket": Bk,
+                   "l2": "flushed before every step outside the timed events",
+                   "launch": "bigcn_layer_forward_bucketed (pack rows, pack weights, product, "
+                             "aggregation)"},
+        "components": {"product_us": 1e3 * statistics.fmean(prod_ms),
+                       "layer_us": 1e3 * statistics.fmean(layer_ms)},
+        "roofline": {"kernel": "bucketed product", "bound": "alu", "achieved": achieved,
+                     "peak": peak, "unit": "T bit-ops/s (N K F)", "frac": achieved / peak,
+                     "traffic": None,
+                     "peak_source": "derived: 16 POPC/clk/SM x 32 bits x 152 SMs x 2070 MHz"},
+        "cpu_baseline": None, "e2e": None, "gpu_launches": 4 * args.steps,
+        "clocks": clocks.summary(),
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def run_forward_only(args):
     """R plain forwards of the workload on cuda:0, nothing timed or printed."""
     import torch
@@ -887,6 +979,9 @@ def main(argv=None):
     ap.add_argument("--inductive", choices=["gcn", "mean", "sage"], default=None,
                     help="time layer 1 as a binarized inductive layer "
                          "(bigcn_inductive_layer_forward) instead")
+    ap.add_argument("--bucket", type=int, default=0, metavar="B",
+                    help="time layer 1 with sub-row bucketing, buckets of B features "
+                         "(a multiple of 64; bigcn_layer_forward_bucketed) instead")
     ap.add_argument("--forward-only", type=int, default=0, metavar="R",
                     help="run R plain forwards (no graph, no timing, no output) and exit: "
                          "a fixed launch sequence for profilers")
@@ -902,6 +997,8 @@ def main(argv=None):
         return run_ablation(args, rank, world, local_rank)
     if args.inductive is not None:
         return run_inductive(args, rank, world, local_rank)
+    if args.bucket > 0:
+        return run_bucketed(args, rank, world, local_rank)
     if args.workload.startswith("C5_"):
         return run_sweep(args, rank, world, local_rank)
     if args.backward:

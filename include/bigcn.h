@@ -353,8 +353,8 @@ bigcn_status bigcn_layer_forward_ablation(int32_t binarize, const float *X, int6
  * Sub-row bucketing (Sec. 4.1: the matrix split into buckets of B consecutive
  * values, each scaled separately). Bucket b of a node row / weight column
  * holds entries k in [bB, min(K, (b + 1)B)); nb = ceil(K / B). B must be a
- * positive multiple of 64 (a bucket is whole packed words); B >= K is one
- * bucket, i.e. Bi-GCN. The packed signs are bigcn_pack_rows' /
+ * positive multiple of 64 (a bucket is whole packed words) with nb <= 65535;
+ * B >= K is one bucket, i.e. Bi-GCN. The packed signs are bigcn_pack_rows' /
  * bigcn_pack_weights'; the scales gain a bucket index:
  *
  *   alpha[i * nb + b] = mean over bucket b of |y_ik|   (N x nb)

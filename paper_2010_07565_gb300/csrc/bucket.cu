@@ -11,12 +11,13 @@
 // gain a bucket index (alpha: N x nb, beta: F x nb, nb = ceil(K / B)).
 //
 // Kernels:
-// * pack_rows_bucketed_kernel: one warp per row, lane l of chunk c owns
-//   feature 32c + l; eight chunks of loads in flight; one ballot per chunk
-//   gives half a word; the |y| of a bucket are summed per lane and reduced
-//   across the warp when the bucket ends.
-// * pack_weights_bucketed_kernel: one thread per (column, bucket), the 64
-//   entries of each word read down the column (coalesced across columns).
+// * pack_rows_bucketed_kernel: one warp per (row, bucket), lane l of chunk c
+//   owns feature 32c + l; eight chunks of loads in flight; one ballot per
+//   chunk gives half a word; the bucket's |y| summed per lane, then across
+//   the warp.
+// * pack_weights_bucketed_kernel: one block per (32 columns, bucket), the
+//   bucket's words spread over eight row groups, each word's 64 entries read
+//   down the column (coalesced across columns), beta added in group order.
 // * xnor_gemm_bucket_kernel: the CUDA-core product of xnor_gemm.cu's shape
 //   (128 x 16 TN tiles, 8-word k-steps staged in shared memory) whose integer
 //   mismatch counts are folded into fp32 accumulators with the bucket's
@@ -35,6 +36,11 @@ namespace cg = cooperative_groups;
 constexpr int kPackWarps = 8;
 constexpr int kUnroll = 8;       // chunks of 32 features in flight per warp
 
+// One warp per (row, bucket) -- grid y is the bucket, grid x strides over
+// rows: the bucket's 2 bw chunks of 32 features, eight
+// chunks (with their centring) loaded before any is used; one ballot per
+// chunk gives half a packed word; the bucket's |y| are summed per lane and
+// reduced across the warp at the end.
 __global__ void __launch_bounds__(32 * kPackWarps)
 pack_rows_bucketed_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
                           const float *__restrict__ scale, const float *__restrict__ shift,
@@ -45,80 +51,94 @@ pack_rows_bucketed_kernel(const float *__restrict__ X, int64_t N, int K, int64_t
     const int64_t nwarps = int64_t(gridDim.x) * kPackWarps;
     const int nchunks = (K + 31) / 32;
     const int bchunks = 2 * bw;                      // chunks per bucket
+    const int b = blockIdx.y;                        // this block's bucket
     for (int64_t row = int64_t(blockIdx.x) * kPackWarps + (threadIdx.x >> 5); row < N;
          row += nwarps) {
         const float *x = X + row * ldx;
-        float part = 0.0f;           // this lane's |y| in the current bucket
+        const int cb = b * bchunks, ce = min(nchunks, cb + bchunks);
+        float part = 0.0f;           // this lane's |y| in the bucket
         uint32_t lo = 0;             // ballot of the word's even chunk
-        for (int c0 = 0; c0 < nchunks; c0 += kUnroll) {
-            float v[kUnroll];
+        for (int c0 = cb; c0 < ce; c0 += kUnroll) {
+            float v[kUnroll], sc[kUnroll], sh[kUnroll];
 #pragma unroll
             for (int u = 0; u < kUnroll; ++u) {
                 const int k = 32 * (c0 + u) + lane;
-                v[u] = k < K ? __ldg(x + k) : 0.0f;
+                const bool in = c0 + u < ce && k < K;
+                v[u] = in ? __ldg(x + k) : 0.0f;
+                sc[u] = (in && scale != nullptr) ? __ldg(scale + k) : 1.0f;
+                sh[u] = (in && scale != nullptr) ? __ldg(shift + k) : 0.0f;
             }
 #pragma unroll
             for (int u = 0; u < kUnroll; ++u) {
                 const int c = c0 + u;
-                if (c >= nchunks) break;
-                const int k = 32 * c + lane;
-                float y = v[u];
-                if (scale != nullptr && k < K) y = __fmaf_rn(y, __ldg(scale + k), __ldg(shift + k));
-                const bool in = k < K;
+                if (c >= ce) break;
+                const bool in = 32 * c + lane < K;
+                const float y = scale != nullptr ? __fmaf_rn(v[u], sc[u], sh[u]) : v[u];
                 const uint32_t m = __ballot_sync(kFullMask, in && y >= 0.0f);
                 if (in) part += fabsf(y);
                 if ((c & 1) == 0) {
                     lo = m;
-                    if (c == nchunks - 1 && lane == 0)
-                        bits[row * words + c / 2] = uint64_t(lo);
+                    if (c == ce - 1 && lane == 0) bits[row * words + c / 2] = uint64_t(lo);
                 } else if (lane == 0) {
                     bits[row * words + c / 2] = uint64_t(lo) | (uint64_t(m) << 32);
                 }
-                if ((c + 1) % bchunks == 0 || c == nchunks - 1) {     // the bucket ends
-                    const int b = c / bchunks;
-                    const int len = min(K, (b + 1) * 64 * bw) - b * 64 * bw;
-                    const float sum = warp_sum(part);
-                    if (lane == 0) alpha[row * nb + b] = sum / float(len);
-                    part = 0.0f;
-                }
             }
         }
-        if (lane == 0)                               // words past the row's chunks
-            for (int w = (nchunks + 1) / 2; w < words; ++w) bits[row * words + w] = 0ull;
+        const int len = min(K, (b + 1) * 64 * bw) - b * 64 * bw;
+        const float sum = warp_sum(part);
+        if (lane == 0) {
+            alpha[row * nb + b] = sum / float(len);
+            if (b == nb - 1)                         // words past the row's chunks
+                for (int w = (nchunks + 1) / 2; w < words; ++w) bits[row * words + w] = 0ull;
+        }
     }
 }
 
-__global__ void __launch_bounds__(256)
+constexpr int kWGroups = 8;      // row groups of the weight-packing block
+
+// One block per (32 columns, bucket): thread (c, g) packs words w0 + g,
+// w0 + g + 8, ... of the bucket for column c (each word's 64 entries read
+// down the column, coalesced across the 32 columns) and sums their |W|; the
+// eight group sums of a column are added in group order.
+__global__ void __launch_bounds__(32 * kWGroups)
 pack_weights_bucketed_kernel(const float *__restrict__ Wt, int K, int F, int64_t ldw, int bw,
                              uint64_t *__restrict__ bits, int words, float *__restrict__ beta,
                              int nb) {
-    const int64_t idx = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
-    if (idx >= int64_t(F) * nb) return;
-    const int j = int(idx % F), b = int(idx / F);
+    __shared__ float part[kWGroups][32];
+    const int c = threadIdx.x & 31, grp = threadIdx.x >> 5;
+    const int j = blockIdx.x * 32 + c;
+    const int b = blockIdx.y;
+    const int w0 = b * bw, w1 = min((K + 63) / 64, (b + 1) * bw);
     float sum = 0.0f;
-    const int w0 = b * bw, w1 = min(words, (b + 1) * bw);
-    for (int w = w0; w < w1; ++w) {
-        uint64_t word = 0ull;
-        float v[64];
+    if (j < F) {
+        for (int w = w0 + grp; w < w1; w += kWGroups) {
+            float v[64];
 #pragma unroll
-        for (int e = 0; e < 64; ++e) {
-            const int k = 64 * w + e;
-            v[e] = k < K ? __ldg(Wt + int64_t(k) * ldw + j) : 0.0f;
-        }
-#pragma unroll
-        for (int e = 0; e < 64; ++e) {
-            const int k = 64 * w + e;
-            if (k < K) {
-                if (v[e] >= 0.0f) word |= uint64_t(1) << e;
-                sum += fabsf(v[e]);
+            for (int e = 0; e < 64; ++e) {
+                const int k = 64 * w + e;
+                v[e] = k < K ? __ldg(Wt + int64_t(k) * ldw + j) : 0.0f;
             }
+            uint64_t word = 0ull;
+#pragma unroll
+            for (int e = 0; e < 64; ++e) {
+                if (64 * w + e < K) {
+                    if (v[e] >= 0.0f) word |= uint64_t(1) << e;
+                    sum += fabsf(v[e]);
+                }
+            }
+            bits[int64_t(j) * words + w] = word;
         }
-        bits[int64_t(j) * words + w] = word;
     }
-    const int len = min(K, (b + 1) * 64 * bw) - b * 64 * bw;
-    beta[int64_t(j) * nb + b] = len > 0 ? sum / float(len) : 0.0f;
-    if (b == nb - 1)                                 // words past the last bucket
-        for (int w = w1; w < words; ++w) bits[int64_t(j) * words + w] = 0ull;
+    part[grp][c] = sum;
+    __syncthreads();
+    if (grp == 0 && j < F) {
+        float t = 0.0f;
+        for (int g = 0; g < kWGroups; ++g) t += part[g][c];
+        const int len = min(K, (b + 1) * 64 * bw) - b * 64 * bw;
+        beta[int64_t(j) * nb + b] = t / float(len);
+        if (b == nb - 1)                             // words past the last bucket
+            for (int w = w1; w < words; ++w) bits[int64_t(j) * words + w] = 0ull;
+    }
 }
 
 constexpr int kBM = 128;     // rows per block tile
@@ -311,18 +331,20 @@ void launch_pack_rows_bucketed(const float *X, int64_t N, int K, int64_t ldx, co
                                float *alpha, const DeviceInfo &dev, cudaStream_t stream) {
     if (N == 0) return;
     const int nb = (K + 64 * bw - 1) / (64 * bw);
+    // Grid y = the bucket; grid x strides over rows, about 16 blocks per SM in all.
     const int64_t want = (N + kPackWarps - 1) / kPackWarps;
-    const int64_t cap = int64_t(dev.sm_count) * 16;
-    pack_rows_bucketed_kernel<<<unsigned(want < cap ? want : cap), 32 * kPackWarps, 0, stream>>>(
-        X, N, K, ldx, scale, shift, bw, bits, words, alpha, nb);
+    int64_t cap = int64_t(dev.sm_count) * 16 / nb;
+    if (cap < 1) cap = 1;
+    pack_rows_bucketed_kernel<<<dim3(unsigned(want < cap ? want : cap), unsigned(nb)),
+                                32 * kPackWarps, 0, stream>>>(X, N, K, ldx, scale, shift, bw,
+                                                             bits, words, alpha, nb);
 }
 
 void launch_pack_weights_bucketed(const float *Wt, int K, int F, int64_t ldw, int bw,
                                   uint64_t *bits, int words, float *beta, cudaStream_t stream) {
     const int nb = (K + 64 * bw - 1) / (64 * bw);
-    const int64_t n = int64_t(F) * nb;
-    pack_weights_bucketed_kernel<<<unsigned((n + 255) / 256), 256, 0, stream>>>(
-        Wt, K, F, ldw, bw, bits, words, beta, nb);
+    pack_weights_bucketed_kernel<<<dim3(unsigned((F + 31) / 32), unsigned(nb)), 32 * kWGroups, 0,
+                                   stream>>>(Wt, K, F, ldw, bw, bits, words, beta, nb);
 }
 
 void launch_xnor_gemm_bucketed(const BucketGemmArgs &g, const DeviceInfo &dev,
@@ -343,6 +365,8 @@ size_t bround(size_t x) { return (x + kBAlign - 1) / kBAlign * kBAlign; }
 
 int bucket_words(int32_t B) { return (B > 0 && B % 64 == 0) ? B / 64 : 0; }
 int64_t bucket_count(int32_t K, int32_t B) { return (int64_t(K) + B - 1) / B; }
+// The packing kernels put the bucket on the grid's y dimension.
+constexpr int64_t kMaxBuckets = 65535;
 
 // Workspace of bigcn_layer_forward_bucketed: A bits, alpha (N x nb), B bits,
 // beta (F x nb), Z' (N x F fp32).
@@ -353,6 +377,7 @@ struct BucketWorkspace {
 bool bucket_workspace(int64_t N, int32_t K, int32_t F, int32_t B, BucketWorkspace *w) {
     if (N < 0 || K < 1 || F < 1 || bucket_words(B) == 0) return false;
     const int64_t words = bigcn_words(K), nb = bucket_count(K, B);
+    if (nb > kMaxBuckets) return false;
     const int64_t widest = words > F ? (words > nb ? words : nb) : (F > nb ? F : nb);
     if (N > kMaxElems / widest) return false;
     size_t off = 0;
@@ -376,6 +401,7 @@ extern "C" bigcn_status bigcn_pack_rows_bucketed(const float *X, int64_t N, int3
         return BIGCN_ERR_INVALID_ARG;
     if ((scale == nullptr) != (shift == nullptr)) return BIGCN_ERR_INVALID_ARG;
     const int64_t nb = bucket_count(K, B);
+    if (nb > kMaxBuckets) return BIGCN_ERR_INVALID_ARG;
     if (N > 0 && (N > kMaxElems / ldx || N > kMaxElems / words || N > kMaxElems / nb))
         return BIGCN_ERR_INVALID_ARG;
     if (N == 0) return BIGCN_OK;
@@ -406,6 +432,7 @@ extern "C" bigcn_status bigcn_pack_weights_bucketed(const float *Wt, int32_t K, 
     if (!aligned_to(Wt, 4) || !aligned_to(bits, 8) || !aligned_to(beta, 4))
         return BIGCN_ERR_MISALIGNED;
     const int64_t nb = bucket_count(K, B);
+    if (nb > kMaxBuckets) return BIGCN_ERR_INVALID_ARG;
     const size_t wb = span_bytes(K, F, ldw, 4), bb = size_t(F) * words * 8,
                  eb = size_t(F) * size_t(nb) * 4;
     if (overlaps(bits, bb, Wt, wb) || overlaps(beta, eb, Wt, wb) || overlaps(beta, eb, bits, bb))
