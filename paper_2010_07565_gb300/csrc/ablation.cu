@@ -206,6 +206,7 @@ struct MixParams {
     int64_t ldz;
     const int64_t *rowptr;   // nullable: rows scaled by 1/sqrt(dhat_i)
     int split;               // KS: CTAs of a cluster sharing a tile's k-blocks
+    bool clip;               // store z where |z| < 1, else 0 (Eq. bp-H)
 };
 
 // Shared-memory plan. Weights binarized (A real): kStages operand stages of
@@ -336,7 +337,10 @@ __device__ __forceinline__ void mix_epilogue(const MixParams &p, unsigned char *
         return rs;
     };
     auto scaled = [&](float rs, int col, float acc) {
-        return kRealA ? rs * (__ldg(p.beta + col) * acc) : rs * acc;
+        float z = kRealA ? rs * ((p.beta != nullptr ? __ldg(p.beta + col) : 1.0f) * acc)
+                         : rs * acc;
+        if (p.clip && !(fabsf(z) < 1.0f)) z = 0.0f;
+        return z;
     };
     const bool vec_z = (p.ldz & 3) == 0 && (reinterpret_cast<uintptr_t>(p.Z) & 15) == 0;
 
@@ -543,7 +547,7 @@ real_binary_tc_kernel(const MixParams p) {
                 for (int e = 0; e < 8; ++e) {
                     const bool in = k + e < p.K;      // y = fmaf(0, 0, 0) = 0 past K
                     sv[e] = in ? __ldg(p.scale + k + e) : 0.0f;
-                    tv[e] = in ? __ldg(p.shift + k + e) : 0.0f;
+                    tv[e] = (in && p.shift != nullptr) ? __ldg(p.shift + k + e) : 0.0f;
                 }
             }
         };
@@ -787,6 +791,7 @@ void launch_real_binary_gemm(const RealBinaryArgs &g, const DeviceInfo &dev, cud
     p.Z = g.Z;
     p.ldz = g.ldz;
     p.rowptr = g.rowptr;
+    p.clip = g.clip;
     if (g.F <= 64) launch_mix<64, true>(p, dev, stream, pdl);
     else if (g.F <= 128) launch_mix<128, true>(p, dev, stream, pdl);
     else launch_mix<256, true>(p, dev, stream, pdl);

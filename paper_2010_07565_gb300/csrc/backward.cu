@@ -12,10 +12,14 @@
 // (alpha: per-node scale, the paper's beta; beta: per-column scale, the
 // paper's alpha; B = sign(W).) The signs come packed from the forward's own
 // kernels (the rows re-packed from X with the same centring, the columns
-// from W). Both products multiply a +-1 matrix by an fp32 one; they run on
-// the CUDA cores in fp32 (the tensor cores' bf16 / tf32 inputs would round
-// G): 64 x 64 output tiles, each thread a 4 x 4 register block that adds
-// +-v for the signs of one packed word.
+// from W). Both products multiply a +-1 matrix by an fp32 one. dH~ runs on
+// the tensor cores through the real x binary product of ablation.cu: the
+// real operand G (times beta_j, applied as its centring scale and rounded
+// once) split into three bf16 parts, the signs of W's rows (W packed row by
+// row over its F columns) exact in bf16, fp32 accumulators, and the clip of
+// Eq. bp-H in the epilogue. dW~ runs on the CUDA cores in fp32: 64 x 64
+// output tiles, each thread a 4 x 4 register block that adds +-v for the
+// signs of one packed word.
 //
 // dW~ sums over all N rows: the rows are split into S chunks (grid z) whose
 // partial sums are added, chunk by chunk in order, by a second kernel, so
@@ -99,79 +103,47 @@ sum_partials_kernel(const float *__restrict__ partial, int S, int64_t n, float *
     }
 }
 
-// dL/dH (Eq. bp-H) for tile (it, kt) of the N x K output: thread (ti, tk)
-// owns rows 64 it + 4 ti + 0..3 and k = 64 kt + 4 tk + 0..3; the sum over j
-// walks the F columns of G (times beta_j) and the signs of W's column j.
-__global__ void __launch_bounds__(kBwThreads)
-grad_input_kernel(const float *__restrict__ G, int64_t ldg, const float *__restrict__ beta,
-                  const uint64_t *__restrict__ wbits, int words, int64_t N, int K, int F,
-                  float *__restrict__ dX, int64_t lddx) {
-    __shared__ __align__(16) float sG[kRowsPerStage][kTile];    // beta_j G[i, j], [j][row]
-    __shared__ uint64_t sW[kRowsPerStage];                      // column j's word of the k-tile
-    const int tid = threadIdx.x, ti = tid / 16, tk = tid % 16;
-    const int64_t i0 = int64_t(blockIdx.x) * kTile;
-    const int kt = blockIdx.y;
-    float acc[4][4] = {};
-    for (int j0 = 0; j0 < F; j0 += kRowsPerStage) {
-        __syncthreads();
-        for (int q = tid; q < kRowsPerStage * kTile; q += kBwThreads) {
-            const int jj = q / kTile, r = q % kTile;
-            const int64_t i = i0 + r;
-            const int j = j0 + jj;
-            sG[jj][r] = (i < N && j < F) ? __ldg(beta + j) * __ldg(G + i * ldg + j) : 0.0f;
-        }
-        for (int jj = tid; jj < kRowsPerStage; jj += kBwThreads) {
-            const int j = j0 + jj;
-            sW[jj] = j < F ? __ldg(wbits + int64_t(j) * words + kt) : 0ull;
-        }
-        __syncthreads();
-        const int n = F - j0 < kRowsPerStage ? F - j0 : kRowsPerStage;
-        for (int jj = 0; jj < n; ++jj) {
-            const uint64_t w = sW[jj];
-            const float4 g = *reinterpret_cast<const float4 *>(&sG[jj][4 * ti]);
-            float s[4];
-#pragma unroll
-            for (int b = 0; b < 4; ++b) s[b] = pm1(w, 4 * tk + b);
-#pragma unroll
-            for (int b = 0; b < 4; ++b) {
-                acc[0][b] = fmaf(g.x, s[b], acc[0][b]);
-                acc[1][b] = fmaf(g.y, s[b], acc[1][b]);
-                acc[2][b] = fmaf(g.z, s[b], acc[2][b]);
-                acc[3][b] = fmaf(g.w, s[b], acc[3][b]);
-            }
-        }
+constexpr int kColGroups = 32;   // row groups of the column-sum block (1024 threads)
+
+// Eq. bp-W, first term's sum: c_j = sum_k dW~_kj B_kj. One block per 32
+// columns: thread (c, g) sums rows g, g + 32, ... of column c (coalesced
+// across the 32 columns), and the 32 group sums are added in group order.
+__global__ void __launch_bounds__(32 * kColGroups)
+weight_colsum_kernel(const float *__restrict__ Wg, const uint64_t *__restrict__ wbits, int words,
+                     int K, int F, float *__restrict__ csum) {
+    __shared__ float part[kColGroups][32];
+    const int cl = threadIdx.x & 31, g = threadIdx.x >> 5;
+    const int j = blockIdx.x * 32 + cl;
+    float acc = 0.0f;
+    if (j < F) {
+        const uint64_t *wb = wbits + int64_t(j) * words;
+        for (int k = g; k < K; k += kColGroups)
+            acc = fmaf(__ldg(Wg + int64_t(k) * F + j), pm1(__ldg(wb + k / 64), k % 64), acc);
     }
-#pragma unroll
-    for (int a = 0; a < 4; ++a) {
-        const int64_t i = i0 + 4 * ti + a;
-        if (i >= N) continue;
-#pragma unroll
-        for (int b = 0; b < 4; ++b) {
-            const int k = kt * kTile + 4 * tk + b;
-            if (k < K) dX[i * lddx + k] = fabsf(acc[a][b]) < 1.0f ? acc[a][b] : 0.0f;
-        }
+    part[g][cl] = acc;
+    __syncthreads();
+    if (g == 0 && j < F) {
+        float t = 0.0f;
+        for (int q = 0; q < kColGroups; ++q) t += part[q][cl];
+        csum[j] = t;
     }
 }
 
-// Eq. bp-W, one warp per column j: c_j = sum_k dW~_kj B_kj (lane-strided,
-// then a fixed shuffle tree), then every entry of the column.
+// Eq. bp-W, every entry: dW_kj = B_kj c_j / K + beta_j dW~_kj 1(|W_kj| < 1).
 __global__ void __launch_bounds__(kBwThreads)
 grad_weight_kernel(const float *__restrict__ Wg, const uint64_t *__restrict__ wbits, int words,
-                   const float *__restrict__ beta, const float *__restrict__ Wt, int64_t ldw,
-                   int K, int F, float *__restrict__ dW, int64_t lddw) {
-    const int lane = threadIdx.x & 31;
-    const int j = blockIdx.x * (kBwThreads / 32) + (threadIdx.x >> 5);
-    if (j >= F) return;
-    const uint64_t *wb = wbits + int64_t(j) * words;
-    float c = 0.0f;
-    for (int k = lane; k < K; k += 32) c = fmaf(__ldg(Wg + int64_t(k) * F + j), pm1(__ldg(wb + k / 64), k % 64), c);
-    c = warp_sum(c);
-    const float bj = __ldg(beta + j), cK = c / float(K);
-    for (int k = lane; k < K; k += 32) {
+                   const float *__restrict__ beta, const float *__restrict__ csum,
+                   const float *__restrict__ Wt, int64_t ldw, int K, int F,
+                   float *__restrict__ dW, int64_t lddw) {
+    const int64_t n = int64_t(K) * F;
+    for (int64_t q = int64_t(blockIdx.x) * kBwThreads + threadIdx.x; q < n;
+         q += int64_t(gridDim.x) * kBwThreads) {
+        const int k = int(q / F), j = int(q % F);
         const float w = __ldg(Wt + int64_t(k) * ldw + j);
         const float ste = fabsf(w) < 1.0f ? 1.0f : 0.0f;
-        dW[int64_t(k) * lddw + j] =
-            pm1(__ldg(wb + k / 64), k % 64) * cK + bj * __ldg(Wg + int64_t(k) * F + j) * ste;
+        const float b = pm1(__ldg(wbits + int64_t(j) * words + k / 64), k % 64);
+        dW[int64_t(k) * lddw + j] = b * (__ldg(csum + j) / float(K)) +
+                                    __ldg(beta + j) * __ldg(Wg + q) * ste;
     }
 }
 
@@ -197,7 +169,7 @@ int wtilde_chunks(int64_t N, int K, int F, const DeviceInfo &dev) {
 }
 
 struct BackwardWorkspace {
-    size_t bits, alpha, wbits, beta, g, wg, partial, total;
+    size_t bits, alpha, wbits, beta, g, wg, partial, wrows, wrow_scale, csum, total;
 };
 
 bool backward_workspace(int64_t N, int32_t K, int32_t F, BackwardWorkspace *w) {
@@ -213,6 +185,9 @@ bool backward_workspace(int64_t N, int32_t K, int32_t F, BackwardWorkspace *w) {
     w->g = take(size_t(N) * F * 4);
     w->wg = take(size_t(K) * F * 4);
     w->partial = take(size_t(max_chunks(K, F)) * K * F * 4);
+    w->wrows = take(size_t(K) * size_t(bigcn_words(F)) * 8);   // W's rows packed over F
+    w->wrow_scale = take(size_t(K) * 4);                         // (their row scales, unused)
+    w->csum = take(size_t(F) * 4);
     w->total = off;
     return true;
 }
@@ -299,10 +274,22 @@ extern "C" bigcn_status bigcn_layer_backward(
                                        ? (kf + kBwThreads - 1) / kBwThreads : 4096),
                           kBwThreads, 0, s>>>(partial, S, kf, Wg);
     if (dX) {
-        const dim3 gi(unsigned((N + kTile - 1) / kTile), unsigned((K + kTile - 1) / kTile));
-        grad_input_kernel<<<gi, kBwThreads, 0, s>>>(G, F, beta, wbits, words, N, K, F, dX, lddx);
+        // dH~ = (G diag(beta)) sign(W)^T with the clip of Eq. bp-H: contraction
+        // over F, one output column per feature k.
+        uint64_t *wrows = reinterpret_cast<uint64_t *>(ws + w.wrows);
+        float *wrow_scale = reinterpret_cast<float *>(ws + w.wrow_scale);
+        const int fwords = bigcn_words(F);
+        launch_pack_rows(Wt, K, F, ldw, nullptr, nullptr, wrows, fwords, wrow_scale, dev, s);
+        RealBinaryArgs gi{G, F, beta, nullptr, wrows, nullptr, N, F, K, fwords, dX, lddx,
+                          nullptr};
+        gi.clip = true;
+        launch_real_binary_gemm(gi, dev, s);
     }
-    grad_weight_kernel<<<unsigned((F + kBwThreads / 32 - 1) / (kBwThreads / 32)), kBwThreads, 0,
-                         s>>>(Wg, wbits, words, beta, Wt, ldw, K, F, dW, lddw);
+    float *csum = reinterpret_cast<float *>(ws + w.csum);
+    weight_colsum_kernel<<<unsigned((F + 31) / 32), 32 * kColGroups, 0, s>>>(Wg, wbits, words, K,
+                                                                            F, csum);
+    const int64_t kfs = (int64_t(K) * F + kBwThreads - 1) / kBwThreads;
+    grad_weight_kernel<<<unsigned(kfs < 4096 ? kfs : 4096), kBwThreads, 0, s>>>(
+        Wg, wbits, words, beta, csum, Wt, ldw, K, F, dW, lddw);
     return launch_status();
 }

@@ -190,9 +190,9 @@ struct RealBinaryArgs {      // weights binarized: Z = Y W~
     const float *X;          // N x K (row stride ldx), centred by scale/shift
     int64_t ldx;
     const float *scale;      // nullable (identity)
-    const float *shift;
+    const float *shift;      // nullable with scale non-null: y = x * scale (rounded once)
     const uint64_t *b_bits;  // F x words
-    const float *beta;       // F
+    const float *beta;       // F; nullable: column scales of 1
     int64_t N;
     int K;
     int F;
@@ -200,6 +200,7 @@ struct RealBinaryArgs {      // weights binarized: Z = Y W~
     float *Z;                // N x F (row stride ldz)
     int64_t ldz;
     const int64_t *rowptr;   // nullable: scale row i by 1/sqrt(1 + deg_i)
+    bool clip = false;       // store z where |z| < 1, else 0 (Eq. bp-H)
 };
 void launch_real_binary_gemm(const RealBinaryArgs &args, const DeviceInfo &dev,
                              cudaStream_t stream, bool pdl = false);
