@@ -726,6 +726,175 @@ binary_real_tc_kernel(const MixParams p) {
     mix_finish<NT, false, kStages>(p, tiles, tmem, m0, n0, rank, kb1 > kb0, sy);
 }
 
+// ---- transposed signs x real: P_s = sum over nodes i of chunk s of
+//      (alpha_i sign(y_ik)) G_ij  (dL/dW~ = H~^T G of Algorithm 1) ----
+//
+// M = the features k (128 per tile), N = the columns j (NT per tile), the
+// contraction over nodes in k-blocks of 64, split over S CTAs (grid z) that
+// each write a fp32 partial; the partials are added in order afterwards.
+// A (K-major: a row per feature, 64 nodes along it) is built from the nodes'
+// packed words: a producer warp takes 32 consecutive features of one 8-node
+// chunk, so its eight word loads are broadcasts, and gathers bit k of each
+// node into a byte of signs. B holds alpha_i G_ij (rounded once) as three
+// bf16 parts, read coalesced across the columns. Warp roles and barriers are
+// those of the ablation products.
+template <int NT>
+struct SignTShape {
+    static constexpr int kTileA = kUmmaM * 128;
+    static constexpr int kTileB = NT * 128;
+    static constexpr int kStage = kTileA + kParts * kTileB;
+    static constexpr int kStages = NT <= 64 ? 4 : (NT <= 128 ? 3 : 2);
+    static constexpr size_t kSmem = 1024 + size_t(kStages) * kStage;
+    static_assert(kSmem <= 227 * 1024, "shared memory per CTA");
+};
+
+struct SignTParams {
+    const uint64_t *bits;    // N x words packed node signs (K features)
+    int words;
+    const float *alpha;      // N
+    const float *G;          // N x F (row stride ldg)
+    int64_t ldg;
+    int64_t N;
+    int K;
+    int F;
+    float *partial;          // S x K x F (row stride F)
+    int per;                 // k-blocks (of 64 nodes) per split
+};
+
+template <int NT>
+__global__ void __launch_bounds__(kMixThreads, 1)
+sign_t_real_tc_kernel(const SignTParams p) {
+    using S = SignTShape<NT>;
+    constexpr int kStages = S::kStages;
+    extern __shared__ unsigned char smem_raw[];
+    __shared__ __align__(8) MixSync<kStages> sy;
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int m0 = blockIdx.x * kUmmaM;         // first feature of the tile
+    const int n0 = blockIdx.y * NT;             // first column
+    const int split = blockIdx.z;
+    const int64_t KB = (p.N + kMixK - 1) / kMixK;
+    const int64_t kb0 = min(KB, int64_t(split) * p.per), kb1 = min(KB, kb0 + p.per);
+    const uint32_t raw_addr = smem_addr(smem_raw);
+    const uint32_t base = (raw_addr + 1023u) & ~1023u;
+    unsigned char *tiles = smem_raw + (base - raw_addr);
+
+    const uint32_t tmem = mix_setup<NT, kStages>(sy);
+    grid_dependency_wait();     // packed rows and G come from earlier kernels
+
+    if (warp == kMmaWarp) {
+        constexpr uint32_t idesc = bf16_idesc(NT);
+        mma_loop<kStages>(sy, int(kb1 - kb0), [&](int it, int s) {
+            const uint32_t a0 = base + s * S::kStage, b0 = a0 + S::kTileA;
+#pragma unroll
+            for (int k = 0; k < kMixK / 16; ++k)
+#pragma unroll
+                for (int part = 0; part < kParts; ++part)
+                    mma_bf16(tmem, sw128_desc(a0 + 32u * k),
+                             sw128_desc(b0 + part * S::kTileB + 32u * k), idesc,
+                             (it > 0 || k > 0 || part > 0) ? 1u : 0u);
+        });
+    } else {
+#pragma unroll 1
+        for (int64_t kb = kb0; kb < kb1; ++kb) {
+            const int it = int(kb - kb0);
+            const int s = it % kStages;
+            if (it >= kStages &&
+                !wait_or_abort(smem_addr(&sy.empty[s]), uint32_t(it / kStages - 1) & 1u,
+                               &sy.abort)) {
+                sy.abort = 1u;
+                break;
+            }
+            unsigned char *sa = tiles + s * S::kStage;
+            unsigned char *sb = sa + S::kTileA;
+            const int64_t i0 = kb * kMixK;
+            // A: 4 x 8 (feature group, node chunk) tasks of 32 features x 8 nodes.
+            for (int t = warp; t < 32; t += kProducerWarps) {
+                const int c = t & 7, mh = t >> 3;
+                const int m = 32 * mh + lane, f = m0 + m;
+                const int wi = (m0 + 32 * mh) / 64;          // the same word for the warp
+                uint32_t byte = 0;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    const int64_t i = i0 + 8 * c + e;
+                    const uint64_t w =
+                        (i < p.N && wi < p.words) ? __ldg(p.bits + i * p.words + wi) : 0ull;
+                    byte |= uint32_t((w >> (f & 63)) & 1ull) << e;
+                }
+                *reinterpret_cast<uint4 *>(sa + sw128_offset(m, c)) = signs8_to_bf16(byte);
+            }
+            // B: (NT / 32) x 8 (column group, node chunk) tasks of 32 columns x 8 nodes.
+            for (int t = warp; t < (NT / 32) * 8; t += kProducerWarps) {
+                const int c = t & 7, jh = t >> 3;
+                const int r = 32 * jh + lane, j = n0 + r;
+                float v[8];
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    const int64_t i = i0 + 8 * c + e;
+                    v[e] = (i < p.N && j < p.F) ? __ldg(p.alpha + i) * __ldg(p.G + i * p.ldg + j)
+                                                : 0.0f;
+                }
+                uint32_t h[4], mi[4], lo[4];
+#pragma unroll
+                for (int w = 0; w < 4; ++w) split3x2(v[2 * w], v[2 * w + 1], h[w], mi[w], lo[w]);
+                const uint32_t off = sw128_offset(r, c);
+                *reinterpret_cast<uint4 *>(sb + off) = make_uint4(h[0], h[1], h[2], h[3]);
+                *reinterpret_cast<uint4 *>(sb + S::kTileB + off) =
+                    make_uint4(mi[0], mi[1], mi[2], mi[3]);
+                *reinterpret_cast<uint4 *>(sb + 2 * S::kTileB + off) =
+                    make_uint4(lo[0], lo[1], lo[2], lo[3]);
+            }
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            mbar_arrive(smem_addr(&sy.full[s]));
+        }
+    }
+    // The last MMA is done once `done` completes; then warps 0-15 move the
+    // partial tile (rows = features, zeros for an empty split) to memory.
+    const bool done = mbar_wait(smem_addr(&sy.done), 0u);
+    const bool ok = __syncthreads_and(done && sy.abort == 0u) != 0;
+    if (!ok && tid == 0) atomicAdd(&g_mix_timeouts, 1u);
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    if (ok && warp < kProducerWarps) {
+        const int quad = warp & 3, group = warp >> 2;
+        const int f = m0 + 32 * quad + lane;
+        const uint32_t taddr = tmem + (uint32_t(32 * quad) << 16);
+        const bool has_acc = kb1 > kb0;
+        float *prow = p.partial + (int64_t(split) * p.K + f) * p.F;
+#pragma unroll 1
+        for (int c0 = 16 * group; c0 < NT; c0 += 64) {
+            uint32_t acc[16];
+            if (has_acc) tmem_ld16(taddr + uint32_t(c0), acc);
+            else {
+#pragma unroll
+                for (int j = 0; j < 16; ++j) acc[j] = 0u;
+            }
+            if (f >= p.K) continue;
+#pragma unroll
+            for (int j = 0; j < 16; ++j)
+                if (n0 + c0 + j < p.F) prow[n0 + c0 + j] = __uint_as_float(acc[j]);
+        }
+    }
+    mix_teardown<NT>(tmem);
+}
+
+template <int NT>
+int launch_sign_t(SignTParams p, int max_split, const DeviceInfo &dev, cudaStream_t stream) {
+    using S = SignTShape<NT>;
+    const int mt = (p.K + kUmmaM - 1) / kUmmaM, nt = (p.F + NT - 1) / NT;
+    const int64_t KB = (p.N + kMixK - 1) / kMixK;
+    int64_t want = (int64_t(dev.sm_count) + int64_t(mt) * nt - 1) / (int64_t(mt) * nt);
+    if (want > max_split) want = max_split;
+    if (want > KB) want = KB;
+    if (want < 1) want = 1;
+    p.per = int((KB + want - 1) / want);
+    const int splits = int((KB + p.per - 1) / p.per);
+    cudaFuncSetAttribute(sign_t_real_tc_kernel<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         int(S::kSmem));
+    launch_kernel(sign_t_real_tc_kernel<NT>, dim3(unsigned(mt), unsigned(nt), unsigned(splits)),
+                  dim3(kMixThreads), S::kSmem, stream, false, dim3(1, 1, 1), p);
+    return splits;
+}
+
 // W (K x F, row stride ldw) -> wparts[p][j][k], the three bf16 parts of
 // W[k][j], zero for k >= K (k < words * 64). Thread (j, 8-element chunk).
 __global__ void __launch_bounds__(256)
@@ -819,6 +988,15 @@ void launch_binary_real_gemm(const BinaryRealArgs &g, const DeviceInfo &dev, cud
     p.ldz = g.ldz;
     p.rowptr = g.rowptr;
     launch_mix<64, false>(p, dev, stream, pdl);
+}
+
+int launch_sign_t_real_gemm(const SignTRealArgs &a, int max_split, const DeviceInfo &dev,
+                            cudaStream_t stream) {
+    if (a.N == 0) return 0;
+    SignTParams p{a.bits, a.words, a.alpha, a.G, a.ldg, a.N, a.K, a.F, a.partial, 0};
+    if (a.F <= 64) return launch_sign_t<64>(p, max_split, dev, stream);
+    if (a.F <= 128) return launch_sign_t<128>(p, max_split, dev, stream);
+    return launch_sign_t<256>(p, max_split, dev, stream);
 }
 
 uint32_t take_mix_timeouts() {

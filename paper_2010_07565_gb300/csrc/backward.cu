@@ -17,9 +17,9 @@
 // real operand G (times beta_j, applied as its centring scale and rounded
 // once) split into three bf16 parts, the signs of W's rows (W packed row by
 // row over its F columns) exact in bf16, fp32 accumulators, and the clip of
-// Eq. bp-H in the epilogue. dW~ runs on the CUDA cores in fp32: 64 x 64
-// output tiles, each thread a 4 x 4 register block that adds +-v for the
-// signs of one packed word.
+// Eq. bp-H in the epilogue. dW~ runs on the tensor cores too
+// (sign_t_real_tc_kernel in ablation.cu): the node signs gathered
+// feature-major from the packed rows, alpha_i G_ij as three bf16 parts.
 //
 // dW~ sums over all N rows: the rows are split into S chunks (grid z) whose
 // partial sums are added, chunk by chunk in order, by a second kernel, so
@@ -31,65 +31,10 @@ namespace {
 
 constexpr int kBwThreads = 256;
 constexpr int kTile = 64;        // output tile edge
-constexpr int kRowsPerStage = 32;
 
 // +1.0f where bit b of w is set, else -1.0f.
 __device__ __forceinline__ float pm1(uint64_t w, int b) {
     return ((w >> b) & 1ull) ? 1.0f : -1.0f;
-}
-
-// Partial dW~ over the rows [chunk start, chunk end): tile (kt, jt) of the
-// K x F output, thread (tk, tj) owning k = 64 kt + 4 tk + 0..3 and
-// j = 64 jt + 4 tj + 0..3.
-__global__ void __launch_bounds__(kBwThreads)
-grad_wtilde_kernel(const uint64_t *__restrict__ bits, int words, const float *__restrict__ alpha,
-                   const float *__restrict__ G, int64_t ldg, int64_t N, int K, int F,
-                   int64_t chunk, float *__restrict__ partial) {
-    __shared__ __align__(16) float sV[kRowsPerStage][kTile];    // alpha_i G[i, j-tile]
-    __shared__ uint64_t sB[kRowsPerStage];                      // row i's word of the k-tile
-    const int tid = threadIdx.x, tk = tid / 16, tj = tid % 16;
-    const int kt = blockIdx.x, jt = blockIdx.y;
-    const int64_t r0 = int64_t(blockIdx.z) * chunk;
-    const int64_t r1 = r0 + chunk < N ? r0 + chunk : N;
-    float acc[4][4] = {};
-    for (int64_t base = r0; base < r1; base += kRowsPerStage) {
-        __syncthreads();
-        for (int q = tid; q < kRowsPerStage * kTile; q += kBwThreads) {
-            const int r = q / kTile, c = q % kTile;
-            const int64_t i = base + r;
-            const int j = jt * kTile + c;
-            sV[r][c] = (i < r1 && j < F) ? __ldg(alpha + i) * __ldg(G + i * ldg + j) : 0.0f;
-        }
-        for (int r = tid; r < kRowsPerStage; r += kBwThreads) {
-            const int64_t i = base + r;
-            sB[r] = i < r1 ? __ldg(bits + i * words + kt) : 0ull;
-        }
-        __syncthreads();
-        const int n = int(r1 - base < kRowsPerStage ? r1 - base : kRowsPerStage);
-        for (int r = 0; r < n; ++r) {
-            const uint64_t w = sB[r];
-            const float4 v = *reinterpret_cast<const float4 *>(&sV[r][4 * tj]);
-#pragma unroll
-            for (int a = 0; a < 4; ++a) {
-                const float s = pm1(w, 4 * tk + a);
-                acc[a][0] = fmaf(s, v.x, acc[a][0]);
-                acc[a][1] = fmaf(s, v.y, acc[a][1]);
-                acc[a][2] = fmaf(s, v.z, acc[a][2]);
-                acc[a][3] = fmaf(s, v.w, acc[a][3]);
-            }
-        }
-    }
-    float *out = partial + int64_t(blockIdx.z) * K * F;
-#pragma unroll
-    for (int a = 0; a < 4; ++a) {
-        const int k = kt * kTile + 4 * tk + a;
-        if (k >= K) continue;
-#pragma unroll
-        for (int b = 0; b < 4; ++b) {
-            const int j = jt * kTile + 4 * tj + b;
-            if (j < F) out[int64_t(k) * F + j] = acc[a][b];
-        }
-    }
 }
 
 // dW~ = the S partial sums added in chunk order.
@@ -156,16 +101,6 @@ int64_t max_chunks(int K, int F) {
     const int64_t tiles = int64_t((K + kTile - 1) / kTile) * ((F + kTile - 1) / kTile);
     const int64_t s = (512 + tiles - 1) / tiles;
     return s < 64 ? s : 64;
-}
-
-// Row chunks of the dW~ reduction: about two blocks per SM in all.
-int wtilde_chunks(int64_t N, int K, int F, const DeviceInfo &dev) {
-    const int64_t tiles = int64_t((K + kTile - 1) / kTile) * ((F + kTile - 1) / kTile);
-    int64_t S = (2 * int64_t(dev.sm_count) + tiles - 1) / tiles;
-    const int64_t max_s = (N + kRowsPerStage - 1) / kRowsPerStage;
-    if (S > max_s) S = max_s;
-    if (S > max_chunks(K, F)) S = max_chunks(K, F);
-    return int(S < 1 ? 1 : S);
 }
 
 struct BackwardWorkspace {
@@ -265,10 +200,9 @@ extern "C" bigcn_status bigcn_layer_backward(
     launch_pack_weights(Wt, K, F, ldw, wbits, words, beta, s);
     SpmmArgs a{rowptr, colidx, N, nnz, dH, ldg, F, G, F, false, false};
     launch_spmm_norm(a, dev, s);                                   // G = A~ dH
-    const int S = wtilde_chunks(N, K, F, dev);
-    const int64_t chunk = (N + S - 1) / S;
-    const dim3 gw(unsigned((K + kTile - 1) / kTile), unsigned((F + kTile - 1) / kTile), unsigned(S));
-    grad_wtilde_kernel<<<gw, kBwThreads, 0, s>>>(bits, words, alpha, G, F, N, K, F, chunk, partial);
+    // dL/dW~ = H~^T G on the tensor cores, in node chunks added in order.
+    SignTRealArgs gw{bits, words, alpha, G, F, N, K, F, partial};
+    const int S = launch_sign_t_real_gemm(gw, int(max_chunks(K, F)), dev, s);
     const int64_t kf = int64_t(K) * F;
     sum_partials_kernel<<<unsigned((kf + kBwThreads - 1) / kBwThreads < 4096
                                        ? (kf + kBwThreads - 1) / kBwThreads : 4096),

@@ -220,6 +220,23 @@ struct BinaryRealArgs {      // features binarized: Z = H~ W
 void launch_binary_real_gemm(const BinaryRealArgs &args, const DeviceInfo &dev,
                              cudaStream_t stream, bool pdl = false);
 
+// Transposed signs x real (ablation.cu): partial[s] = sum over the nodes of
+// chunk s of alpha_i sign(y_ik) G_ij (K x F each; dL/dW~ = H~^T G is their
+// sum in order). Returns the number of chunks written (<= max_split).
+struct SignTRealArgs {
+    const uint64_t *bits;    // N x words packed node signs (K features)
+    int words;
+    const float *alpha;      // N
+    const float *G;          // N x F (row stride ldg)
+    int64_t ldg;
+    int64_t N;
+    int K;
+    int F;
+    float *partial;          // max_split x K x F
+};
+int launch_sign_t_real_gemm(const SignTRealArgs &args, int max_split, const DeviceInfo &dev,
+                            cudaStream_t stream);
+
 // Bytes of the bf16 parts of a K x F weight matrix, and the kernel that
 // writes them (parts[p][j][k], zero for k >= K up to bigcn_words(K) * 64).
 size_t weight_parts_bytes(int K, int F);
