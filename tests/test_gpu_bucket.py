@@ -2,7 +2,9 @@
 with their own scales) against the oracle, through the C ABI: packed signs
 bit-exact, per-bucket scales and products within |g - o| <= 1e-6 + 1e-4 *
 max(|o|, scale) (scale = the sum of the |terms|, the products being sums of
-per-bucket terms with both signs), the plain form required of all but 0.1 %.
+per-bucket terms with both signs); the plain form is required wherever
+1e-4 |o| exceeds sqrt(n) 2^-24 scale, the typical rounding error of an fp32
+sum of n terms.
 Buckets from one word (64) to more than K (one bucket: Bi-GCN), K and F
 ragged, a last bucket shorter than B, few tiles (the k-steps split over a
 cluster) and many, extra words in the packed rows.
@@ -24,7 +26,7 @@ def rng(seed):
     return np.random.Generator(np.random.PCG64(seed))
 
 
-def check(gpu, ref, scale, what, plain_misses_allowed=0.001):
+def check(gpu, ref, scale, what, nterms):
     gpu = np.asarray(gpu, np.float64)
     err = np.abs(gpu - ref)
     bound = ATOL + RTOL * np.maximum(np.abs(ref), scale)
@@ -33,8 +35,13 @@ def check(gpu, ref, scale, what, plain_misses_allowed=0.001):
         q = np.unravel_index(np.argmax(err - bound), err.shape)
         raise AssertionError(f"{what}: {int(bad.sum())} of {bad.size} out of tolerance; worst "
                              f"at {q}: gpu={gpu[q]!r} oracle={ref[q]!r} scale={scale[q]!r}")
+    # The |o|-relative form is required wherever RTOL |o| exceeds the typical
+    # rounding error of an fp32 sum of `nterms` terms, sqrt(nterms) 2^-24 scale;
+    # below that the terms have cancelled to under what fp32 resolves.
     plain = err > ATOL + RTOL * np.abs(ref)
-    assert plain.mean() <= plain_misses_allowed, f"{what}: {plain.mean():.2%} miss |o|-relative"
+    resolved = RTOL * np.abs(ref) > np.sqrt(nterms) * 2.0 ** -24 * scale
+    stray = plain & resolved
+    assert not stray.any(), f"{what}: {int(stray.sum())} |o|-relative misses outside cancellation"
 
 
 PACK_CASES = [(1, 1, 64), (37, 63, 64), (20, 64, 64), (19, 65, 64), (300, 200, 128),
@@ -93,7 +100,7 @@ def test_xnor_gemm_bucketed(cuda_device, N, K, F, B):
     B_.bigcn_xnor_gemm_bucketed(to_dev(oracle.pack(SF)), to_dev(alpha), to_dev(oracle.pack(SB)),
                                 to_dev(beta), K, B, Z)
     torch.cuda.synchronize()
-    check(Z.cpu().numpy(), ref, mag, f"bucketed product {N}x{K}x{F}, B={B}")
+    check(Z.cpu().numpy(), ref, mag, f"bucketed product {N}x{K}x{F}, B={B}", nterms=K)
 
 
 LAYER_CASES = [(300, 70, 6, 64, 4.0, 0), (2708, 1433, 64, 256, 4.0, 0),
@@ -114,11 +121,12 @@ def test_layer_forward_bucketed(cuda_device, N, K, F, B, deg, hub):
     torch.cuda.synchronize()
     ref = oracle.layer_forward_bucketed(case["X"], case["W"], case["rowptr"], case["colidx"], B,
                                         case["s"], case["t"])
-    check(H.cpu().numpy(), ref["H"], ref["scale"], f"bucketed layer B={B}")
+    nt = K + int(np.diff(case["rowptr"]).max(initial=0)) + 1
+    check(H.cpu().numpy(), ref["H"], ref["scale"], f"bucketed layer B={B}", nterms=nt)
     if B >= K:       # one bucket: Bi-GCN's layer
         bi = oracle.layer_forward(case["X"], case["W"], case["rowptr"], case["colidx"],
                                   case["s"], case["t"])
-        check(H.cpu().numpy(), bi["H"], ref["scale"], "one bucket = Bi-GCN")
+        check(H.cpu().numpy(), bi["H"], ref["scale"], "one bucket = Bi-GCN", nterms=nt)
 
 
 def test_bucketed_argument_errors(cuda_device):

@@ -5,7 +5,8 @@ aggregator) against the oracle, through the C ABI.
 The products are exact integers scaled by fp32 alpha and beta; the
 aggregation's fp32 sums are compared with |gpu - oracle| <= 1e-6 + 1e-4 *
 max(|oracle|, scale), scale = the sum of the |terms| of the aggregation, the
-plain |oracle|-relative form required of all but 0.1 % of the entries.
+plain |oracle|-relative form required wherever 1e-4 |oracle| exceeds
+sqrt(n) 2^-24 scale, the typical rounding error of an fp32 sum of n terms.
 Graphs: isolated nodes (GraphSAGE's mean is then 0), a hub heavy enough for
 the whole-block path, mean degree past 8 (eight dots per lane), no edges; K
 past 32767 (the product kept in fp32 instead of 16-bit dots); F not a
@@ -24,7 +25,7 @@ pytestmark = pytest.mark.gpu
 RTOL, ATOL = 1e-4, 1e-6
 
 
-def check(gpu, ref, scale, what, plain_misses_allowed=0.001):
+def check(gpu, ref, scale, what, nterms):
     gpu = np.asarray(gpu, np.float64)
     err = np.abs(gpu - ref)
     bound = ATOL + RTOL * np.maximum(np.abs(ref), scale)
@@ -33,9 +34,18 @@ def check(gpu, ref, scale, what, plain_misses_allowed=0.001):
         q = np.unravel_index(np.argmax(err - bound), err.shape)
         raise AssertionError(f"{what}: {int(bad.sum())} of {bad.size} out of tolerance; worst "
                              f"at {q}: gpu={gpu[q]!r} oracle={ref[q]!r} scale={scale[q]!r}")
+    # The |o|-relative form is required wherever RTOL |o| exceeds the typical
+    # rounding error of an fp32 sum of `nterms` terms, sqrt(nterms) 2^-24 scale;
+    # below that the terms have cancelled to under what fp32 resolves.
     plain = err > ATOL + RTOL * np.abs(ref)
-    assert plain.mean() <= plain_misses_allowed, f"{what}: {plain.mean():.2%} miss |o|-relative"
+    resolved = RTOL * np.abs(ref) > np.sqrt(nterms) * 2.0 ** -24 * scale
+    stray = plain & resolved
+    assert not stray.any(), f"{what}: {int(stray.sum())} |o|-relative misses outside cancellation"
     assert np.isfinite(gpu).all()
+
+
+def maxdeg(case):
+    return int(np.diff(case["rowptr"]).max(initial=0)) + 1
 
 
 def run(agg, case, Wn=None, ldh=None, dev=None):
@@ -75,7 +85,7 @@ def test_inductive_layer_matches_oracle(cuda_device, agg, N, K, F, deg, hub):
     H, _ = run(agg, case, Wn, dev=cuda_device)
     ref = oracle.layer_forward_inductive(case["X"], case["W"], case["rowptr"], case["colidx"],
                                          agg, case["s"], case["t"], W_neigh=Wn)
-    check(H, ref["H"], ref["absterm"], f"{agg} layer {N}x{K}x{F}")
+    check(H, ref["H"], ref["absterm"], f"{agg} layer {N}x{K}x{F}", nterms=K + maxdeg(case))
     assert B.device_timeouts() == 0
 
 
@@ -87,7 +97,7 @@ def test_inductive_layer_past_the_16_bit_dots(cuda_device, agg):
     H, _ = run(agg, case, Wn, dev=cuda_device)
     ref = oracle.layer_forward_inductive(case["X"], case["W"], case["rowptr"], case["colidx"],
                                          agg, case["s"], case["t"], W_neigh=Wn)
-    check(H, ref["H"], ref["absterm"], f"{agg} layer, K = {K}")
+    check(H, ref["H"], ref["absterm"], f"{agg} layer, K = {K}", nterms=K + maxdeg(case))
 
 
 def test_inductive_layer_padded_output_and_gcn_mode(cuda_device):
@@ -98,7 +108,7 @@ def test_inductive_layer_padded_output_and_gcn_mode(cuda_device):
     assert torch.all(buf[:, F:] == -3.0)
     ref = oracle.layer_forward_inductive(case["X"], case["W"], case["rowptr"], case["colidx"],
                                          "sage", case["s"], case["t"], W_neigh=Wn)
-    check(H, ref["H"], ref["absterm"], "sage layer, padded H")
+    check(H, ref["H"], ref["absterm"], "sage layer, padded H", nterms=K + maxdeg(case))
     # The "gcn" aggregator is bigcn_layer_forward.
     d = {k: to_dev(v) for k, v in case.items()}
     ws = torch.empty(B.bigcn_inductive_layer_workspace_bytes("gcn", N, K, F), dtype=torch.uint8,
