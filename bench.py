@@ -610,11 +610,13 @@ def run_backward(args, rank, world, local_rank):
         return 0
     peaks, peak_kind = load_peaks()
     mean_ms = max_ms / args.steps
-    # The two +-1 x fp32 products dominate: N K F fused multiply-adds each,
-    # on the CUDA cores. fp32 FMA peak from the unit counts: 152 SMs x 128
-    # lanes x 2 flops x 2070 MHz.
+    # The two +-1 x fp32 products (dL/dW~ and dL/dH~, N K F multiply-adds each)
+    # run on the tensor cores, fp32-accurate through three bf16 parts: their
+    # ceiling is the measured bf16 peak / 3. The rate is taken over the whole
+    # step (pack, aggregation, products, sums), so it is a lower bound.
     flops = 2.0 * 2.0 * N * K * F
-    fma_peak = 152 * 128 * 2 * 2.070e9 / 1e12
+    tc_peak = float(peaks.get("bf16_tflops", 1900.0)) / 3.0
+    achieved = flops / (mean_ms * 1e-3) / 1e12
     line = {
         "metric": "Bi-GCN layer backward nodes/s (Algorithm 1, Eqs. bp-H, bp-W)",
         "value": units / (max_ms * 1e-3), "unit": "nodes/s", "n_gpus": world,
@@ -624,13 +626,14 @@ def run_backward(args, rank, world, local_rank):
         "config": {"workload": w.description + " -- layer 1 backward", "name": w.name, "N": N,
                    "K": K, "F": F, "nnz": int(data["colidx"].shape[0]),
                    "l2": "flushed before every step outside the timed events",
-                   "launch": "bigcn_layer_backward (7 kernels)"},
-        "roofline": {"kernel": "whole backward", "bound": "alu",
-                     "achieved": flops / (mean_ms * 1e-3) / 1e12,
-                     "peak": fma_peak, "unit": "TFLOP/s (fp32 FMA, the two +-1 x fp32 products)",
-                     "frac": flops / (mean_ms * 1e-3) / 1e12 / fma_peak, "traffic": None,
-                     "peak_source": "derived: 152 SMs x 128 FMA/clk x 2 x 2070 MHz"},
-        "cpu_baseline": None, "e2e": None, "gpu_launches": 7 * args.steps,
+                   "launch": "bigcn_layer_backward (9 kernels)"},
+        "roofline": {"kernel": "whole backward step (the two products' flops over the step's "
+                               "time)", "bound": "tensor", "achieved": achieved,
+                     "peak": tc_peak,
+                     "unit": "TFLOP/s (2 N K F per product; fp32-accurate = 3 bf16 MMAs)",
+                     "frac": achieved / tc_peak, "traffic": None,
+                     "peak_source": f"{peak_kind} MEASURED_PEAKS.json bf16_tflops / 3"},
+        "cpu_baseline": None, "e2e": None, "gpu_launches": 9 * args.steps,
         "clocks": clocks.summary(),
     }
     print(json.dumps(line), flush=True)
