@@ -1,7 +1,6 @@
-// Shared-memory mbarriers and 1-D bulk async copies (the TMA's untiled
-// form), as inline PTX for sm_103a. Every wait is bounded: it gives up after
-// kWaitLimit polls and reports false, so that a kernel can record the failure
-// and return instead of hanging.
+// Shared-memory mbarriers as inline PTX for sm_103a. Every wait is bounded:
+// it gives up after kWaitLimit polls and reports false, so that a kernel can
+// record the failure and return instead of hanging.
 #pragma once
 
 #include <cstdint>
@@ -44,23 +43,6 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
 // One arrival (release semantics for this thread's earlier accesses).
 __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
-
-// One arrival that also raises the phase's expected transaction bytes.
-__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
-                 : "memory");
-}
-
-// Copies `bytes` (a multiple of 16) from global `src` (16-byte aligned) to
-// shared `dst` (16-byte aligned); completion is counted on mbarrier `bar`.
-__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t bytes,
-                                         uint32_t bar) {
-    asm volatile(
-        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::
-            "r"(dst),
-        "l"(src), "r"(bytes), "r"(bar)
-        : "memory");
 }
 
 }  // namespace bigcn

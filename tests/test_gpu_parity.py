@@ -317,11 +317,11 @@ def test_forward_2layer_matches_oracle(cuda_device, N, K, Fh, Fo, deg, hub):
     assert torch.equal(out, out2)
 
 
-# The layer-1 front streams whole rows of X into shared memory with bulk
-# copies of each row's 16-byte-aligned interior; these cases move the row
-# starts off that alignment (odd row strides, a base 4 bytes past a 16-byte
-# boundary), make rows too short to have an interior, and give every CTA
-# many more rows than its ring has stages.
+# Rows of X whose starts sit off every vector alignment (odd row strides, a
+# base 4 or 12 bytes past a 16-byte boundary), rows shorter than one 32-wide
+# chunk or than 16 bytes, Citeseer-shaped rows on the split front (several
+# warps per row), more row groups than resident CTAs, and rows too long for the fused front (80 KB:
+# packing and product as separate kernels).
 @pytest.mark.parametrize("N,K,ldx,offset,Fh,centred", [
     (333, 1, 1, 0, 8, True),          # one feature: no interior at all
     (333, 3, 5, 1, 8, False),         # rows shorter than 16 bytes, odd stride
