@@ -320,16 +320,16 @@ def test_forward_2layer_matches_oracle(cuda_device, N, K, Fh, Fo, deg, hub):
 # Rows of X whose starts sit off every vector alignment (odd row strides, a
 # base 4 or 12 bytes past a 16-byte boundary), rows shorter than one 32-wide
 # chunk or than 16 bytes, Citeseer-shaped rows on the split front (several
-# warps per row), more row groups than resident CTAs, and rows too long for the fused front (80 KB:
-# packing and product as separate kernels).
+# warps per row), more row groups than resident CTAs, and rows too long for
+# the fused front (80 KB: packing and product as separate kernels).
 @pytest.mark.parametrize("N,K,ldx,offset,Fh,centred", [
-    (333, 1, 1, 0, 8, True),          # one feature: no interior at all
+    (333, 1, 1, 0, 8, True),          # one feature per row
     (333, 3, 5, 1, 8, False),         # rows shorter than 16 bytes, odd stride
-    (200, 9, 9, 1, 33, True),         # interior of at most one 16-byte unit
+    (200, 9, 9, 1, 33, True),         # one partial chunk, 33 hidden columns
     (700, 3703, 3703, 0, 64, True),   # Citeseer-shaped rows (stride 14812 bytes)
     (700, 3703, 3705, 3, 64, True),   # same rows, odd stride, base 12 bytes past
-    (5000, 1433, 1437, 1, 16, True),  # many rows per CTA: the stage ring wraps
-    (64, 20000, 20001, 1, 128, True), # rows of 80 KB: two stages
+    (5000, 1433, 1437, 1, 16, True),  # more row groups than resident CTAs
+    (64, 20000, 20001, 1, 128, True), # rows of 80 KB: packing, then the product
 ])
 def test_forward_2layer_front_unaligned_rows(cuda_device, N, K, ldx, offset, Fh, centred):
     Fo = 5
