@@ -175,9 +175,11 @@ int front_rows(int64_t N, const DeviceInfo &dev) {
 // after the block's first rows have been streamed.
 
 // Shared memory: F x pitch packed columns, 16 x pitch packed rows, and the
-// centring affine as K (scale, shift) pairs.
+// centring affine as K (scale, shift) pairs; at most kSplitMaxSmem, so that
+// two blocks (with the 1 KB each that the SM reserves) share an SM's 228 KB.
 constexpr int kSplitThreads = 512;
 constexpr int kSplitWarps = kSplitThreads / 32;
+constexpr size_t kSplitMaxSmem = 112 * 1024;
 
 size_t split_smem(int F, int K, int words, bool affine) {
     return (size_t(F) + size_t(kSplitWarps)) * size_t(words | 1) * 8 +
@@ -294,7 +296,8 @@ front_split_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
 
 bool split_supported(int64_t N, int K, int F, const DeviceInfo &dev) {
     return F >= 1 && F <= 128 && split_warps(N, K, dev) > 1 &&
-           split_smem(F, K, (K + 63) / 64, true) <= kFrontMaxSmem / 2;
+           split_smem(F, K, (K + 63) / 64, true) <= kSplitMaxSmem &&
+           split_smem(F, K, (K + 63) / 64, true) <= size_t(dev.max_smem_optin);
 }
 
 void launch_split(const FrontArgs &a, const DeviceInfo &dev, cudaStream_t s, bool pdl) {

@@ -70,6 +70,7 @@ CASES = [
     (300, 70, 6, 4.0, 0),
     (400, 90, 13, 1.0, 0),           # many isolated nodes
     (2708, 1433, 64, 4.0, 0),        # Cora-shaped layer 1
+    (3327, 3703, 64, 2.8, 0),        # Citeseer-shaped: GraphSAGE on the split front
     (5000, 300, 33, 6.0, 900),       # a hub on the whole-block path
     (3000, 200, 128, 12.0, 0),       # mean degree past 8: eight dots per lane
     (50, 20, 5, 0.0, 0),             # no edges
