@@ -1,0 +1,72 @@
+"""bench.py's command-line contract, checked on the CPU: the reference arm
+(the oracle timed on the host cores) prints one JSON line with the keys the
+benchmark contract names, prints it once under a two-rank launch, the
+warm-up rule is enforced, and the CUDA arm fails loudly instead of falling
+back to the CPU when no GPU is present."""
+import json
+import os
+import socket
+import subprocess
+import sys
+
+import pytest
+import torch
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+BENCH = os.path.join(ROOT, "bench.py")
+
+
+def run(args, timeout=300):
+    return subprocess.run([sys.executable, *args], cwd=ROOT, capture_output=True, text=True,
+                          timeout=timeout)
+
+
+def json_lines(stdout):
+    return [json.loads(l) for l in stdout.splitlines() if l.startswith("{")]
+
+
+def free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def test_reference_arm_prints_the_contract_line():
+    r = run([BENCH, "--impl", "reference", "--steps", "1", "--warmup", "3"])
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = json_lines(r.stdout)
+    assert len(lines) == 1
+    d = lines[0]
+    assert d["impl"] == "reference"
+    assert d["unit"] == "nodes/s" and d["value"] > 0 and d["higher_is_better"] is True
+    assert d["n_gpus"] == 1 and d["steps"] == 1 and d["warmup"] == 3
+    assert d["ms_per_step"] > 0 and d["data"] == "synthetic"
+    assert isinstance(d["config"]["workload"], str) and d["config"]["workload"]
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"]
+    assert cb["unit"] == d["unit"] and cb["sample"]
+    e2e = d["e2e"]
+    assert e2e["value"] == d["value"] and e2e["unit"] == d["unit"]
+    assert e2e["h2d_bytes_per_step"] == 0 and e2e["d2h_bytes_per_step"] == 0
+
+
+def test_reference_arm_under_two_ranks_prints_once():
+    r = run(["-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node", "2",
+             "--master-addr", "127.0.0.1", "--master-port", str(free_port()), BENCH,
+             "--impl", "reference", "--gpus", "2", "--steps", "1", "--warmup", "3"])
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = json_lines(r.stdout)
+    assert len(lines) == 1 and lines[0]["impl"] == "reference" and lines[0]["n_gpus"] == 2
+
+
+def test_fewer_than_three_warmup_steps_are_refused():
+    r = run([BENCH, "--impl", "reference", "--steps", "1", "--warmup", "2"])
+    assert r.returncode != 0 and "warmup" in r.stderr
+    assert not json_lines(r.stdout)
+
+
+@pytest.mark.skipif(torch.cuda.is_available(), reason="checks the behaviour without a GPU")
+def test_cuda_arm_fails_without_a_gpu():
+    r = run([BENCH, "--steps", "1", "--warmup", "3"])
+    assert r.returncode != 0
+    assert not json_lines(r.stdout)
