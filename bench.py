@@ -9,12 +9,13 @@ call (5 kernels for the usual widths), replayed as a CUDA graph with timing
 events around it. Per-kernel durations come from a second pass of the same
 forward with an event between kernels.
 
-Default workload: C2 (the Citeseer-shaped 2-layer configuration: N=3327,
-K=3703, hidden 64, out 6). Its inputs (49 MB) fit in L2, so L2 is flushed
-before every step, outside the timed events: a 256 MiB buffer is written and
-its first half read back, which leaves L2 holding clean lines of that buffer
-(the inputs come from HBM, and the step does not pay for writing back the
-flush's dirty lines).
+Default workload: C4 (the Reddit-shaped 2-layer configuration: N=232965,
+K=602, hidden 128, out 41, 114.6M CSR entries), the largest configuration
+that runs as a 2-layer forward on one GPU. Smaller workloads (C1..C3) fit in
+L2, so L2 is flushed before every step, outside the timed events: a 256 MiB
+buffer is written and its first half read back, which leaves L2 holding clean
+lines of that buffer (the inputs come from HBM, and the step does not pay for
+writing back the flush's dirty lines).
 
 Prints one JSON line (rank 0): nodes/s of the device-resident forward, the
 same through host buffers (e2e), per-kernel times and the dominant kernel's
@@ -45,9 +46,12 @@ if ROOT not in sys.path:
 import numpy as np  # noqa: E402
 
 METRIC = "Bi-GCN layer fwd nodes/s; XNOR-GEMM bit-ops/s; SpMM GB/s as % of GB300 peak"
-DEFAULT_WORKLOAD = "C2"
+DEFAULT_WORKLOAD = "C4"
 L2_FLUSH_BYTES = 256 << 20
-POPC_PER_CLK_PER_SM = 16          # 32-bit population counts per clock per SM
+# 32-bit population counts per clock per SM, as measured on GB300 by
+# tests/probes/instruction_rates.cu (profiles/xnor_gemm_instruction_rates.txt:
+# 151.8 T bit-ops/s over 152 SMs at 2070 MHz); the ALU ceiling of the POPC products.
+POPC_PER_CLK_PER_SM = 15.1
 FALLBACK_HBM_GBS = 6800.0
 
 
@@ -167,13 +171,16 @@ def profiled_traffic(name, workload):
 
 
 class ClockSampler:
-    """nvidia-smi clock / throttle samples every 200 ms while running."""
+    """nvidia-smi clock / throttle samples every ``interval_ms`` while running
+    (the bench opens it before the warm-up steps, so that short timed regions
+    still see samples under load)."""
     QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
-    def __init__(self, gpu_index: int):
+    def __init__(self, gpu_index: int, interval_ms: int = 100):
         self.gpu = gpu_index
+        self.interval = interval_ms
         self.proc = None
         self.out = None
 
@@ -182,7 +189,7 @@ class ClockSampler:
             self.out = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.QUERY}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", str(self.interval)],
                 stdout=self.out, stderr=subprocess.DEVNULL)
         except (OSError, FileNotFoundError):
             self.proc = None
@@ -223,6 +230,20 @@ def build_workload(name):
     W1, W2 = inputs.layer_weights(w)
     rowptr, colidx = inputs.graph(w)
     return w, dict(X=X, s=s, t=t, W1=W1, W2=W2, rowptr=rowptr, colidx=colidx)
+
+
+def oracle_block_nodes(w, data, budget_s):
+    """Nodes of a block whose induced subgraph the CPU oracle's 2-layer
+    forward finishes in about a third of ``budget_s`` (calibrated on a
+    256-node block; the whole graph if that is smaller)."""
+    import oracle
+    cal = min(w.N, 256)
+    rp, ci = induced_subgraph(data["rowptr"], data["colidx"], 0, cal)
+    t0 = time.perf_counter()
+    oracle.forward_2layer(np.ascontiguousarray(data["X"][:cal]), data["s"], data["t"],
+                          data["W1"], data["W2"], rp, ci)
+    per_node = max((time.perf_counter() - t0) / cal, 1e-9)
+    return int(max(cal, min(w.N, budget_s / 3.0 / per_node)))
 
 
 def time_oracle(w, data, budget_s, rows=None):
@@ -282,7 +303,7 @@ def run_reference(args, rank, world):
             "scaling": "weak", "vs_baseline": None, "dtype": "f32+b1", "data": "synthetic",
             "config": {"workload": w.description, "name": w.name, "nodes_per_step": n},
             "cpu_baseline": {"value": value, "unit": "nodes/s", "cores": 1, "kind": "oracle",
-                             "sample": sample},
+                             "sample": sample, "host_cores": os.cpu_count()},
             "e2e": {"value": value, "unit": "nodes/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -324,16 +345,17 @@ def run_gpu(args, rank, world, local_rank):
         flush_half.sum()
 
     ea, eb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    for _ in range(args.warmup):
-        flush_l2()
-        model.replay()
-    torch.cuda.synchronize()
-    if world > 1:
-        dist.barrier()
-    torch.cuda.synchronize()
-
     step_ms = []
+    # Clocks are sampled from the warm-up on: a short timed region alone may
+    # see no sample.
     with ClockSampler(local_rank) as clocks:
+        for _ in range(args.warmup):
+            flush_l2()
+            model.replay()
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
         for _ in range(args.steps):
             flush_l2()
             ea.record()
@@ -412,9 +434,11 @@ def run_gpu(args, rank, world, local_rank):
 
     cpu_baseline = None
     if world == 1 and not args.no_cpu_baseline:
-        v, sample = time_oracle(w, data, budget_s=args.cpu_seconds)
+        rows = oracle_block_nodes(w, data, args.cpu_seconds)
+        v, sample = time_oracle(w, data, budget_s=args.cpu_seconds, rows=rows)
         cpu_baseline = {"value": v, "unit": "nodes/s", "cores": 1, "kind": "oracle",
-                        "sample": sample}
+                        "sample": sample, "host_cores": os.cpu_count(),
+                        "note": "the oracle is single-threaded: 1 of the host's cores"}
 
     dims = [w.K, w.hidden, w.out]
     line = {
@@ -922,7 +946,10 @@ def run_bucketed(args, rank, world, local_rank):
         return 0
     prod_s = statistics.fmean(prod_ms) * 1e-3
     bitops = float(N) * K * F
-    peak = POPC_PER_CLK_PER_SM * 32 * 152 * 2.070e9 / 1e12
+    peaks, _ = load_peaks()
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    sm_max = float(peaks.get("sm_max_mhz", 2070.0))
+    peak = POPC_PER_CLK_PER_SM * 32 * sms * sm_max * 1e6 / 1e12
     achieved = bitops / prod_s / 1e12
     line = {
         "metric": f"Bi-GCN bucketed layer fwd nodes/s (buckets of {Bk} features)",
@@ -940,7 +967,8 @@ def run_bucketed(args, rank, world, local_rank):
         "roofline": {"kernel": "bucketed product", "bound": "alu", "achieved": achieved,
                      "peak": peak, "unit": "T bit-ops/s (N K F)", "frac": achieved / peak,
                      "traffic": None,
-                     "peak_source": "derived: 16 POPC/clk/SM x 32 bits x 152 SMs x 2070 MHz"},
+                     "peak_source": f"measured {POPC_PER_CLK_PER_SM} POPC/clk/SM x 32 bits x "
+                                    f"{sms} SMs x {sm_max:.0f} MHz"},
         "cpu_baseline": None, "e2e": None, "gpu_launches": 4 * args.steps,
         "clocks": clocks.summary(),
     }
@@ -972,7 +1000,7 @@ def main(argv=None):
     ap.add_argument("--impl", choices=["bigcn", "reference"], default="bigcn")
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD,
                     help="C1..C4, or a one-layer sweep point such as C5_K4096_F256")
-    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--backward", action="store_true",
                     help="time layer 1's back-propagation (bigcn_layer_backward) instead")

@@ -199,6 +199,11 @@ size_t bigcn_layer_workspace_bytes(int64_t N, int32_t K, int32_t F);
  *            bytes, 256-byte aligned, not overlapping any argument; its
  *            contents on entry do not matter and on exit are unspecified.
  * H must not overlap the workspace; it may not be X either.
+ * The tensor-core product (many rows) waits on shared-memory barriers a
+ * bounded number of times: a tile whose wait runs out leaves its part of the
+ * product, and so of H, unwritten while the call still returns BIGCN_OK
+ * (the call is asynchronous). bigcn_device_timeouts() reports such waits;
+ * callers that must know call it after the layer (it synchronizes).
  */
 bigcn_status bigcn_layer_forward(const float *X, int64_t N, int32_t K, int64_t ldx,
                                  const float *scale, const float *shift,
@@ -479,8 +484,14 @@ bigcn_status bigcn_layer_backward(const float *X, int64_t N, int32_t K, int64_t 
  * Arguments, results and errors are those of bigcn_layer_forward minus
  * `workspace` and `ws_bytes`, plus: when bigcn_layer_workspace_bytes(N, K, F)
  * exceeds BIGCN_STATIC_SCRATCH_BYTES the call returns
- * BIGCN_ERR_SCRATCH_LIMIT and enqueues nothing. (Roughly: N * (K/8 + 4F)
- * bytes must fit, e.g. 90,000 nodes with K = 602 and F = 64.)
+ * BIGCN_ERR_SCRATCH_LIMIT and enqueues nothing. The exact test is
+ * bigcn_layer_workspace_bytes(N, K, F) <= BIGCN_STATIC_SCRATCH_BYTES. Per
+ * node that is 8*ceil(K/64) + 2*round_up(F, 8) + 8 bytes when K <= 32767
+ * (the dots kept as 16-bit integers) and 8*ceil(K/64) + 4*F + 4 bytes above,
+ * plus the packed weights: about 155,000 nodes fit with K = 602 and F = 64.
+ * As in bigcn_layer_forward, a bounded device wait that runs out leaves
+ * part of H unwritten while the call returns BIGCN_OK; bigcn_device_timeouts()
+ * (which synchronizes) reports it.
  *
  * The first call on a device, with that device current, looks up the array's
  * device address (cudaGetSymbolAddress) and caches it for the device; make

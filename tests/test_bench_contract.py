@@ -32,7 +32,7 @@ def free_port():
 
 
 def test_reference_arm_prints_the_contract_line():
-    r = run([BENCH, "--impl", "reference", "--steps", "1", "--warmup", "3"])
+    r = run([BENCH, "--impl", "reference", "--workload", "C1", "--steps", "1", "--warmup", "3"])
     assert r.returncode == 0, r.stderr[-2000:]
     lines = json_lines(r.stdout)
     assert len(lines) == 1
@@ -45,6 +45,7 @@ def test_reference_arm_prints_the_contract_line():
     cb = d["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"]
     assert cb["unit"] == d["unit"] and cb["sample"]
+    assert cb["host_cores"] == os.cpu_count()
     e2e = d["e2e"]
     assert e2e["value"] == d["value"] and e2e["unit"] == d["unit"]
     assert e2e["h2d_bytes_per_step"] == 0 and e2e["d2h_bytes_per_step"] == 0
@@ -53,20 +54,21 @@ def test_reference_arm_prints_the_contract_line():
 def test_reference_arm_under_two_ranks_prints_once():
     r = run(["-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node", "2",
              "--master-addr", "127.0.0.1", "--master-port", str(free_port()), BENCH,
-             "--impl", "reference", "--gpus", "2", "--steps", "1", "--warmup", "3"])
+             "--impl", "reference", "--workload", "C1", "--gpus", "2", "--steps", "1",
+             "--warmup", "3"])
     assert r.returncode == 0, r.stderr[-2000:]
     lines = json_lines(r.stdout)
     assert len(lines) == 1 and lines[0]["impl"] == "reference" and lines[0]["n_gpus"] == 2
 
 
 def test_fewer_than_three_warmup_steps_are_refused():
-    r = run([BENCH, "--impl", "reference", "--steps", "1", "--warmup", "2"])
+    r = run([BENCH, "--impl", "reference", "--workload", "C1", "--steps", "1", "--warmup", "2"])
     assert r.returncode != 0 and "warmup" in r.stderr
     assert not json_lines(r.stdout)
 
 
 @pytest.mark.skipif(torch.cuda.is_available(), reason="checks the behaviour without a GPU")
 def test_cuda_arm_fails_without_a_gpu():
-    r = run([BENCH, "--steps", "1", "--warmup", "3"])
+    r = run([BENCH, "--workload", "C1", "--steps", "1", "--warmup", "3"])
     assert r.returncode != 0
     assert not json_lines(r.stdout)

@@ -7,8 +7,10 @@ deployments that fix their memory footprint at load time. Instead of a
 workspace argument it uses a 32 MiB array compiled into the library.
 
 Checked here through the C ABI: its output equals that of
-bigcn_layer_forward with a caller-allocated workspace (within the parity
-tolerance of the other GPU tests), on two calls in a row per case and across
+bigcn_layer_forward with a caller-allocated workspace bit for bit (both run
+the same kernels on 256-byte aligned scratch, so any difference would be a
+stale or misplaced scratch read), with no bounded device wait run out, on
+two calls in a row per case and across
 cases of different sizes, so a call must not depend on what the previous
 call left in the shared array; and a layer whose workspace would not fit is
 refused with BIGCN_ERR_SCRATCH_LIMIT before anything runs. The file is named
@@ -58,11 +60,14 @@ def test_static_scratch_layer_matches_workspace_layer(cuda_device):
         B.bigcn_layer_forward(d["X"], d["s"], d["t"], d["W"], d["rowptr"], d["colidx"], ws,
                               H_ref)
         ref = H_ref.cpu().numpy().astype(np.float64)
+        assert B.device_timeouts() == 0
         for call in range(2):
             H = torch.full((N, F), float("nan"), dtype=torch.float32, device=cuda_device)
             assert call_static(d, H) == 0, f"call {call} on N={N}, K={K}, F={F}"
             torch.cuda.synchronize()
+            assert B.device_timeouts() == 0, f"call {call} on N={N}, K={K}, F={F}"
             assert_close(H, ref, f"static-scratch layer, call {call}, N={N} K={K} F={F}")
+            assert torch.equal(H, H_ref), f"call {call} on N={N}, K={K}, F={F}: not bit-equal"
 
 
 def test_static_scratch_refuses_a_layer_that_does_not_fit(cuda_device):
