@@ -23,3 +23,35 @@ def cuda_device():
     from paper_2010_07565_gb300 import binding
     binding.lib()  # raises if libbigcn.so has not been built
     return torch.device("cuda", 0)
+
+
+@pytest.fixture(scope="session")
+def c4():
+    """The Reddit-shaped workload C4 (N = 232965, K = 602, 114.6M CSR entries,
+    hidden 128, out 41) as host arrays, generated once per session:
+    (workload, dict of X, s, t, W1, W2, rowptr, colidx)."""
+    from paper_2010_07565_gb300 import inputs
+    w = inputs.get_workload("C4")
+    X = inputs.features(w)
+    s, t = inputs.bn_stats(X)
+    W1, W2 = inputs.layer_weights(w)
+    rowptr, colidx = inputs.graph(w)
+    return w, dict(X=X, s=s, t=t, W1=W1, W2=W2, rowptr=rowptr, colidx=colidx)
+
+
+def pytest_terminal_summary(terminalreporter):
+    """Elements of the GPU parity checks that met the tolerance only by the
+    cancellation exemption of gpu_helpers.check_sum (flagged, not hidden)."""
+    mod = sys.modules.get("gpu_helpers")
+    ex = getattr(mod, "EXEMPTIONS", None) if mod is not None else None
+    if not ex:
+        return
+    terminalreporter.section("cancellation exemptions (|oracle|-relative misses inside the "
+                             "fp32 cancellation zone)")
+    total_e = total_n = 0
+    for what in sorted(ex):
+        e, n = ex[what]
+        total_e += e
+        total_n += n
+        terminalreporter.write_line(f"{e:>8} of {n:>11}  {what}")
+    terminalreporter.write_line(f"{total_e:>8} of {total_n:>11}  all checks")

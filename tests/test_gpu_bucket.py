@@ -14,34 +14,17 @@ import pytest
 import torch
 
 import oracle
-from gpu_helpers import assert_bits_equal, assert_close, to_dev
+from gpu_helpers import check_sum as check, assert_bits_equal, assert_close, to_dev
 from paper_2010_07565_gb300 import binding as B_
 from paper_2010_07565_gb300 import inputs
 
 pytestmark = pytest.mark.gpu
-RTOL, ATOL = 1e-4, 1e-6
 
 
 def rng(seed):
     return np.random.Generator(np.random.PCG64(seed))
 
 
-def check(gpu, ref, scale, what, nterms):
-    gpu = np.asarray(gpu, np.float64)
-    err = np.abs(gpu - ref)
-    bound = ATOL + RTOL * np.maximum(np.abs(ref), scale)
-    bad = err > bound
-    if bad.any():
-        q = np.unravel_index(np.argmax(err - bound), err.shape)
-        raise AssertionError(f"{what}: {int(bad.sum())} of {bad.size} out of tolerance; worst "
-                             f"at {q}: gpu={gpu[q]!r} oracle={ref[q]!r} scale={scale[q]!r}")
-    # The |o|-relative form is required wherever RTOL |o| exceeds the typical
-    # rounding error of an fp32 sum of `nterms` terms, sqrt(nterms) 2^-24 scale;
-    # below that the terms have cancelled to under what fp32 resolves.
-    plain = err > ATOL + RTOL * np.abs(ref)
-    resolved = RTOL * np.abs(ref) > np.sqrt(nterms) * 2.0 ** -24 * scale
-    stray = plain & resolved
-    assert not stray.any(), f"{what}: {int(stray.sum())} |o|-relative misses outside cancellation"
 
 
 PACK_CASES = [(1, 1, 64), (37, 63, 64), (20, 64, 64), (19, 65, 64), (300, 200, 128),

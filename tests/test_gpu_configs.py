@@ -21,7 +21,8 @@ import pytest
 import torch
 
 import oracle
-from gpu_helpers import ATOL, RTOL, assert_bits_equal, assert_close, bits_np, to_dev
+from gpu_helpers import (ATOL, RTOL, assert_bits_equal, assert_close, bits_np, check_sum,
+                         to_dev)
 from paper_2010_07565_gb300 import inputs
 from paper_2010_07565_gb300.runner import GCN2Forward
 
@@ -85,11 +86,6 @@ def sample_rows(N, n, seed):
     return rows
 
 
-@pytest.fixture(scope="module")
-def c4():
-    return workload_data("C4")
-
-
 def test_c4_layer1_sampled(cuda_device, c4):
     w, d = c4
     m = run_model(w, d, cuda_device)
@@ -133,25 +129,47 @@ def test_c4_layer2_sampled(cuda_device, c4):
     assert_close(m.logits.cpu().numpy()[rows], ref2["H"], "fused logits (sampled)")
 
 
-@pytest.mark.parametrize("K,F", [(512, 64), (4096, 256)])
-def test_c5_sweep_point_sampled(cuda_device, K, F):
-    """One layer on 2^20 nodes; features drawn on the device by torch's seeded
-    generator (the host would need tens of GB), sampled rows copied back as
-    the oracle's input."""
+@pytest.fixture(scope="module")
+def c5_graph():
+    """The sweep's Erdos-Renyi graph (one seed for every sweep point)."""
+    return inputs.graph(inputs.sweep_workload(512, 64))
+
+
+C5_POINTS = [(K, F) for K in (512, 1024, 4096, 8192) for F in (64, 256)]
+
+
+@pytest.mark.parametrize("K,F", C5_POINTS)
+def test_c5_sweep_point_sampled(cuda_device, c5_graph, K, F):
+    """One layer on 2^20 nodes at every sweep point; features drawn on the
+    device by torch's seeded generator (the host would need up to 34 GB),
+    sampled rows copied back as the oracle's input. Both the step calls and
+    bigcn_layer_forward -- the kernels the sweep benchmark times, Z kept
+    factored as 16-bit dots and a row scale -- are checked: packed bits and
+    dots bit-exact, alpha and Z on 2048 sampled rows, and H of 2048 sampled
+    rows against the oracle's aggregation of the exact dots (neighbours'
+    dots and alpha from the GPU, per-step parity)."""
     from paper_2010_07565_gb300 import binding as B
     w = inputs.sweep_workload(K, F)
     gen = torch.Generator(device=cuda_device)
     gen.manual_seed(1000 + w.index)
     X = torch.randn((w.N, K), device=cuda_device, generator=gen)
     Wt = inputs.weights(K, F, 3000 + w.index)
-    rowptr, colidx = inputs.graph(w)
+    rowptr, colidx = c5_graph
     rows = sample_rows(w.N, 2048, 46)
+    rp_d, ci_d, W_d = to_dev(rowptr), to_dev(colidx), to_dev(Wt)
     bits, alpha = B.pack_rows(X)
-    wbits, beta = B.pack_weights(to_dev(Wt))
+    wbits, beta = B.pack_weights(W_d)
     Z, dots = B.xnor_gemm(bits, alpha, wbits, beta, K, with_dots=True)
-    H = B.spmm_norm(to_dev(rowptr), to_dev(colidx), Z)
+    H = B.spmm_norm(rp_d, ci_d, Z)
+    ws = torch.empty(B.bigcn_layer_workspace_bytes(w.N, K, F), dtype=torch.uint8,
+                     device=cuda_device)
+    H_layer = torch.empty((w.N, F), device=cuda_device)
+    B.bigcn_layer_forward(X, None, None, W_d, rp_d, ci_d, ws, H_layer)
     torch.cuda.synchronize()
+    assert B.device_timeouts() == 0
     Xs = X[torch.from_numpy(rows).to(cuda_device)].cpu().numpy()
+    del X, ws
+    torch.cuda.empty_cache()
     Y = oracle.centre(Xs)
     SF = oracle.sign(Y)
     assert_bits_equal(bits_np(bits)[rows], oracle.pack(SF), "packed rows (sampled)")
@@ -159,9 +177,16 @@ def test_c5_sweep_point_sampled(cuda_device, K, F):
     SB, ref_beta = oracle.weight_binarize(Wt)
     assert_bits_equal(wbits, oracle.pack(SB), "packed weights")
     ref_dot = oracle.binary_dot(SF, SB)
-    assert np.array_equal(dots.cpu().numpy()[rows], ref_dot)
+    dots_h = dots.cpu().numpy()
+    assert np.array_equal(dots_h[rows], ref_dot)
     assert_close(Z.cpu().numpy()[rows], oracle.zeta(ref_dot, oracle.row_scale(Y), ref_beta),
                  "Z (sampled)")
     Zg = Z.cpu().numpy().astype(np.float64)
-    assert_close(H.cpu().numpy()[rows],
-                 oracle.aggregate(rowptr, colidx, Zg, rows=rows), "H (sampled)")
+    nterms = int(np.diff(rowptr)[rows].max()) + 1
+    Href, absterm = oracle.aggregate(rowptr, colidx, Zg, rows=rows, with_absterm=True)
+    check_sum(H.cpu().numpy()[rows], Href, absterm, f"C5 K={K} F={F} step H (sampled)", nterms)
+    # The layer: the oracle's zeta of the exact dots, alpha_j and beta.
+    zeta = oracle.zeta(dots_h, alpha.cpu().numpy(), beta.cpu().numpy())
+    Hl, absl = oracle.aggregate(rowptr, colidx, zeta, rows=rows, with_absterm=True)
+    check_sum(H_layer.cpu().numpy()[rows], Hl, absl, f"C5 K={K} F={F} layer H (sampled)",
+              nterms)
