@@ -3,6 +3,7 @@
 // reductions. Not part of the public interface (include/bigcn.h).
 #pragma once
 
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 
 #include <cstddef>
@@ -131,6 +132,14 @@ class EventMarks {
     bool ok_ = true;
     bool failed_ = false;
 };
+
+// A dot of Eqs. 11-12 in the compressed forms of a factored product: uint16
+// with a bias of 32768 (|dot| <= 32767), or fp16 bits when `f16` (exact for
+// |dot| <= 2048); `valid` false gives the zero dot of a padding column.
+__device__ __forceinline__ uint16_t encode_dot(int dot, bool valid, bool f16) {
+    if (f16) return valid ? __half_as_ushort(__int2half_rn(dot)) : uint16_t(0);
+    return uint16_t(valid ? dot + 32768 : 32768);
+}
 
 // 1 / sqrt(1 + row length): the D^-1/2 factor of A + I (Sec. 3.1, Eq. 1),
 // with IEEE-rounded sqrt and division.

@@ -15,6 +15,11 @@
 // not fit the fused kernel (hidden width not a multiple of 4 or above 128, or
 // more than 64 outputs). Every step runs on the GPU either way.
 //
+// When K <= 2048 (layer 1's dots exact in fp16), Fh <= 128 and Fo <= 64, the
+// products stay factored as fp16 dots with a row scale and both
+// aggregations run on the tensor cores (spmm_tc.cu): step 2 writes layer 2's
+// dots D2 and row scale s2 instead of fp32 Z2', and step 3 multiplies by beta2.
+//
 // Every kernel after the first is launched with programmatic serialization:
 // it may start while its predecessor drains, and waits (griddepcontrol) only
 // before it reads what an earlier kernel wrote -- the fused front streams and
@@ -29,6 +34,14 @@ size_t round_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 // Largest K (or Fh) whose dots the compressed uint16 form holds.
 constexpr int32_t kMaxDots16K = 32767;
+// Largest K whose dots fp16 holds exactly: the tensor-core aggregation's input.
+constexpr int32_t kMaxDotsF16K = 2048;
+
+// The tensor-core path: layer 1's dots as fp16, both aggregations on
+// spmm_tc.cu, layer 2's product kept factored as fp16 dots as well.
+bool forward2_tc(int32_t K, int32_t Fh, int32_t Fo) {
+    return K <= kMaxDotsF16K && spmm_tc_pack_gemm_supported(Fh, Fo);
+}
 
 // Workspace carve-up. Layer 1's Z' is fp32 (N x Fh) or, when K <= 32767,
 // compressed: uint16 dots (N x Fh8, Fh8 = Fh rounded up to 8) and a row
@@ -36,8 +49,9 @@ constexpr int32_t kMaxDots16K = 32767;
 // 4 (its rows are narrow: the extra row-scale read would cost more than the
 // bytes a compressed row saves).
 struct Forward2Workspace {
-    size_t bits1, alpha1, wbits1, beta1, z1, s1, wbits2, beta2, z2, h1, bits2, alpha2, total;
-    bool c16;
+    size_t bits1, alpha1, wbits1, beta1, z1, s1, wbits2, beta2, z2, h1, bits2, alpha2, d2, s2,
+        total;
+    bool c16, tc;
 };
 
 bool forward2_workspace(int64_t N, int32_t K, int32_t Fh, int32_t Fo, Forward2Workspace *w) {
@@ -49,13 +63,15 @@ bool forward2_workspace(int64_t N, int32_t K, int32_t Fh, int32_t Fo, Forward2Wo
     if (Fo4 > widest) widest = Fo4;
     if (N > kMaxElems / widest) return false;
     w->c16 = K <= kMaxDots16K;
+    w->tc = forward2_tc(K, Fh, Fo);
+    const int64_t Fh16 = (int64_t(Fh) + 15) / 16 * 16, Fo16 = (int64_t(Fo) + 15) / 16 * 16;
     size_t off = 0;
     auto take = [&](size_t bytes) { size_t at = off; off = round_up(off + bytes); return at; };
     w->bits1 = take(size_t(N) * w1 * 8);
     w->alpha1 = take(size_t(N) * 4);
     w->wbits1 = take(size_t(Fh) * w1 * 8);
     w->beta1 = take(size_t(Fh) * 4);
-    w->z1 = take(w->c16 ? size_t(N) * Fh8 * 2 : size_t(N) * Fh * 4);
+    w->z1 = take(w->tc ? size_t(N) * Fh16 * 2 : w->c16 ? size_t(N) * Fh8 * 2 : size_t(N) * Fh * 4);
     w->s1 = take(size_t(N) * 4);
     w->wbits2 = take(size_t(Fo) * w2 * 8);
     w->beta2 = take(size_t(Fo) * 4);
@@ -63,6 +79,8 @@ bool forward2_workspace(int64_t N, int32_t K, int32_t Fh, int32_t Fo, Forward2Wo
     w->h1 = take(size_t(N) * Fh * 4);
     w->bits2 = take(size_t(N) * w2 * 8);
     w->alpha2 = take(size_t(N) * 4);
+    w->d2 = take(w->tc ? size_t(N) * Fo16 * 2 : 0);
+    w->s2 = take(w->tc ? size_t(N) * 4 : 0);
     w->total = off;
     return true;
 }
@@ -83,7 +101,7 @@ extern "C" int32_t bigcn_forward_2layer_launches(int64_t N, int32_t K, int32_t F
     DeviceInfo dev;
     if (current_device(&dev) != BIGCN_OK) return -1;
     return 1 + (front_supported(N, K, Fh, dev) ? 1 : 2) +
-           (spmm_pack_gemm_supported(Fh, Fo) ? 1 : 3) + 1;
+           (forward2_tc(K, Fh, Fo) || spmm_pack_gemm_supported(Fh, Fo) ? 1 : 3) + 1;
 }
 
 extern "C" bigcn_status bigcn_forward_2layer(
@@ -144,6 +162,8 @@ extern "C" bigcn_status bigcn_forward_2layer(
     float *Z2 = static_cast<float *>(at(w.z2));
     const int words1 = bigcn_words(K), words2 = bigcn_words(Fh);
     const int64_t Fh8 = (Fh + 7) / 8 * 8, Fo4 = (Fo + 3) / 4 * 4;
+    const int64_t Fh16 = (Fh + 15) / 16 * 16, Fo16 = (Fo + 15) / 16 * 16;
+    const int64_t ldd1 = w.tc ? Fh16 : Fh8;     // layer 1's compressed row stride
     const bool fused = spmm_pack_gemm_supported(Fh, Fo);
     uint16_t *D1 = w.c16 ? static_cast<uint16_t *>(Z1) : nullptr;
     float *Z1f = w.c16 ? nullptr : static_cast<float *>(Z1);
@@ -161,8 +181,9 @@ extern "C" bigcn_status bigcn_forward_2layer(
         FrontArgs fr{X, N, K, ldx, scale, shift, wbits1, beta1, Fh, words1, rowptr, Z1f, Fh};
         if (w.c16) {
             fr.D16 = D1;
-            fr.ldd16 = Fh8;
+            fr.ldd16 = ldd1;
             fr.rowscale = s1;
+            fr.dots_f16 = w.tc;
         }
         launch_front(fr, dev, s, true);
         mark();
@@ -172,11 +193,27 @@ extern "C" bigcn_status bigcn_forward_2layer(
         GemmArgs g1{bits1, alpha1, N, wbits1, beta1, Fh, K, words1, Z1f, Fh, nullptr, rowptr};
         if (w.c16) {
             g1.dots16 = D1;
-            g1.ldd16 = Fh8;
+            g1.ldd16 = ldd1;
             g1.rowscale = s1;
+            g1.dots_f16 = w.tc;
         }
         launch_xnor_gemm(g1, dev, s, true);
         mark();
+    }
+    if (w.tc) {
+        // Both aggregations on the tensor cores: layer 1's fused with layer 2's
+        // binarization and product (fp16 dots D2 and row scale s2), then layer 2's.
+        uint16_t *D2 = static_cast<uint16_t *>(at(w.d2));
+        float *s2 = static_cast<float *>(at(w.s2));
+        SpmmTcPackGemmArgs f{rowptr, colidx, N, nnz, D1, ldd1, s1, Fh, beta1, H1, ldh1,
+                             wbits2, Fo, D2, Fo16, s2};
+        launch_spmm_tc_pack_gemm(f, dev, s, true);
+        mark();
+        SpmmTcArgs a2{rowptr, colidx, N, nnz, D2, Fo16, s2, Fo, out, ldo, beta2, pred};
+        launch_spmm_tc(a2, dev, s, true);
+        mark();
+        const bigcn_status ls = launch_status();
+        return marks.failed() ? BIGCN_ERR_CUDA : ls;
     }
     if (fused) {
         SpmmPackGemmArgs f{rowptr, colidx, N, nnz, Z1f, D1, Fh8, s1, beta1, Fh, H1, ldh1,

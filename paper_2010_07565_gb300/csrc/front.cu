@@ -48,7 +48,7 @@ front_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
              const float *__restrict__ scale, const float *__restrict__ shift,
              const uint64_t *__restrict__ wbits, const float *__restrict__ beta, int F, int words,
              const int64_t *__restrict__ rowptr, float *__restrict__ Z, int64_t ldz,
-             uint16_t *__restrict__ D16, int64_t ldd16, float *__restrict__ rowscale) {
+             uint16_t *__restrict__ D16, int64_t ldd16, float *__restrict__ rowscale, bool f16) {
     constexpr int BM = 16 * RI;
     extern __shared__ __align__(16) unsigned char smem[];
     const int pitch = words + 1;
@@ -120,9 +120,7 @@ front_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
 #pragma unroll
             for (int j = 0; j < CJ; ++j) {
                 const int col = cg + 16 * j;
-                if (col < ldd16)
-                    D16[row * ldd16 + col] =
-                        uint16_t(col < F ? K - 2 * mism[i][j] + 32768 : 32768);
+                if (col < ldd16) D16[row * ldd16 + col] = encode_dot(K - 2 * mism[i][j], col < F, f16);
             }
             continue;
         }
@@ -141,7 +139,7 @@ void launch_ri_cj(const FrontArgs &a, int BM, size_t smem, cudaStream_t s, bool 
                          int(smem));
     launch_kernel(front_kernel<RI, CJ>, dim3(grid), dim3(kFrontThreads), smem, s, pdl,
                   dim3(1, 1, 1), a.X, a.N, a.K, a.ldx, a.scale, a.shift, a.wbits, a.beta, a.F,
-                  a.words, a.rowptr, a.Z, a.ldz, a.D16, a.ldd16, a.rowscale);
+                  a.words, a.rowptr, a.Z, a.ldz, a.D16, a.ldd16, a.rowscale, a.dots_f16);
 }
 
 template <int RI>
@@ -207,7 +205,7 @@ front_split_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
                    const uint64_t *__restrict__ wbits, const float *__restrict__ beta, int F,
                    int words, const int64_t *__restrict__ rowptr, float *__restrict__ Z,
                    int64_t ldz, uint16_t *__restrict__ D16, int64_t ldd16,
-                   float *__restrict__ rowscale, int P) {
+                   float *__restrict__ rowscale, int P, bool f16) {
     extern __shared__ __align__(16) unsigned char smem[];
     __shared__ float part[kSplitWarps];
     constexpr int R = kSplitWarps / G;       // rows per group
@@ -284,7 +282,7 @@ front_split_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
                 for (int o = 1; o < P; o <<= 1) mism += __shfl_xor_sync(kFullMask, mism, o);
                 if (sub != 0 || c >= Fw) continue;
                 if (D16 != nullptr)
-                    D16[row2 * ldd16 + c] = uint16_t(c < F ? K - 2 * mism + 32768 : 32768);
+                    D16[row2 * ldd16 + c] = encode_dot(K - 2 * mism, c < F, f16);
                 else
                     Z[row2 * ldz + c] = ai * (__ldg(beta + c) * float(K - 2 * mism));
             }
@@ -311,7 +309,7 @@ void launch_split(const FrontArgs &a, const DeviceInfo &dev, cudaStream_t s, boo
     const size_t smem = split_smem(a.F, a.K, a.words, affine);
     void (*kernel)(const float *, int64_t, int, int64_t, const float *, const float *,
                    const uint64_t *, const float *, int, int, const int64_t *, float *, int64_t,
-                   uint16_t *, int64_t, float *, int);
+                   uint16_t *, int64_t, float *, int, bool);
     if (G == 2) kernel = affine ? front_split_kernel<2, true> : front_split_kernel<2, false>;
     else if (G == 4) kernel = affine ? front_split_kernel<4, true> : front_split_kernel<4, false>;
     else kernel = affine ? front_split_kernel<8, true> : front_split_kernel<8, false>;
@@ -326,7 +324,7 @@ void launch_split(const FrontArgs &a, const DeviceInfo &dev, cudaStream_t s, boo
     launch_kernel(kernel, dim3(unsigned(groups < resident ? groups : resident)),
                   dim3(kSplitThreads), smem, s, pdl, dim3(1, 1, 1), a.X, a.N, a.K, a.ldx, a.scale,
                   a.shift, a.wbits, a.beta, a.F, a.words, a.rowptr, a.Z, a.ldz, a.D16, a.ldd16,
-                  a.rowscale, P);
+                  a.rowscale, P, a.dots_f16);
 }
 
 }  // namespace

@@ -60,6 +60,9 @@ struct GemmArgs {
     uint16_t *dots16 = nullptr;
     int64_t ldd16 = 0;
     float *rowscale = nullptr;
+    // With dots_f16 the compressed dots are fp16 bits instead (exact for
+    // K <= 2048), padding columns zero: the input of launch_spmm_tc.
+    bool dots_f16 = false;
 };
 
 // Step 4 on the tensor cores (xnor_gemm_tc.cu): +-1 signs as FP8 E4M3,
@@ -136,6 +139,7 @@ struct FrontArgs {
     uint16_t *D16 = nullptr;
     int64_t ldd16 = 0;
     float *rowscale = nullptr;
+    bool dots_f16 = false;   // as in GemmArgs
 };
 
 // Whether the fused pack + XNOR-GEMM kernel fits (F <= 128, packed tiles in
@@ -183,6 +187,57 @@ bool spmm_pack_gemm_supported(int Fh, int Fo);
 // Layer-1 step 5 fused with layer-2 steps 2 and 4 (see spmm.cu).
 void launch_spmm_pack_gemm(const SpmmPackGemmArgs &args, const DeviceInfo &dev,
                            cudaStream_t stream, bool pdl = false);
+
+// Step 5 on the tensor cores (spmm_tc.cu) over a product kept factored as
+// fp16 integer dots (exact for |dot| <= 2048): H_if = colscale_f *
+// (1/sqrt(dhat_i)) * sum_{j in N(i) u {i}} rowscale_j * D[j, f], with
+// rowscale_j carrying 1/sqrt(dhat_j). D's rows hold ldd halves (a multiple of
+// 8, at least F rounded up to 16); features F .. round_up(F, 16) must hold
+// zero dots. F <= 128.
+struct SpmmTcArgs {
+    const int64_t *rowptr;
+    const int32_t *colidx;
+    int64_t N;
+    int64_t nnz;
+    const uint16_t *D;       // fp16 bits
+    int64_t ldd;
+    const float *rowscale;   // N
+    int F;
+    float *H;                // N x F (row stride ldh)
+    int64_t ldh;
+    const float *colscale;   // nullable: 1
+    int32_t *pred;           // nullable: each row's argmax (lowest index on ties)
+};
+bool spmm_tc_supported(int F);
+void launch_spmm_tc(const SpmmTcArgs &args, const DeviceInfo &dev, cudaStream_t stream,
+                    bool pdl = false);
+
+// Layer 1's tensor-core aggregation fused with layer 2's binarization and
+// XNOR product (spmm_tc.cu): from layer 1's fp16 dots D1 (row scale s1,
+// column scale beta1) to layer 2's fp16 dots D2 (rows of ldd2 halves, a
+// multiple of 8 >= Fo rounded up to 16, zeros past Fo) and row scale s2
+// (alpha2_i / sqrt(dhat_i)); H1 (nullable) receives layer 1's output.
+struct SpmmTcPackGemmArgs {
+    const int64_t *rowptr;
+    const int32_t *colidx;
+    int64_t N;
+    int64_t nnz;
+    const uint16_t *D1;
+    int64_t ldd1;
+    const float *s1;
+    int Fh;
+    const float *beta1;
+    float *H1;
+    int64_t ldh1;
+    const uint64_t *wbits2;  // Fo x ceil(Fh / 64)
+    int Fo;
+    uint16_t *D2;
+    int64_t ldd2;
+    float *s2;
+};
+bool spmm_tc_pack_gemm_supported(int Fh, int Fo);
+void launch_spmm_tc_pack_gemm(const SpmmTcPackGemmArgs &args, const DeviceInfo &dev,
+                              cudaStream_t stream, bool pdl = false);
 
 // Ablation products of step 4 (ablation.cu): one operand real, the other
 // binarized, on the tensor cores with the real operand as three bf16 parts.

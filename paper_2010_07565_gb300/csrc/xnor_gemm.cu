@@ -43,7 +43,8 @@ xnor_gemm_popc_kernel(const uint64_t *__restrict__ A, const float *__restrict__ 
                       const uint64_t *__restrict__ B, const float *__restrict__ beta, int F,
                       int K, int words, float *__restrict__ Z, int64_t ldz,
                       int32_t *__restrict__ dots, const int64_t *__restrict__ rowptr,
-                      uint16_t *__restrict__ dots16, int64_t ldd16, float *__restrict__ rowscale) {
+                      uint16_t *__restrict__ dots16, int64_t ldd16, float *__restrict__ rowscale,
+                      bool f16) {
     constexpr int BN = 16 * TN;
     constexpr int kALoads = kBM * kBKW / kThreads;                         // 4
     constexpr int kBLoads = (BN * kBKW + kThreads - 1) / kThreads;          // 1..2
@@ -148,9 +149,7 @@ xnor_gemm_popc_kernel(const uint64_t *__restrict__ A, const float *__restrict__ 
 #pragma unroll
             for (int j = 0; j < TN; ++j) {
                 const int col = n0 + tx + 16 * j;
-                if (col < ldd16)
-                    dots16[row * ldd16 + col] =
-                        uint16_t(col < F ? K - 2 * mism[i][j] + 32768 : 32768);
+                if (col < ldd16) dots16[row * ldd16 + col] = encode_dot(K - 2 * mism[i][j], col < F, f16);
             }
             continue;
         }
@@ -183,12 +182,12 @@ void launch_tn(const GemmArgs &g, const DeviceInfo &dev, cudaStream_t s, bool pd
     if (S == 1) {
         launch_kernel(xnor_gemm_popc_kernel<TN, kDeg, false>, dim3(gx, gy), dim3(kThreads), 0, s,
                       pdl, dim3(1, 1, 1), g.A, g.alpha, g.N, g.B, g.beta, g.F, g.K, g.words, g.Z,
-                      g.ldz, g.dots, g.rowptr, g.dots16, g.ldd16, g.rowscale);
+                      g.ldz, g.dots, g.rowptr, g.dots16, g.ldd16, g.rowscale, g.dots_f16);
         return;
     }
     launch_kernel(xnor_gemm_popc_kernel<TN, kDeg, true>, dim3(gx, gy, S), dim3(kThreads), 0, s,
                   pdl, dim3(1, 1, S), g.A, g.alpha, g.N, g.B, g.beta, g.F, g.K, g.words, g.Z,
-                  g.ldz, g.dots, g.rowptr, g.dots16, g.ldd16, g.rowscale);
+                  g.ldz, g.dots, g.rowptr, g.dots16, g.ldd16, g.rowscale, g.dots_f16);
 }
 
 template <bool kDeg>

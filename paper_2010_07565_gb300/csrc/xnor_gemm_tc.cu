@@ -47,7 +47,7 @@ xnor_gemm_tc_kernel(const uint64_t *__restrict__ A, const float *__restrict__ al
                     const uint64_t *__restrict__ B, const float *__restrict__ beta, int F, int K,
                     int words, float *__restrict__ Z, int64_t ldz, int32_t *__restrict__ dots,
                     const int64_t *__restrict__ rowptr, uint16_t *__restrict__ dots16,
-                    int64_t ldd16, float *__restrict__ rowscale) {
+                    int64_t ldd16, float *__restrict__ rowscale, bool f16) {
     constexpr int kStageA = kUmmaM * kTcKBytes;
     constexpr int kStageB = NT * kTcKBytes;
     constexpr int kStage = kStageA + kStageB;
@@ -192,7 +192,7 @@ xnor_gemm_tc_kernel(const uint64_t *__restrict__ A, const float *__restrict__ al
             tmem_ld16(taddr + uint32_t(c0), acc);
             if (row >= N) continue;
             const int col0 = n0 + c0;
-            if (dots16 != nullptr) {        // compressed output: biased dots, 4 per store
+            if (dots16 != nullptr) {        // compressed output: 16-bit dots, 4 per store
                 uint16_t *dr = dots16 + row * ldd16 + col0;
 #pragma unroll
                 for (int q = 0; q < 4; ++q) {
@@ -201,9 +201,8 @@ xnor_gemm_tc_kernel(const uint64_t *__restrict__ A, const float *__restrict__ al
 #pragma unroll
                     for (int e = 0; e < 4; ++e) {
                         const int col = col0 + 4 * q + e;
-                        u[e] = col < F ? uint32_t(__float2int_rn(__uint_as_float(acc[4 * q + e])) +
-                                                  32768)
-                                       : 32768u;
+                        u[e] = encode_dot(__float2int_rn(__uint_as_float(acc[4 * q + e])), col < F,
+                                          f16);
                     }
                     *reinterpret_cast<uint2 *>(dr + 4 * q) =
                         make_uint2(u[0] | (u[1] << 16), u[2] | (u[3] << 16));
@@ -264,7 +263,7 @@ void launch_nt(const GemmArgs &g, cudaStream_t s, bool pdl) {
     const dim3 grid(unsigned((g.N + kUmmaM - 1) / kUmmaM), unsigned((g.F + NT - 1) / NT));
     launch_kernel(xnor_gemm_tc_kernel<NT, kDeg>, grid, dim3(kTcThreads), smem, s, pdl,
                   dim3(1, 1, 1), g.A, g.alpha, g.N, g.B, g.beta, g.F, g.K, g.words, g.Z, g.ldz,
-                  g.dots, g.rowptr, g.dots16, g.ldd16, g.rowscale);
+                  g.dots, g.rowptr, g.dots16, g.ldd16, g.rowscale, g.dots_f16);
 }
 
 template <bool kDeg>

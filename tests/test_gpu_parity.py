@@ -414,7 +414,10 @@ def test_forward_2layer_records_one_event_per_kernel_boundary(cuda_device):
     d = {k: to_dev(v) for k, v in case.items()}
     W2 = to_dev(inputs.weights(Fh, Fo, seed=4))
     n = B.bigcn_forward_2layer_launches(N, K, Fh, Fo)
-    assert n == 4 and B.bigcn_forward_2layer_launches(N, K, 30, 7) == 6
+    # K <= 2048: both aggregations on the tensor cores, any Fh <= 128 fused
+    assert n == 4 and B.bigcn_forward_2layer_launches(N, K, 30, 7) == 4
+    # longer rows keep the CUDA-core aggregation, fused only for Fh % 4 == 0
+    assert B.bigcn_forward_2layer_launches(N, 3000, 30, 7) == 6
     assert B.bigcn_forward_2layer_launches(N, 3000, 64, 7) == 4
     assert B.bigcn_forward_2layer_launches(N, 3000, 200, 7) == 7
     assert B.bigcn_forward_2layer_launches(N, 8192, 256, 7) == 7
@@ -529,3 +532,33 @@ def test_xnor_gemm_tensor_core_degree_scaled(cuda_device):
                       beta.astype(np.float64)) * dinv[:, None]
     assert_close(Z, ref, "Z'")
     assert B.device_timeouts() == 0
+
+
+# The tensor-core aggregations on long rows: one-row windows (mean degree at
+# least 24), hub rows split over a whole block, widths that are not multiples
+# of 16 (padding tiles), and K at the fp16 limit of the dots (2048).
+@pytest.mark.parametrize("N,K,Fh,Fo,deg,hub", [
+    (3000, 602, 128, 41, 40.0, 2500),    # Reddit-like widths, hubs on the block path
+    (2000, 2048, 64, 7, 30.0, 0),        # largest K of the fp16 dots
+    (1500, 300, 40, 17, 60.0, 1200),     # widths not multiples of 16
+    (800, 100, 16, 3, 24.0, 700),        # one tile each side
+])
+def test_forward_2layer_long_rows(cuda_device, N, K, Fh, Fo, deg, hub):
+    case = inputs.layer_case(N, K, Fh, seed=N + K + Fh, mean_degree=deg, hub_degree=hub)
+    W2 = inputs.weights(Fh, Fo, seed=N + Fo)
+    d = {k: to_dev(v) for k, v in case.items()}
+    ws = torch.empty(B.bigcn_forward_2layer_workspace_bytes(N, K, Fh, Fo), dtype=torch.uint8,
+                     device=cuda_device)
+    H1 = torch.full((N, Fh), float("nan"), device=cuda_device)
+    out = torch.full((N, Fo), float("nan"), device=cuda_device)
+    pred = torch.full((N,), -7, dtype=torch.int32, device=cuda_device)
+    B.bigcn_forward_2layer(d["X"], d["s"], d["t"], d["W"], to_dev(W2), d["rowptr"],
+                           d["colidx"], ws, out, H1=H1, pred=pred)
+    torch.cuda.synchronize()
+    assert B.device_timeouts() == 0
+    ref1 = oracle.layer_forward(case["X"], case["W"], case["rowptr"], case["colidx"],
+                                case["s"], case["t"])
+    assert_close(H1, ref1["H"], "H1")
+    ref2 = oracle.layer_forward(H1.cpu().numpy(), W2, case["rowptr"], case["colidx"])
+    assert_close(out, ref2["H"], "logits")
+    assert np.array_equal(pred.cpu().numpy(), np.argmax(out.cpu().numpy(), axis=1))
