@@ -115,6 +115,7 @@ struct TcParams {
     int64_t ldd;             // halves; a multiple of 8, >= 16 * FT
     const float *rowscale;   // s_j
     int64_t heavy_degree;    // rows with more neighbours are walked by whole blocks
+    bool off32;              // N * ldd * 2 < 2^32: row byte offsets fit 32 bits
     int heavy_blocks;        // blocks [0, heavy_blocks) walk the heavy rows
     int light_first;         // blocks [light_first, grid) walk the light windows
 };
@@ -189,16 +190,24 @@ __device__ __forceinline__ void walk_window(const TcParams &P, const Window<ROWS
     float *wslot = reinterpret_cast<float *>(ring + G::NS * G::STAGE);   // NS x 16 scales
     int *cslot = reinterpret_cast<int *>(wslot + G::NS * 16);            // NS x 16 indices
     const uint32_t wslot_s = smem_addr(wslot), cslot_s = smem_addr(cslot);
-    // Copy plan of one block's rows: chunk c = lane + 32 k -> row c / CH, piece c % CH.
+    // Copy plan of one block's rows: chunk c = lane + 32 k -> row c / CH, piece
+    // c % CH (for CH a power of two: row lane / CH + k 32 / CH, piece lane % CH,
+    // so the destinations differ by constants).
     int crow[FT], cpo[FT];
     uint32_t cdst[FT];
 #pragma unroll
     for (int k = 0; k < FT; ++k) {
-        const int c = lane + 32 * k;
-        crow[k] = c / G::CH;
-        cpo[k] = (c % G::CH) * 8;
-        cdst[k] = uint32_t(crow[k] * G::PITCH + (c % G::CH) * 16);
+        if constexpr ((G::CH & (G::CH - 1)) == 0) {
+            crow[k] = lane / G::CH + k * (32 / G::CH);
+            cpo[k] = (lane % G::CH) * 16;
+        } else {
+            crow[k] = (lane + 32 * k) / G::CH;
+            cpo[k] = ((lane + 32 * k) % G::CH) * 16;
+        }
+        cdst[k] = uint32_t(crow[k] * G::PITCH + cpo[k]);
     }
+    const char *Dbytes = reinterpret_cast<const char *>(P.D);
+    const uint32_t row_bytes = uint32_t(P.ldd) * 2u;
     // ldmatrix address of this lane within a stage: matrices (entries 0-7 |
     // 8-15) x (features 0-7 | 8-15) of a tile.
     const uint32_t lofs =
@@ -228,10 +237,21 @@ __device__ __forceinline__ void walk_window(const TcParams &P, const Window<ROWS
     // A block's rows and row scales (column j per lane) -> stage `st`.
     auto copy_rows = [&](int st, int j) {
         const uint32_t base = rows_s + uint32_t(st * G::STAGE);
+        if (P.off32) {          // each lane's row byte offset, shuffled once per copy
+            const uint32_t ro = j >= 0 ? uint32_t(j) * row_bytes : 0xffffffffu;
 #pragma unroll
-        for (int k = 0; k < FT; ++k) {
-            const int jj = __shfl_sync(kFullMask, j, crow[k]);
-            cp_async16(base + cdst[k], P.D + int64_t(jj >= 0 ? jj : 0) * P.ldd + cpo[k], jj >= 0);
+            for (int k = 0; k < FT; ++k) {
+                const uint32_t r = __shfl_sync(kFullMask, ro, crow[k]);
+                const bool live = r != 0xffffffffu;
+                cp_async16(base + cdst[k], Dbytes + (live ? r : 0u) + cpo[k], live);
+            }
+        } else {
+#pragma unroll
+            for (int k = 0; k < FT; ++k) {
+                const int jj = __shfl_sync(kFullMask, j, crow[k]);
+                cp_async16(base + cdst[k], Dbytes + int64_t(jj >= 0 ? jj : 0) * row_bytes + cpo[k],
+                           jj >= 0);
+            }
         }
         if (lane < 16)
             asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(
@@ -685,7 +705,7 @@ void launch_rows(const TcParams &P0, const Epi &epi, const DeviceInfo &dev, cuda
     const int64_t resident = int64_t(per_sm) * dev.sm_count;
     const int64_t chunks = (P.N + 31) / 32;
     int64_t blocks;
-    if (need > 2 * resident) {          // persistent: every block does both
+    if (need > 4 * resident) {          // persistent: every block does both
         blocks = resident;
         P.heavy_blocks = int(resident);
         P.light_first = 0;
@@ -702,13 +722,11 @@ void launch_rows(const TcParams &P0, const Epi &epi, const DeviceInfo &dev, cuda
 template <int FT, class Epi>
 void launch_ft(const TcParams &P, const Epi &epi, const DeviceInfo &dev, cudaStream_t s,
                bool pdl) {
-    // Long rows: one-row windows with a ring of as many stages as fit about
-    // 12 KB per warp (3 to 8), so that narrow rows keep as many bytes in
-    // flight as wide ones. Short rows: four-row windows, three stages (a
-    // window is only a few blocks long).
-    constexpr int kStage = 16 * (32 * FT + 16);
-    constexpr int kDeep = 12288 / kStage < 3 ? 3 : 12288 / kStage > 8 ? 8 : 12288 / kStage;
-    if (tc_rows(P.N, P.nnz) == 1) launch_rows<FT, 1, kDeep>(P, epi, dev, s, pdl);
+    // Three stages: deeper rings (up to 12 KB per warp for narrow rows) were
+    // measured slower on the Reddit-shaped graph (layer 2: 2.04 -> 2.19 ms);
+    // the walk is bound by L2 sector throughput and issue, not by the bytes a
+    // warp keeps in flight.
+    if (tc_rows(P.N, P.nnz) == 1) launch_rows<FT, 1, 3>(P, epi, dev, s, pdl);
     else launch_rows<FT, kTcRows, 3>(P, epi, dev, s, pdl);
 }
 
@@ -718,7 +736,8 @@ bool spmm_tc_supported(int F) { return F >= 1 && F <= 128; }
 
 void launch_spmm_tc(const SpmmTcArgs &a, const DeviceInfo &dev, cudaStream_t s, bool pdl) {
     if (a.N == 0) return;
-    TcParams P{a.rowptr, a.colidx, a.N, a.nnz, a.D, a.ldd, a.rowscale, 0, 0, 0};
+    TcParams P{a.rowptr, a.colidx, a.N, a.nnz, a.D, a.ldd, a.rowscale, 0,
+               a.N * a.ldd * 2 < (int64_t(1) << 32), 0, 0};
     switch ((a.F + 15) / 16) {
 #define BIGCN_TC_CASE(ft)                                                                   \
     case ft:                                                                                \
@@ -744,7 +763,8 @@ bool spmm_tc_pack_gemm_supported(int Fh, int Fo) {
 void launch_spmm_tc_pack_gemm(const SpmmTcPackGemmArgs &a, const DeviceInfo &dev,
                               cudaStream_t s, bool pdl) {
     if (a.N == 0) return;
-    TcParams P{a.rowptr, a.colidx, a.N, a.nnz, a.D1, a.ldd1, a.s1, 0, 0, 0};
+    TcParams P{a.rowptr, a.colidx, a.N, a.nnz, a.D1, a.ldd1, a.s1, 0,
+               a.N * a.ldd1 * 2 < (int64_t(1) << 32), 0, 0};
     const int words2 = (a.Fh + 63) / 64;
     switch ((a.Fh + 15) / 16) {
 #define BIGCN_TCPG_CASE(ft)                                                                 \
