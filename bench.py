@@ -98,17 +98,46 @@ def induced_subgraph(rowptr, colidx, lo: int, hi: int):
     return out, (cols[keep] - lo).astype(np.int32)
 
 
+# Random row gathers from an L2-resident buffer (63 MB), plain 16-byte loads,
+# every SM busy: bytes/s by row size, measured on GB300 by
+# tests/probes/l2_gather.cu (profiles/l2_gather_rates.txt).
+L2_GATHER_GBS = {16: 900.0, 64: 8897.0, 128: 20469.0, 256: 21319.0, 512: 21529.0}
+
+
+def l2_gather_peak(row_bytes):
+    """The measured L2 gather ceiling for rows of this size (the entry for the
+    smallest measured row size at least this large)."""
+    for size in sorted(L2_GATHER_GBS):
+        if row_bytes <= size:
+            return L2_GATHER_GBS[size], size
+    return L2_GATHER_GBS[512], 512
+
+
+def tensor_core_aggregation(w):
+    from paper_2010_07565_gb300 import binding as B
+    return B.bigcn_forward_2layer_aggregation(w.K, w.hidden, w.out) == 1
+
+
+def z_rows(w):
+    """Bytes per node of layer 1's and layer 2's factored products as the
+    forward keeps them (dot rows + row scale): fp16 dots in rows padded to 16
+    on the tensor-core path; else uint16 dots (rows padded to 8) or fp32 for
+    layer 1 and fp32 rows padded to 4 for layer 2."""
+    K, Fh, Fo = w.K, w.hidden, w.out
+    if tensor_core_aggregation(w):
+        return 2.0 * ((Fh + 15) // 16 * 16) + 4.0, 2.0 * ((Fo + 15) // 16 * 16) + 4.0
+    z1 = 2.0 * ((Fh + 7) // 8 * 8) + 4.0 if K <= 32767 else 4.0 * Fh
+    return z1, 4.0 * ((Fo + 3) // 4 * 4)
+
+
 def kernel_work(w, nnz, name):
     """Algorithmic work of one launch of the named kernel of the 2-layer
     forward: (amount, unit, bound)."""
     N, K, Fh, Fo = w.N, w.K, w.hidden, w.out
     W1, W2 = (K + 63) // 64, (Fh + 63) // 64
     csr = 8.0 * (N + 1) + 4.0 * nnz
-    Fh4, Fo4 = (Fh + 3) // 4 * 4, (Fo + 3) // 4 * 4
-    # Layer 1's Z' as the forward keeps it: uint16 dots + a row scale when
-    # K <= 32767, else fp32; layer 2's Z' is fp32 with rows padded to Fo4.
-    z1 = 2.0 * N * Fh4 + 4.0 * N if K <= 32767 else 4.0 * N * Fh
-    z2 = 4.0 * N * Fo4
+    r1, r2 = z_rows(w)
+    z1, z2 = N * r1, N * r2
     table = {
         "pack_weights(W1,W2)": (4.0 * K * Fh + 8.0 * Fh * W1 + 4.0 * Fh + 4.0 * Fh * Fo
                                 + 8.0 * Fo * W2 + 4.0 * Fo, "bytes", "hbm"),
@@ -142,13 +171,20 @@ KERNEL_FILES = {"pack_rows": "pack.cu", "pack_weights": "pack.cu", "xnor_gemm": 
                 "L1.spmm+L2.pack_rows+L2.xnor_gemm": "spmm.cu"}
 
 
-def source_hash(name):
-    path = os.path.join(ROOT, "paper_2010_07565_gb300", "csrc", KERNEL_FILES[name])
+def kernel_file(name, w=None):
+    if w is not None and name in ("L1.spmm+L2.pack_rows+L2.xnor_gemm", "L2.spmm") and \
+            tensor_core_aggregation(w):
+        return "spmm_tc.cu"
+    return KERNEL_FILES[name]
+
+
+def source_hash(name, w=None):
+    path = os.path.join(ROOT, "paper_2010_07565_gb300", "csrc", kernel_file(name, w))
     with open(path, "rb") as f:
         return hashlib.sha256(f.read()).hexdigest()[:16]
 
 
-def profiled_traffic(name, workload):
+def profiled_traffic(name, workload, w=None):
     """DRAM bytes per launch from a committed ncu summary, if it was taken on
     the current source of the kernel (profiles/<kernel>_<workload>.txt lines
     'source_sha256_16: ...' and 'dram_bytes_per_launch: ...')."""
@@ -162,7 +198,7 @@ def profiled_traffic(name, workload):
             if ":" in line:
                 k, v = line.split(":", 1)
                 fields[k.strip()] = v.strip()
-    if fields.get("source_sha256_16") != source_hash(name):
+    if fields.get("source_sha256_16") != source_hash(name, w):
         return None
     try:
         return float(fields["dram_bytes_per_launch"])
@@ -420,17 +456,25 @@ def run_gpu(args, rank, world, local_rank):
         achieved, peak, unit = rate / 1e9, hbm, "GB/s"
     else:
         achieved, peak, unit = rate / 1e12, popc_peak / 1e12, "T bit-ops/s"
-    traffic = profiled_traffic(dom["name"], w.name)
+    traffic = profiled_traffic(dom["name"], w.name, w)
     by_name = {r["name"]: r for r in kernels}
     gemm1 = by_name.get("L1.xnor_gemm") or by_name["L1.pack_rows+L1.xnor_gemm"]
     agg1 = by_name.get("L1.spmm+L2.pack_rows+L2.xnor_gemm") or by_name["L1.spmm"]
     spmm_gbs = kernel_work(w, nnz, agg1["name"])[0] / (agg1["mean_us"] * 1e-6) / 1e9
-    # Bytes the layer-1 aggregation gathers: one row of Z1' (and its row scale
-    # when factored) per CSR entry and self-loop, plus the CSR itself -- what
-    # a graph without reuse moves, served from L2 where rows repeat.
-    row1 = 2 * ((w.hidden + 7) // 8 * 8) + 4 if w.K <= 32767 else 4 * w.hidden
-    gather1 = float(nnz + w.N) * row1 + 8.0 * (w.N + 1) + 4.0 * nnz
-    gather_gbs = gather1 / (agg1["mean_us"] * 1e-6) / 1e9
+    # Bytes an aggregation gathers: one row of the factored product (with its
+    # row scale) and one column index per CSR entry and self-loop -- what a
+    # graph without reuse moves, served from L2 where rows repeat -- against
+    # the measured L2 gather ceiling for rows of that size.
+    r1, r2 = z_rows(w)
+    gathers = {}
+    for label, r, rec in (("layer1", r1, agg1), ("layer2", r2, by_name["L2.spmm"])):
+        gb = (float(nnz + w.N) * (r + 4.0) + 8.0 * (w.N + 1)) / (rec["mean_us"] * 1e-6) / 1e9
+        peak_g, size = l2_gather_peak(r)
+        gathers[label] = {"kernel": rec["name"], "gathered_gbs": gb, "row_bytes": r,
+                          "l2_gather_peak_gbs": peak_g, "frac": gb / peak_g,
+                          "peak_source": f"measured random {size}-byte row gathers from a "
+                                         "63 MB L2-resident buffer (profiles/l2_gather_rates.txt)"}
+    gather_gbs = gathers["layer1"]["gathered_gbs"]
 
     cpu_baseline = None
     if world == 1 and not args.no_cpu_baseline:
@@ -457,8 +501,9 @@ def run_gpu(args, rank, world, local_rank):
             "spmm_gbs": spmm_gbs, "spmm_pct_of_hbm_peak": 100.0 * spmm_gbs / hbm,
             "l1_aggregation_gather_gbs": gather_gbs,
             "l1_aggregation_gather_frac_of_hbm": gather_gbs / hbm,
-            "l1_aggregation_gather_note": "every neighbour row (and row scale) of Z1' the "
-                                          "layer-1 aggregation reads, per second; rows that "
+            "aggregation_gathers": gathers,
+            "l1_aggregation_gather_note": "every neighbour row (and row scale) of the factored "
+                                          "product an aggregation reads, per second; rows that "
                                           "repeat are served from L2, so this can exceed HBM",
             "per_kernel_us": {r["name"]: round(r["mean_us"], 3) for r in kernels},
             "per_kernel_note": "from a second pass of the same graph with an event node "
@@ -466,6 +511,8 @@ def run_gpu(args, rank, world, local_rank):
         "roofline": {"kernel": dom["name"], "bound": dom["bound"],
                      "achieved": achieved, "peak": peak, "unit": unit, "frac": achieved / peak,
                      "traffic": traffic,
+                     "l2_gather": next((g for g in gathers.values() if g["kernel"] == dom["name"]),
+                                       None),
                      "peak_source": (f"{peak_kind} MEASURED_PEAKS.json hbm_gbs"
                                      if dom["bound"] == "hbm" else
                                      f"{POPC_PER_CLK_PER_SM} POPC/clk/SM x {props.multi_processor_count}"

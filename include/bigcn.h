@@ -247,7 +247,11 @@ bigcn_status bigcn_layer_forward_timed(const float *X, int64_t N, int32_t K, int
  * computes layer 2's XNOR product while the row is in registers, so H1 never
  * goes through memory. When K <= 32767, layer 1's Z' stays factored in the
  * workspace (integer dots as biased uint16 and a row scale, as in
- * bigcn_layer_forward), so its aggregation gathers half-size rows. The call
+ * bigcn_layer_forward), so its aggregation gathers half-size rows. When
+ * K <= 2048 (the dots exact in fp16), Fh <= 128 and Fo <= 64, both products
+ * stay factored as fp16 dots and a row scale and both aggregations run on the
+ * tensor cores (bigcn_forward_2layer_aggregation); layer 1's aggregation then
+ * binarizes H1 and computes layer 2's dots for any Fh <= 128. The call
  * launches 4 to 7 kernels (bigcn_forward_2layer_launches).
  *
  * X N x K (ldx), W1 K x Fh (ldw1), W2 Fh x Fo (ldw2), CSR as in
@@ -269,6 +273,12 @@ size_t bigcn_forward_2layer_workspace_bytes(int64_t N, int32_t K, int32_t Fh, in
 /* Kernel launches bigcn_forward_2layer makes for these sizes on the current
  * device (4 to 7), or -1 on invalid sizes or a device error. */
 int32_t bigcn_forward_2layer_launches(int64_t N, int32_t K, int32_t Fh, int32_t Fo);
+
+/* Which aggregation bigcn_forward_2layer runs for these widths: 1 = both on
+ * the tensor cores over fp16 dots, 0 = on the CUDA cores, -1 = invalid sizes.
+ * An interface query with no counterpart in the paper (it selects how the
+ * sums of Eq. 13 are evaluated, not what they are); needs no device. */
+int32_t bigcn_forward_2layer_aggregation(int32_t K, int32_t Fh, int32_t Fo);
 
 bigcn_status bigcn_forward_2layer(const float *X, int64_t N, int32_t K, int64_t ldx,
                                   const float *scale, const float *shift,
@@ -464,6 +474,27 @@ bigcn_status bigcn_layer_backward(const float *X, int64_t N, int32_t K, int64_t 
                                   const float *dH, int64_t ldg, float *dX, int64_t lddx,
                                   float *dW, int64_t lddw, void *workspace, size_t ws_bytes,
                                   void *stream);
+
+/*
+ * The aggregation of Eq. 13 for a block of output rows whose neighbours'
+ * pre-scaled rows come from a separate table: a shard of the graph in a
+ * multi-GPU layer (rows partitioned across GPUs, every GPU holding its own rows
+ * of Z' followed by the rows of the neighbours other GPUs own -- its halo).
+ *
+ *   H_i = (1/sqrt(dhat_i)) * sum over q in N(i) u {i} of Z'[q]      i < n_rows
+ *
+ * rowptr (n_rows + 1) and colidx (nnz) describe the block's rows in the
+ * table's numbering: entries of a row are indices into Z' (0 <= q < n_cols),
+ * the self-loop of row i is Z'[i] (a block's own rows come first), and dhat_i
+ * = 1 + the row's length (its full degree in the whole graph). Z' rows must
+ * already carry their own 1/sqrt(dhat_q) (bigcn_xnor_gemm_degscaled on the
+ * owning GPU). n_cols >= n_rows; other arguments, layouts and errors as in
+ * bigcn_spmm_prescaled, which it equals when n_cols == n_rows.
+ */
+bigcn_status bigcn_spmm_prescaled_rows(const int64_t *rowptr, const int32_t *colidx,
+                                       int64_t n_rows, int64_t n_cols, int64_t nnz,
+                                       const float *Z, int64_t ldz, int32_t F, float *H,
+                                       int64_t ldh, void *stream);
 
 /* Bytes of the device scratch array behind bigcn_layer_forward_static. */
 #define BIGCN_STATIC_SCRATCH_BYTES ((size_t)32 << 20)

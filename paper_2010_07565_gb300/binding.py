@@ -55,6 +55,9 @@ SIGNATURES = {
                               _i64, _p, _i64, _p, _i64, _p, _sz, _p], ctypes.c_int),
     "bigcn_forward_2layer_workspace_bytes": ([_i64, _i32, _i32, _i32], _sz),
     "bigcn_forward_2layer_launches": ([_i64, _i32, _i32, _i32], _i32),
+    "bigcn_forward_2layer_aggregation": ([_i32, _i32, _i32], _i32),
+    "bigcn_spmm_prescaled_rows": ([_p, _p, _i64, _i64, _i64, _p, _i64, _i32, _p, _i64, _p],
+                                  ctypes.c_int),
     "bigcn_forward_2layer": ([_p, _i64, _i32, _i64, _p, _p, _p, _i32, _i64, _p, _i32, _i64, _p,
                               _p, _i64, _p, _sz, _p, _i64, _p, _i64, _p, _p, _i32, _p],
                              ctypes.c_int),
@@ -204,6 +207,15 @@ def bigcn_spmm_prescaled(rowptr, colidx, Z, H, stream=None):
     _check("bigcn_spmm_prescaled", lib().bigcn_spmm_prescaled(
         _ptr(rowptr), _ptr(colidx) if colidx.numel() else None, N, colidx.numel(), _ptr(Z),
         _ld(Z), F, _ptr(H), _ld(H), _stream(stream)))
+
+
+def bigcn_spmm_prescaled_rows(rowptr, colidx, Z, H, stream=None):
+    """A block of output rows (H: n_rows x F) aggregated over a table of
+    pre-scaled rows (Z: n_cols x F, the block's own rows first)."""
+    n_rows, n_cols = H.shape[0], Z.shape[0]
+    _check("bigcn_spmm_prescaled_rows", lib().bigcn_spmm_prescaled_rows(
+        _ptr(rowptr), _ptr(colidx) if colidx.numel() else None, n_rows, n_cols, colidx.numel(),
+        _ptr(Z), _ld(Z), Z.shape[1], _ptr(H), _ld(H), _stream(stream)))
 
 
 def bigcn_layer_workspace_bytes(N: int, K: int, F: int) -> int:
@@ -367,6 +379,15 @@ def bigcn_forward_2layer_launches(N: int, K: int, Fh: int, Fo: int) -> int:
     n = int(lib().bigcn_forward_2layer_launches(N, K, Fh, Fo))
     if n < 0:
         raise BigcnError("bigcn_forward_2layer_launches", 1)
+    return n
+
+
+def bigcn_forward_2layer_aggregation(K: int, Fh: int, Fo: int) -> int:
+    """1 when bigcn_forward_2layer aggregates on the tensor cores (fp16 dots),
+    0 on the CUDA cores."""
+    n = int(lib().bigcn_forward_2layer_aggregation(K, Fh, Fo))
+    if n < 0:
+        raise BigcnError("bigcn_forward_2layer_aggregation", 1)
     return n
 
 

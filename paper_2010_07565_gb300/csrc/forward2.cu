@@ -96,6 +96,11 @@ extern "C" size_t bigcn_forward_2layer_workspace_bytes(int64_t N, int32_t K, int
     return forward2_workspace(N, K, Fh, Fo, &w) ? w.total : 0;
 }
 
+extern "C" int32_t bigcn_forward_2layer_aggregation(int32_t K, int32_t Fh, int32_t Fo) {
+    if (K < 1 || Fh < 1 || Fo < 1) return -1;
+    return forward2_tc(K, Fh, Fo) ? 1 : 0;
+}
+
 extern "C" int32_t bigcn_forward_2layer_launches(int64_t N, int32_t K, int32_t Fh, int32_t Fo) {
     if (N < 0 || K < 1 || Fh < 1 || Fo < 1) return -1;
     DeviceInfo dev;

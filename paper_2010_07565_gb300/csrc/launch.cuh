@@ -63,7 +63,15 @@ struct GemmArgs {
     // With dots_f16 the compressed dots are fp16 bits instead (exact for
     // K <= 2048), padding columns zero: the input of launch_spmm_tc.
     bool dots_f16 = false;
+    // Nullable device scratch of xnor_gemm_tc_bexp_bytes(K, F) bytes (16-byte
+    // aligned): the tensor-core product then expands B's signs to FP8 once
+    // into it, and each CTA copies its tiles instead of expanding them.
+    uint8_t *b_e4m3 = nullptr;
 };
+
+// Bytes of the pre-expanded B of the tensor-core product (0 when it would
+// not be used for these widths).
+size_t xnor_gemm_tc_bexp_bytes(int K, int F);
 
 // Step 4 on the tensor cores (xnor_gemm_tc.cu): +-1 signs as FP8 E4M3,
 // tcgen05.mma with fp32 accumulators in tensor memory. Used by
@@ -112,6 +120,10 @@ struct SpmmArgs {
     int agg = kAggGcn;
     const void *Zs = nullptr;
     const float *colscale_s = nullptr;
+    // Rows of Z when they differ from the N output rows (a shard's own rows
+    // followed by its halo rows): column indices must lie below it. 0: N.
+    // Needs pre-scaled rows or dots with a row scale (no neighbour degree is read).
+    int64_t ncols = 0;
 };
 
 // Step 5: H = D^-1/2 (A + I) D^-1/2 Z (Eqs. 1, 13); launches one kernel, or

@@ -101,6 +101,7 @@ struct SpmmParams {
     int agg = 0;
     const void *Zs = nullptr;
     const float *colscale_s = nullptr;
+    int64_t ncols = 0;       // rows of Z (column indices must lie below); N when 0
 };
 
 // How a lane loads VEC consecutive entries of a row of Z and adds them,
@@ -199,7 +200,7 @@ __device__ __forceinline__ void gather(const SpmmParams &p, int64_t i, int64_t b
         const int64_t q = base + lane;
         if (q < q1) {
             j = (q == 0) ? int(i) : __ldg(p.colidx + b + q - 1);
-            if (j < 0 || j >= p.N) j = -1;
+            if (j < 0 || j >= p.ncols) j = -1;
             if (j >= 0)
                 wj = S == kPre ? 1.0f
                                : S == kDots16
@@ -596,7 +597,7 @@ void launch_cfg(const SpmmArgs &a, const DeviceInfo &dev, int Fload, cudaStream_
     SpmmParams p{a.rowptr, a.colidx, a.N, a.nnz, Z, a.ldz, Fload, a.F, a.H, a.ldh,
                  heavy_block_count(a.N, dev), heavy_degree(a.N, a.nnz, (32 / L) * U), vec_store,
                  a.rowscale, a.colscale, one_slab ? a.pred : nullptr, a.agg, a.Zs,
-                 a.colscale_s};
+                 a.colscale_s, a.ncols > 0 ? a.ncols : a.N};
     dim3 grid(unsigned(p.heavy_blocks + (a.N + kSpmmWarps - 1) / kSpmmWarps),
               unsigned((a.F + SLAB - 1) / SLAB));
     launch_kernel(spmm_norm_kernel<VEC, L, NV, U, S, AGG>, grid, dim3(kSpmmThreads), 0, s, pdl,
@@ -693,6 +694,7 @@ void launch_spmm_pack_gemm(const SpmmPackGemmArgs &a, const DeviceInfo &dev, cud
     SpmmParams p{a.rowptr, a.colidx, a.N, a.nnz, Z1, c16 ? a.ldz1 : a.Fh, Fload, a.Fh, nullptr, 0,
                  heavy_block_count(a.N, dev), heavy_degree(a.N, a.nnz, (32 / L) * U), false,
                  a.s1, nullptr, nullptr};
+    p.ncols = a.N;
     FusedLayer2 f{a.H1, a.ldh, nullptr, nullptr, nullptr, a.Fo, (a.Fh + 63) / 64, a.Z2, a.ldz2};
     const dim3 grid(unsigned(p.heavy_blocks + (a.N + kSpmmWarps - 1) / kSpmmWarps));
     const dim3 one(1, 1, 1), block(kSpmmThreads);
@@ -745,6 +747,34 @@ bigcn_status spmm_entry(const int64_t *rowptr, const int32_t *colidx, int64_t N,
     return launch_status();
 }
 }  // namespace
+
+extern "C" bigcn_status bigcn_spmm_prescaled_rows(const int64_t *rowptr, const int32_t *colidx,
+                                                  int64_t n_rows, int64_t n_cols, int64_t nnz,
+                                                  const float *Z, int64_t ldz, int32_t F,
+                                                  float *H, int64_t ldh, void *stream) {
+    if (n_rows < 0 || n_rows > int64_t(INT32_MAX) || n_cols < n_rows ||
+        n_cols > int64_t(INT32_MAX) || nnz < 0 || F < 1 || ldz < F || ldh < F)
+        return BIGCN_ERR_INVALID_ARG;
+    if (n_rows > 0 && (n_cols > kMaxElems / ldz || n_rows > kMaxElems / ldh))
+        return BIGCN_ERR_INVALID_ARG;
+    if (n_rows == 0) return BIGCN_OK;
+    if (!rowptr || !Z || !H || (nnz > 0 && !colidx)) return BIGCN_ERR_INVALID_ARG;
+    if (!aligned_to(rowptr, 8) || (colidx && !aligned_to(colidx, 4)) || !aligned_to(Z, 4) ||
+        !aligned_to(H, 4))
+        return BIGCN_ERR_MISALIGNED;
+    const size_t hb = span_bytes(n_rows, F, ldh, 4);
+    if (overlaps(H, hb, Z, span_bytes(n_cols, F, ldz, 4)) ||
+        overlaps(H, hb, rowptr, size_t(n_rows + 1) * 8) ||
+        overlaps(H, hb, colidx, size_t(nnz) * 4))
+        return BIGCN_ERR_INVALID_ARG;
+    DeviceInfo dev;
+    bigcn_status st = current_device(&dev);
+    if (st != BIGCN_OK) return st;
+    SpmmArgs a{rowptr, colidx, n_rows, nnz, Z, ldz, F, H, ldh, true, false};
+    a.ncols = n_cols;
+    launch_spmm_norm(a, dev, as_stream(stream));
+    return launch_status();
+}
 
 extern "C" bigcn_status bigcn_spmm_norm(const int64_t *rowptr, const int32_t *colidx,
                                         int64_t N, int64_t nnz, const float *Z, int64_t ldz,

@@ -116,6 +116,7 @@ struct TcParams {
     const float *rowscale;   // s_j
     int64_t heavy_degree;    // rows with more neighbours are walked by whole blocks
     bool off32;              // N * ldd * 2 < 2^32: row byte offsets fit 32 bits
+    int f_base;              // first feature of this launch (column slab y: f_base + 16 FT y)
     int heavy_blocks;        // blocks [0, heavy_blocks) walk the heavy rows
     int light_first;         // blocks [light_first, grid) walk the light windows
 };
@@ -206,7 +207,8 @@ __device__ __forceinline__ void walk_window(const TcParams &P, const Window<ROWS
         }
         cdst[k] = uint32_t(crow[k] * G::PITCH + cpo[k]);
     }
-    const char *Dbytes = reinterpret_cast<const char *>(P.D);
+    const char *Dbytes = reinterpret_cast<const char *>(P.D) +
+                         2 * (int64_t(P.f_base) + int64_t(blockIdx.y) * G::FP);
     const uint32_t row_bytes = uint32_t(P.ldd) * 2u;
     // ldmatrix address of this lane within a stage: matrices (entries 0-7 |
     // 8-15) x (features 0-7 | 8-15) of a tile.
@@ -409,15 +411,17 @@ struct TcRows {
     }
 };
 
-// Epilogue of the plain aggregation: H_if = dinv_i * (c_f * sum_f) for f < F,
-// with an optional argmax of each row (lowest index on ties).
+// Epilogue of the plain aggregation: H_if = dinv_i * (c_f * sum_f) for f < F
+// (features f0 .. f0 + 16 FT - 1 of the block's column slab), with an
+// optional argmax of each row (lowest index on ties; one slab only).
 template <int FT>
 struct TcStore {
     float *H;
     int64_t ldh;
     int F;
     const float *colscale;   // nullable: 1
-    int32_t *pred;           // nullable
+    int32_t *pred;           // nullable (one column slab only)
+    int f_base;              // first feature of the launch's slab 0
     static constexpr size_t kSmemFloats = 0;
     __device__ __forceinline__ void prologue(float *) {}
     __device__ __forceinline__ void operator()(const TcRows &rows, const TcRowSums<FT> &s) const {
@@ -425,6 +429,7 @@ struct TcStore {
         const int g = lane >> 2, t = lane & 3;
         const int64_t i = rows.of(t);
         const float di = rows.dinv_of(t);
+        const int f0 = f_base + int(blockIdx.y) * 16 * FT;
         float bestv = 0.0f;
         int best = -1;
         if (i >= 0) {
@@ -432,7 +437,7 @@ struct TcStore {
             for (int T = 0; T < FT; ++T)
 #pragma unroll
                 for (int h = 0; h < 2; ++h) {
-                    const int f = 16 * T + g + 8 * h;
+                    const int f = f0 + 16 * T + g + 8 * h;
                     if (f < F) {
                         const float c = colscale != nullptr ? __ldg(colscale + f) : 1.0f;
                         const float o = di * (c * s.v[T][h]);
@@ -685,8 +690,8 @@ int64_t tc_heavy_degree(int64_t N, int64_t nnz) {
 }
 
 template <int FT, int ROWS, int NS, class Epi>
-void launch_rows(const TcParams &P0, const Epi &epi, const DeviceInfo &dev, cudaStream_t s,
-                 bool pdl) {
+void launch_rows(const TcParams &P0, const Epi &epi, int slabs, const DeviceInfo &dev,
+                 cudaStream_t s, bool pdl) {
     TcParams P = P0;
     P.heavy_degree = tc_heavy_degree(P.N, P.nnz);
     const size_t smem = tc_smem<FT, NS>(Epi::kSmemFloats);
@@ -715,33 +720,45 @@ void launch_rows(const TcParams &P0, const Epi &epi, const DeviceInfo &dev, cuda
         P.light_first = int(hb);
         blocks = hb + need;
     }
-    const dim3 grid(static_cast<unsigned>(blocks));
+    const dim3 grid(static_cast<unsigned>(blocks), static_cast<unsigned>(slabs));
     launch_kernel(kernel, grid, dim3(kTcThreads), smem, s, pdl, dim3(1, 1, 1), P, epi);
 }
 
 template <int FT, class Epi>
 void launch_ft(const TcParams &P, const Epi &epi, const DeviceInfo &dev, cudaStream_t s,
-               bool pdl) {
+               bool pdl, int slabs = 1) {
     // Three stages: deeper rings (up to 12 KB per warp for narrow rows) were
     // measured slower on the Reddit-shaped graph (layer 2: 2.04 -> 2.19 ms);
     // the walk is bound by L2 sector throughput and issue, not by the bytes a
     // warp keeps in flight.
-    if (tc_rows(P.N, P.nnz) == 1) launch_rows<FT, 1, 3>(P, epi, dev, s, pdl);
-    else launch_rows<FT, kTcRows, 3>(P, epi, dev, s, pdl);
+    if (tc_rows(P.N, P.nnz) == 1) launch_rows<FT, 1, 3>(P, epi, slabs, dev, s, pdl);
+    else launch_rows<FT, kTcRows, 3>(P, epi, slabs, dev, s, pdl);
 }
 
 }  // namespace
 
-bool spmm_tc_supported(int F) { return F >= 1 && F <= 128; }
+bool spmm_tc_supported(int F) { return F >= 1; }
 
+// Column slabs of 128 features (FT = 8) in one launch, then the remaining
+// F mod 128 features in a second launch with as many 16-feature tiles as they
+// need (or one launch of ceil(F / 16) tiles when F <= 128).
 void launch_spmm_tc(const SpmmTcArgs &a, const DeviceInfo &dev, cudaStream_t s, bool pdl) {
     if (a.N == 0) return;
     TcParams P{a.rowptr, a.colidx, a.N, a.nnz, a.D, a.ldd, a.rowscale, 0,
-               a.N * a.ldd * 2 < (int64_t(1) << 32), 0, 0};
-    switch ((a.F + 15) / 16) {
-#define BIGCN_TC_CASE(ft)                                                                   \
-    case ft:                                                                                \
-        launch_ft<ft>(P, TcStore<ft>{a.H, a.ldh, a.F, a.colscale, a.pred}, dev, s, pdl);   \
+               a.N * a.ldd * 2 < (int64_t(1) << 32), 0, 0, 0};
+    const int full = a.F > 128 ? a.F / 128 : 0;
+    if (full > 0) {
+        launch_ft<8>(P, TcStore<8>{a.H, a.ldh, a.F, a.colscale, nullptr, 0}, dev, s, pdl, full);
+        pdl = true;         // the remainder launch follows on the same stream
+    }
+    const int rest = a.F - 128 * full;
+    if (rest == 0) return;
+    P.f_base = 128 * full;
+    int32_t *pred = full == 0 ? a.pred : nullptr;
+    switch ((rest + 15) / 16) {
+#define BIGCN_TC_CASE(ft)                                                                     \
+    case ft:                                                                                  \
+        launch_ft<ft>(P, TcStore<ft>{a.H, a.ldh, a.F, a.colscale, pred, P.f_base}, dev, s, pdl); \
         break;
         BIGCN_TC_CASE(1)
         BIGCN_TC_CASE(2)
@@ -764,7 +781,7 @@ void launch_spmm_tc_pack_gemm(const SpmmTcPackGemmArgs &a, const DeviceInfo &dev
                               cudaStream_t s, bool pdl) {
     if (a.N == 0) return;
     TcParams P{a.rowptr, a.colidx, a.N, a.nnz, a.D1, a.ldd1, a.s1, 0,
-               a.N * a.ldd1 * 2 < (int64_t(1) << 32), 0, 0};
+               a.N * a.ldd1 * 2 < (int64_t(1) << 32), 0, 0, 0};
     const int words2 = (a.Fh + 63) / 64;
     switch ((a.Fh + 15) / 16) {
 #define BIGCN_TCPG_CASE(ft)                                                                 \

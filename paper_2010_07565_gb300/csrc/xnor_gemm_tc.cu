@@ -18,7 +18,13 @@
 // once (and the next k-block's while the MMAs are issued), and turns every
 // four signs into four E4M3 bytes with one multiply and three logic ops.
 // A stage is reused only after the tcgen05.commit of the MMAs that read it
-// has arrived on its mbarrier.
+// has arrived on its mbarrier. With a caller's scratch for it, B's signs are
+// instead expanded once per launch (expand_b_kernel) into the stage images of
+// every (column tile, k-block), and thread 0 copies each k-block's image into
+// its stage with one bulk copy (completion counted on a second mbarrier per
+// stage) while the CTA expands only A. (A separate five-stage ring for B, 3
+// k-blocks ahead, was measured slower: it leaves one CTA per SM instead of two,
+// 2.77 -> 3.82 ms on 2^20 x 8192 x 256.)
 // Every mbarrier wait is bounded; a wait that runs out is counted in
 // g_tc_timeouts (see bigcn_device_timeouts), the CTA skips its epilogue,
 // frees its tensor memory and returns.
@@ -41,13 +47,14 @@ constexpr int kTcThreads = 256;
 constexpr int kTcKBytes = 128;
 constexpr int kTcStages = 2;
 
-template <int NT, bool kDeg>
-__global__ void __launch_bounds__(kTcThreads)
+template <int NT, bool kDeg, bool kBexp>
+__global__ void __launch_bounds__(kTcThreads, NT == 256 ? 2 : 4)
 xnor_gemm_tc_kernel(const uint64_t *__restrict__ A, const float *__restrict__ alpha, int64_t N,
                     const uint64_t *__restrict__ B, const float *__restrict__ beta, int F, int K,
                     int words, float *__restrict__ Z, int64_t ldz, int32_t *__restrict__ dots,
                     const int64_t *__restrict__ rowptr, uint16_t *__restrict__ dots16,
-                    int64_t ldd16, float *__restrict__ rowscale, bool f16) {
+                    int64_t ldd16, float *__restrict__ rowscale, bool f16,
+                    const uint8_t *__restrict__ bexp) {
     constexpr int kStageA = kUmmaM * kTcKBytes;
     constexpr int kStageB = NT * kTcKBytes;
     constexpr int kStage = kStageA + kStageB;
@@ -56,6 +63,7 @@ xnor_gemm_tc_kernel(const uint64_t *__restrict__ A, const float *__restrict__ al
     constexpr int kBChunks = NT / kRowsPerPass;           // 2, 4 or 8 rows of B per thread
     extern __shared__ unsigned char smem_raw[];
     __shared__ __align__(8) uint64_t bars[kTcStages];
+    __shared__ __align__(8) uint64_t full[kTcStages];       // B tile landed (kBexp)
     __shared__ uint32_t tmem_base;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -72,7 +80,10 @@ xnor_gemm_tc_kernel(const uint64_t *__restrict__ A, const float *__restrict__ al
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
     }
     if (tid == 0) {
-        for (int s = 0; s < kTcStages; ++s) mbar_init(smem_addr(&bars[s]), 1);
+        for (int s = 0; s < kTcStages; ++s) {
+            mbar_init(smem_addr(&bars[s]), 1);
+            mbar_init(smem_addr(&full[s]), 1);
+        }
         mbar_fence_init();
     }
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -95,9 +106,12 @@ xnor_gemm_tc_kernel(const uint64_t *__restrict__ A, const float *__restrict__ al
 #pragma unroll
         for (int q = 0; q < kBChunks; ++q) {
             const int col = n0 + r0 + kRowsPerPass * q;
-            wb[q] = (col < F && k0 < K) ? __ldg(B + int64_t(col) * words + (k0 >> 6)) : 0ull;
+            wb[q] = (!kBexp && col < F && k0 < K)
+                        ? __ldg(B + int64_t(col) * words + (k0 >> 6)) : 0ull;
         }
     };
+    const uint8_t *btiles = kBexp ? bexp + size_t(blockIdx.y) * KB * kStageB : nullptr;
+    int issued = -1, landed = -1;       // thread 0: last k-block copied / seen landing
     // 16 signs from bit `sh` of w as E4M3 bytes, zero past `valid` signs.
     auto expand = [&](uint64_t w, int sh, int valid) {
         const uint32_t bits = uint32_t(w >> sh);
@@ -130,6 +144,18 @@ xnor_gemm_tc_kernel(const uint64_t *__restrict__ A, const float *__restrict__ al
         }
         unsigned char *sa = tiles + s * kStage;
         unsigned char *sb = sa + kStageA;
+        if (kBexp && tid == 0) {    // B's tile of this k-block: one bulk copy
+            const uint32_t fb = smem_addr(&full[s]);
+            asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(fb),
+                         "r"(uint32_t(kStageB))
+                         : "memory");
+            asm volatile(
+                "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], "
+                "%2, [%3];" ::"r"(smem_addr(sb)),
+                "l"(btiles + size_t(kb) * kStageB), "r"(uint32_t(kStageB)), "r"(fb)
+                : "memory");
+            issued = kb;
+        }
         const int k0 = kb * kTcKBytes + c * 16;
         const int sh = k0 & 63;
         const int valid = min(max(K - k0, 0), 16);
@@ -140,14 +166,27 @@ xnor_gemm_tc_kernel(const uint64_t *__restrict__ A, const float *__restrict__ al
             *reinterpret_cast<uint4 *>(sa + sw128_offset(r, c)) =
                 live ? expand(wa[q], sh, valid) : make_uint4(0u, 0u, 0u, 0u);
         }
+        if (!kBexp) {
 #pragma unroll
-        for (int q = 0; q < kBChunks; ++q) {
-            const int r = r0 + kRowsPerPass * q;
-            *reinterpret_cast<uint4 *>(sb + sw128_offset(r, c)) = expand(wb[q], sh, 16);
+            for (int q = 0; q < kBChunks; ++q) {
+                const int r = r0 + kRowsPerPass * q;
+                *reinterpret_cast<uint4 *>(sb + sw128_offset(r, c)) = expand(wb[q], sh, 16);
+            }
         }
         if (kb + 1 < KB) load_words(kb + 1);      // in flight across the barrier and MMAs
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         __syncthreads();
+        if (kBexp) {                // B's tile has landed (bounded wait, as for the MMAs)
+            bool here = true;
+            if (tid == 0) {
+                here = mbar_wait(smem_addr(&full[s]), uint32_t(kb >> 1) & 1u);
+                if (here) landed = kb;
+            }
+            if (!__syncthreads_and(here)) {
+                ok = false;
+                break;
+            }
+        }
         if (tid == 0) {
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
             const uint32_t a0 = smem_addr(sa), b0 = smem_addr(sb);
@@ -164,6 +203,11 @@ xnor_gemm_tc_kernel(const uint64_t *__restrict__ A, const float *__restrict__ al
     }
     // Every MMA issued is done once the last commit has arrived (waited for
     // even after a failed wait, so that no MMA is in flight at deallocation).
+    // B copies whose landing was not seen (a wait ran out, or the loop ended
+    // early) are waited for too, bounded, before the shared memory is given up.
+    if (kBexp && tid == 0)
+        for (int kbp = landed + 1; kbp <= issued; ++kbp)
+            mbar_wait(smem_addr(&full[kbp & 1]), uint32_t(kbp >> 1) & 1u);
     bool done = true;
     if (committed >= 0)
         done = mbar_wait(smem_addr(&bars[committed & 1]), uint32_t(committed >> 1) & 1u);
@@ -250,20 +294,70 @@ xnor_gemm_tc_kernel(const uint64_t *__restrict__ A, const float *__restrict__ al
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(NT));
 }
 
+// B's signs as the product's FP8 tiles: tile (n-tile y, k-block kb) is NT
+// rows (columns n0 + r of W, zero rows past F) x 128 signs (zero past K) in
+// the 128B-swizzled layout of a stage, NT * 128 bytes, tiles in (y, kb) order.
 template <int NT>
+__global__ void __launch_bounds__(kTcThreads)
+expand_b_kernel(const uint64_t *__restrict__ B, int F, int K, int words, int KB,
+                uint8_t *__restrict__ out) {
+    grid_dependency_wait();     // the packed columns come from the previous kernel
+    const int tile = blockIdx.x;
+    const int y = tile / KB, kb = tile % KB;
+    uint8_t *dst = out + size_t(tile) * NT * kTcKBytes;
+    for (int q = threadIdx.x; q < NT * 8; q += kTcThreads) {
+        const int r = q >> 3, c = q & 7;
+        const int col = y * NT + r;
+        const int k0 = kb * kTcKBytes + c * 16;
+        uint4 v = make_uint4(0u, 0u, 0u, 0u);
+        if (col < F && k0 < K) {
+            const uint32_t bits = uint32_t(__ldg(B + int64_t(col) * words + (k0 >> 6)) >> (k0 & 63));
+            v = make_uint4(signs4_to_e4m3(bits & 15u), signs4_to_e4m3((bits >> 4) & 15u),
+                           signs4_to_e4m3((bits >> 8) & 15u), signs4_to_e4m3((bits >> 12) & 15u));
+            const int valid = K - k0;
+            if (valid < 16) {
+                uint32_t *e = reinterpret_cast<uint32_t *>(&v);
+#pragma unroll
+                for (int p = 0; p < 4; ++p) {
+                    const int keep = valid - 4 * p;
+                    if (keep <= 0) e[p] = 0u;
+                    else if (keep < 4) e[p] &= (1u << (8 * keep)) - 1u;
+                }
+            }
+        }
+        *reinterpret_cast<uint4 *>(dst + sw128_offset(r, c)) = v;
+    }
+}
+
+int tc_nt(int F) { return F <= 64 ? 64 : F <= 128 ? 128 : 256; }
+
+template <int NT, bool kBexp = false>
 size_t tc_smem() {
     return 1024 + size_t(kTcStages) * (kUmmaM * kTcKBytes + NT * kTcKBytes);
 }
 
+template <int NT, bool kDeg, bool kBexp>
+void launch_nt2(const GemmArgs &g, cudaStream_t s, bool pdl) {
+    const size_t smem = tc_smem<NT, kBexp>();
+    auto kernel = xnor_gemm_tc_kernel<NT, kDeg, kBexp>;
+    cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+    const dim3 grid(unsigned((g.N + kUmmaM - 1) / kUmmaM), unsigned((g.F + NT - 1) / NT));
+    if (kBexp) {
+        const int KB = (g.K + kTcKBytes - 1) / kTcKBytes;
+        launch_kernel(expand_b_kernel<NT>, dim3(grid.y * unsigned(KB)), dim3(kTcThreads), 0, s,
+                      pdl, dim3(1, 1, 1), g.B, g.F, g.K, g.words, KB, g.b_e4m3);
+    }
+    launch_kernel(kernel, grid, dim3(kTcThreads), smem, s, pdl || kBexp, dim3(1, 1, 1), g.A,
+                  g.alpha, g.N, g.B, g.beta, g.F, g.K, g.words, g.Z, g.ldz, g.dots, g.rowptr,
+                  g.dots16, g.ldd16, g.rowscale, g.dots_f16, static_cast<const uint8_t *>(g.b_e4m3));
+}
+
 template <int NT, bool kDeg>
 void launch_nt(const GemmArgs &g, cudaStream_t s, bool pdl) {
-    const size_t smem = tc_smem<NT>();
-    cudaFuncSetAttribute(xnor_gemm_tc_kernel<NT, kDeg>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         int(smem));
-    const dim3 grid(unsigned((g.N + kUmmaM - 1) / kUmmaM), unsigned((g.F + NT - 1) / NT));
-    launch_kernel(xnor_gemm_tc_kernel<NT, kDeg>, grid, dim3(kTcThreads), smem, s, pdl,
-                  dim3(1, 1, 1), g.A, g.alpha, g.N, g.B, g.beta, g.F, g.K, g.words, g.Z, g.ldz,
-                  g.dots, g.rowptr, g.dots16, g.ldd16, g.rowscale, g.dots_f16);
+    if (g.b_e4m3 != nullptr && xnor_gemm_tc_bexp_bytes(g.K, g.F) > 0)
+        launch_nt2<NT, kDeg, true>(g, s, pdl);
+    else
+        launch_nt2<NT, kDeg, false>(g, s, pdl);
 }
 
 template <bool kDeg>
@@ -275,10 +369,20 @@ void launch_deg(const GemmArgs &g, cudaStream_t s, bool pdl) {
 
 }  // namespace
 
+size_t xnor_gemm_tc_bexp_bytes(int K, int F) {
+    // Expanding W once pays where its share of the per-k-block expansion is
+    // large (256-column tiles) and the k-blocks are many; measured on 2^20
+    // rows: K = 8192, F = 256: 3637 -> 2773 us; K = 512, F = 64: 168 -> 232 us.
+    if (K < 128 || F < 32 || !((F > 128 && K >= 1024) || K >= 4096)) return 0;
+    const int NT = tc_nt(F);
+    return size_t((F + NT - 1) / NT) * size_t((K + kTcKBytes - 1) / kTcKBytes) * size_t(NT) *
+           kTcKBytes;
+}
+
 bool xnor_gemm_tc_supported(int64_t N, int K, int F, const DeviceInfo &dev) {
     // Enough 128-row tiles to give every SM one, and shared memory for two stages.
     return K >= 128 && F >= 32 && (N + kUmmaM - 1) / kUmmaM >= dev.sm_count &&
-           size_t(dev.max_smem_optin) >= tc_smem<256>();
+           size_t(dev.max_smem_optin) >= tc_smem<256, true>();
 }
 
 void launch_xnor_gemm_tc(const GemmArgs &g, const DeviceInfo &, cudaStream_t stream, bool pdl) {

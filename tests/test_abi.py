@@ -60,15 +60,23 @@ def test_words_and_status_strings(lib):
 def test_workspace_bytes(lib):
     assert lib.bigcn_layer_workspace_bytes(0, 0, 5) == 0
     assert lib.bigcn_layer_workspace_bytes(-1, 10, 5) == 0
-    # K <= 32767: Z kept factored as uint16 dots (rows padded to 4) plus a row scale
+    # K <= 2048, F <= 128: Z kept factored as fp16 dots (rows padded to 16) plus
+    # a row scale
     n = lib.bigcn_layer_workspace_bytes(1000, 130, 62)
     need = 1000 * 3 * 8 + 1000 * 4 + 62 * 3 * 8 + 62 * 4 + 1000 * 64 * 2 + 1000 * 4
-    assert need <= n <= need + 6 * 256 and n % 256 == 0
+    assert need <= n <= need + 7 * 256 and n % 256 == 0
     assert lib.bigcn_layer_workspace_bytes(2000, 130, 62) > n
+    # K > 2048: uint16 dots (rows padded to 8); K >= 4096: also the weight signs
+    # as the tensor-core product's FP8 tiles (one 64-column tile x 33 k-blocks
+    # of 128 bytes a row)
+    n = lib.bigcn_layer_workspace_bytes(1000, 4100, 62)
+    need = (1000 * 65 * 8 + 1000 * 4 + 62 * 65 * 8 + 62 * 4 + 1000 * 64 * 2 + 1000 * 4 +
+            1 * 33 * 64 * 128)
+    assert need <= n <= need + 7 * 256 and n % 256 == 0
     # larger K: fp32 Z
     n = lib.bigcn_layer_workspace_bytes(100, 40000, 5)
     need = 100 * 625 * 8 + 100 * 4 + 5 * 625 * 8 + 5 * 4 + 100 * 5 * 4
-    assert need <= n <= need + 6 * 256 and n % 256 == 0
+    assert need <= n <= need + 7 * 256 and n % 256 == 0
 
 
 def test_pack_rows_argument_checks(lib):
@@ -131,3 +139,18 @@ def test_layer_forward_argument_checks(lib):
     assert f(*args(ws=X)) == INVALID                                              # overlaps X
     assert f(*args(H=ws + 256)) == INVALID                                        # H in workspace
     assert f(*args(H=X)) == INVALID
+
+
+def test_forward_2layer_aggregation_query(lib):
+    """The 2-layer forward aggregates on the tensor cores exactly when layer 1's
+    dots fit fp16 (K <= 2048), Fh <= 128 and Fo <= 64; the query needs no GPU."""
+    from paper_2010_07565_gb300 import binding as B
+    assert B.bigcn_forward_2layer_aggregation(602, 128, 41) == 1      # Reddit-shaped
+    assert B.bigcn_forward_2layer_aggregation(1433, 64, 7) == 1       # Cora-shaped
+    assert B.bigcn_forward_2layer_aggregation(2048, 30, 64) == 1
+    assert B.bigcn_forward_2layer_aggregation(3703, 64, 6) == 0       # Citeseer-shaped
+    assert B.bigcn_forward_2layer_aggregation(2049, 64, 7) == 0
+    assert B.bigcn_forward_2layer_aggregation(500, 129, 7) == 0
+    assert B.bigcn_forward_2layer_aggregation(500, 64, 65) == 0
+    with pytest.raises(B.BigcnError):
+        B.bigcn_forward_2layer_aggregation(0, 64, 7)
