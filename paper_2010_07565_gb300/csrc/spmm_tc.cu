@@ -52,16 +52,26 @@ constexpr int kTcThreads = 256;
 constexpr int kTcWarps = kTcThreads / 32;
 constexpr int kTcRows = 4;          // output rows per light window
 
-template <int FT, int NSTAGES>
+// Entries per block: 32 for narrow rows in one-row windows (every lane owns
+// an entry, and the per-block work -- index copies, waits, scales, B
+// fragments -- covers twice the entries; two MMA k-steps per block; layer 2 on
+// the Reddit-shaped graph: 2.04 -> 1.93 ms), else 16 (wide rows would leave one
+// block per SM; in four-row windows 32 was measured slower: 835 -> 1215 us on
+// 2^20 nodes of mean degree 16).
+constexpr int tc_entries_per_block(int FT, int ROWS) { return ROWS == 1 && FT <= 4 ? 32 : 16; }
+
+template <int FT, int NSTAGES, int EBLOCK>
 struct TcGeom {
     static constexpr int FP = 16 * FT;             // features per staged row
     static constexpr int CH = 2 * FT;              // 16-byte copies per row
     static constexpr int PITCH = FP * 2 + 16;      // bytes per staged row (conflict-free ldmatrix)
-    static constexpr int STAGE = 16 * PITCH;       // one block of 16 entries
+    static constexpr int EB = EBLOCK;              // entries per block (16 or 32)
+    static constexpr int KCH = EB * CH / 32;       // 16-byte row copies per lane and block
+    static constexpr int STAGE = EB * PITCH;       // one block of EB entries
     static constexpr int NS = NSTAGES;             // ring depth (blocks of 16 entries)
     static constexpr int D = NS - 1;               // blocks copied ahead
-    // one warp's ring: NS row stages, then NS x 16 row scales and NS x 16 column indices
-    static constexpr int WARP = NS * STAGE + NS * 16 * 8;
+    // one warp's ring: NS row stages, then NS x EB row scales and NS x EB column indices
+    static constexpr int WARP = NS * STAGE + NS * EB * 8;
 };
 
 __device__ __forceinline__ uint32_t smem_addr(const void *p) {
@@ -170,34 +180,35 @@ struct TcRowSums {
 };
 
 // Walks a window's position stream and leaves its sums in `out`. The warp's
-// ring `ring` (shared, TcGeom<FT, NS>::WARP bytes) is free on entry and on exit.
+// ring `ring` (shared, TcGeom<FT, NS, EB>::WARP bytes) is free on entry and on exit.
 //
-// Pipeline (blocks of 16 positions; lane e16 = lane & 15 owns position e16 of
-// a block; lanes 16-31 repeat lanes 0-15): group n, committed in iteration n,
+// Pipeline (blocks of EB positions; lane e = lane mod EB owns position e of a
+// block; with EB = 16 lanes 16-31 repeat lanes 0-15): group n, committed in iteration n,
 // copies block n + D's rows and row scales and block n + 2D's column indices,
 // so iteration n finds block n (rows, scales) and block n + D's indices landed
 // after waiting for all but the last D - 1 groups. No register of the loop
 // waits on a global load. Block b uses ring stage b mod NS.
-template <int FT, int ROWS, int NS>
+template <int FT, int ROWS, int NS, int EBLOCK>
 __device__ __forceinline__ void walk_window(const TcParams &P, const Window<ROWS> &w,
                                            uint8_t *ring, TcRowSums<FT> &out) {
-    using G = TcGeom<FT, NS>;
+    using G = TcGeom<FT, NS, EBLOCK>;
     const int lane = threadIdx.x & 31;
     const int g = lane >> 2, t = lane & 3;
-    const int e16 = lane & 15;
+    constexpr int EB = G::EB;
+    const int e16 = lane & (EB - 1);        // this lane's entry of a block
     const int total = w.off[ROWS];
-    const int nblk = (total + 15) >> 4;
+    const int nblk = (total + EB - 1) / EB;
     const uint32_t rows_s = smem_addr(ring);
-    float *wslot = reinterpret_cast<float *>(ring + G::NS * G::STAGE);   // NS x 16 scales
-    int *cslot = reinterpret_cast<int *>(wslot + G::NS * 16);            // NS x 16 indices
+    float *wslot = reinterpret_cast<float *>(ring + G::NS * G::STAGE);   // NS x EB scales
+    int *cslot = reinterpret_cast<int *>(wslot + G::NS * EB);            // NS x EB indices
     const uint32_t wslot_s = smem_addr(wslot), cslot_s = smem_addr(cslot);
     // Copy plan of one block's rows: chunk c = lane + 32 k -> row c / CH, piece
     // c % CH (for CH a power of two: row lane / CH + k 32 / CH, piece lane % CH,
     // so the destinations differ by constants).
-    int crow[FT], cpo[FT];
-    uint32_t cdst[FT];
+    int crow[G::KCH], cpo[G::KCH];
+    uint32_t cdst[G::KCH];
 #pragma unroll
-    for (int k = 0; k < FT; ++k) {
+    for (int k = 0; k < G::KCH; ++k) {
         if constexpr ((G::CH & (G::CH - 1)) == 0) {
             crow[k] = lane / G::CH + k * (32 / G::CH);
             cpo[k] = (lane % G::CH) * 16;
@@ -217,23 +228,23 @@ __device__ __forceinline__ void walk_window(const TcParams &P, const Window<ROWS
 
     // Block b's column indices -> index slot `st` (zeros for self / dead entries).
     auto copy_cols = [&](int b, int st) {
-        const int p = b * 16 + e16;
+        const int p = b * EB + e16;
         const int tg = tag_of(w, p);
         const bool live = p < total && p != pick<ROWS>(w.selfp, tg);
         const int32_t *src = P.colidx + (live ? pick<ROWS>(w.cbase, tg) + p : 0);
-        if (lane < 16)
+        if (lane < EB)
             asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(
-                             cslot_s + uint32_t((st * 16 + e16) * 4)),
+                             cslot_s + uint32_t((st * EB + e16) * 4)),
                          "l"(src), "r"(live ? 4 : 0)
                          : "memory");
     };
     // Column of block b's entry of this lane, from its landed index slot `st`.
     auto column = [&](int b, int st) -> int {
-        const int p = b * 16 + e16;
+        const int p = b * EB + e16;
         if (p >= total) return -1;
         const int tg = tag_of(w, p);
         const int64_t j = p == pick<ROWS>(w.selfp, tg) ? pick<ROWS>(w.row, tg)
-                                                        : int64_t(cslot[st * 16 + e16]);
+                                                        : int64_t(cslot[st * EB + e16]);
         return (j >= 0 && j < P.N) ? int(j) : -1;
     };
     // A block's rows and row scales (column j per lane) -> stage `st`.
@@ -242,22 +253,22 @@ __device__ __forceinline__ void walk_window(const TcParams &P, const Window<ROWS
         if (P.off32) {          // each lane's row byte offset, shuffled once per copy
             const uint32_t ro = j >= 0 ? uint32_t(j) * row_bytes : 0xffffffffu;
 #pragma unroll
-            for (int k = 0; k < FT; ++k) {
+            for (int k = 0; k < G::KCH; ++k) {
                 const uint32_t r = __shfl_sync(kFullMask, ro, crow[k]);
                 const bool live = r != 0xffffffffu;
                 cp_async16(base + cdst[k], Dbytes + (live ? r : 0u) + cpo[k], live);
             }
         } else {
 #pragma unroll
-            for (int k = 0; k < FT; ++k) {
+            for (int k = 0; k < G::KCH; ++k) {
                 const int jj = __shfl_sync(kFullMask, j, crow[k]);
                 cp_async16(base + cdst[k], Dbytes + int64_t(jj >= 0 ? jj : 0) * row_bytes + cpo[k],
                            jj >= 0);
             }
         }
-        if (lane < 16)
+        if (lane < EB)
             asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(
-                             wslot_s + uint32_t((st * 16 + e16) * 4)),
+                             wslot_s + uint32_t((st * EB + e16) * 4)),
                          "l"(P.rowscale + (j >= 0 ? j : 0)), "r"(j >= 0 ? 4 : 0)
                          : "memory");
     };
@@ -276,7 +287,7 @@ __device__ __forceinline__ void walk_window(const TcParams &P, const Window<ROWS
 #pragma unroll
     for (int k = 0; k < G::D; ++k) {
         copy_cols(G::D + k, (G::D + k) % G::NS);
-        copy_rows(k, fetch_col(P, w, 16 * k + e16));
+        copy_rows(k, fetch_col(P, w, EB * k + e16));
         cp_async_commit();
     }
 
@@ -293,8 +304,8 @@ __device__ __forceinline__ void walk_window(const TcParams &P, const Window<ROWS
         cp_async_commit();
 
         // This block's weights and the scale exponent of each row they belong to.
-        const float w0 = wslot[st * 16 + e16];      // 0 for dead entries
-        uint32_t b0, b1;
+        const float w0 = wslot[st * EB + e16];      // 0 for dead entries
+        uint32_t b0[EB / 16], b1[EB / 16];
         if constexpr (ROWS == 1) {
             const int e = exponent_of(__reduce_max_sync(kFullMask, __float_as_uint(w0)));
             if (e > E[0]) {     // keep the sums on the row's current scale
@@ -311,18 +322,21 @@ __device__ __forceinline__ void walk_window(const TcParams &P, const Window<ROWS
             const uint32_t pw = uint32_t(__half_as_ushort(hi)) | (uint32_t(__half_as_ushort(lo)) << 16);
             // B fragment: column 0 = hi, column 1 = lo, columns 2-7 zero; entries
             // 2t, 2t+1 (b0) and 2t+8, 2t+9 (b1).
-            const uint32_t v0 = __shfl_sync(kFullMask, pw, 2 * t);
-            const uint32_t v1 = __shfl_sync(kFullMask, pw, 2 * t + 1);
-            const uint32_t v2 = __shfl_sync(kFullMask, pw, 2 * t + 8);
-            const uint32_t v3 = __shfl_sync(kFullMask, pw, 2 * t + 9);
             const uint32_t sel = g == 0 ? 0x5410u : 0x7632u;
-            b0 = g < 2 ? __byte_perm(v0, v1, sel) : 0u;
-            b1 = g < 2 ? __byte_perm(v2, v3, sel) : 0u;
+#pragma unroll
+            for (int kk = 0; kk < EB / 16; ++kk) {
+                const uint32_t v0 = __shfl_sync(kFullMask, pw, 16 * kk + 2 * t);
+                const uint32_t v1 = __shfl_sync(kFullMask, pw, 16 * kk + 2 * t + 1);
+                const uint32_t v2 = __shfl_sync(kFullMask, pw, 16 * kk + 2 * t + 8);
+                const uint32_t v3 = __shfl_sync(kFullMask, pw, 16 * kk + 2 * t + 9);
+                b0[kk] = g < 2 ? __byte_perm(v0, v1, sel) : 0u;
+                b1[kk] = g < 2 ? __byte_perm(v2, v3, sel) : 0u;
+            }
         } else {
-            const int pos = n * 16 + e16;
+            const int pos = n * EB + e16;
             const int tg = pos < total ? tag_of(w, pos) : ROWS;
-            const int tlo = tag_of(w, n * 16);
-            const int thi = tag_of(w, min(n * 16 + 15, total - 1));
+            const int tlo = tag_of(w, n * EB);
+            const int thi = tag_of(w, min(n * EB + EB - 1, total - 1));
             bool grew = false;
             int Enew[ROWS];
 #pragma unroll
@@ -364,17 +378,22 @@ __device__ __forceinline__ void walk_window(const TcParams &P, const Window<ROWS
                 const uint32_t h = __byte_perm(va, vb, sel);
                 return (ta == sel_row ? (h & 0xffffu) : 0u) | (tb == sel_row ? (h & 0xffff0000u) : 0u);
             };
-            b0 = pair(2 * t);
-            b1 = pair(2 * t + 8);
+#pragma unroll
+            for (int kk = 0; kk < EB / 16; ++kk) {
+                b0[kk] = pair(16 * kk + 2 * t);
+                b1[kk] = pair(16 * kk + 2 * t + 8);
+            }
         }
 
         const uint32_t sa = rows_s + uint32_t(st * G::STAGE) + lofs;
 #pragma unroll
-        for (int T = 0; T < FT; ++T) {
-            uint32_t a[4];
-            ldsm_x4_trans(sa + uint32_t(T * 32), a);
-            mma_16816(acc[T], a, b0, b1);
-        }
+        for (int kk = 0; kk < EB / 16; ++kk)
+#pragma unroll
+            for (int T = 0; T < FT; ++T) {
+                uint32_t a[4];
+                ldsm_x4_trans(sa + uint32_t(kk * 16 * G::PITCH + T * 32), a);
+                mma_16816(acc[T], a, b0[kk], b1[kk]);
+            }
         __syncwarp();           // stage st is refilled in iteration n + 1
         st = st == G::NS - 1 ? 0 : st + 1;
     }
@@ -536,7 +555,7 @@ struct TcPackGemm {
 };
 
 // One light window: rows first .. first + ROWS - 1, leaving out heavy ones.
-template <int FT, int ROWS, int NS, class Epi>
+template <int FT, int ROWS, int NS, int EBLOCK, class Epi>
 __device__ __forceinline__ void light_window(const TcParams &P, const Epi &epi, uint8_t *ring,
                                              int64_t first) {
     Window<ROWS> w;
@@ -573,17 +592,17 @@ __device__ __forceinline__ void light_window(const TcParams &P, const Epi &epi, 
     }
     w.off[ROWS] = pos;
     TcRowSums<FT> s;
-    walk_window<FT, ROWS, NS>(P, w, ring, s);
+    walk_window<FT, ROWS, NS, EBLOCK>(P, w, ring, s);
     epi(out, s);
 }
 
 // Heavy rows (blocks take chunks of 32 rows in turn): every warp of the block
 // walks an eighth of the row's list (a one-row window), and warp 0 adds the
 // eight partial rows in warp order.
-template <int FT, int NS, class Epi>
+template <int FT, int NS, int EBLOCK, class Epi>
 __device__ __forceinline__ void heavy_rows(const TcParams &P, const Epi &epi, uint8_t *ring,
                                            float *part) {
-    using G = TcGeom<FT, NS>;
+    using G = TcGeom<FT, NS, EBLOCK>;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int g = lane >> 2, t = lane & 3;
     for (int64_t base = int64_t(blockIdx.x) * 32; base < P.N;
@@ -613,7 +632,7 @@ __device__ __forceinline__ void heavy_rows(const TcParams &P, const Epi &epi, ui
             w.off[0] = 0;
             w.off[1] = int(q1 - q0);
             TcRowSums<FT> s;
-            walk_window<FT, 1, NS>(P, w, ring, s);
+            walk_window<FT, 1, NS, EBLOCK>(P, w, ring, s);
             if (t == 0) {
 #pragma unroll
                 for (int T = 0; T < FT; ++T) {
@@ -649,7 +668,8 @@ __device__ __forceinline__ void heavy_rows(const TcParams &P, const Epi &epi, ui
 template <int FT, int ROWS, int NS, class Epi>
 __global__ void __launch_bounds__(kTcThreads, 2)
 spmm_tc_kernel(TcParams P, Epi epi) {
-    using G = TcGeom<FT, NS>;
+    constexpr int EB = tc_entries_per_block(FT, ROWS);
+    using G = TcGeom<FT, NS, EB>;
     extern __shared__ __align__(128) uint8_t smem[];
     uint8_t *rings = smem;
     float *part = reinterpret_cast<float *>(smem + kTcWarps * G::WARP);
@@ -664,17 +684,17 @@ spmm_tc_kernel(TcParams P, Epi epi) {
     // persistent blocks does both (a block per window would hold its SM until
     // its longest row ended, most of its warps idle). Few windows: a warp per
     // window, with separate leading blocks for the heavy rows.
-    if (int(blockIdx.x) < P.heavy_blocks) heavy_rows<FT, NS>(P, epi, ring, part);
+    if (int(blockIdx.x) < P.heavy_blocks) heavy_rows<FT, NS, EB>(P, epi, ring, part);
     if (int(blockIdx.x) < P.light_first) return;
     const int64_t windows = (P.N + ROWS - 1) / ROWS;
     for (int64_t wi = int64_t(int(blockIdx.x) - P.light_first) * kTcWarps + warp; wi < windows;
          wi += int64_t(int(gridDim.x) - P.light_first) * kTcWarps)
-        light_window<FT, ROWS, NS>(P, epi, ring, wi * ROWS);
+        light_window<FT, ROWS, NS, EB>(P, epi, ring, wi * ROWS);
 }
 
-template <int FT, int NS>
+template <int FT, int NS, int EB>
 size_t tc_smem(size_t extra_floats) {
-    using G = TcGeom<FT, NS>;
+    using G = TcGeom<FT, NS, EB>;
     return size_t(kTcWarps) * G::WARP + size_t(kTcWarps) * G::FP * 4 + extra_floats * 4;
 }
 
@@ -694,7 +714,7 @@ void launch_rows(const TcParams &P0, const Epi &epi, int slabs, const DeviceInfo
                  cudaStream_t s, bool pdl) {
     TcParams P = P0;
     P.heavy_degree = tc_heavy_degree(P.N, P.nnz);
-    const size_t smem = tc_smem<FT, NS>(Epi::kSmemFloats);
+    const size_t smem = tc_smem<FT, NS, tc_entries_per_block(FT, ROWS)>(Epi::kSmemFloats);
     auto kernel = spmm_tc_kernel<FT, ROWS, NS, Epi>;
     cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
     // One wave of resident blocks, or fewer when the windows do not need them.
