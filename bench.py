@@ -171,9 +171,17 @@ KERNEL_FILES = {"pack_rows": "pack.cu", "pack_weights": "pack.cu", "xnor_gemm": 
                 "L1.spmm+L2.pack_rows+L2.xnor_gemm": "spmm.cu"}
 
 
+def sweep_tensor_core_aggregation(w):
+    """The one-layer entry points keep fp16 dots and aggregate on the tensor
+    cores for K <= 2048 and F <= 128 (csrc/layer.cu)."""
+    return w.K <= 2048 and w.hidden <= 128
+
+
 def kernel_file(name, w=None):
     if w is not None and name in ("L1.spmm+L2.pack_rows+L2.xnor_gemm", "L2.spmm") and \
             tensor_core_aggregation(w):
+        return "spmm_tc.cu"
+    if w is not None and name == "spmm" and w.layers == 1 and sweep_tensor_core_aggregation(w):
         return "spmm_tc.cu"
     return KERNEL_FILES[name]
 
@@ -550,6 +558,11 @@ def run_sweep(args, rank, world, local_rank):
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
     w = inputs.get_workload(args.workload)
+    if args.sweep_nodes:    # a smaller case of the same sweep point (profiler captures)
+        import dataclasses
+        w = dataclasses.replace(w, N=args.sweep_nodes, undirected_edges=8 * args.sweep_nodes,
+                                description=w.description.replace("N=2^20",
+                                                                  f"N={args.sweep_nodes}"))
     N, K, F = w.N, w.K, w.hidden
     gen = torch.Generator(device=dev)
     gen.manual_seed(1000 + w.index)
@@ -587,8 +600,14 @@ def run_sweep(args, rank, world, local_rank):
     hbm = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
     mean_us = [1e3 * statistics.fmean(t) for t in per_kernel]
     words = (K + 63) // 64
-    # The layer keeps Z factored (uint16 dots + a row scale) when K <= 32767.
-    z_bytes = 2.0 * N * ((F + 3) // 4 * 4) + 4.0 * N if K <= 32767 else 4.0 * N * F
+    # The layer keeps Z factored when K <= 32767: fp16 dots in rows padded to
+    # 16 (K <= 2048, F <= 128) or uint16 dots in rows padded to 8, plus a row scale.
+    if sweep_tensor_core_aggregation(w):
+        z_bytes = 2.0 * N * ((F + 15) // 16 * 16) + 4.0 * N
+    elif K <= 32767:
+        z_bytes = 2.0 * N * ((F + 7) // 8 * 8) + 4.0 * N
+    else:
+        z_bytes = 4.0 * N * F
     work = {"pack_rows": (4.0 * N * K + 8.0 * N * words + 4.0 * N, "bytes", "hbm"),
             "pack_weights": (4.0 * K * F + 8.0 * F * words + 4.0 * F, "bytes", "hbm"),
             "xnor_gemm": (float(N) * K * F, "bit-ops", "tensor"),
@@ -621,7 +640,7 @@ def run_sweep(args, rank, world, local_rank):
             "spmm_gbs": work["spmm"][0] / (mean_us[3] * 1e-6) / 1e9},
         "roofline": {"kernel": name, "bound": bound, "achieved": achieved, "peak": peak,
                      "unit": runit, "frac": achieved / peak,
-                     "traffic": profiled_traffic(name, w.name), "peak_source": src},
+                     "traffic": profiled_traffic(name, w.name, w), "peak_source": src},
         "cpu_baseline": None, "e2e": None,
         "note": "sweep point: one layer, kernel-level timing; no host-buffer run (the features "
                 "alone are up to 34 GB)",
@@ -1060,6 +1079,9 @@ def main(argv=None):
     ap.add_argument("--bucket", type=int, default=0, metavar="B",
                     help="time layer 1 with sub-row bucketing, buckets of B features "
                          "(a multiple of 64; bigcn_layer_forward_bucketed) instead")
+    ap.add_argument("--sweep-nodes", type=int, default=0, metavar="N",
+                    help="run a sweep point on N nodes (mean degree 16) instead of 2^20: a "
+                         "smaller case of the same kernels for profiler captures")
     ap.add_argument("--forward-only", type=int, default=0, metavar="R",
                     help="run R plain forwards (no graph, no timing, no output) and exit: "
                          "a fixed launch sequence for profilers")
