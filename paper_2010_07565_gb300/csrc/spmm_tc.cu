@@ -31,10 +31,12 @@
 // holds row t's sums for features 16 T + g and 16 T + g + 8 of every tile T.
 // Gathered rows are staged by cp.async (16 bytes per copy; positions past the
 // end of the stream and out-of-range column indices copy zeros and carry zero
-// weight) in a three-stage ring: the copies of blocks n + 1 and n + 2 and the
-// column indices of blocks n + 3 and n + 4 are in flight while block n is
-// multiplied; the column indices and row scales go through shared memory too,
-// so the loop never waits on a register loaded from global memory.
+// weight) in a per-warp ring of two (or three) blocks, XOR-swizzled so that
+// ldmatrix reads are free of bank conflicts without padding the rows: the
+// copies of the next block(s) are in flight while block n is multiplied, and
+// the column indices, copied two blocks further ahead, and the row scales go
+// through shared memory too, so the loop never waits on a register loaded
+// from global memory.
 //
 // Rows with more than `heavy_degree` neighbours are each walked by all 8 warps
 // of one block, whose fp32 partial rows are added in warp order
@@ -64,14 +66,26 @@ template <int FT, int NSTAGES, int EBLOCK>
 struct TcGeom {
     static constexpr int FP = 16 * FT;             // features per staged row
     static constexpr int CH = 2 * FT;              // 16-byte copies per row
-    static constexpr int PITCH = FP * 2 + 16;      // bytes per staged row (conflict-free ldmatrix)
+    // Bytes per staged row: the row's 32 FT bytes rounded up to a multiple of
+    // 128, its 16-byte chunk c stored at slot c ^ (r & 7) of staged row r. The
+    // eight rows an ldmatrix reads then fall in eight different bank groups,
+    // and the two halves of every 32-byte sector of a gathered row stay in one
+    // aligned 32-byte slot pair (a padded pitch of 32 FT + 16 bytes split a
+    // sector over two shared-memory lines on every other row: 256-byte rows
+    // gathered at 13.7 TB/s instead of 20.6 TB/s, 96-byte rows at 8.8 instead
+    // of 13.0 TB/s, 24 warps per SM).
+    static constexpr int PITCH = (FP * 2 + 127) / 128 * 128;
     static constexpr int EB = EBLOCK;              // entries per block (16 or 32)
     static constexpr int KCH = EB * CH / 32;       // 16-byte row copies per lane and block
     static constexpr int STAGE = EB * PITCH;       // one block of EB entries
-    static constexpr int NS = NSTAGES;             // ring depth (blocks of 16 entries)
-    static constexpr int D = NS - 1;               // blocks copied ahead
-    // one warp's ring: NS row stages, then NS x EB row scales and NS x EB column indices
-    static constexpr int WARP = NS * STAGE + NS * EB * 8;
+    static constexpr int NS = NSTAGES;             // row ring depth (blocks)
+    static constexpr int D = NS - 1;               // blocks of rows copied ahead
+    static constexpr int DI = 2;                   // groups between a block's index copy and its row copy
+    static constexpr int NI = DI + 1;              // index slots
+    // one warp's ring: NS row stages, NS x EB row scales, NI x EB column
+    // indices (a multiple of 128 bytes, so that every stage starts on a
+    // 128-byte line)
+    static constexpr int WARP = (NS * STAGE + NS * EB * 4 + NI * EB * 4 + 127) / 128 * 128;
 };
 
 __device__ __forceinline__ uint32_t smem_addr(const void *p) {
@@ -183,11 +197,13 @@ struct TcRowSums {
 // ring `ring` (shared, TcGeom<FT, NS, EB>::WARP bytes) is free on entry and on exit.
 //
 // Pipeline (blocks of EB positions; lane e = lane mod EB owns position e of a
-// block; with EB = 16 lanes 16-31 repeat lanes 0-15): group n, committed in iteration n,
-// copies block n + D's rows and row scales and block n + 2D's column indices,
-// so iteration n finds block n (rows, scales) and block n + D's indices landed
-// after waiting for all but the last D - 1 groups. No register of the loop
-// waits on a global load. Block b uses ring stage b mod NS.
+// block; with EB = 16 lanes 16-31 repeat lanes 0-15). Group m of cp.async
+// copies holds block m + D's rows and row scales and block m + D + DI's column
+// indices. Iteration n first waits for group n - DI (block n + D's indices),
+// issues group n -- so that its rows are in flight while the warp waits for
+// block n -- then waits for group n - D (block n's rows) and multiplies. No
+// register of the loop waits on a global load. Block b uses row stage b mod NS
+// and index slot b mod NI.
 template <int FT, int ROWS, int NS, int EBLOCK>
 __device__ __forceinline__ void walk_window(const TcParams &P, const Window<ROWS> &w,
                                            uint8_t *ring, TcRowSums<FT> &out) {
@@ -200,31 +216,53 @@ __device__ __forceinline__ void walk_window(const TcParams &P, const Window<ROWS
     const int nblk = (total + EB - 1) / EB;
     const uint32_t rows_s = smem_addr(ring);
     float *wslot = reinterpret_cast<float *>(ring + G::NS * G::STAGE);   // NS x EB scales
-    int *cslot = reinterpret_cast<int *>(wslot + G::NS * EB);            // NS x EB indices
+    int *cslot = reinterpret_cast<int *>(wslot + G::NS * EB);            // NI x EB indices
     const uint32_t wslot_s = smem_addr(wslot), cslot_s = smem_addr(cslot);
-    // Copy plan of one block's rows: chunk c = lane + 32 k -> row c / CH, piece
-    // c % CH (for CH a power of two: row lane / CH + k 32 / CH, piece lane % CH,
-    // so the destinations differ by constants).
-    int crow[G::KCH], cpo[G::KCH];
-    uint32_t cdst[G::KCH];
+    const uint32_t n32 = uint32_t(P.N);     // N <= INT32_MAX
+    // Copy plan of one block's rows: chunk q = lane + 32 k -> row q / CH, piece
+    // q % CH, stored at slot piece ^ (row & 7) of the staged row. For CH a power
+    // of two a lane's rows are r0 + k S (S = 32 / CH) and its slots repeat with
+    // period 8 / S, so only that many destinations are kept.
+    constexpr bool kPow2 = (G::CH & (G::CH - 1)) == 0;
+    constexpr int kStep = kPow2 ? 32 / G::CH : 0;
+    constexpr int kPer = kPow2 ? (kStep >= 8 ? 1 : 8 / kStep) : G::KCH;
+    constexpr int kArr = kPow2 ? 1 : G::KCH;
+    int crow[kArr], cpo[kArr];
+    uint32_t cdst[kPer];
+    if constexpr (kPow2) {
+        const int r0 = lane / G::CH, piece = lane % G::CH;
+        crow[0] = r0;
+        cpo[0] = piece * 16;
 #pragma unroll
-    for (int k = 0; k < G::KCH; ++k) {
-        if constexpr ((G::CH & (G::CH - 1)) == 0) {
-            crow[k] = lane / G::CH + k * (32 / G::CH);
-            cpo[k] = (lane % G::CH) * 16;
-        } else {
+        for (int m = 0; m < kPer; ++m)
+            cdst[m] = uint32_t(r0 * G::PITCH + ((piece ^ ((r0 + m * kStep) & 7)) * 16));
+    } else {
+#pragma unroll
+        for (int k = 0; k < G::KCH; ++k) {
+            const int piece = (lane + 32 * k) % G::CH;
             crow[k] = (lane + 32 * k) / G::CH;
-            cpo[k] = ((lane + 32 * k) % G::CH) * 16;
+            cpo[k] = piece * 16;
+            cdst[k] = uint32_t(crow[k] * G::PITCH + ((piece ^ (crow[k] & 7)) * 16));
         }
-        cdst[k] = uint32_t(crow[k] * G::PITCH + cpo[k]);
     }
+    auto plan_row = [&](int k) { return kPow2 ? crow[0] + k * kStep : crow[k]; };
+    auto plan_src = [&](int k) { return kPow2 ? cpo[0] : cpo[k]; };
+    auto plan_dst = [&](int k) {
+        return kPow2 ? cdst[k % kPer] + uint32_t(k * kStep * G::PITCH) : cdst[k];
+    };
     const char *Dbytes = reinterpret_cast<const char *>(P.D) +
                          2 * (int64_t(P.f_base) + int64_t(blockIdx.y) * G::FP);
     const uint32_t row_bytes = uint32_t(P.ldd) * 2u;
-    // ldmatrix address of this lane within a stage: matrices (entries 0-7 |
-    // 8-15) x (features 0-7 | 8-15) of a tile.
-    const uint32_t lofs =
-        uint32_t(((lane & 7) + 8 * (lane >> 4)) * G::PITCH + ((lane >> 3) & 1) * 16);
+    // ldmatrix addresses of this lane: matrices (entries 0-7 | 8-15) x
+    // (features 0-7 | 8-15) of a tile; lane l supplies entry e = (l & 7) +
+    // 8 (l >> 4), chunk c = 2 T + b with b = (l >> 3) & 1, stored at slot
+    // c ^ (e & 7) = 2 (T ^ y) + (b ^ x0) with x0 = l & 1, y = (l >> 1) & 3.
+    // Stages start on 128-byte lines and the row pitch is a multiple of 128,
+    // so the address is ((stage + tl) ^ 32 (T & 3)) + 128 (T >> 2) with
+    // tl = e PITCH + 16 (b ^ x0) + 32 y.
+    constexpr int kTq = FT < 4 ? FT : 4;
+    const uint32_t tl = uint32_t(((lane & 7) + 8 * (lane >> 4)) * G::PITCH +
+                                 16 * (((lane >> 3) & 1) ^ (lane & 1)) + 32 * ((lane >> 1) & 3));
 
     // Block b's column indices -> index slot `st` (zeros for self / dead entries).
     auto copy_cols = [&](int b, int st) {
@@ -243,27 +281,30 @@ __device__ __forceinline__ void walk_window(const TcParams &P, const Window<ROWS
         const int p = b * EB + e16;
         if (p >= total) return -1;
         const int tg = tag_of(w, p);
-        const int64_t j = p == pick<ROWS>(w.selfp, tg) ? pick<ROWS>(w.row, tg)
-                                                        : int64_t(cslot[st * EB + e16]);
-        return (j >= 0 && j < P.N) ? int(j) : -1;
+        const int j = p == pick<ROWS>(w.selfp, tg) ? int(pick<ROWS>(w.row, tg))
+                                                    : cslot[st * EB + e16];
+        return uint32_t(j) < n32 ? j : -1;
     };
-    // A block's rows and row scales (column j per lane) -> stage `st`.
+    // A block's rows and row scales (column j per lane; -1: dead) -> stage `st`.
+    // Dead entries copy zeros and read nothing (pointing them all at one real
+    // row instead made that row's L2 line a hot spot: 2.7 -> 4.5 ms on the
+    // Reddit-shaped graph).
     auto copy_rows = [&](int st, int j) {
         const uint32_t base = rows_s + uint32_t(st * G::STAGE);
         if (P.off32) {          // each lane's row byte offset, shuffled once per copy
             const uint32_t ro = j >= 0 ? uint32_t(j) * row_bytes : 0xffffffffu;
 #pragma unroll
             for (int k = 0; k < G::KCH; ++k) {
-                const uint32_t r = __shfl_sync(kFullMask, ro, crow[k]);
+                const uint32_t r = __shfl_sync(kFullMask, ro, plan_row(k));
                 const bool live = r != 0xffffffffu;
-                cp_async16(base + cdst[k], Dbytes + (live ? r : 0u) + cpo[k], live);
+                cp_async16(base + plan_dst(k), Dbytes + (live ? r : 0u) + plan_src(k), live);
             }
         } else {
 #pragma unroll
             for (int k = 0; k < G::KCH; ++k) {
-                const int jj = __shfl_sync(kFullMask, j, crow[k]);
-                cp_async16(base + cdst[k], Dbytes + int64_t(jj >= 0 ? jj : 0) * row_bytes + cpo[k],
-                           jj >= 0);
+                const int jj = __shfl_sync(kFullMask, j, plan_row(k));
+                cp_async16(base + plan_dst(k),
+                           Dbytes + int64_t(jj >= 0 ? jj : 0) * row_bytes + plan_src(k), jj >= 0);
             }
         }
         if (lane < EB)
@@ -282,26 +323,30 @@ __device__ __forceinline__ void walk_window(const TcParams &P, const Window<ROWS
 #pragma unroll
     for (int r = 0; r < ROWS; ++r) E[r] = kNoScale;
 
-    // Prologue: the groups of iterations -D .. -1 (blocks 0 .. D-1 with their
-    // indices read directly, the index copies of blocks D .. 2D-1).
+    // Prologue: groups -DI .. -1 (the index copies of blocks D .. D + DI - 1;
+    // from group -D on also the rows of blocks 0 .. D - 1, whose indices are
+    // read directly).
 #pragma unroll
-    for (int k = 0; k < G::D; ++k) {
-        copy_cols(G::D + k, (G::D + k) % G::NS);
-        copy_rows(k, fetch_col(P, w, EB * k + e16));
+    for (int m = -G::DI; m < 0; ++m) {
+        if (m + G::D >= 0) copy_rows(m + G::D, fetch_col(P, w, EB * (m + G::D) + e16));
+        copy_cols(m + G::D + G::DI, (m + G::D + G::DI) % G::NI);
         cp_async_commit();
     }
 
-    int st = 0;                 // stage of block n (n mod NS)
+    int st = 0;                             // row stage of block n (n mod NS)
+    int si = G::D % G::NI;                  // index slot of block n + D
     for (int n = 0; n < nblk; ++n) {
-        const int stD = st == 0 ? G::NS - 1 : st - 1;       // block n + D (and n - 1)
-        const int st2D = stD == 0 ? G::NS - 1 : stD - 1;    // block n + 2D's indices
-        cp_async_wait<G::D - 1>();  // group n - D: block n, and block n + D's indices
+        const int stD = st == 0 ? G::NS - 1 : st - 1;       // row stage of block n + D (= n - 1)
+        const int siI = si == 0 ? G::NI - 1 : si - 1;       // index slot of block n + D + DI
+        cp_async_wait<G::DI - 1>();     // group n - DI: block n + D's indices
         __syncwarp();
-        const int jD = column(n + G::D, stD);
-        __syncwarp();           // every lane has read index slot stD before it is reused
+        const int jD = column(n + G::D, si);
+        __syncwarp();           // every lane has read index slot si before it is reused
         copy_rows(stD, jD);
-        copy_cols(n + 2 * G::D, st2D);
+        copy_cols(n + G::D + G::DI, siI);
         cp_async_commit();
+        cp_async_wait<G::D>();          // group n - D: block n's rows and scales
+        __syncwarp();
 
         // This block's weights and the scale exponent of each row they belong to.
         const float w0 = wslot[st * EB + e16];      // 0 for dead entries
@@ -385,17 +430,21 @@ __device__ __forceinline__ void walk_window(const TcParams &P, const Window<ROWS
             }
         }
 
-        const uint32_t sa = rows_s + uint32_t(st * G::STAGE) + lofs;
+        const uint32_t sl = rows_s + uint32_t(st * G::STAGE) + tl;
+        uint32_t tq[kTq];
+#pragma unroll
+        for (int m = 0; m < kTq; ++m) tq[m] = sl ^ uint32_t(32 * m);
 #pragma unroll
         for (int kk = 0; kk < EB / 16; ++kk)
 #pragma unroll
             for (int T = 0; T < FT; ++T) {
                 uint32_t a[4];
-                ldsm_x4_trans(sa + uint32_t(kk * 16 * G::PITCH + T * 32), a);
+                ldsm_x4_trans(tq[T & 3] + uint32_t(kk * 16 * G::PITCH + 128 * (T >> 2)), a);
                 mma_16816(acc[T], a, b0[kk], b1[kk]);
             }
         __syncwarp();           // stage st is refilled in iteration n + 1
         st = st == G::NS - 1 ? 0 : st + 1;
+        si = si == G::NI - 1 ? 0 : si + 1;
     }
     cp_async_wait<0>();         // the ring is idle before the next window
     __syncwarp();
@@ -598,13 +647,15 @@ __device__ __forceinline__ void light_window(const TcParams &P, const Epi &epi, 
 
 // Heavy rows (blocks take chunks of 32 rows in turn): every warp of the block
 // walks an eighth of the row's list (a one-row window), and warp 0 adds the
-// eight partial rows in warp order.
+// eight partial rows in warp order. A warp's partial row goes to the start of
+// its own ring, which is idle between walks.
 template <int FT, int NS, int EBLOCK, class Epi>
-__device__ __forceinline__ void heavy_rows(const TcParams &P, const Epi &epi, uint8_t *ring,
-                                           float *part) {
+__device__ __forceinline__ void heavy_rows(const TcParams &P, const Epi &epi, uint8_t *rings) {
     using G = TcGeom<FT, NS, EBLOCK>;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int g = lane >> 2, t = lane & 3;
+    uint8_t *ring = rings + warp * G::WARP;
+    auto part = [&](int q) { return reinterpret_cast<float *>(rings + q * G::WARP); };
     for (int64_t base = int64_t(blockIdx.x) * 32; base < P.N;
          base += int64_t(P.heavy_blocks) * 32) {
         const int64_t r = base + lane;
@@ -636,8 +687,8 @@ __device__ __forceinline__ void heavy_rows(const TcParams &P, const Epi &epi, ui
             if (t == 0) {
 #pragma unroll
                 for (int T = 0; T < FT; ++T) {
-                    part[warp * G::FP + 16 * T + g] = s.v[T][0];
-                    part[warp * G::FP + 16 * T + g + 8] = s.v[T][1];
+                    part(warp)[16 * T + g] = s.v[T][0];
+                    part(warp)[16 * T + g + 8] = s.v[T][1];
                 }
             }
             __syncthreads();
@@ -647,7 +698,7 @@ __device__ __forceinline__ void heavy_rows(const TcParams &P, const Epi &epi, ui
 #pragma unroll
                     for (int h = 0; h < 2; ++h) {
                         float a = 0.0f;
-                        for (int q = 0; q < kTcWarps; ++q) a += part[q * G::FP + 16 * T + g + 8 * h];
+                        for (int q = 0; q < kTcWarps; ++q) a += part(q)[16 * T + g + 8 * h];
                         s.v[T][h] = a;
                     }
                 TcRows out;
@@ -660,20 +711,24 @@ __device__ __forceinline__ void heavy_rows(const TcParams &P, const Epi &epi, ui
                 }
                 epi(out, s);
             }
-            __syncthreads();    // part[] is rewritten by the next heavy row
+            __syncthreads();    // the rings are walked again by the next heavy row
         }
     }
 }
 
+// Blocks per SM the kernel is compiled for: three with two-stage rings (at
+// most 80 registers a thread), two with three stages.
+constexpr int tc_min_blocks(int NS) { return NS == 2 ? 3 : 2; }
+
 template <int FT, int ROWS, int NS, class Epi>
-__global__ void __launch_bounds__(kTcThreads, 2)
+__global__ void __launch_bounds__(kTcThreads, tc_min_blocks(NS))
 spmm_tc_kernel(TcParams P, Epi epi) {
     constexpr int EB = tc_entries_per_block(FT, ROWS);
     using G = TcGeom<FT, NS, EB>;
     extern __shared__ __align__(128) uint8_t smem[];
-    uint8_t *rings = smem;
-    float *part = reinterpret_cast<float *>(smem + kTcWarps * G::WARP);
-    float *extra = part + kTcWarps * G::FP;
+    // The rings start on a 128-byte line (the ldmatrix addressing relies on it).
+    uint8_t *rings = smem + ((128u - (smem_addr(smem) & 127u)) & 127u);
+    float *extra = reinterpret_cast<float *>(rings + kTcWarps * G::WARP);
     grid_dependency_wait();     // the dots and row scales come from the previous kernel
     epi.prologue(extra);
     __syncthreads();
@@ -684,7 +739,7 @@ spmm_tc_kernel(TcParams P, Epi epi) {
     // persistent blocks does both (a block per window would hold its SM until
     // its longest row ended, most of its warps idle). Few windows: a warp per
     // window, with separate leading blocks for the heavy rows.
-    if (int(blockIdx.x) < P.heavy_blocks) heavy_rows<FT, NS, EB>(P, epi, ring, part);
+    if (int(blockIdx.x) < P.heavy_blocks) heavy_rows<FT, NS, EB>(P, epi, rings);
     if (int(blockIdx.x) < P.light_first) return;
     const int64_t windows = (P.N + ROWS - 1) / ROWS;
     for (int64_t wi = int64_t(int(blockIdx.x) - P.light_first) * kTcWarps + warp; wi < windows;
@@ -695,7 +750,9 @@ spmm_tc_kernel(TcParams P, Epi epi) {
 template <int FT, int NS, int EB>
 size_t tc_smem(size_t extra_floats) {
     using G = TcGeom<FT, NS, EB>;
-    return size_t(kTcWarps) * G::WARP + size_t(kTcWarps) * G::FP * 4 + extra_floats * 4;
+    static_assert(G::FP * 4 <= G::WARP, "a warp's partial row must fit its ring");
+    static_assert(G::WARP % 16 == 0, "rings must keep 16-byte alignment");
+    return 128 + size_t(kTcWarps) * G::WARP + extra_floats * 4;
 }
 
 // Rows per light window: one when rows are long (a window's blocks then all
@@ -747,12 +804,14 @@ void launch_rows(const TcParams &P0, const Epi &epi, int slabs, const DeviceInfo
 template <int FT, class Epi>
 void launch_ft(const TcParams &P, const Epi &epi, const DeviceInfo &dev, cudaStream_t s,
                bool pdl, int slabs = 1) {
-    // Three stages: deeper rings (up to 12 KB per warp for narrow rows) were
-    // measured slower on the Reddit-shaped graph (layer 2: 2.04 -> 2.19 ms);
-    // the walk is bound by L2 sector throughput and issue, not by the bytes a
-    // warp keeps in flight.
-    if (tc_rows(P.N, P.nnz) == 1) launch_rows<FT, 1, 3>(P, epi, slabs, dev, s, pdl);
-    else launch_rows<FT, kTcRows, 3>(P, epi, slabs, dev, s, pdl);
+    // Two-stage rings and three blocks (24 warps) per SM: on the Reddit-shaped
+    // graph 3109 -> 3000 us (layer 1) and 1927 -> 1869 us (layer 2) against
+    // three stages at two blocks per SM; four-row windows 846 -> 782 us (2^20
+    // nodes of mean degree 16, 64 features). Four-row windows of more than 64
+    // features keep three stages: at 80 registers they would spill.
+    constexpr int kNs4 = FT <= 4 ? 2 : 3;
+    if (tc_rows(P.N, P.nnz) == 1) launch_rows<FT, 1, 2>(P, epi, slabs, dev, s, pdl);
+    else launch_rows<FT, kTcRows, kNs4>(P, epi, slabs, dev, s, pdl);
 }
 
 }  // namespace
