@@ -8,6 +8,9 @@
 //     and the loaded words are summed so that nothing is dead code;
 //   - cp.async gathers: the same rows copied 16 bytes per lane into a
 //     per-warp shared-memory buffer (two stages), then read back and summed;
+//   - cp.async gathers into staged rows of a given pitch, plain or with the
+//     16-byte chunk c of staged row r at slot c ^ (r & 7) (the layout the
+//     tensor-core aggregation reads with ldmatrix), 24 warps per SM;
 //   - the warp-level f16 tensor-core MMA (m16n8k16, fp32 accumulate), the
 //     instruction a tensor-core form of the aggregation would issue.
 // Every index lies in [0, rows) and every row lies inside the buffer, so all
@@ -146,6 +149,58 @@ gather_cpasync(const uint8_t *__restrict__ buf, int64_t pitch, const int *__rest
     out[blockIdx.x * kThreads + threadIdx.x] = acc;
 }
 
+
+// cp.async gathers of ROWB-byte rows into staged rows PITCH bytes apart: a
+// warp stages R rows per step in S steps' worth of buffers; chunk q = lane +
+// 32 k of a step -> row q / (ROWB / 16), chunk q % (ROWB / 16), stored at slot
+// chunk (SWZ = 0) or chunk ^ (row & 7) (SWZ = 1).
+template <int R, int S, int ROWB, int PITCH, int SWZ>
+__global__ void __launch_bounds__(kThreads)
+gather_staged(const uint8_t *__restrict__ buf, const int *__restrict__ idx, int64_t per_warp,
+              float *out) {
+    extern __shared__ __align__(16) uint8_t smem[];
+    constexpr int CH = ROWB / 16;
+    constexpr int kStage = R * PITCH;
+    constexpr int KCH = R * CH / 32;
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    uint8_t *mine = smem + wid * S * kStage;
+    const uint32_t base_s = uint32_t(__cvta_generic_to_shared(mine));
+    const int64_t warp = (int64_t(blockIdx.x) * kThreads + threadIdx.x) >> 5;
+    const int *my = idx + warp * per_warp;
+    float acc = 0.0f;
+    const int64_t steps = per_warp / R;
+    auto issue = [&](int64_t st) {
+        const int j = lane < R ? __ldg(my + st * R + lane) : 0;
+        const uint32_t dst = base_s + uint32_t(st % S) * kStage;
+#pragma unroll
+        for (int k = 0; k < KCH; ++k) {
+            const int q = lane + 32 * k, r = q / CH, c = q % CH;
+            const int jj = __shfl_sync(0xffffffffu, j, r);
+            const int slot = SWZ ? (c ^ (r & 7)) : c;
+            cp_async16(dst + uint32_t(r * PITCH + slot * 16), buf + int64_t(jj) * ROWB + c * 16);
+        }
+        asm volatile("cp.async.commit_group;");
+    };
+    for (int s = 0; s < S - 1; ++s)
+        if (s < steps) issue(s);
+        else asm volatile("cp.async.commit_group;");
+    for (int64_t st = 0; st < steps; ++st) {
+        if (st + S - 1 < steps) issue(st + S - 1);
+        else asm volatile("cp.async.commit_group;");
+        asm volatile("cp.async.wait_group %0;" ::"n"(S - 1));
+        __syncwarp();
+        const float4 *s = reinterpret_cast<const float4 *>(mine + (st % S) * kStage);
+#pragma unroll
+        for (int q = lane; q < kStage / 16; q += 32) {
+            const float4 v = s[q];
+            acc += (v.x + v.y) + (v.z + v.w);
+        }
+        __syncwarp();
+    }
+    asm volatile("cp.async.wait_group 0;");
+    out[blockIdx.x * kThreads + threadIdx.x] = acc;
+}
+
 // Warp-level f16 MMA m16n8k16 with fp32 accumulators: 8 independent chains.
 __global__ void __launch_bounds__(kThreads) mma_f16(const uint32_t *in, float *out, int iters) {
     const int lane = threadIdx.x & 31;
@@ -232,6 +287,25 @@ void run_cpasync(Ctx &c, int64_t ws_bytes, int64_t nidx) {
            ws_bytes / 1e6, occ, ms, gathered / ms / 1e6);
 }
 
+template <int R, int S, int ROWB, int PITCH, int SWZ>
+void run_staged(Ctx &c, int64_t ws_bytes, int64_t nidx) {
+    const int64_t rows = ws_bytes / ROWB;
+    const int smem = (kThreads / 32) * S * R * PITCH;
+    auto k = gather_staged<R, S, ROWB, PITCH, SWZ>;
+    CK(cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+    int occ = 0;
+    CK(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k, kThreads, smem));
+    const int blocks = c.sms * occ;
+    const int64_t warps = int64_t(blocks) * (kThreads / 32);
+    const int64_t per_warp = (nidx / warps) / 32 * 32;
+    fill_idx<<<1024, 256>>>(c.idx, warps * per_warp, rows, 31);
+    const float ms = best_ms(c, [&] { k<<<blocks, kThreads, smem>>>(c.buf, c.idx, per_warp, c.out); });
+    const double gathered = double(warps * per_warp) * ROWB;
+    printf("cp.async row %4d B  staged pitch %3d B  swizzle %d  set %7.1f MB  blocks/SM %d: %8.3f ms"
+           "  gathered %7.0f GB/s\n",
+           ROWB, PITCH, SWZ, ws_bytes / 1e6, occ, ms, gathered / ms / 1e6);
+}
+
 int main() {
     Ctx c;
     CK(cudaDeviceGetAttribute(&c.sms, cudaDevAttrMultiProcessorCount, 0));
@@ -262,6 +336,13 @@ int main() {
         run_ldg<16, 512, 4>(c, ws, nidx);
         run_cpasync(c, ws, nidx);
     }
+    // Staged layouts (two steps of 16 or 32 rows per warp, as many blocks per SM as fit).
+    const int64_t ws63 = int64_t(60) << 20, ws25 = int64_t(24) << 20;
+    run_staged<16, 2, 256, 256, 0>(c, ws63, nidx);
+    run_staged<16, 2, 256, 272, 0>(c, ws63, nidx);
+    run_staged<16, 2, 256, 256, 1>(c, ws63, nidx);
+    run_staged<32, 2, 96, 112, 0>(c, ws25, nidx);
+    run_staged<32, 2, 96, 128, 1>(c, ws25, nidx);
 
     uint32_t *in;
     CK(cudaMalloc(&in, 256 * sizeof(uint32_t)));
