@@ -500,7 +500,10 @@ TC_CASES = [(128, 32, 128), (129, 33, 129), (300, 64, 200), (1000, 128, 1000),
 
 @pytest.mark.parametrize("N,F,K", TC_CASES)
 def test_xnor_gemm_tensor_core_path(cuda_device, N, F, K):
-    """K >= 128 and F >= 32 take the tcgen05 FP8 path: dots must still be exact."""
+    """Shapes at and around the tensor-core product's K and F thresholds with
+    fewer 128-row tiles than SMs, which the POPC kernel takes: dots exact at
+    +-K. The tcgen05 kernels themselves, at the row counts that select them:
+    test_gpu_tc_product.py."""
     g = rng(N + 7 * F + 13 * K)
     SF, SB = random_signs(g, N, K), random_signs(g, F, K)
     if N >= 2 and F >= 2:
