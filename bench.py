@@ -277,17 +277,22 @@ def build_workload(name):
 
 
 def oracle_block_nodes(w, data, budget_s):
-    """Nodes of a block whose induced subgraph the CPU oracle's 2-layer
-    forward finishes in about a third of ``budget_s`` (calibrated on a
-    256-node block; the whole graph if that is smaller)."""
+    """Nodes of a block (the first n nodes, their induced subgraph) whose CPU
+    oracle 2-layer forward takes at most about ``budget_s``: the block is
+    doubled from 256 nodes while four times the last measured time still fits
+    (an induced subgraph's edges grow with the square of its nodes, so a
+    per-node rate from a small block would overshoot on dense graphs)."""
     import oracle
-    cal = min(w.N, 256)
-    rp, ci = induced_subgraph(data["rowptr"], data["colidx"], 0, cal)
-    t0 = time.perf_counter()
-    oracle.forward_2layer(np.ascontiguousarray(data["X"][:cal]), data["s"], data["t"],
-                          data["W1"], data["W2"], rp, ci)
-    per_node = max((time.perf_counter() - t0) / cal, 1e-9)
-    return int(max(cal, min(w.N, budget_s / 3.0 / per_node)))
+    n = min(w.N, 256)
+    while True:
+        rp, ci = induced_subgraph(data["rowptr"], data["colidx"], 0, n)
+        t0 = time.perf_counter()
+        oracle.forward_2layer(np.ascontiguousarray(data["X"][:n]), data["s"], data["t"],
+                              data["W1"], data["W2"], rp, ci)
+        t = time.perf_counter() - t0
+        if n >= w.N or 4.0 * t > budget_s:
+            return n
+        n = min(w.N, 2 * n)
 
 
 def time_oracle(w, data, budget_s, rows=None):
@@ -319,15 +324,9 @@ def run_reference(args, rank, world):
         return 0
     import oracle
     w, data = build_workload(args.workload)
-    # seconds per node of the oracle, from a small calibration block
-    cal = min(w.N, 128)
-    rp, ci = induced_subgraph(data["rowptr"], data["colidx"], 0, cal)
-    t0 = time.perf_counter()
-    oracle.forward_2layer(np.ascontiguousarray(data["X"][:cal]), data["s"], data["t"],
-                          data["W1"], data["W2"], rp, ci)
-    sec_per_node = (time.perf_counter() - t0) / cal
-    per_step = 150.0 / max(args.steps + args.warmup, 1)
-    n = int(max(16, min(w.N, per_step / max(sec_per_node, 1e-9))))
+    # the largest block (by doubling) whose forward fits a step's share of
+    # about two and a half minutes
+    n = oracle_block_nodes(w, data, 150.0 / max(args.steps + args.warmup, 1))
     times = []
     for step in range(args.warmup + args.steps):
         lo = (step * n) % max(w.N - n + 1, 1)
@@ -424,6 +423,23 @@ def run_gpu(args, rank, world, local_rank):
             for k in range(len(names)):
                 per_kernel[k].append(kev[k].elapsed_time(kev[k + 1]))
 
+    # The chain's launch and dependency latency: the same CUDA-graph forward
+    # (same widths) on a one-node graph without edges.
+    floor = GCN2Forward(1, w.K, w.hidden, w.out, 0, dev)
+    floor.load(non_blocking=False, X=host["X"][:1], s=host["s"], t=host["t"], W1=host["W1"],
+               W2=host["W2"], rowptr=torch.zeros(2, dtype=torch.int64))
+    floor.capture()
+    for _ in range(20):
+        floor.replay()
+    torch.cuda.synchronize()
+    floor_ms = []
+    for _ in range(200):
+        ea.record()
+        floor.replay()
+        eb.record()
+        eb.synchronize()
+        floor_ms.append(ea.elapsed_time(eb))
+
     # End to end through host buffers: pinned inputs -> device, forward, logits -> host.
     logits_host = torch.empty((w.N, w.out), dtype=torch.float32).pin_memory()
     h2d = sum(int(v.numel() * v.element_size()) for v in host.values())
@@ -515,7 +531,12 @@ def run_gpu(args, rank, world, local_rank):
                                           "repeat are served from L2, so this can exceed HBM",
             "per_kernel_us": {r["name"]: round(r["mean_us"], 3) for r in kernels},
             "per_kernel_note": "from a second pass of the same graph with an event node "
-                               "between kernels (each node adds a few us)"},
+                               "between kernels (each node adds a few us)",
+            "latency_floor": {"us": 1e3 * statistics.median(floor_ms),
+                              "kernels": len(floor.kernel_names),
+                              "note": "median step of the same CUDA-graph forward on a one-node "
+                                      "graph without edges (same widths): the launch and "
+                                      "dependency latency of the kernel chain"}},
         "roofline": {"kernel": dom["name"], "bound": dom["bound"],
                      "achieved": achieved, "peak": peak, "unit": unit, "frac": achieved / peak,
                      "traffic": traffic,
