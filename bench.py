@@ -214,6 +214,42 @@ def profiled_traffic(name, workload, w=None):
         return None
 
 
+def sources_hash(files):
+    """sha-256 (16 hex digits) of the listed kernel source files, in order."""
+    h = hashlib.sha256()
+    for f in files:
+        with open(os.path.join(ROOT, "paper_2010_07565_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def profile_file_traffic(fname, files):
+    """DRAM bytes per launch from profiles/<fname> if its 'source_sha256_16'
+    is the hash of the listed sources as they are now; else None."""
+    path = os.path.join(ROOT, "profiles", fname)
+    if not os.path.exists(path):
+        return None
+    fields = {}
+    with open(path) as f:
+        for line in f:
+            if ":" in line:
+                k, v = line.split(":", 1)
+                fields[k.strip()] = v.strip()
+    if fields.get("source_sha256_16", "").split(" ")[0] != sources_hash(files):
+        return None
+    try:
+        return float(fields["dram_bytes_per_launch"].split(" ")[0])
+    except (KeyError, ValueError):
+        return None
+
+
+INDUCTIVE_SOURCES = {
+    "gcn": ["inductive.cu", "pack.cu", "xnor_gemm.cu", "xnor_gemm_tc.cu", "layer.cu", "spmm_tc.cu"],
+    "mean": ["inductive.cu", "pack.cu", "xnor_gemm.cu", "xnor_gemm_tc.cu", "spmm.cu"],
+    "sage": ["inductive.cu", "pack.cu", "xnor_gemm.cu", "xnor_gemm_tc.cu", "spmm.cu"]}
+BACKWARD_SOURCES = ["backward.cu", "pack.cu", "spmm.cu", "ablation.cu"]
+
+
 class ClockSampler:
     """nvidia-smi clock / throttle samples every ``interval_ms`` while running
     (the bench opens it before the warm-up steps, so that short timed regions
@@ -742,7 +778,10 @@ def run_backward(args, rank, world, local_rank):
                                "time)", "bound": "tensor", "achieved": achieved,
                      "peak": tc_peak,
                      "unit": "TFLOP/s (2 N K F per product; fp32-accurate = 3 bf16 MMAs)",
-                     "frac": achieved / tc_peak, "traffic": None,
+                     "frac": achieved / tc_peak,
+                     "traffic": profile_file_traffic(f"backward_step_{w.name}.txt",
+                                                     BACKWARD_SOURCES),
+                     "traffic_note": "DRAM bytes of one whole call (its 9 kernels)",
                      "peak_source": f"{peak_kind} MEASURED_PEAKS.json bf16_tflops / 3"},
         "cpu_baseline": None, "e2e": None, "gpu_launches": 9 * args.steps,
         "clocks": clocks.summary(),
@@ -860,7 +899,9 @@ def run_ablation(args, rank, world, local_rank):
                 "unit": "TFLOP/s (2 N K F; fp32-accurate = 3 bf16 MMAs per multiply-add)",
                 "peak_source": f"{peak_kind} MEASURED_PEAKS.json bf16_tflops / 3"}
     roof.update({"kernel": f"product ({'Y W~' if mode == 'weights' else 'H~ W'})",
-                 "frac": roof["achieved"] / roof["peak"], "traffic": None,
+                 "frac": roof["achieved"] / roof["peak"],
+                 "traffic": profile_file_traffic(f"ablation_product_{mode}_{w.name}.txt",
+                                                 ["ablation.cu"]),
                  "other_bound_frac": (t_tc if roof["bound"] == "hbm" else t_hbm) / prod_s})
     line = {
         "metric": f"Bi-GCN ablation layer fwd nodes/s ({mode} binarized only)",
@@ -957,7 +998,10 @@ def run_inductive(args, rank, world, local_rank):
                              "product, aggregation" + (", plus the weight concatenation copies"
                                                        if agg == "sage" else "") + ")"},
         "roofline": {"kernel": "whole layer", "bound": "hbm", "achieved": achieved, "peak": hbm,
-                     "unit": "GB/s", "frac": achieved / hbm, "traffic": None,
+                     "unit": "GB/s", "frac": achieved / hbm,
+                     "traffic": profile_file_traffic(f"inductive_layer_{agg}_{w.name}.txt",
+                                                     INDUCTIVE_SOURCES[agg]),
+                     "traffic_note": "DRAM bytes of one whole call (its 4 kernels)",
                      "peak_source": f"{peak_kind} MEASURED_PEAKS.json hbm_gbs",
                      "algorithmic_bytes": layer_bytes},
         "cpu_baseline": None, "e2e": None, "gpu_launches": 4 * args.steps,
@@ -1053,7 +1097,8 @@ def run_bucketed(args, rank, world, local_rank):
                        "layer_us": 1e3 * statistics.fmean(layer_ms)},
         "roofline": {"kernel": "bucketed product", "bound": "alu", "achieved": achieved,
                      "peak": peak, "unit": "T bit-ops/s (N K F)", "frac": achieved / peak,
-                     "traffic": None,
+                     "traffic": profile_file_traffic(f"bucketed_product_B{Bk}_{w.name}.txt",
+                                                     ["bucket.cu"]),
                      "peak_source": f"measured {POPC_PER_CLK_PER_SM} POPC/clk/SM x 32 bits x "
                                     f"{sms} SMs x {sm_max:.0f} MHz"},
         "cpu_baseline": None, "e2e": None, "gpu_launches": 4 * args.steps,
