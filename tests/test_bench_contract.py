@@ -72,3 +72,46 @@ def test_cuda_arm_fails_without_a_gpu():
     r = run([BENCH, "--workload", "C1", "--steps", "1", "--warmup", "3"])
     assert r.returncode != 0
     assert not json_lines(r.stdout)
+
+
+def _profile_fields(path):
+    fields = {}
+    with open(path) as f:
+        for line in f:
+            if ":" in line:
+                k, v = line.split(":", 1)
+                fields[k.strip()] = v.strip()
+    return fields
+
+
+def test_kernel_profiles_name_their_command_sources_and_traffic():
+    """Every committed per-kernel ncu summary gives the full command (ncu with
+    --clock-control none after a plain run of the same command), the source
+    files it was taken on with their hash, and the DRAM bytes per launch."""
+    import glob
+    paths = [p for p in glob.glob(os.path.join(ROOT, "profiles", "*.txt"))
+             if "source_sha256_16" in _profile_fields(p)]
+    assert len(paths) >= 20
+    for p in paths:
+        f = _profile_fields(p)
+        cmd = f.get("command", "")
+        assert "ncu" in cmd and "--clock-control none" in cmd, p
+        assert cmd.split("&&")[0].strip().startswith("python bench.py"), p
+        assert "source_file" in f or "source_files" in f, p
+        assert float(f["dram_bytes_per_launch"].split(" ")[0]) > 0, p
+
+
+def test_profile_traffic_needs_the_current_source(monkeypatch):
+    """bench.py reports a summary's DRAM bytes only while the hash of the
+    kernel sources it names is the one recorded in it."""
+    sys.path.insert(0, ROOT)
+    import bench
+    name = "backward_step_C4.txt"
+    f = _profile_fields(os.path.join(ROOT, "profiles", name))
+    recorded = f["source_sha256_16"].split(" ")[0]
+    files = ["backward.cu", "pack.cu", "spmm.cu", "ablation.cu"]
+    monkeypatch.setattr(bench, "sources_hash", lambda fs: recorded)
+    assert bench.profile_file_traffic(name, files) == float(f["dram_bytes_per_launch"].split(" ")[0])
+    monkeypatch.setattr(bench, "sources_hash", lambda fs: "0" * 16)
+    assert bench.profile_file_traffic(name, files) is None
+    assert bench.profile_file_traffic("no_such_profile.txt", files) is None
