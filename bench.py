@@ -101,7 +101,7 @@ def induced_subgraph(rowptr, colidx, lo: int, hi: int):
 # Random row gathers from an L2-resident buffer (63 MB), plain 16-byte loads,
 # every SM busy: bytes/s by row size, measured on GB300 by
 # tests/probes/l2_gather.cu (profiles/l2_gather_rates.txt).
-L2_GATHER_GBS = {16: 900.0, 64: 8897.0, 128: 20469.0, 256: 21319.0, 512: 21529.0}
+L2_GATHER_GBS = {16: 900.0, 64: 8867.0, 128: 20304.0, 256: 21238.0, 512: 21334.0}
 
 
 def l2_gather_peak(row_bytes):
