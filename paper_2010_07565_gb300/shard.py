@@ -13,9 +13,15 @@ halo -- and sends the rows of its own block that other ranks reference.
                    which own rows go to which rank
   exchange_rows    the halo exchange, one all-to-all of the requested rows
                    (torch.distributed: NCCL between GPUs, gloo on the CPU)
+  exchange_packed_rows
+                   the other form of the exchange: the requested rows' packed
+                   signs and row scales (8 ceil(K/64) + 4 bytes a row instead
+                   of 4 F), from which the receiving rank computes the halo's
+                   product itself (the halo rows' degrees come with the plan)
   layer_forward_sharded
                    the layer on one rank: the library's kernels for steps 1-4
-                   on its block, the exchange, then bigcn_spmm_prescaled_rows
+                   on its block, the exchange (the smaller of the two forms by
+                   default), then bigcn_spmm_prescaled_rows
 
 The degree of every row (dhat = 1 + row length) is known to the rank that
 owns the row, which also applies 1/sqrt(dhat_j) to its product rows before
@@ -54,6 +60,9 @@ class ShardPlan:
     recv_counts[r]: halo rows that come from rank r (halo is sorted, so they
     are consecutive and in rank order). send_index: the own rows (local
     indices) other ranks need, grouped by destination rank with send_counts.
+    halo_rowptr: cumulative degrees of the halo rows (halo_rowptr[h + 1] -
+    halo_rowptr[h] = row length of halo[h] in the whole graph), so that the
+    degree-scaled product of received packed rows runs as for own rows.
     """
     rank: int
     bounds: np.ndarray
@@ -65,6 +74,7 @@ class ShardPlan:
     recv_counts: np.ndarray
     send_index: np.ndarray
     send_counts: np.ndarray
+    halo_rowptr: np.ndarray = None
 
     @property
     def n_own(self) -> int:
@@ -118,8 +128,15 @@ def build_plan(rowptr: np.ndarray, colidx: np.ndarray, bounds: np.ndarray, rank:
     dist.all_to_all_single(asked, req, output_split_sizes=send_counts.tolist(),
                            input_split_sizes=recv.tolist(), group=group)
     send_index = asked.cpu().numpy() - lo
+    # The degrees of the rows this rank sends, answered the same way.
+    own_deg = np.diff(rp)
+    sent_deg = torch.from_numpy(own_deg[send_index].astype(np.int64)).to(dev)
+    halo_deg = torch.empty(int(halo.shape[0]), dtype=torch.int64, device=dev)
+    dist.all_to_all_single(halo_deg, sent_deg, output_split_sizes=recv.tolist(),
+                           input_split_sizes=send_counts.tolist(), group=group)
+    halo_rowptr = np.concatenate([[0], np.cumsum(halo_deg.cpu().numpy())]).astype(np.int64)
     return ShardPlan(rank, np.asarray(bounds, np.int64), lo, int(bounds[rank + 1]), rp, ci, halo,
-                     recv, send_index.astype(np.int64), send_counts)
+                     recv, send_index.astype(np.int64), send_counts, halo_rowptr)
 
 
 def _collective_device(group=None):
@@ -145,22 +162,63 @@ def exchange_rows(own: torch.Tensor, plan: ShardPlan, group=None) -> torch.Tenso
     return table
 
 
-def layer_forward_sharded(X_own, scale, shift, Wt, plan: ShardPlan, group=None):
+def exchange_packed_rows(bits: torch.Tensor, alpha: torch.Tensor, plan: ShardPlan, group=None):
+    """The packed form of the halo exchange: returns the halo rows' packed
+    signs (n_halo x words, int64) and row scales alpha (n_halo), received from
+    their owners. ``bits`` / ``alpha`` are this rank's own rows."""
+    import torch.distributed as dist
+    idx = torch.from_numpy(plan.send_index).to(bits.device)
+    n_halo = int(plan.halo.shape[0])
+    halo_bits = torch.empty((n_halo, bits.shape[1]), dtype=bits.dtype, device=bits.device)
+    halo_alpha = torch.empty(n_halo, dtype=alpha.dtype, device=alpha.device)
+    splits = dict(output_split_sizes=plan.recv_counts.tolist(),
+                  input_split_sizes=plan.send_counts.tolist(), group=group)
+    dist.all_to_all_single(halo_bits, bits[idx].contiguous(), **splits)
+    dist.all_to_all_single(halo_alpha, alpha[idx].contiguous(), **splits)
+    return halo_bits, halo_alpha
+
+
+def exchange_bytes_per_row(K: int, F: int, packed: bool) -> int:
+    """Bytes a halo row costs in the exchange: the product row (4 F) or the
+    packed signs and the row scale (8 ceil(K/64) + 4)."""
+    return 8 * ((K + 63) // 64) + 4 if packed else 4 * F
+
+
+def layer_forward_sharded(X_own, scale, shift, Wt, plan: ShardPlan, group=None,
+                          exchange: str = "auto"):
     """One Bi-GCN layer on this rank's block of rows (X_own: n_own x K on this
     rank's GPU): the product of its rows with 1/sqrt(dhat) applied (Eqs. 10-12,
     bigcn_xnor_gemm_degscaled on the block's CSR, whose row lengths are the
     rows' full degrees), the halo exchange (NCCL), and the aggregation of its
-    rows (Eq. 13, bigcn_spmm_prescaled_rows). Returns H_own (n_own x F)."""
+    rows (Eq. 13, bigcn_spmm_prescaled_rows). ``exchange``: "rows" sends the
+    halo's product rows, "packed" their packed signs and row scales (the
+    receiving rank then runs the same degree-scaled product on them, with the
+    halo degrees from the plan), "auto" the one with fewer bytes a row.
+    Returns H_own (n_own x F)."""
     from . import binding as B
     dev = X_own.device
     K, F = Wt.shape
+    if exchange == "auto":
+        exchange = "packed" if exchange_bytes_per_row(K, F, True) < \
+            exchange_bytes_per_row(K, F, False) else "rows"
+    if exchange not in ("rows", "packed"):
+        raise ValueError("exchange must be 'rows', 'packed' or 'auto'")
     rowptr = torch.from_numpy(plan.rowptr).to(dev)
     colidx = torch.from_numpy(plan.colidx).to(dev)
     bits, alpha = B.pack_rows(X_own, scale, shift)
     wbits, beta = B.pack_weights(Wt)
-    Zp = torch.empty((plan.n_own, F), dtype=torch.float32, device=dev)
-    B.bigcn_xnor_gemm_degscaled(bits, alpha, wbits, beta, K, rowptr, Zp)
-    table = exchange_rows(Zp, plan, group)
+    if exchange == "rows":
+        Zp = torch.empty((plan.n_own, F), dtype=torch.float32, device=dev)
+        B.bigcn_xnor_gemm_degscaled(bits, alpha, wbits, beta, K, rowptr, Zp)
+        table = exchange_rows(Zp, plan, group)
+    else:
+        halo_bits, halo_alpha = exchange_packed_rows(bits, alpha, plan, group)
+        table = torch.empty((plan.n_cols, F), dtype=torch.float32, device=dev)
+        B.bigcn_xnor_gemm_degscaled(bits, alpha, wbits, beta, K, rowptr, table[:plan.n_own])
+        if plan.n_cols > plan.n_own:
+            B.bigcn_xnor_gemm_degscaled(halo_bits, halo_alpha, wbits, beta, K,
+                                        torch.from_numpy(plan.halo_rowptr).to(dev),
+                                        table[plan.n_own:])
     H = torch.empty((plan.n_own, F), dtype=torch.float32, device=dev)
     B.bigcn_spmm_prescaled_rows(rowptr, colidx, table, H)
     return H

@@ -1,10 +1,12 @@
 """The sharded layer's host logic on the CPU: the row partition, each rank's
 renumbered CSR and halo, and the halo exchange over two (and three) gloo
-ranks. The products are the oracle's (no GPU here): each rank takes the
-oracle's product of its own rows with 1/sqrt(dhat) applied, exchanges rows
-with exchange_rows, and aggregates its block by the plain definition of
-Eq. 13 over its table; the blocks, put back together, must equal the oracle's
-whole-graph layer."""
+ranks, in both forms. The products are the oracle's (no GPU here): each rank
+takes the oracle's product of its own rows with 1/sqrt(dhat) applied and
+either exchanges those rows (exchange_rows) or exchanges the packed signs and
+row scales of its rows (exchange_packed_rows) and computes the halo's product
+itself, with the halo degrees the plan carries; it then aggregates its block
+by the plain definition of Eq. 13 over its table. The blocks, put back
+together, must equal the oracle's whole-graph layer."""
 import os
 import socket
 
@@ -55,7 +57,16 @@ def test_local_plan_renumbers_and_lists_the_halo():
         assert np.array_equal(table[lci], ci[rp[lo]:rp[hi]])
 
 
-def _rank_main(rank, world, port, result_path):
+def unpack_signs(bits, K):
+    """Signs (+-1, int8) of packed rows (bit k of a row at word k / 64,
+    position k % 64)."""
+    w = np.ascontiguousarray(bits).view(np.uint64)
+    k = np.arange(K)
+    b = (w[:, k // 64] >> (k % 64).astype(np.uint64)) & np.uint64(1)
+    return np.where(b == 1, 1, -1).astype(np.int8)
+
+
+def _rank_main(rank, world, port, result_path, packed=False):
     os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
     dist.init_process_group("gloo", rank=rank, world_size=world)
     try:
@@ -64,13 +75,23 @@ def _rank_main(rank, world, port, result_path):
         b = shard.partition_rows(rp, world)
         plan = shard.build_plan(rp, ci, b, rank)
         lo, hi = plan.lo, plan.hi
+        assert np.array_equal(np.diff(plan.halo_rowptr), np.diff(rp)[plan.halo])
         # This rank's product rows (the oracle's), with 1/sqrt(dhat_j) applied.
         Y = oracle.centre(c["X"][lo:hi], c["s"], c["t"])
+        SF, alpha = oracle.sign(Y), oracle.row_scale(Y)
         SB, beta = oracle.weight_binarize(c["W"])
-        z = oracle.zeta(oracle.binary_dot(oracle.sign(Y), SB), oracle.row_scale(Y), beta)
+        z = oracle.zeta(oracle.binary_dot(SF, SB), alpha, beta)
         dhat = np.diff(plan.rowptr) + 1.0
-        zp = torch.from_numpy(z / np.sqrt(dhat)[:, None])
-        table = shard.exchange_rows(zp, plan).numpy()
+        zp = z / np.sqrt(dhat)[:, None]
+        if packed:
+            K = c["X"].shape[1]
+            bits = torch.from_numpy(np.ascontiguousarray(oracle.pack(SF)).view(np.int64))
+            hb, ha = shard.exchange_packed_rows(bits, torch.from_numpy(alpha), plan)
+            zh = oracle.zeta(oracle.binary_dot(unpack_signs(hb.numpy(), K), SB), ha.numpy(), beta)
+            zh = zh / np.sqrt(np.diff(plan.halo_rowptr) + 1.0)[:, None]
+            table = np.concatenate([zp, zh])
+        else:
+            table = shard.exchange_rows(torch.from_numpy(zp), plan).numpy()
         # Eq. 13 on the block: H_i = dhat_i^-1/2 (Z'_i + sum over the row's entries of Z'_q).
         H = np.empty((plan.n_own, z.shape[1]))
         for i in range(plan.n_own):
@@ -81,13 +102,24 @@ def _rank_main(rank, world, port, result_path):
         dist.destroy_process_group()
 
 
-@pytest.mark.parametrize("world", [2, 3])
-def test_sharded_layer_equals_the_whole_graph_layer(tmp_path, world):
+@pytest.mark.parametrize("world,packed", [(2, False), (3, False), (2, True), (3, True)])
+def test_sharded_layer_equals_the_whole_graph_layer(tmp_path, world, packed):
     path = str(tmp_path / "H")
-    mp.start_processes(_rank_main, args=(world, free_port(), path), nprocs=world,
+    mp.start_processes(_rank_main, args=(world, free_port(), path, packed), nprocs=world,
                        start_method="spawn")
     c = case()
     ref = oracle.layer_forward(c["X"], c["W"], c["rowptr"], c["colidx"], c["s"], c["t"])["H"]
     H = np.concatenate([np.load(f"{path}.{r}.npy") for r in range(world)])
     assert H.shape == ref.shape
     assert np.allclose(H, ref, rtol=1e-12, atol=1e-12)
+
+
+def test_exchange_bytes_choose_the_smaller_form():
+    # C1's widths: packed signs (23 words) + scale, 188 B a row, against 256 B
+    assert shard.exchange_bytes_per_row(1433, 64, True) == 188
+    assert shard.exchange_bytes_per_row(1433, 64, False) == 256
+    # C4's layer 1: 84 B against 512 B; layer 2 (K = 128, F = 41): 20 against 164
+    assert shard.exchange_bytes_per_row(602, 128, True) == 84
+    assert shard.exchange_bytes_per_row(128, 41, True) < shard.exchange_bytes_per_row(128, 41, False)
+    # wide rows of few features: the product rows are smaller
+    assert shard.exchange_bytes_per_row(8192, 16, True) > shard.exchange_bytes_per_row(8192, 16, False)
