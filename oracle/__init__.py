@@ -11,6 +11,8 @@ order:
     step 3  B = sign(W), column scale (Eq. 3, Eq. 4)    oracle_weight_binarize
     step 4  zeta = alpha beta (F . B) (Eq. 11, Eq. 12)  oracle_binary_dot, oracle_zeta
     step 5  H = A~ zeta (Eq. 13, Eq. 1)                 oracle_aggregate
+            ... with a weighted A (Sec. 3)              oracle_degree_weighted,
+                                                        oracle_aggregate_weighted
 
 the ablation variants of step 4 (Sec. 6.3, one operand kept real):
 
@@ -116,6 +118,11 @@ def lib() -> ctypes.CDLL:
             h.oracle_zeta_bucketed.restype = None
             h.oracle_grad_weight.argtypes = [_f64p, _i8p, _f64p, _f32p, _i32, _i32, _i64, _f64p]
             h.oracle_grad_weight.restype = None
+            h.oracle_degree_weighted.argtypes = [_i64p, _f64p, _i64, _f64p]
+            h.oracle_degree_weighted.restype = None
+            h.oracle_aggregate_weighted.argtypes = [_i64p, _i32p, _f64p, _i64, _f64p, _i32,
+                                                    _vp, _i64, _f64p, _vp]
+            h.oracle_aggregate_weighted.restype = ctypes.c_int
             _lib = h
     return _lib
 
@@ -272,6 +279,50 @@ def forward_2layer(X, s, t, W1, W2, rowptr, colidx) -> dict:
     H1 = l1["H"].astype(np.float32)
     l2 = layer_forward(H1, W2, rowptr, colidx)
     return dict(layer1=l1, layer2=l2, H1=H1, logits=l2["H"])
+
+
+# ---------------------------------------------------- weighted adjacency ----
+def degree_weighted(rowptr, values) -> np.ndarray:
+    """Sec. 3 with a weighted A: dhat_i = sum_j (A + I)_ij = 1 + the sum of
+    row i's CSR values (float64)."""
+    rowptr, v = _c(rowptr, np.int64), _c(values, np.float64)
+    N = rowptr.shape[0] - 1
+    d = np.empty(N, np.float64)
+    lib().oracle_degree_weighted(rowptr, v if v.size else np.zeros(1), N, d)
+    return d
+
+
+def aggregate_weighted(rowptr, colidx, values, zeta_, rows=None, with_absterm=False):
+    """Eq. 13 with Eq. 1's operator on a weighted A (values[e] = a_ij of CSR
+    entry e): H_i = zeta_i / dhat_i + sum_e a_ij zeta_j / sqrt(dhat_i dhat_j),
+    float64. Weights must be finite and >= 0."""
+    rowptr, colidx = _c(rowptr, np.int64), _c(colidx, np.int32)
+    v, z = _c(values, np.float64), _c(zeta_, np.float64)
+    N, F = z.shape
+    assert rowptr.shape[0] == N + 1 and v.shape == colidx.shape
+    keep, nrows, rp = _rows_arg(rows, N)
+    H = np.empty((nrows, F), np.float64)
+    A = np.empty((nrows, F), np.float64) if with_absterm else None
+    if colidx.size == 0:
+        colidx, v = np.zeros(1, np.int32), np.zeros(1, np.float64)
+    if lib().oracle_aggregate_weighted(rowptr, colidx, v, N, z, F, rp, nrows, H,
+                                       None if A is None else A.ctypes.data) != 0:
+        raise ValueError("malformed CSR, row index or weight")
+    return (H, A) if with_absterm else H
+
+
+def layer_forward_weighted(X, Wt, rowptr, colidx, values, s=None, t=None, rows=None) -> dict:
+    """One binarized layer (Eqs. 10-13) over a weighted adjacency: the steps
+    of ``layer_forward`` with ``aggregate_weighted`` as step 5."""
+    Y = centre(X, s, t)
+    SF = sign(Y)
+    alpha = row_scale(Y)
+    SB, beta = weight_binarize(Wt)
+    dot = binary_dot(SF, SB)
+    z = zeta(dot, alpha, beta)
+    H, absterm = aggregate_weighted(rowptr, colidx, values, z, rows=rows, with_absterm=True)
+    return dict(Y=Y, SF=SF, alpha=alpha, SB=SB, beta=beta, dot=dot, zeta=z,
+                dhat=degree_weighted(rowptr, values), H=H, absterm=absterm)
 
 
 # ------------------------------------------------------ ablation variants ----

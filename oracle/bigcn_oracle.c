@@ -11,7 +11,9 @@
  *   scales .......... Eq. 4 (weight column), Eq. 7 (node row), both read as the
  *                     mean absolute value over the d_in entries of the bucket
  *   binary product .. Eq. 11 / Eq. 12 (dot of +-1 vectors, then scaled)
- *   aggregation ..... Eq. 13 with the operator of Eq. 1, D^-1/2 (A+I) D^-1/2
+ *   aggregation ..... Eq. 13 with the operator of Eq. 1, D^-1/2 (A+I) D^-1/2,
+ *                     for a 0/1 adjacency and for a weighted one (Sec. 3's
+ *                     A = [a_ij], D^_ii = sum_j a^_ij)
  *   back-propagation  Algorithm 1 (A~^T dH, H~^T G, G W~^T), Eq. bp-H (the
  *                     gradient of the layer input, clipped to |.| < 1) and
  *                     Eq. bp-W (the weight gradient through the column scale
@@ -356,6 +358,60 @@ int oracle_aggregate_sage(const int64_t *rowptr, const int32_t *colidx, int64_t 
         for (e = rowptr[i]; e < rowptr[i + 1]; ++e)               /* W_neigh mean_j h_j */
             add_weighted(h, a, zneigh + (int64_t)colidx[e] * F, F, 1.0 / (double)deg);
     }
+    return 0;
+}
+
+/* ---- A weighted adjacency (Sec. 3 notations, Eq. 1) ---- */
+
+void oracle_degree_weighted(const int64_t *rowptr, const double *values, int64_t N,
+                            double *dhat) {
+    int64_t i, e;
+    for (i = 0; i < N; ++i) {
+        double d = 1.0;                         /* the self-loop's a^_ii = 1 */
+        for (e = rowptr[i]; e < rowptr[i + 1]; ++e)
+            d += values[e];
+        dhat[i] = d;
+    }
+}
+
+int oracle_aggregate_weighted(const int64_t *rowptr, const int32_t *colidx,
+                              const double *values, int64_t N, const double *zeta,
+                              int32_t F, const int64_t *rows, int64_t nrows, double *H,
+                              double *absterm) {
+    int64_t r, e, count = (rows != NULL) ? nrows : N;
+    int32_t f;
+    double *dhat;
+    if (csr_check(rowptr, colidx, N) != 0)
+        return -1;
+    for (e = 0; e < rowptr[N]; ++e)
+        if (!(values[e] >= 0.0) || !isfinite(values[e]))
+            return -1;
+    dhat = (double *)malloc(sizeof(double) * (size_t)(N > 0 ? N : 1));
+    if (!dhat)
+        return -1;
+    oracle_degree_weighted(rowptr, values, N, dhat);
+    for (r = 0; r < count; ++r) {
+        int64_t i = (rows != NULL) ? rows[r] : r;
+        double *h = H + r * (int64_t)F;
+        double *a = (absterm != NULL) ? absterm + r * (int64_t)F : NULL;
+        if (i < 0 || i >= N) {
+            free(dhat);
+            return -1;
+        }
+        for (f = 0; f < F; ++f) {
+            h[f] = 0.0;
+            if (a != NULL)
+                a[f] = 0.0;
+        }
+        /* the self-loop of A + I, weight 1 ... */
+        add_weighted(h, a, zeta + i * (int64_t)F, F, 1.0 / sqrt(dhat[i] * dhat[i]));
+        /* ... then each entry a_ij of row i of A */
+        for (e = rowptr[i]; e < rowptr[i + 1]; ++e) {
+            int64_t j = colidx[e];
+            add_weighted(h, a, zeta + j * (int64_t)F, F, values[e] / sqrt(dhat[i] * dhat[j]));
+        }
+    }
+    free(dhat);
     return 0;
 }
 

@@ -146,6 +146,27 @@ int oracle_aggregate_sage(const int64_t *rowptr, const int32_t *colidx, int64_t 
                           const double *zself, const double *zneigh, int32_t F,
                           const int64_t *rows, int64_t nrows, double *H, double *absterm);
 
+/* ---- A weighted adjacency (Sec. 3: A = [a_ij] with general entries, d_i =
+ * sum_j a_ij, A^ = A + I and D^_ii = sum_j a^_ij; Eq. 1's operator on it). The
+ * CSR's values[e] is a_ij for the entry e = (i, colidx[e]); the weights must be
+ * finite and non-negative. ---- */
+
+/* dhat[i] = 1 + sum of values[e] over the entries e of row i. */
+void oracle_degree_weighted(const int64_t *rowptr, const double *values, int64_t N,
+                            double *dhat);
+
+/* Eq. 13 with the weighted operator of Eq. 1: for each requested row
+ * i = rows[r] (rows == NULL: all rows),
+ *   H[r,:] = zeta[i,:] / dhat_i + sum over the entries e of row i of
+ *            values[e] zeta[j,:] / sqrt(dhat_i dhat_j),   j = colidx[e],
+ * the first term being the self-loop that I adds. absterm as in
+ * oracle_aggregate. Returns 0, or -1 for a malformed CSR or row index or a
+ * negative or non-finite weight. */
+int oracle_aggregate_weighted(const int64_t *rowptr, const int32_t *colidx,
+                              const double *values, int64_t N, const double *zeta,
+                              int32_t F, const int64_t *rows, int64_t nrows, double *H,
+                              double *absterm);
+
 /* ---- Sub-row bucketing (Sec. 4.1: buckets of B consecutive values, each
  * scaled separately). Bucket b of a row (column) holds its entries k in
  * [bB, min(K, (b + 1)B)); nb = ceil(K / B) buckets. ---- */
