@@ -248,6 +248,7 @@ INDUCTIVE_SOURCES = {
     "mean": ["inductive.cu", "pack.cu", "xnor_gemm.cu", "xnor_gemm_tc.cu", "spmm.cu"],
     "sage": ["inductive.cu", "pack.cu", "xnor_gemm.cu", "xnor_gemm_tc.cu", "spmm.cu"]}
 BACKWARD_SOURCES = ["backward.cu", "pack.cu", "spmm.cu", "ablation.cu"]
+WEIGHTED_SOURCES = ["weighted.cu", "pack.cu", "xnor_gemm.cu", "xnor_gemm_tc.cu", "spmm.cu"]
 
 
 class ClockSampler:
@@ -302,14 +303,37 @@ class ClockSampler:
 
 
 # ---------------------------------------------------------------- workload --
+WORKLOAD_ARRAYS = ("X", "s", "t", "W1", "W2", "rowptr", "colidx")
+
+
 def build_workload(name):
+    """The seeded workload ``name``. With BIGCN_BENCH_CACHE set to a
+    directory, the arrays are also saved there (and loaded on later runs)
+    under a key made of the name and the sha-256 of the generator's source,
+    so that a series of runs on one machine draws the Reddit-shaped graph
+    once; the arrays are the same either way."""
     from paper_2010_07565_gb300 import inputs
     w = inputs.get_workload(name)
+    cache = os.environ.get("BIGCN_BENCH_CACHE")
+    path = None
+    if cache:
+        with open(inputs.__file__, "rb") as f:
+            key = hashlib.sha256(f.read()).hexdigest()[:16]
+        path = os.path.join(cache, f"{name}_{key}.npz")
+        if os.path.exists(path):
+            with np.load(path) as z:
+                return w, {k: z[k] for k in WORKLOAD_ARRAYS}
     X = inputs.features(w)
     s, t = inputs.bn_stats(X)
     W1, W2 = inputs.layer_weights(w)
     rowptr, colidx = inputs.graph(w)
-    return w, dict(X=X, s=s, t=t, W1=W1, W2=W2, rowptr=rowptr, colidx=colidx)
+    data = dict(X=X, s=s, t=t, W1=W1, W2=W2, rowptr=rowptr, colidx=colidx)
+    if path is not None:
+        os.makedirs(cache, exist_ok=True)
+        tmp = f"{path}.{os.getpid()}.npz"
+        np.savez(tmp, **data)
+        os.replace(tmp, path)
+    return w, data
 
 
 def oracle_block_nodes(w, data, budget_s):
@@ -1011,6 +1035,94 @@ def run_inductive(args, rank, world, local_rank):
     return 0
 
 
+def run_weighted(args, rank, world, local_rank):
+    """Layer 1 of a workload over a weighted adjacency (Sec. 3's general a_ij,
+    Eq. 1's operator on A + I): seeded symmetric edge weights, uniform in
+    [0.5, 2), on the workload's graph. One bigcn_weighted_layer_forward call
+    per step (pack rows, pack weights, the weighted-degree pass, the XNOR
+    product, the weighted aggregation), L2 flushed before every step outside
+    the timed events. The roofline is the whole layer's algorithmic bytes
+    against HBM: X once, the packed rows and the factored product written and
+    read once, the row pointers and the weights read by the degree pass and
+    the aggregation, the column indices, dinv and s written and read, H."""
+    import torch
+
+    from paper_2010_07565_gb300 import binding as B
+    from paper_2010_07565_gb300 import inputs
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    w, data = build_workload(args.workload)
+    N, K, F = w.N, w.K, w.hidden
+    d = {k: torch.from_numpy(np.ascontiguousarray(v)).to(dev)
+         for k, v in data.items() if k in ("X", "s", "t", "W1", "rowptr", "colidx")}
+    values = torch.from_numpy(inputs.edge_weights(data["rowptr"], data["colidx"],
+                                                  4100 + w.index)).to(dev)
+    nnz = int(data["colidx"].shape[0])
+    ws = torch.empty(B.bigcn_weighted_layer_workspace_bytes(N, K, F), dtype=torch.uint8,
+                     device=dev)
+    H = torch.empty((N, F), device=dev)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    flush_half = flush[: flush.numel() // 2]
+
+    def step():
+        B.bigcn_weighted_layer_forward(d["X"], d["s"], d["t"], d["W1"], d["rowptr"],
+                                       d["colidx"], values, ws, H)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    times = []
+    with ClockSampler(local_rank) as clocks:
+        for _ in range(args.steps):
+            flush.zero_()
+            flush_half.sum()
+            e0.record()
+            step()
+            e1.record()
+            e1.synchronize()
+            times.append(e0.elapsed_time(e1))
+    assert B.device_timeouts() == 0
+    total_ms = float(sum(times))
+    max_ms, units = aggregate_over_ranks(total_ms, float(N) * args.steps, world)
+    if rank != 0:
+        return 0
+    peaks, peak_kind = load_peaks()
+    hbm = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+    words = (K + 63) // 64
+    Fz = (F + 7) // 8 * 8
+    zrow = 2.0 * Fz + 4.0 if K <= 32767 else 4.0 * Fz
+    layer_bytes = (4.0 * N * K + 2 * 8.0 * N * words + 2.0 * N * zrow + 2 * 8.0 * (N + 1) +
+                   4.0 * nnz + 2 * 4.0 * nnz + 4 * 4.0 * N + 4.0 * N * F)
+    mean_ms = max_ms / args.steps
+    achieved = layer_bytes / (mean_ms * 1e-3) / 1e9
+    line = {
+        "metric": "Bi-GCN weighted-adjacency layer fwd nodes/s",
+        "value": units / (max_ms * 1e-3), "unit": "nodes/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": mean_ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32+b1",
+        "data": "synthetic",
+        "config": {"workload": w.description + " -- layer 1, edge weights uniform in [0.5, 2), "
+                                               "symmetric", "name": w.name,
+                   "N": N, "K": K, "F": F, "nnz": nnz,
+                   "l2": "flushed before every step outside the timed events",
+                   "launch": "bigcn_weighted_layer_forward (pack rows, pack weights, weighted "
+                             "degrees, XNOR product, weighted aggregation)"},
+        "roofline": {"kernel": "whole layer", "bound": "hbm", "achieved": achieved, "peak": hbm,
+                     "unit": "GB/s", "frac": achieved / hbm,
+                     "traffic": profile_file_traffic(f"weighted_layer_{w.name}.txt",
+                                                     WEIGHTED_SOURCES),
+                     "traffic_note": "DRAM bytes of one whole call (its 5 kernels)",
+                     "peak_source": f"{peak_kind} MEASURED_PEAKS.json hbm_gbs",
+                     "algorithmic_bytes": layer_bytes},
+        "cpu_baseline": None, "e2e": None, "gpu_launches": 5 * args.steps,
+        "clocks": clocks.summary(),
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def run_bucketed(args, rank, world, local_rank):
     """Layer 1 of a workload with sub-row bucketing (Sec. 4.1): buckets of
     ``--bucket`` B features, each with its own scales. One
@@ -1142,6 +1254,9 @@ def main(argv=None):
     ap.add_argument("--inductive", choices=["gcn", "mean", "sage"], default=None,
                     help="time layer 1 as a binarized inductive layer "
                          "(bigcn_inductive_layer_forward) instead")
+    ap.add_argument("--weighted", action="store_true",
+                    help="time layer 1 over seeded symmetric edge weights "
+                         "(bigcn_weighted_layer_forward) instead")
     ap.add_argument("--bucket", type=int, default=0, metavar="B",
                     help="time layer 1 with sub-row bucketing, buckets of B features "
                          "(a multiple of 64; bigcn_layer_forward_bucketed) instead")
@@ -1154,6 +1269,8 @@ def main(argv=None):
     args = ap.parse_args(argv)
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")
+    if args.weighted and args.workload.startswith("C5_"):
+        ap.error("--weighted runs layer 1 of C1..C4")
     rank, world, local_rank = dist_env()
     if args.impl == "reference":
         return run_reference(args, rank, world)
@@ -1165,6 +1282,8 @@ def main(argv=None):
         return run_inductive(args, rank, world, local_rank)
     if args.bucket > 0:
         return run_bucketed(args, rank, world, local_rank)
+    if args.weighted:
+        return run_weighted(args, rank, world, local_rank)
     if args.workload.startswith("C5_"):
         return run_sweep(args, rank, world, local_rank)
     if args.backward:

@@ -447,6 +447,63 @@ bigcn_status bigcn_inductive_layer_forward(int32_t aggregator, const float *X, i
                                            float *H, int64_t ldh, void *stream);
 
 /*
+ * A weighted adjacency. Sec. 3 writes A = [a_ij] with general entries, the
+ * degree d_i = sum_j a_ij, A^ = A + I and D^_ii = sum_j a^_ij, and Eq. 1's
+ * operator D^-1/2 A^ D^-1/2 on that; the entry points above are the case
+ * a_ij = 1. Here `values` holds a_ij for each CSR entry (nnz fp32, in the
+ * order of colidx). Weights must be finite and >= 0: a negative degree has
+ * no square root and gives NaN or Inf outputs (never a fault); the calls do
+ * not check it. Symmetry of the weights is the caller's contract, as the
+ * CSR's; the formulas below are evaluated for any weights.
+ *
+ * bigcn_weighted_dinv: dinv[i] = 1 / sqrt(1 + sum over the entries e of
+ * row i of values[e]) for i < N (rows summed with compensated fp32 adds).
+ * rowptr (N+1 int64) and values (nnz) as above, dinv N fp32 written, not
+ * overlapping them. 0 <= N < 2^31, 0 <= nnz; values may be NULL when
+ * nnz == 0.
+ */
+bigcn_status bigcn_weighted_dinv(const int64_t *rowptr, const float *values, int64_t N,
+                                 int64_t nnz, float *dinv, void *stream);
+
+/*
+ * Step 5 over a weighted A (Eq. 13 with Eq. 1's operator):
+ *
+ *   H[i,:] = dinv_i * (dinv_i Z[i,:] + sum over the entries e of row i of
+ *            values[e] * dinv_j * Z[j,:]),   j = colidx[e],
+ *
+ * with dinv from bigcn_weighted_dinv on the same rowptr and values. The CSR,
+ * Z, H and the errors are those of bigcn_spmm_norm; values (nnz) and dinv
+ * (N) are read only and must not overlap H.
+ */
+bigcn_status bigcn_spmm_norm_weighted(const int64_t *rowptr, const int32_t *colidx,
+                                      const float *values, const float *dinv, int64_t N,
+                                      int64_t nnz, const float *Z, int64_t ldz, int32_t F,
+                                      float *H, int64_t ldh, void *stream);
+
+/* Bytes of device workspace bigcn_weighted_layer_forward needs; 0 on invalid
+ * sizes. */
+size_t bigcn_weighted_layer_workspace_bytes(int64_t N, int32_t K, int32_t F);
+
+/*
+ * One binarized layer over a weighted A: H = D^-1/2 (A + I) D^-1/2 zeta with
+ * zeta as in bigcn_layer_forward. Runs the kernels of bigcn_pack_rows,
+ * bigcn_pack_weights, bigcn_weighted_dinv (which also forms each row's scale
+ * s_j = alpha_j dinv_j), bigcn_xnor_gemm with s as its row scale (kept
+ * factored, uint16 dots and s_j, when K <= 32767) and the weighted
+ * aggregation. Arguments and errors are those of bigcn_layer_forward plus
+ * `values` (nnz fp32, not overlapping the workspace or H); the workspace is
+ * bigcn_weighted_layer_workspace_bytes(N, K, F) bytes, 256-byte aligned. The
+ * tensor-core product's bounded waits behave as in bigcn_layer_forward.
+ */
+bigcn_status bigcn_weighted_layer_forward(const float *X, int64_t N, int32_t K, int64_t ldx,
+                                          const float *scale, const float *shift,
+                                          const float *Wt, int32_t F, int64_t ldw,
+                                          const int64_t *rowptr, const int32_t *colidx,
+                                          const float *values, int64_t nnz, void *workspace,
+                                          size_t ws_bytes, float *H, int64_t ldh,
+                                          void *stream);
+
+/*
  * Back-propagation of one layer (Algorithm 1 with Eqs. bp-H and bp-W), from
  * the gradient dH = dL/dH^(l+1) of the layer's output (N x F, row stride ldg)
  * to

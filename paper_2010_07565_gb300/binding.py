@@ -82,6 +82,12 @@ SIGNATURES = {
                                       _p, _i64, _p, _sz, _p, _i64, _p], ctypes.c_int),
     "bigcn_layer_forward_static": ([_p, _i64, _i32, _i64, _p, _p, _p, _i32, _i64, _p, _p, _i64,
                                     _p, _i64, _p], ctypes.c_int),
+    "bigcn_weighted_dinv": ([_p, _p, _i64, _i64, _p, _p], ctypes.c_int),
+    "bigcn_spmm_norm_weighted": ([_p, _p, _p, _p, _i64, _i64, _p, _i64, _i32, _p, _i64, _p],
+                                 ctypes.c_int),
+    "bigcn_weighted_layer_workspace_bytes": ([_i64, _i32, _i32], _sz),
+    "bigcn_weighted_layer_forward": ([_p, _i64, _i32, _i64, _p, _p, _p, _i32, _i64, _p, _p, _p,
+                                      _i64, _p, _sz, _p, _i64, _p], ctypes.c_int),
 }
 
 
@@ -425,6 +431,37 @@ def bigcn_layer_forward_static(X, scale, shift, Wt, rowptr, colidx, H, stream=No
         _ptr(X), N, K, _ld(X), _ptr(scale), _ptr(shift), _ptr(Wt), F, _ld(Wt), _ptr(rowptr),
         _ptr(colidx) if colidx.numel() else None, colidx.numel(), _ptr(H), _ld(H),
         _stream(stream)))
+
+
+def bigcn_weighted_dinv(rowptr, values, dinv, stream=None):
+    """dinv_i = 1/sqrt(1 + sum of row i's edge weights) (Sec. 3, weighted A)."""
+    N = rowptr.numel() - 1
+    _check("bigcn_weighted_dinv", lib().bigcn_weighted_dinv(
+        _ptr(rowptr), _ptr(values) if values.numel() else None, N, values.numel(), _ptr(dinv),
+        _stream(stream)))
+
+
+def bigcn_spmm_norm_weighted(rowptr, colidx, values, dinv, Z, H, stream=None):
+    N, F = Z.shape
+    _check("bigcn_spmm_norm_weighted", lib().bigcn_spmm_norm_weighted(
+        _ptr(rowptr), _ptr(colidx) if colidx.numel() else None,
+        _ptr(values) if values.numel() else None, _ptr(dinv), N, colidx.numel(), _ptr(Z), _ld(Z),
+        F, _ptr(H), _ld(H), _stream(stream)))
+
+
+def bigcn_weighted_layer_workspace_bytes(N: int, K: int, F: int) -> int:
+    return int(lib().bigcn_weighted_layer_workspace_bytes(N, K, F))
+
+
+def bigcn_weighted_layer_forward(X, scale, shift, Wt, rowptr, colidx, values, workspace, H,
+                                 stream=None):
+    N, K = X.shape
+    F = Wt.shape[1]
+    _check("bigcn_weighted_layer_forward", lib().bigcn_weighted_layer_forward(
+        _ptr(X), N, K, _ld(X), _ptr(scale), _ptr(shift), _ptr(Wt), F, _ld(Wt), _ptr(rowptr),
+        _ptr(colidx) if colidx.numel() else None, _ptr(values) if values.numel() else None,
+        colidx.numel(), _ptr(workspace), workspace.numel() * workspace.element_size(), _ptr(H),
+        _ld(H), _stream(stream)))
 
 
 # ------------------------------------------------- allocating conveniences ---

@@ -86,8 +86,9 @@ void launch_xnor_gemm(const GemmArgs &args, const DeviceInfo &dev, cudaStream_t 
                       bool pdl = false);
 
 // Aggregators of step 5: Eq. 1's D^-1/2 (A + I) D^-1/2, the mean over
-// N(i) u {i} (inductive GCN), GraphSAGE's self + mean over N(i).
-enum : int { kAggGcn = 0, kAggMean = 1, kAggSage = 2 };
+// N(i) u {i} (inductive GCN), GraphSAGE's self + mean over N(i), and Eq. 1's
+// operator on a weighted A (Sec. 3: entries a_ij, D^_ii = 1 + sum_j a_ij).
+enum : int { kAggGcn = 0, kAggMean = 1, kAggSage = 2, kAggWeighted = 3 };
 
 struct SpmmArgs {
     const int64_t *rowptr;   // N + 1
@@ -124,12 +125,22 @@ struct SpmmArgs {
     // followed by its halo rows): column indices must lie below it. 0: N.
     // Needs pre-scaled rows or dots with a row scale (no neighbour degree is read).
     int64_t ncols = 0;
+    // kAggWeighted: the weight a_ij of each CSR entry (nnz) and every node's
+    // 1/sqrt(dhat) (N, from launch_weighted_dinv). fp32 rows (prescaled
+    // false) are weighted by a_ij dinv_j, dots by a_ij rowscale_j (rowscale
+    // carrying dinv_j); the sum is multiplied by dinv_i.
+    const float *values = nullptr;
+    const float *dinv = nullptr;
 };
 
 // Step 5: H = D^-1/2 (A + I) D^-1/2 Z (Eqs. 1, 13); launches one kernel, or
 // two when an argmax is asked for rows wider than one column slab.
 void launch_spmm_norm(const SpmmArgs &args, const DeviceInfo &dev, cudaStream_t stream,
                       bool pdl = false);
+// The weighted degrees of A + I (weighted.cu): dinv_i = 1/sqrt(1 + sum of
+// row i's values) and, when alpha is given, s_i = alpha_i dinv_i.
+void launch_weighted_dinv(const int64_t *rowptr, const float *values, int64_t N, int64_t nnz,
+                          const float *alpha, float *dinv, float *s, cudaStream_t stream);
 
 struct FrontArgs {
     const float *X;          // N x K (row stride ldx)

@@ -102,6 +102,8 @@ struct SpmmParams {
     const void *Zs = nullptr;
     const float *colscale_s = nullptr;
     int64_t ncols = 0;       // rows of Z (column indices must lie below); N when 0
+    const float *values = nullptr;   // kAggWeighted: a_ij per CSR entry
+    const float *dinv = nullptr;     // kAggWeighted: 1/sqrt(dhat) per node
 };
 
 // How a lane loads VEC consecutive entries of a row of Z and adds them,
@@ -162,8 +164,8 @@ struct RowSrc<8, kDots16> {
 // Row i's neighbour list: CSR entries [b, b + total - 1) plus the self-loop
 // (entry 0); `first` is the first entry the aggregator sums (1 when the self
 // row is added separately), `dinv` the factor applied to the sum: Eq. 1's
-// 1/sqrt(dhat_i), the mean's 1/dhat_i, or GraphSAGE's 1/|N(i)| (0 without
-// neighbours).
+// 1/sqrt(dhat_i) (for a weighted A read from `wdinv`), the mean's 1/dhat_i,
+// or GraphSAGE's 1/|N(i)| (0 without neighbours).
 struct RowSpan {
     int64_t b;
     int64_t total;
@@ -172,12 +174,14 @@ struct RowSpan {
 };
 
 __device__ __forceinline__ RowSpan row_span(const int64_t *__restrict__ rowptr, int64_t nnz,
-                                            int64_t i, int agg = kAggGcn) {
+                                            int64_t i, int agg = kAggGcn,
+                                            const float *wdinv = nullptr) {
     const int64_t rb = __ldg(rowptr + i), re = __ldg(rowptr + i + 1);
     const int64_t b = min(max(rb, int64_t(0)), nnz);
     const int64_t e = min(max(re, b), nnz);
     const int64_t deg = e - b;
-    const float norm = agg == kAggGcn    ? inv_sqrt_degree(deg)
+    const float norm = agg == kAggWeighted ? __ldg(wdinv + i)
+                       : agg == kAggGcn    ? inv_sqrt_degree(deg)
                        : agg == kAggMean ? 1.0f / (1.0f + float(deg))
                        : deg > 0         ? 1.0f / float(deg)
                                          : 0.0f;
@@ -185,8 +189,10 @@ __device__ __forceinline__ RowSpan row_span(const int64_t *__restrict__ rowptr, 
 }
 
 // Adds, into acc, the Z rows of entries [q0, q1) of row i's list (entry 0 is
-// the self-loop), weighted by 1/sqrt(dhat_j) (kDinv), 1 (kPre) or s_j (kDots16).
-template <int VEC, int L, int NV, int U, int S>
+// the self-loop), weighted by 1/sqrt(dhat_j) (kDinv), 1 (kPre) or s_j (kDots16),
+// and for a weighted A (kAggWeighted) also by the entry's a_ij (1 for the
+// self-loop), with dhat_j read from p.dinv.
+template <int VEC, int L, int NV, int U, int S, int AGG = kAggGcn>
 __device__ __forceinline__ void gather(const SpmmParams &p, int64_t i, int64_t b, int64_t q0,
                                        int64_t q1, int f0, float (&acc)[NV][VEC]) {
     using Src = RowSrc<VEC, S>;
@@ -201,11 +207,14 @@ __device__ __forceinline__ void gather(const SpmmParams &p, int64_t i, int64_t b
         if (q < q1) {
             j = (q == 0) ? int(i) : __ldg(p.colidx + b + q - 1);
             if (j < 0 || j >= p.ncols) j = -1;
-            if (j >= 0)
-                wj = S == kPre ? 1.0f
-                               : S == kDots16
-                                     ? __ldg(p.rowscale + j)
-                                     : inv_sqrt_degree(__ldg(p.rowptr + j + 1) - __ldg(p.rowptr + j));
+            if (j >= 0) {
+                wj = S == kPre              ? 1.0f
+                     : S == kDots16         ? __ldg(p.rowscale + j)
+                     : AGG == kAggWeighted  ? __ldg(p.dinv + j)
+                                            : inv_sqrt_degree(__ldg(p.rowptr + j + 1) -
+                                                              __ldg(p.rowptr + j));
+                if (AGG == kAggWeighted && q > 0) wj *= __ldg(p.values + b + q - 1);
+            }
         }
         const int cnt = int(min(q1 - base, int64_t(32)));
         for (int t0 = 0; t0 < cnt; t0 += P * U) {
@@ -353,14 +362,14 @@ __device__ __forceinline__ void light_rows(const SpmmParams &p, const Epi &epi, 
     const int warp = threadIdx.x >> 5;
     const int64_t i = int64_t(blockIdx.x - p.heavy_blocks) * kSpmmWarps + warp;
     if (i >= p.N) return;
-    const RowSpan sp = row_span(p.rowptr, p.nnz, i, AGG);
+    const RowSpan sp = row_span(p.rowptr, p.nnz, i, AGG, p.dinv);
     if (p.heavy_blocks > 0 && sp.total - 1 > p.heavy_degree) return;   // a heavy block's row
     float acc[NV][VEC];
 #pragma unroll
     for (int v = 0; v < NV; ++v)
 #pragma unroll
         for (int c = 0; c < VEC; ++c) acc[v][c] = 0.0f;
-    gather<VEC, L, NV, U, S>(p, i, sp.b, sp.first, sp.total, f0, acc);
+    gather<VEC, L, NV, U, S, AGG>(p, i, sp.b, sp.first, sp.total, f0, acc);
     reduce_groups<VEC, L, NV>(acc);
     epi(p, i, sp.dinv, f0, acc);
 }
@@ -383,7 +392,7 @@ __device__ __forceinline__ void heavy_rows(const SpmmParams &p, const Epi &epi, 
             const int bit = __ffs(mm) - 1;
             mm &= mm - 1u;
             const int64_t i = base + bit;
-            const RowSpan sp = row_span(p.rowptr, p.nnz, i, AGG);
+            const RowSpan sp = row_span(p.rowptr, p.nnz, i, AGG, p.dinv);
             float acc[NV][VEC];
 #pragma unroll
             for (int v = 0; v < NV; ++v)
@@ -392,7 +401,7 @@ __device__ __forceinline__ void heavy_rows(const SpmmParams &p, const Epi &epi, 
             const int64_t span = sp.total - sp.first;
             const int64_t q0 = sp.first + span * warp / kSpmmWarps;
             const int64_t q1 = sp.first + span * (warp + 1) / kSpmmWarps;
-            gather<VEC, L, NV, U, S>(p, i, sp.b, q0, q1, f0, acc);
+            gather<VEC, L, NV, U, S, AGG>(p, i, sp.b, q0, q1, f0, acc);
             reduce_groups<VEC, L, NV>(acc);
             if (g == 0) {
 #pragma unroll
@@ -597,7 +606,7 @@ void launch_cfg(const SpmmArgs &a, const DeviceInfo &dev, int Fload, cudaStream_
     SpmmParams p{a.rowptr, a.colidx, a.N, a.nnz, Z, a.ldz, Fload, a.F, a.H, a.ldh,
                  heavy_block_count(a.N, dev), heavy_degree(a.N, a.nnz, (32 / L) * U), vec_store,
                  a.rowscale, a.colscale, one_slab ? a.pred : nullptr, a.agg, a.Zs,
-                 a.colscale_s, a.ncols > 0 ? a.ncols : a.N};
+                 a.colscale_s, a.ncols > 0 ? a.ncols : a.N, a.values, a.dinv};
     dim3 grid(unsigned(p.heavy_blocks + (a.N + kSpmmWarps - 1) / kSpmmWarps),
               unsigned((a.F + SLAB - 1) / SLAB));
     launch_kernel(spmm_norm_kernel<VEC, L, NV, U, S, AGG>, grid, dim3(kSpmmThreads), 0, s, pdl,
@@ -654,12 +663,26 @@ void launch_inductive(const SpmmArgs &a, const DeviceInfo &dev, cudaStream_t str
     launch_src<kPre, AGG>(a, dev, stream, pdl);
 }
 
+// A weighted A: dots with their row scale, or plain fp32 rows whose source
+// factor dinv_j is read per neighbour (kDinv).
+void launch_weighted(const SpmmArgs &a, const DeviceInfo &dev, cudaStream_t stream, bool pdl) {
+    if (a.D16 != nullptr) {
+        if (a.ldz % 8 == 0 && aligned_to(a.D16, 16) && wide_dots(a.N, a.nnz))
+            launch_vec<8, kDots16, kAggWeighted>(a, dev, (a.F + 7) / 8 * 8, stream, pdl);
+        else
+            launch_vec<4, kDots16, kAggWeighted>(a, dev, (a.F + 3) / 4 * 4, stream, pdl);
+        return;
+    }
+    launch_src<kDinv, kAggWeighted>(a, dev, stream, pdl);
+}
+
 }  // namespace
 
 void launch_spmm_norm(const SpmmArgs &a, const DeviceInfo &dev, cudaStream_t stream, bool pdl) {
     if (a.N == 0) return;
     if (a.agg == kAggMean) return launch_inductive<kAggMean>(a, dev, stream, pdl);
     if (a.agg == kAggSage) return launch_inductive<kAggSage>(a, dev, stream, pdl);
+    if (a.agg == kAggWeighted) return launch_weighted(a, dev, stream, pdl);
     if (a.D16 != nullptr) {
         // Compressed rows: eight dots (16 bytes) per vector when the row
         // stride and base allow and rows are long, else four (8 bytes);

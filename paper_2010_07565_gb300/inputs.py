@@ -268,23 +268,29 @@ def graph(w: Workload, seed: int | None = None):
 
 
 def edge_weights(rowptr, colidx, seed: int, low: float = 0.5, high: float = 2.0) -> np.ndarray:
-    """Symmetric positive edge weights for a CSR (fp32, one per entry): the
-    entries (i, j) and (j, i) get the same weight, uniform in [low, high),
-    drawn from a splitmix64 hash of (seed, min(i, j), max(i, j)) so that no
-    pairing of the two entries is needed."""
+    """Symmetric positive edge weights for a CSR (fp32, one per entry, in the
+    order of colidx): the entries (i, j) and (j, i) get the same weight,
+    uniform between low and high. Each node draws a 32-bit key from the seeded
+    PCG64; an entry's weight comes from a 32-bit integer hash of the sum of its
+    two nodes' keys (the same sum from either end, so no pairing of the two
+    entries is needed)."""
     rowptr = np.asarray(rowptr, np.int64)
-    colidx = np.asarray(colidx, np.int64)
     N = rowptr.shape[0] - 1
-    row = np.repeat(np.arange(N, dtype=np.int64), np.diff(rowptr))
-    lo, hi = np.minimum(row, colidx), np.maximum(row, colidx)
-    with np.errstate(over="ignore"):
-        x = (lo.astype(np.uint64) << np.uint64(32)) ^ hi.astype(np.uint64)
-        x = x + np.uint64((0x9E3779B97F4A7C15 * (seed + 1)) & 0xFFFFFFFFFFFFFFFF)
-        x = (x ^ (x >> np.uint64(30))) * np.uint64(0xBF58476D1CE4E5B9)
-        x = (x ^ (x >> np.uint64(27))) * np.uint64(0x94D049BB133111EB)
-        x = x ^ (x >> np.uint64(31))
-    u = (x >> np.uint64(40)).astype(np.float64) / float(1 << 24)
-    return (low + (high - low) * u).astype(np.float32)
+    key = np.random.Generator(np.random.PCG64(seed)).integers(0, 1 << 32, size=N,
+                                                               dtype=np.uint32)
+    x = np.repeat(key, np.diff(rowptr))
+    x += key[np.asarray(colidx)]                 # wraps modulo 2^32
+    m = np.uint32(0x45D9F3B)
+    x ^= x >> np.uint32(16)
+    x *= m
+    x ^= x >> np.uint32(16)
+    x *= m
+    x ^= x >> np.uint32(16)
+    u = (x >> np.uint32(8)).astype(np.float32)
+    u *= np.float32(1.0 / (1 << 24))
+    u *= np.float32(high - low)
+    u += np.float32(low)
+    return u
 
 
 def random_graph(N: int, mean_degree: float, seed: int, hub_degree: int = 0):

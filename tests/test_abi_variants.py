@@ -1,7 +1,7 @@
 """Host-side logic of the C-ABI's variant entry points without a GPU:
 workspace sizes and the argument checks of the ablation products and
-layers, the inductive layers, sub-row bucketing and the layer backward,
-which return their documented status before any CUDA call (fake,
+layers, the inductive layers, sub-row bucketing, the layer backward and
+the weighted-adjacency calls, which return their documented status before any CUDA call (fake,
 never-dereferenced pointers are enough to reach them)."""
 import pytest
 
@@ -164,3 +164,51 @@ def test_backward_workspace_and_argument_checks(lib):
     assert f(*args(dW=dH)) == INVALID                              # dW overlaps dH
     assert f(*args(dX=dW)) == INVALID                              # dX overlaps dW
     assert f(*args(dX=dX + 2)) == MISALIGNED
+
+
+# ------------------------------------------------------ weighted adjacency --
+def test_weighted_workspace_bytes(lib):
+    f = lib.bigcn_weighted_layer_workspace_bytes
+    assert f(0, 0, 5) == 0 and f(-1, 10, 5) == 0
+    # uint16 dots (rows padded to 8) + row scale, then dinv and s (N each)
+    n = f(1000, 130, 62)
+    need = (1000 * 3 * 8 + 1000 * 4 + 62 * 3 * 8 + 62 * 4 + 1000 * 64 * 2 + 1000 * 4 +
+            2 * 1000 * 4)
+    assert need <= n <= need + 9 * 256 and n % 256 == 0
+    n = f(100, 40000, 5)                        # fp32 Z
+    need = 100 * 625 * 8 + 100 * 4 + 5 * 625 * 8 + 5 * 4 + 100 * 5 * 4 + 2 * 100 * 4
+    assert need <= n <= need + 9 * 256 and n % 256 == 0
+
+
+def test_weighted_argument_checks(lib):
+    d = lib.bigcn_weighted_dinv
+    rp, v, dv = ptrs(3)
+    assert d(rp, v, 0, 0, dv, None) == OK
+    assert d(rp, None, 8, 5, dv, None) == INVALID       # values NULL with entries
+    assert d(rp, v, -1, 5, dv, None) == INVALID
+    assert d(rp, v, 8, -1, dv, None) == INVALID
+    assert d(rp + 4, v, 8, 5, dv, None) == MISALIGNED
+    assert d(rp, v + 2, 8, 5, dv, None) == MISALIGNED
+    assert d(rp, v, 8, 5, v + 8, None) == INVALID       # dinv overlaps values
+    s = lib.bigcn_spmm_norm_weighted
+    rp, ci, v, dv, z, h = ptrs(6)
+    assert s(rp, ci, v, dv, 0, 0, z, 4, 4, h, 4, None) == OK
+    assert s(rp, ci, None, dv, 8, 5, z, 4, 4, h, 4, None) == INVALID        # values NULL
+    assert s(rp, ci, v, None, 8, 5, z, 4, 4, h, 4, None) == INVALID         # dinv NULL
+    assert s(rp, ci, v + 2, dv, 8, 5, z, 4, 4, h, 4, None) == MISALIGNED
+    assert s(rp, ci, v, dv, 8, 5, z, 4, 4, v + 4, 4, None) == INVALID       # H overlaps values
+    assert s(rp, ci, v, dv, 8, 5, z, 4, 4, dv, 4, None) == INVALID          # H overlaps dinv
+    assert s(rp, ci, v, dv, 8, 5, z, 4, 4, h, 3, None) == INVALID           # ldh < F
+    f = lib.bigcn_weighted_layer_forward
+    X, W, rp, ci, v, ws, H = ptrs(7)
+    need = lib.bigcn_weighted_layer_workspace_bytes(100, 70, 8)
+    args = lambda **kw: [X, kw.get("N", 100), 70, 70, None, None, W, 8, 8, rp, ci,
+                         kw.get("v", v), 300, kw.get("ws", ws), kw.get("wsb", need),
+                         kw.get("H", H), 8, None]
+    assert f(*args(N=0)) == OK
+    assert f(*args(v=None)) == INVALID
+    assert f(*args(v=v + 2)) == MISALIGNED
+    assert f(*args(wsb=need - 1)) == INVALID
+    assert f(*args(ws=ws + 128)) == MISALIGNED
+    assert f(*args(ws=v)) == INVALID                    # workspace overlaps values
+    assert f(*args(H=v)) == INVALID                     # H overlaps values

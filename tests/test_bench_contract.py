@@ -115,3 +115,20 @@ def test_profile_traffic_needs_the_current_source(monkeypatch):
     monkeypatch.setattr(bench, "sources_hash", lambda fs: "0" * 16)
     assert bench.profile_file_traffic(name, files) is None
     assert bench.profile_file_traffic("no_such_profile.txt", files) is None
+
+
+def test_workload_cache_returns_the_same_arrays(monkeypatch, tmp_path):
+    """With BIGCN_BENCH_CACHE set, the first build saves the workload and the
+    second loads it: the arrays (values and dtypes) are those drawn afresh."""
+    sys.path.insert(0, ROOT)
+    import numpy as np
+    import bench
+    monkeypatch.delenv("BIGCN_BENCH_CACHE", raising=False)
+    _, fresh = bench.build_workload("C1")
+    monkeypatch.setenv("BIGCN_BENCH_CACHE", str(tmp_path))
+    _, first = bench.build_workload("C1")
+    assert len(list(tmp_path.iterdir())) == 1
+    _, second = bench.build_workload("C1")
+    for k in bench.WORKLOAD_ARRAYS:
+        for got in (first[k], second[k]):
+            assert got.dtype == fresh[k].dtype and np.array_equal(got, fresh[k]), k

@@ -3,8 +3,9 @@
 the configuration the benchmark times them: layer 1's back-propagation
 (Algorithm 1 with Eqs. bp-H, bp-W), both ablation layers of Sec. 6.3 (one
 operand of Eq. 11 kept real), the inductive mean and GraphSAGE-mean layers
-(Sec. 6.3, Table 3) and sub-row bucketing with buckets of 128 and 512
-features (Sec. 4.1).
+(Sec. 6.3, Table 3), sub-row bucketing with buckets of 128 and 512
+features (Sec. 4.1) and the layer over a weighted adjacency (Sec. 3's
+general a_ij).
 
 The oracle computes what it can one by one at this size:
   - products (Eq. 11 and its variants) on 2048 seeded sampled rows, from the
@@ -162,6 +163,42 @@ def test_c4_inductive_layer(cuda_device, c4dev, agg):
         check_layer_rows(H, rows, d["rowptr"], d["colidx"], z, np.abs(z),
                          "C4 sage layer H (sampled)", K, agg="sage", zeta_n=zn,
                          zabs_n=np.abs(zn))
+
+
+# ------------------------------------------------------ weighted adjacency ---
+def test_c4_weighted_layer(cuda_device, c4dev):
+    """Layer 1 over seeded symmetric edge weights (Sec. 3's general a_ij), as
+    the benchmark's --weighted line times it: the weighted degrees of every
+    node, the product's dots and H on the sampled rows."""
+    w, d, g, Y = c4dev
+    N, K, F = w.N, w.K, w.hidden
+    rows = sample(N, NSAMPLE, 64)
+    vals = inputs.edge_weights(d["rowptr"], d["colidx"], 4100 + w.index)
+    v_d = to_dev(vals)
+    ws = torch.empty(B.bigcn_weighted_layer_workspace_bytes(N, K, F), dtype=torch.uint8,
+                     device=cuda_device)
+    H = torch.empty((N, F), device=cuda_device)
+    B.bigcn_weighted_layer_forward(g["X"], g["s"], g["t"], g["W1"], g["rowptr"], g["colidx"],
+                                   v_d, ws, H)
+    dinv = torch.empty(N, device=cuda_device)
+    B.bigcn_weighted_dinv(g["rowptr"], v_d, dinv)
+    bits, alpha = B.pack_rows(g["X"], g["s"], g["t"])
+    wbits, beta = B.pack_weights(g["W1"])
+    _, dots = B.xnor_gemm(bits, alpha, wbits, beta, K, with_dots=True)
+    torch.cuda.synchronize()
+    assert B.device_timeouts() == 0
+    del v_d, ws
+    assert_close(dinv, 1.0 / np.sqrt(oracle.degree_weighted(d["rowptr"], vals)),
+                 "C4 weighted dinv", rtol=1e-6, atol=0.0)
+    SF = oracle.sign(Y[rows])
+    SB, _ = oracle.weight_binarize(d["W1"])
+    dh = dots.cpu().numpy()
+    assert np.array_equal(dh[rows], oracle.binary_dot(SF, SB))
+    z = oracle.zeta(dh, alpha.cpu().numpy(), beta.cpu().numpy())
+    ref = oracle.aggregate_weighted(d["rowptr"], d["colidx"], vals, z, rows=rows)
+    scale = oracle.aggregate_weighted(d["rowptr"], d["colidx"], vals, np.abs(z), rows=rows)
+    check_sum(H.cpu().numpy()[rows], ref, scale, "C4 weighted layer H (sampled)",
+              nterms=K + nterms_of(d["rowptr"], rows))
 
 
 # ------------------------------------------------------- sub-row bucketing ---
