@@ -179,8 +179,20 @@ constexpr int kSplitThreads = 512;
 constexpr int kSplitWarps = kSplitThreads / 32;
 constexpr size_t kSplitMaxSmem = 112 * 1024;
 
-size_t split_smem(int F, int K, int words, bool affine) {
-    return (size_t(F) + size_t(kSplitWarps)) * size_t(words | 1) * 8 +
+// Row pitch in 64-bit words. With one lane per output column (P = 1) a lane
+// reads its column two words at a time (16-byte loads): the rows are padded
+// to an even count of words with a zero word, and the pitch is = 2 mod 4
+// words, so that the eight columns of a quarter-warp fall on the eight
+// distinct 16-byte slots of a 128-byte line (conflict-free). Otherwise an
+// odd pitch keeps the 8-byte loads of neighbouring columns conflict-free.
+int split_pitch(int words, int P) {
+    if (P != 1) return words | 1;
+    const int even = (words + 1) & ~1;
+    return even % 4 == 2 ? even : even + 2;
+}
+
+size_t split_smem(int F, int K, int pitch, bool affine) {
+    return (size_t(F) + size_t(kSplitWarps)) * size_t(pitch) * 8 +
            (affine ? size_t(K) * 8 : 0);
 }
 
@@ -205,13 +217,13 @@ front_split_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
                    const uint64_t *__restrict__ wbits, const float *__restrict__ beta, int F,
                    int words, const int64_t *__restrict__ rowptr, float *__restrict__ Z,
                    int64_t ldz, uint16_t *__restrict__ D16, int64_t ldd16,
-                   float *__restrict__ rowscale, int P, bool f16) {
+                   float *__restrict__ rowscale, int P, int pitch, bool f16) {
     extern __shared__ __align__(16) unsigned char smem[];
     __shared__ float part[kSplitWarps];
     constexpr int R = kSplitWarps / G;       // rows per group
     constexpr int T = 32 * G;                // threads per row in the product
     constexpr Affine kA = kAffine ? Affine::kShared : Affine::kNone;
-    const int pitch = words | 1;
+    const int npairs = (words + 1) >> 1;     // P = 1: 16-byte pairs of words per row
     uint64_t *Ws = reinterpret_cast<uint64_t *>(smem);      // F x pitch packed columns
     uint64_t *As = Ws + size_t(F) * pitch;                   // R x pitch packed rows
     float2 *sST = reinterpret_cast<float2 *>(As + size_t(kSplitWarps) * pitch);
@@ -240,7 +252,9 @@ front_split_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
         uint32_t *a32 = reinterpret_cast<uint32_t *>(As + size_t(warp / G) * pitch);
         const float l1 = (row < N) ? pack_share<G, kFrontUnroll, kA>(X + row * ldx, K, nullptr,
                                                                      nullptr, sST, a32,
-                                                                     2 * words, warp % G)
+                                                                     P == 1 ? 4 * npairs
+                                                                            : 2 * words,
+                                                                     warp % G)
                                    : 0.0f;
         if (lane == 0) part[warp] = l1;
         if (!staged) {
@@ -259,6 +273,8 @@ front_split_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
                     if (q < n) Ws[(q / words) * pitch + (q % words)] = v[u];
                 }
             }
+            if (P == 1 && (words & 1))      // the zero word that completes the last pair
+                for (int c = tid; c < F; c += kSplitThreads) Ws[c * pitch + words] = 0ull;
             staged = true;
         }
         __syncthreads();
@@ -274,11 +290,24 @@ front_split_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
                           inv_sqrt_degree(__ldg(rowptr + row2 + 1) - __ldg(rowptr + row2));
             if (D16 != nullptr && tt == 0) rowscale[row2] = ai;
             const uint64_t *a = As + size_t(rr) * pitch;
+            const ulonglong2 *a2 = reinterpret_cast<const ulonglong2 *>(a);
             for (int j = 0; j < passes; ++j) {
                 const int c = tt / P + j * cstep;
                 int mism = 0;
-                if (c < F)
-                    for (int w = sub; w < words; w += P) mism += __popcll(a[w] ^ Ws[c * pitch + w]);
+                if (c < F) {
+                    if (P == 1) {    // a lane per column: two words per 16-byte load
+                        const ulonglong2 *w2 =
+                            reinterpret_cast<const ulonglong2 *>(Ws + size_t(c) * pitch);
+#pragma unroll 4
+                        for (int q = 0; q < npairs; ++q) {
+                            const ulonglong2 x = a2[q], y = w2[q];
+                            mism += __popcll(x.x ^ y.x) + __popcll(x.y ^ y.y);
+                        }
+                    } else {
+                        for (int w = sub; w < words; w += P)
+                            mism += __popcll(a[w] ^ Ws[c * pitch + w]);
+                    }
+                }
                 for (int o = 1; o < P; o <<= 1) mism += __shfl_xor_sync(kFullMask, mism, o);
                 if (sub != 0 || c >= Fw) continue;
                 if (D16 != nullptr)
@@ -293,9 +322,12 @@ front_split_kernel(const float *__restrict__ X, int64_t N, int K, int64_t ldx,
 }
 
 bool split_supported(int64_t N, int K, int F, const DeviceInfo &dev) {
-    return F >= 1 && F <= 128 && split_warps(N, K, dev) > 1 &&
-           split_smem(F, K, (K + 63) / 64, true) <= kSplitMaxSmem &&
-           split_smem(F, K, (K + 63) / 64, true) <= size_t(dev.max_smem_optin);
+    const int words = (K + 63) / 64;
+    const int pitch = split_pitch(words, 1) > split_pitch(words, 2) ? split_pitch(words, 1)
+                                                                     : split_pitch(words, 2);
+    const size_t smem = split_smem(F, K, pitch, true);
+    return F >= 1 && F <= 128 && split_warps(N, K, dev) > 1 && smem <= kSplitMaxSmem &&
+           smem <= size_t(dev.max_smem_optin);
 }
 
 void launch_split(const FrontArgs &a, const DeviceInfo &dev, cudaStream_t s, bool pdl) {
@@ -306,10 +338,11 @@ void launch_split(const FrontArgs &a, const DeviceInfo &dev, cudaStream_t s, boo
     if (P < 1) P = 1;
     if (P > 32) P = 32;
     const bool affine = a.scale != nullptr;
-    const size_t smem = split_smem(a.F, a.K, a.words, affine);
+    const int pitch = split_pitch(a.words, P);
+    const size_t smem = split_smem(a.F, a.K, pitch, affine);
     void (*kernel)(const float *, int64_t, int, int64_t, const float *, const float *,
                    const uint64_t *, const float *, int, int, const int64_t *, float *, int64_t,
-                   uint16_t *, int64_t, float *, int, bool);
+                   uint16_t *, int64_t, float *, int, int, bool);
     if (G == 2) kernel = affine ? front_split_kernel<2, true> : front_split_kernel<2, false>;
     else if (G == 4) kernel = affine ? front_split_kernel<4, true> : front_split_kernel<4, false>;
     else kernel = affine ? front_split_kernel<8, true> : front_split_kernel<8, false>;
@@ -324,7 +357,7 @@ void launch_split(const FrontArgs &a, const DeviceInfo &dev, cudaStream_t s, boo
     launch_kernel(kernel, dim3(unsigned(groups < resident ? groups : resident)),
                   dim3(kSplitThreads), smem, s, pdl, dim3(1, 1, 1), a.X, a.N, a.K, a.ldx, a.scale,
                   a.shift, a.wbits, a.beta, a.F, a.words, a.rowptr, a.Z, a.ldz, a.D16, a.ldd16,
-                  a.rowscale, P, a.dots_f16);
+                  a.rowscale, P, pitch, a.dots_f16);
 }
 
 }  // namespace
