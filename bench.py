@@ -48,6 +48,10 @@ import numpy as np  # noqa: E402
 METRIC = "Bi-GCN layer fwd nodes/s; XNOR-GEMM bit-ops/s; SpMM GB/s as % of GB300 peak"
 DEFAULT_WORKLOAD = "C4"
 L2_FLUSH_BYTES = 256 << 20
+L2_BYTES = 129 << 20        # the GB300's L2
+TOPS_STYLE_NOTE = ("2 N K F / t in 10^12 per second: each bit-MAC counted as a multiply and "
+                   "an add, as dense-GEMM TOPS are; the bit-ops/s figure counts one XNOR + "
+                   "count per (i, j, k)")
 # 32-bit population counts per clock per SM, as measured on GB300 by
 # tests/probes/instruction_rates.cu (profiles/xnor_gemm_instruction_rates.txt:
 # 151.8 T bit-ops/s over 152 SMs at 2070 MHz); the ALU ceiling of the POPC products.
@@ -152,6 +156,16 @@ def kernel_work(w, nnz, name):
         "L2.spmm": (csr + z2 + 4.0 * N * Fo, "bytes", "hbm"),
     }
     return table[name][:3]
+
+
+def workload_bytes(w, nnz):
+    """Bytes a 2-layer forward touches: the features, the CSR, both weight
+    matrices, both layers' factored products (16-bit dots and a row scale)
+    and the logits."""
+    pad16 = lambda f: (f + 15) // 16 * 16
+    return (4.0 * w.N * w.K + 8.0 * (w.N + 1) + 4.0 * nnz + 4.0 * w.K * w.hidden +
+            4.0 * w.hidden * w.out + w.N * (2.0 * pad16(w.hidden) + 4.0) +
+            w.N * (2.0 * pad16(w.out) + 4.0) + 4.0 * w.N * w.out)
 
 
 def kernel_bitops(w, name):
@@ -473,6 +487,23 @@ def run_gpu(args, rank, world, local_rank):
     max_ms, units = aggregate_over_ranks(total_ms, float(w.N) * args.steps, world)
     value = units / (max_ms * 1e-3)
 
+    # Warm L2: workloads whose inputs and intermediates fit L2 also timed with
+    # no flush between steps (a reported figure beside the flushed one).
+    warm = None
+    if workload_bytes(w, nnz) < L2_BYTES:
+        warm_ms = []
+        for _ in range(args.steps):
+            ea.record()
+            model.replay()
+            eb.record()
+            eb.synchronize()
+            warm_ms.append(ea.elapsed_time(eb))
+        wmax, wunits = aggregate_over_ranks(float(sum(warm_ms)), float(w.N) * args.steps, world)
+        warm = {"value": wunits / (wmax * 1e-3), "unit": "nodes/s",
+                "ms_per_step": wmax / args.steps,
+                "note": "the same graph replayed with no L2 flush between steps: the "
+                        "workload's bytes fit the 129 MB L2"}
+
     # Per-kernel durations (events between kernels, L2 flushed before each pass).
     per_kernel = [[] for _ in names]
     for i in range(min(args.steps, 300) + 3):
@@ -582,6 +613,10 @@ def run_gpu(args, rank, world, local_rank):
                    "parallelism": "replicas" if world > 1 else "single GPU"},
         "components": {
             "xnor_gemm_bitops_per_s": kernel_bitops(w, gemm1["name"]) / (gemm1["mean_us"] * 1e-6),
+            "xnor_gemm_tops_style": 2.0 * kernel_bitops(w, gemm1["name"]) /
+                                    (gemm1["mean_us"] * 1e-6) / 1e12,
+            "xnor_gemm_tops_style_note": TOPS_STYLE_NOTE,
+            "warm_l2": warm,
             "spmm_gbs": spmm_gbs, "spmm_pct_of_hbm_peak": 100.0 * spmm_gbs / hbm,
             "l1_aggregation_gather_gbs": gather_gbs,
             "l1_aggregation_gather_frac_of_hbm": gather_gbs / hbm,
@@ -718,6 +753,8 @@ def run_sweep(args, rank, world, local_rank):
             "per_kernel_us": {n: round(t, 3) for n, t in zip(SWEEP_KERNELS, mean_us)},
             "pack_rows_gbs": work["pack_rows"][0] / (mean_us[0] * 1e-6) / 1e9,
             "xnor_gemm_bitops_per_s": work["xnor_gemm"][0] / (mean_us[2] * 1e-6),
+            "xnor_gemm_tops_style": 2.0 * work["xnor_gemm"][0] / (mean_us[2] * 1e-6) / 1e12,
+            "xnor_gemm_tops_style_note": TOPS_STYLE_NOTE,
             "spmm_gbs": work["spmm"][0] / (mean_us[3] * 1e-6) / 1e9},
         "roofline": {"kernel": name, "bound": bound, "achieved": achieved, "peak": peak,
                      "unit": runit, "frac": achieved / peak,

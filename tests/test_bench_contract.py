@@ -132,3 +132,16 @@ def test_workload_cache_returns_the_same_arrays(monkeypatch, tmp_path):
     for k in bench.WORKLOAD_ARRAYS:
         for got in (first[k], second[k]):
             assert got.dtype == fresh[k].dtype and np.array_equal(got, fresh[k]), k
+
+
+def test_warm_l2_lines_are_for_workloads_that_fit_l2():
+    """The 2-layer line adds a warm-L2 figure only where the forward's bytes
+    fit the 129 MB L2: the Cora-, Citeseer- and PubMed-shaped workloads, not
+    the Reddit-shaped one."""
+    sys.path.insert(0, ROOT)
+    import bench
+    from paper_2010_07565_gb300 import inputs
+    nnz = {"C1": 10556, "C2": 9228, "C3": 88648, "C4": 114600000}
+    for name, fits in (("C1", True), ("C2", True), ("C3", True), ("C4", False)):
+        w = inputs.get_workload(name)
+        assert (bench.workload_bytes(w, nnz[name]) < bench.L2_BYTES) == fits, name
