@@ -6,7 +6,8 @@ either exchanges those rows (exchange_rows) or exchanges the packed signs and
 row scales of its rows (exchange_packed_rows) and computes the halo's product
 itself, with the halo degrees the plan carries; it then aggregates its block
 by the plain definition of Eq. 13 over its table. The blocks, put back
-together, must equal the oracle's whole-graph layer."""
+together, must equal the oracle's whole-graph layer -- also with more ranks
+than rows (empty blocks) and on a graph without edges (no halo)."""
 import os
 import socket
 
@@ -26,8 +27,26 @@ def free_port():
         return s.getsockname()[1]
 
 
-def case():
-    return inputs.layer_case(600, 150, 12, seed=77, mean_degree=6.0, hub_degree=250)
+# Graphs: a hub of degree 250 (most rows' halos cross ranks), three rows on
+# more ranks than rows (an empty block), and no edges at all (no halo).
+CASES = {"hub": dict(N=600, K=150, F=12, seed=77, mean_degree=6.0, hub_degree=250),
+         "tiny": dict(N=3, K=70, F=5, seed=5, mean_degree=2.0),
+         "edgeless": dict(N=50, K=40, F=7, seed=9, mean_degree=0.0)}
+
+
+def case(name="hub"):
+    return inputs.layer_case(**CASES[name])
+
+
+def test_partition_of_fewer_rows_than_ranks_leaves_empty_blocks():
+    rp = case("tiny")["rowptr"]
+    b = shard.partition_rows(rp, 5)
+    assert b.tolist()[0] == 0 and b.tolist()[-1] == 3 and np.all(np.diff(b) >= 0)
+    assert int((np.diff(b) == 0).sum()) == 2          # five ranks, three rows
+    empty = int(np.flatnonzero(np.diff(b) == 0)[0])
+    lrp, lci, halo, recv = shard.local_plan(rp, case("tiny")["colidx"], b, empty)
+    assert lrp.tolist() == [0] and lci.size == 0 and halo.size == 0 and recv.sum() == 0
+    assert shard.partition_rows(np.zeros(1, np.int64), 3).tolist() == [0, 0, 0, 0]
 
 
 def test_partition_balances_work_and_covers_every_row():
@@ -66,11 +85,11 @@ def unpack_signs(bits, K):
     return np.where(b == 1, 1, -1).astype(np.int8)
 
 
-def _rank_main(rank, world, port, result_path, packed=False):
+def _rank_main(rank, world, port, result_path, packed=False, name="hub"):
     os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
     dist.init_process_group("gloo", rank=rank, world_size=world)
     try:
-        c = case()
+        c = case(name)
         rp, ci = c["rowptr"], c["colidx"]
         b = shard.partition_rows(rp, world)
         plan = shard.build_plan(rp, ci, b, rank)
@@ -102,12 +121,15 @@ def _rank_main(rank, world, port, result_path, packed=False):
         dist.destroy_process_group()
 
 
-@pytest.mark.parametrize("world,packed", [(2, False), (3, False), (2, True), (3, True)])
-def test_sharded_layer_equals_the_whole_graph_layer(tmp_path, world, packed):
+@pytest.mark.parametrize("world,packed,name", [(2, False, "hub"), (3, False, "hub"),
+                                               (2, True, "hub"), (3, True, "hub"),
+                                               (4, False, "tiny"), (4, True, "tiny"),
+                                               (3, True, "edgeless")])
+def test_sharded_layer_equals_the_whole_graph_layer(tmp_path, world, packed, name):
     path = str(tmp_path / "H")
-    mp.start_processes(_rank_main, args=(world, free_port(), path, packed), nprocs=world,
+    mp.start_processes(_rank_main, args=(world, free_port(), path, packed, name), nprocs=world,
                        start_method="spawn")
-    c = case()
+    c = case(name)
     ref = oracle.layer_forward(c["X"], c["W"], c["rowptr"], c["colidx"], c["s"], c["t"])["H"]
     H = np.concatenate([np.load(f"{path}.{r}.npy") for r in range(world)])
     assert H.shape == ref.shape
