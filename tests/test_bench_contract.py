@@ -145,3 +145,24 @@ def test_warm_l2_lines_are_for_workloads_that_fit_l2():
     for name, fits in (("C1", True), ("C2", True), ("C3", True), ("C4", False)):
         w = inputs.get_workload(name)
         assert (bench.workload_bytes(w, nnz[name]) < bench.L2_BYTES) == fits, name
+
+
+def test_roofline_work_matches_the_profile_summaries():
+    """The algorithmic bytes bench.py divides by a kernel's time are the ones
+    the committed ncu summaries state for the same kernel and workload, and
+    the L2 gather ceiling is the measured entry for the next row size up."""
+    sys.path.insert(0, ROOT)
+    import bench
+    from paper_2010_07565_gb300 import inputs
+    cases = [("C4", 114600000, "L1.spmm+L2.pack_rows+L2.xnor_gemm",
+              "L1.spmm_L2.pack_rows_L2.xnor_gemm_C4.txt"),
+             ("C4", 114600000, "L2.spmm", "L2.spmm_C4.txt"),
+             ("C2", 9356, "L1.pack_rows+L1.xnor_gemm", "L1.pack_rows_L1.xnor_gemm_C2.txt")]
+    for name, nnz, kernel, fname in cases:
+        f = _profile_fields(os.path.join(ROOT, "profiles", fname))
+        stated = float(f["algorithmic_bytes_per_launch"].split(" ")[0])
+        work, unit, bound = bench.kernel_work(inputs.get_workload(name), nnz, kernel)
+        assert (unit, bound) == ("bytes", "hbm") and work == stated, (name, kernel, work, stated)
+    assert bench.l2_gather_peak(260) == (bench.L2_GATHER_GBS[512], 512)
+    assert bench.l2_gather_peak(100) == (bench.L2_GATHER_GBS[128], 128)
+    assert bench.l2_gather_peak(4096) == (bench.L2_GATHER_GBS[512], 512)
